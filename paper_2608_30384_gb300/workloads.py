@@ -1,0 +1,175 @@
+"""Seeded synthetic workloads (inputs only; none of the codec arithmetic).
+
+These generators stand in for the paper's datasets (glove D=100, bigann
+D=128, openai D=1536, wiki D=3072/384; Sec. 4.2, Table "Overview of
+Evaluated Datasets"), which are not available: Gaussian-mixture vectors with
+the same dimensionalities and scale of N, optionally unit-normalised (like
+the text-embedding sets) or with log-normal norms (non-normalised MIPS).
+
+Every random stream is a numpy PCG64 generator seeded by
+``SeedSequence(seed, spawn_key=(stream, chunk))`` so that any chunk of rows
+can be regenerated on its own.  Streams: 0 mixture centers, 1 component ids,
+2 noise, 3 norms (database rows); 5, 6, 7 the same for queries.
+
+Recipe of a row: component k ~ uniform{0..P-1}; y = center_k + sigma * eps,
+eps ~ N(0, I); then y / ||y|| when ``normalize``; rho * y / ||y|| with
+rho ~ LogNormal(0, lognormal_sigma) when ``lognormal_sigma`` is set.  The
+IVF assignment of a row is its generating component.  Centroids are either
+the true centers or the member means of the generated rows.
+"""
+
+from __future__ import annotations
+
+import math
+from dataclasses import dataclass, replace
+
+import numpy as np
+
+CHUNK = 1 << 16  # rows per independently seeded chunk
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    N: int
+    D: int
+    P: int                    # mixture components = IVF partitions
+    sigma: float
+    normalize: bool
+    lognormal_sigma: float | None
+    centroids: str            # 'true' or 'mean'
+    nq: int
+    bits: int
+    rescore_bits: int
+    nprobe: int
+    k: int                    # stage-1 top-K
+    k_final: int              # final top-k (== k without rescoring)
+    seed: int = 0
+    description: str = ""
+
+    def scaled(self, **kw) -> "Workload":
+        """A copy with some fields replaced (smaller parity cases)."""
+        return replace(self, **kw)
+
+
+WORKLOADS = {
+    "C1": Workload("C1", 10_000, 128, 16, 0.3, False, None, "true", 100, 4, 0, 4, 10, 10,
+                   description="N=1e4 d=128 16-Gaussian mixture sigma=0.3, IVF16 true centers, "
+                               "4-bit codes, 100 queries, nprobe=4, top-10"),
+    "C2": Workload("C2", 1_000_000, 96, 1024, 0.5, False, None, "true", 10_000, 2, 4, 32, 100, 10,
+                   description="N=1e6 d=96 1024-Gaussian mixture sigma=0.5, IVF1024 true centers, "
+                               "2-bit scoring + 4-bit rescoring, 1e4 queries, nprobe=32, "
+                               "top-100 -> top-10"),
+    "C3": Workload("C3", 1_000_000, 768, 2048, 0.5, True, None, "mean", 10_000, 1, 4, 64, 100, 10,
+                   description="N=1e6 d=768 unit-normalised 2048-Gaussian mixture, IVF2048 "
+                               "member means, 1-bit scoring + 4-bit rescoring, 1e4 queries, "
+                               "nprobe=64, top-100 -> top-10"),
+    "C4": Workload("C4", 10_000_000, 128, 8192, 0.5, False, 0.5, "mean", 100_000, 4, 0, 64, 10, 10,
+                   description="N=1e7 d=128 8192-Gaussian mixture with log-normal(0, 0.5) norms, "
+                               "IVF8192 member means, 4-bit codes, 1e5 queries, nprobe=64, top-10"),
+    "C5": Workload("C5", 5_000_000, 1536, 4096, 0.5, True, None, "mean", 50_000, 2, 4, 128, 200, 10,
+                   description="N=5e6 d=1536 unit-normalised 4096-Gaussian mixture, IVF4096 member "
+                               "means, 2-bit scoring + 4-bit rescoring, 5e4 queries, nprobe=128, "
+                               "top-200 -> top-10"),
+}
+
+
+def _rng(seed: int, stream: int, chunk: int = 0) -> np.random.Generator:
+    return np.random.Generator(np.random.PCG64(np.random.SeedSequence(seed, spawn_key=(stream, chunk))))
+
+
+def centers(w: Workload) -> np.ndarray:
+    """Mixture centers, P x D float32, ~ N(0, I)."""
+    return _rng(w.seed, 0).standard_normal((w.P, w.D), dtype=np.float32)
+
+
+def _rows(w: Workload, ctr: np.ndarray, n: int, base: int, chunk: int):
+    comp = _rng(w.seed, base + 1, chunk).integers(0, w.P, size=n, dtype=np.int64)
+    y = ctr[comp] + np.float32(w.sigma) * _rng(w.seed, base + 2, chunk).standard_normal(
+        (n, w.D), dtype=np.float32)
+    if w.normalize or w.lognormal_sigma is not None:
+        nrm = np.sqrt(np.einsum("ij,ij->i", y.astype(np.float64), y.astype(np.float64)))
+        nrm = np.where(nrm > 0, nrm, 1.0)
+        scale = 1.0 / nrm
+        if w.lognormal_sigma is not None:
+            rho = _rng(w.seed, base + 3, chunk).lognormal(0.0, w.lognormal_sigma, size=n)
+            scale = scale * rho
+        y = (y.astype(np.float64) * scale[:, None]).astype(np.float32)
+    return y, comp.astype(np.int32)
+
+
+def chunk_rows(w: Workload, chunk: int, ctr: np.ndarray | None = None):
+    """Rows [chunk*CHUNK, min(N, (chunk+1)*CHUNK)) and their components."""
+    ctr = centers(w) if ctr is None else ctr
+    lo = chunk * CHUNK
+    n = max(0, min(w.N, lo + CHUNK) - lo)
+    return _rows(w, ctr, n, 0, chunk)
+
+
+def n_chunks(w: Workload) -> int:
+    return math.ceil(w.N / CHUNK)
+
+
+def rows(w: Workload, ids, ctr: np.ndarray | None = None):
+    """Rows with the given ids (regenerating only the chunks they live in)."""
+    ids = np.asarray(ids, dtype=np.int64)
+    ctr = centers(w) if ctr is None else ctr
+    X = np.zeros((ids.size, w.D), dtype=np.float32)
+    A = np.zeros(ids.size, dtype=np.int32)
+    for c in np.unique(ids // CHUNK):
+        sel = np.nonzero(ids // CHUNK == c)[0]
+        Xc, Ac = chunk_rows(w, int(c), ctr)
+        X[sel] = Xc[ids[sel] - c * CHUNK]
+        A[sel] = Ac[ids[sel] - c * CHUNK]
+    return X, A
+
+
+def database(w: Workload):
+    """All N rows (float32) and their components (int32)."""
+    ctr = centers(w)
+    X = np.empty((w.N, w.D), dtype=np.float32)
+    A = np.empty(w.N, dtype=np.int32)
+    for c in range(n_chunks(w)):
+        Xc, Ac = chunk_rows(w, c, ctr)
+        X[c * CHUNK:c * CHUNK + len(Ac)] = Xc
+        A[c * CHUNK:c * CHUNK + len(Ac)] = Ac
+    return X, A
+
+
+def member_means(w: Workload, X: np.ndarray, A: np.ndarray, ctr: np.ndarray) -> np.ndarray:
+    """Per-component mean of the rows (float32); empty components keep the center."""
+    sums = np.zeros((w.P, w.D))
+    cnt = np.bincount(A, minlength=w.P)
+    for lo in range(0, X.shape[0], CHUNK):
+        a = A[lo:lo + CHUNK]
+        o = np.argsort(a, kind="stable")
+        a_sorted = a[o]
+        starts = np.r_[0, np.nonzero(np.diff(a_sorted))[0] + 1]
+        part = np.add.reduceat(X[lo:lo + CHUNK][o].astype(np.float64), starts, axis=0)
+        sums[a_sorted[starts]] += part
+    out = ctr.astype(np.float64).copy()
+    nz = cnt > 0
+    out[nz] = sums[nz] / cnt[nz, None]
+    return out.astype(np.float32)
+
+
+def ivf_centroids(w: Workload, X: np.ndarray | None = None, A: np.ndarray | None = None) -> np.ndarray:
+    """IVF centroids: the true centers, or the member means of the data."""
+    ctr = centers(w)
+    if w.centroids == "true":
+        return ctr
+    if X is None:
+        X, A = database(w)
+    return member_means(w, X, A, ctr)
+
+
+def queries(w: Workload, nq: int | None = None) -> np.ndarray:
+    """The first ``nq`` (default all) queries, drawn from the same mixture."""
+    nq = w.nq if nq is None else nq
+    ctr = centers(w)
+    out = np.empty((nq, w.D), dtype=np.float32)
+    for c in range(math.ceil(nq / CHUNK)):
+        lo = c * CHUNK
+        n = min(nq, lo + CHUNK) - lo
+        out[lo:lo + n] = _rows(w, ctr, n, 4, c)[0]
+    return out
