@@ -1,0 +1,28 @@
+// launch.h -- host launchers of the librslm kernels.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "rslm_internal.h"
+
+namespace rslm {
+
+cudaError_t launch_rotate_rows(const RotSpec& rot, const float* in, int64_t n, float* out, int Dp,
+                               cudaStream_t s);
+cudaError_t launch_encode(const rslm_index* ix, const float* x, int64_t row_begin, int64_t rows,
+                          cudaStream_t s);
+cudaError_t launch_export_import(const rslm_index* ix, int which, int64_t row_begin, int64_t rows,
+                                 uint8_t* codes, uint16_t* lscale, uint16_t* gscale, bool import,
+                                 cudaStream_t s);
+// Top-kk of every row of S [rows * n] by (value desc, column asc).
+cudaError_t launch_select_topn(const float* S, int64_t rows, int n, int kk, int32_t* out_idx,
+                               float* out_val, cudaStream_t s);
+cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, const int32_t* probes,
+                        const float* cs, int nprobe, int k, int out_k, int64_t* out_ids,
+                        float* out_scores, cudaStream_t s);
+cudaError_t launch_rescore(const rslm_index* ix, const float* qrot2, int64_t nq,
+                           const int64_t* cand_ids, const float* cand_scores, int k, int k_final,
+                           int64_t* out_ids, float* out_scores, cudaStream_t s);
+
+}  // namespace rslm

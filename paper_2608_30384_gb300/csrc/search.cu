@@ -1,0 +1,484 @@
+// search.cu -- probe selection, code scan with per-query top-k, rescoring.
+//
+// Scan (Sec. 5.5.1 step 3 with the scores of Sec. 3.5): one CTA per query.
+// The query, already rotated (Sec. 5.4), becomes a lookup table
+// T[group][code] = <q_group, codeword_code> in shared memory, so that the
+// dot product <R q, uhat> of a row is the sum of one table entry per 4-bit
+// code.  Warps stream 128-row tiles of the probed partitions; every lane
+// owns 4 rows of a tile and reads 16-byte chunks that are contiguous across
+// the warp (tile-interleaved layout).  The epilogue applies the scales,
+// s = G (cs + L dot) (Sec. 3.5.2), and feeds a per-warp top-k list; the
+// lists are merged by a block sort at the end.
+#include <cuda_runtime.h>
+#include <math_constants.h>
+
+#include <climits>
+
+#include "device_common.cuh"
+#include "launch.h"
+
+namespace rslm {
+namespace {
+
+// ------------------------------------------------------------ probe select
+__global__ void select_topn_kernel(const float* __restrict__ S, int n, int kk,
+                                   int32_t* __restrict__ out_idx, float* __restrict__ out_val) {
+  extern __shared__ uint32_t xsm[];
+  __shared__ uint32_t hist[256];
+  __shared__ int scratch[32];
+  __shared__ uint32_t sh_prefix, sh_rem, sh_gt;
+  int p2 = 1;
+  while (p2 < kk) p2 <<= 1;
+  uint32_t* skey = xsm;
+  int32_t* sidx = reinterpret_cast<int32_t*>(xsm + p2);
+  const float* s = S + int64_t(blockIdx.x) * n;
+  const int tid = threadIdx.x;
+
+  // Radix select of the kk-th largest order key, 8 bits at a time.
+  uint32_t prefix = 0, mask = 0, rem = uint32_t(kk);
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (int i = tid; i < n; i += blockDim.x) {
+      const uint32_t key = float_order_key(s[i]);
+      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      uint32_t cum = 0;
+      int b = 255;
+      for (; b > 0; --b) {
+        if (cum + hist[b] >= rem) break;
+        cum += hist[b];
+      }
+      sh_rem = rem - cum;
+      sh_prefix = prefix | (uint32_t(b) << shift);
+    }
+    __syncthreads();
+    rem = sh_rem;
+    prefix = sh_prefix;
+    mask |= 255u << shift;
+    __syncthreads();
+  }
+  // prefix is now the kk-th largest key; rem of its copies are taken.
+  const uint32_t T = prefix;
+  const int ngt = kk - int(rem);
+  if (tid == 0) sh_gt = 0;
+  __syncthreads();
+  for (int i = tid; i < n; i += blockDim.x) {
+    const uint32_t key = float_order_key(s[i]);
+    if (key > T) {
+      const uint32_t slot = atomicAdd(&sh_gt, 1u);
+      skey[slot] = key;
+      sidx[slot] = i;
+    }
+  }
+  // Copies of T in column order (lower column first).
+  int taken = 0;
+  for (int base = 0; base < n && taken < int(rem); base += blockDim.x) {
+    const int i = base + tid;
+    const int e = (i < n && float_order_key(s[i]) == T) ? 1 : 0;
+    int tot;
+    const int ex = block_exclusive_scan(e, scratch, &tot);
+    if (e && taken + ex < int(rem)) {
+      skey[ngt + taken + ex] = T;
+      sidx[ngt + taken + ex] = i;
+    }
+    taken += tot;
+  }
+  for (int i = kk + tid; i < p2; i += blockDim.x) {
+    skey[i] = 0;
+    sidx[i] = INT_MAX;
+  }
+  block_bitonic_sort(skey, sidx, p2);
+  for (int i = tid; i < kk; i += blockDim.x) {
+    out_idx[int64_t(blockIdx.x) * kk + i] = sidx[i];
+    out_val[int64_t(blockIdx.x) * kk + i] = float_from_order_key(skey[i]);
+  }
+}
+
+// ------------------------------------------------------------------- scan
+struct ScanArgs {
+  const float* qrot;
+  int Dp;
+  const int32_t* probes;
+  const float* cs;
+  int nprobe;
+  int k;
+  int out_k;
+  const uint8_t* codes;
+  const uint32_t* scales;
+  const int64_t* ids;
+  const int64_t* part_off;
+  const int32_t* part_n;
+  int nlist;
+  int stride;
+  int lut_groups;  // 2 * stride: one table row per nibble position of a row
+  int ngroups;
+  int g;
+  float cb[64];
+  int64_t* out_ids;
+  float* out_scores;
+  int* err;
+  int lut_region;  // bytes of the table / merge region
+};
+
+template <int CH>
+__device__ __forceinline__ void load_chunk(const uint8_t* p, uint32_t (&w)[CH / 4]) {
+  if constexpr (CH == 16) {
+    const uint4 v = __ldg(reinterpret_cast<const uint4*>(p));
+    w[0] = v.x;
+    w[1] = v.y;
+    w[2] = v.z;
+    w[3] = v.w;
+  } else if constexpr (CH == 8) {
+    const uint2 v = __ldg(reinterpret_cast<const uint2*>(p));
+    w[0] = v.x;
+    w[1] = v.y;
+  } else {
+    w[0] = __ldg(reinterpret_cast<const uint32_t*>(p));
+  }
+}
+
+// Insert (s, p) into a warp's list sorted by (score desc, position asc).
+// Every lane calls with the same (s, p).
+__device__ __forceinline__ void warp_insert(float* sc, int* ps, int& cnt, int k, float s, int p,
+                                            int lane) {
+  int at = 0;
+  for (int base = 0; base < cnt; base += 32) {
+    const int i = base + lane;
+    bool b = false;
+    if (i < cnt) {
+      const float v = sc[i];
+      b = v > s || (v == s && ps[i] < p);
+    }
+    at += __popc(__ballot_sync(kFull, b));
+  }
+  if (at >= k) return;
+  const int newcnt = cnt + 1 < k ? cnt + 1 : k;
+  for (int end = newcnt - 1; end > at; end -= 32) {
+    const int i = end - lane;
+    const bool act = i > at;
+    float v = 0.0f;
+    int pp = 0;
+    if (act) {
+      v = sc[i - 1];
+      pp = ps[i - 1];
+    }
+    __syncwarp();
+    if (act) {
+      sc[i] = v;
+      ps[i] = pp;
+    }
+    __syncwarp();
+  }
+  if (lane == 0) {
+    sc[at] = s;
+    ps[at] = p;
+  }
+  __syncwarp();
+  cnt = newcnt;
+}
+
+template <int CH>
+__global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanArgs a) {
+  extern __shared__ __align__(16) uint8_t ssm[];
+  __shared__ int scratch[32];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, W = blockDim.x >> 5;
+  const int64_t q = blockIdx.x;
+  float* lut = reinterpret_cast<float*>(ssm);
+  float* wsc = reinterpret_cast<float*>(ssm + a.lut_region);
+  int* wps = reinterpret_cast<int*>(wsc + W * a.k);
+  int* wcnt = wps + W * a.k;
+  int* pid = wcnt + W;
+  int* tpref = pid + a.nprobe;
+
+  // Query lookup table: T[group][code] = <q_group, C[code]>.
+  const float* qr = a.qrot + q * a.Dp;
+  for (int e = tid; e < a.lut_groups * 16; e += blockDim.x) {
+    const int grp = e >> 4, code = e & 15;
+    float v = 0.0f;
+    if (grp < a.ngroups)
+      for (int j = 0; j < a.g; ++j) v = fmaf(qr[grp * a.g + j], a.cb[code * a.g + j], v);
+    lut[e] = v;
+  }
+  // Probe list -> tiles to visit.
+  int run = 0;
+  for (int base = 0; base < a.nprobe; base += blockDim.x) {
+    const int j = base + tid;
+    int nt = 0;
+    if (j < a.nprobe) {
+      const int p = a.probes[q * a.nprobe + j];
+      if (p < 0 || p >= a.nlist) {
+        set_device_error(a.err, kErrBadProbe);
+        pid[j] = -1;
+      } else {
+        pid[j] = p;
+        nt = (a.part_n[p] + kTile - 1) / kTile;
+      }
+    }
+    int tot;
+    const int ex = block_exclusive_scan(nt, scratch, &tot);
+    if (j < a.nprobe) tpref[j] = run + ex;
+    run += tot;
+  }
+  if (tid == 0) tpref[a.nprobe] = run;
+  if (tid < W) wcnt[tid] = 0;
+  __syncthreads();
+
+  const int total = tpref[a.nprobe];
+  int cnt = 0;
+  float thr = -CUDART_INF_F;
+  int thr_pos = INT_MAX;
+  float* msc = wsc + warp * a.k;
+  int* mps = wps + warp * a.k;
+  const int nch = a.stride / CH;
+  int j = 0;
+  for (int it = warp; it < total; it += W) {
+    while (tpref[j + 1] <= it) ++j;
+    const int p = pid[j];
+    const int t = it - tpref[j];
+    const int64_t slot0 = a.part_off[p] + int64_t(t) * kTile;
+    const int nvalid = min(kTile, a.part_n[p] - t * kTile);
+    const float csj = a.cs[q * a.nprobe + j];
+    const uint8_t* tp = a.codes + slot0 * a.stride;
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    for (int c = 0; c < nch; ++c) {
+      const float* lc = lut + c * (2 * CH) * 16;
+      uint32_t w[4][CH / 4];
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+        load_chunk<CH>(tp + (size_t(c) * kTile + r * 32 + lane) * CH, w[r]);
+#pragma unroll
+      for (int r = 0; r < 4; ++r)
+#pragma unroll
+        for (int v = 0; v < CH / 4; ++v)
+#pragma unroll
+          for (int n = 0; n < 8; ++n) acc[r] += lc[(v * 8 + n) * 16 + ((w[r][v] >> (4 * n)) & 15u)];
+    }
+#pragma unroll
+    for (int r = 0; r < 4; ++r) {
+      const int row = r * 32 + lane;
+      const bool valid = row < nvalid;
+      const int pos = int(slot0) + row;
+      float s = -CUDART_INF_F;
+      if (valid) {
+        const uint32_t sc = __ldg(a.scales + slot0 + row);
+        s = ue4m12_to_f32(sc >> 16) * fmaf(ue7m9_to_f32(sc & 0xffffu), acc[r], csj);
+      }
+      const bool cand = valid && (cnt < a.k || s > thr || (s == thr && pos < thr_pos));
+      unsigned m = __ballot_sync(kFull, cand);
+      while (m) {
+        const int src = __ffs(m) - 1;
+        m &= m - 1;
+        const float s2 = __shfl_sync(kFull, s, src);
+        const int p2 = __shfl_sync(kFull, pos, src);
+        if (cnt < a.k || s2 > thr || (s2 == thr && p2 < thr_pos)) {
+          warp_insert(msc, mps, cnt, a.k, s2, p2, lane);
+          if (cnt == a.k) {
+            thr = msc[a.k - 1];
+            thr_pos = mps[a.k - 1];
+          }
+        }
+      }
+    }
+  }
+  if (lane == 0) wcnt[warp] = cnt;
+  __syncthreads();
+
+  // Merge the warp lists: block sort by (score desc, row id asc).
+  const int tot = W * a.k;
+  int np2 = 1;
+  while (np2 < tot) np2 <<= 1;
+  float* mkey = lut;
+  int64_t* mid = reinterpret_cast<int64_t*>(ssm + ((size_t(np2) * 4 + 15) & ~size_t(15)));
+  for (int e = tid; e < np2; e += blockDim.x) {
+    float kv = -CUDART_INF_F;
+    int64_t iv = LLONG_MAX;
+    if (e < tot) {
+      const int w = e / a.k, i = e - w * a.k;
+      if (i < wcnt[w]) {
+        kv = wsc[w * a.k + i];
+        iv = a.ids[wps[w * a.k + i]];
+      }
+    }
+    mkey[e] = kv;
+    mid[e] = iv;
+  }
+  block_bitonic_sort(mkey, mid, np2);
+  for (int e = tid; e < a.out_k; e += blockDim.x) {
+    const int64_t id = mid[e];
+    const bool ok = id != LLONG_MAX;
+    a.out_ids[q * a.out_k + e] = ok ? id : -1;
+    a.out_scores[q * a.out_k + e] = ok ? mkey[e] : -CUDART_INF_F;
+  }
+}
+
+// ---------------------------------------------------------------- rescore
+struct RescoreArgs {
+  const float* qrot2;
+  int Dp2;
+  const int64_t* cand_ids;
+  const float* cand_scores;
+  int k;
+  int kf;
+  const int32_t* slot_of_row;
+  int64_t n_rows;
+  const uint8_t* codes2;
+  const uint32_t* scales2;
+  int stride2;
+  int code_bytes2;
+  float lv[16];
+  int64_t* out_ids;
+  float* out_scores;
+  int* err;
+};
+
+__global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ RescoreArgs a) {
+  extern __shared__ __align__(16) uint8_t rsm2[];
+  __shared__ float lv[16];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, W = blockDim.x >> 5;
+  const int64_t q = blockIdx.x;
+  int np2 = 1;
+  while (np2 < a.k) np2 <<= 1;
+  const int qlen = 2 * a.stride2;
+  float* q2 = reinterpret_cast<float*>(rsm2);
+  float* key = q2 + qlen;
+  int64_t* idv = reinterpret_cast<int64_t*>(rsm2 + ((size_t(qlen + np2) * 4 + 15) & ~size_t(15)));
+  if (tid < 16) lv[tid] = a.lv[tid];
+  for (int d = tid; d < qlen; d += blockDim.x) q2[d] = d < a.Dp2 ? a.qrot2[q * a.Dp2 + d] : 0.0f;
+  __syncthreads();
+  for (int j = warp; j < np2; j += W) {
+    float s2 = -CUDART_INF_F;
+    int64_t id = LLONG_MAX;
+    if (j < a.k) {
+      const int64_t cid = a.cand_ids[q * a.k + j];
+      if (cid >= a.n_rows || cid < -1) set_device_error(a.err, kErrBadCandidate);
+      if (cid >= 0 && cid < a.n_rows) {
+        const int64_t slot = a.slot_of_row[cid];
+        const uint8_t* row = a.codes2 + slot * a.stride2;
+        float acc = 0.0f;
+        for (int b = lane * 4; b < a.code_bytes2; b += 128) {
+          const uint32_t w = __ldg(reinterpret_cast<const uint32_t*>(row + b));
+#pragma unroll
+          for (int n = 0; n < 8; ++n) acc = fmaf(lv[(w >> (4 * n)) & 15u], q2[2 * b + n], acc);
+        }
+        acc = warp_sum(acc);
+        const uint32_t sc = __ldg(a.scales2 + slot);
+        const float s1 = a.cand_scores[q * a.k + j];
+        s2 = ue4m12_to_f32(sc >> 16) * fmaf(ue7m9_to_f32(sc & 0xffffu), acc, s1);
+        id = cid;
+      }
+    }
+    if (lane == 0) {
+      key[j] = s2;
+      idv[j] = id;
+    }
+  }
+  block_bitonic_sort(key, idv, np2);
+  for (int e = tid; e < a.kf; e += blockDim.x) {
+    const bool ok = idv[e] != LLONG_MAX;
+    a.out_ids[q * a.kf + e] = ok ? idv[e] : -1;
+    a.out_scores[q * a.kf + e] = ok ? key[e] : -CUDART_INF_F;
+  }
+}
+
+template <int CH>
+cudaError_t launch_scan_ch(const ScanArgs& a, int64_t nq, size_t smem, cudaStream_t s) {
+  cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       int(smem));
+  if (e != cudaSuccess) return e;
+  scan_kernel<CH><<<unsigned(nq), 256, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_select_topn(const float* S, int64_t rows, int n, int kk, int32_t* out_idx,
+                               float* out_val, cudaStream_t s) {
+  if (rows == 0) return cudaSuccess;
+  int p2 = 1;
+  while (p2 < kk) p2 <<= 1;
+  const size_t smem = size_t(p2) * 8;
+  cudaError_t e = cudaFuncSetAttribute(select_topn_kernel,
+                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  select_topn_kernel<<<unsigned(rows), 256, smem, s>>>(S, n, kk, out_idx, out_val);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, const int32_t* probes,
+                        const float* cs, int nprobe, int k, int out_k, int64_t* out_ids,
+                        float* out_scores, cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  ScanArgs a;
+  a.qrot = qrot;
+  a.Dp = ix->cs1.Dp;
+  a.probes = probes;
+  a.cs = cs;
+  a.nprobe = nprobe;
+  a.k = k;
+  a.out_k = out_k;
+  a.codes = ix->codes1;
+  a.scales = ix->scales1;
+  a.ids = ix->ids;
+  a.part_off = ix->part_off;
+  a.part_n = ix->part_n;
+  a.nlist = ix->nlist;
+  a.stride = ix->cs1.stride;
+  a.lut_groups = 2 * ix->cs1.stride;
+  a.ngroups = ix->cs1.ngroups;
+  a.g = ix->cs1.g;
+  for (int i = 0; i < 64; ++i) a.cb[i] = ix->cs1.cbf[i];
+  a.out_ids = out_ids;
+  a.out_scores = out_scores;
+  a.err = ix->d_err;
+  const int W = 8;
+  int np2 = 1;
+  while (np2 < W * k) np2 <<= 1;
+  const size_t lut_bytes = size_t(a.lut_groups) * 16 * 4;
+  const size_t merge_bytes = ((size_t(np2) * 4 + 15) & ~size_t(15)) + size_t(np2) * 8;
+  size_t region = lut_bytes > merge_bytes ? lut_bytes : merge_bytes;
+  region = (region + 15) & ~size_t(15);
+  a.lut_region = int(region);
+  const size_t smem = region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
+  switch (ix->cs1.chunk) {
+    case 16: return launch_scan_ch<16>(a, nq, smem, s);
+    case 8: return launch_scan_ch<8>(a, nq, smem, s);
+    default: return launch_scan_ch<4>(a, nq, smem, s);
+  }
+}
+
+cudaError_t launch_rescore(const rslm_index* ix, const float* qrot2, int64_t nq,
+                           const int64_t* cand_ids, const float* cand_scores, int k, int k_final,
+                           int64_t* out_ids, float* out_scores, cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  RescoreArgs a;
+  a.qrot2 = qrot2;
+  a.Dp2 = ix->cs2.Dp;
+  a.cand_ids = cand_ids;
+  a.cand_scores = cand_scores;
+  a.k = k;
+  a.kf = k_final;
+  a.slot_of_row = ix->slot_of_row;
+  a.n_rows = ix->n_rows;
+  a.codes2 = ix->codes2;
+  a.scales2 = ix->scales2;
+  a.stride2 = ix->cs2.stride;
+  a.code_bytes2 = ix->cs2.code_bytes;
+  for (int i = 0; i < 16; ++i) a.lv[i] = ix->cs2.cbf[i];
+  a.out_ids = out_ids;
+  a.out_scores = out_scores;
+  a.err = ix->d_err;
+  int np2 = 1;
+  while (np2 < k) np2 <<= 1;
+  const size_t smem = ((size_t(2 * a.stride2 + np2) * 4 + 15) & ~size_t(15)) + size_t(np2) * 8;
+  cudaError_t e = cudaFuncSetAttribute(rescore_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                       int(smem));
+  if (e != cudaSuccess) return e;
+  rescore_kernel<<<unsigned(nq), 256, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+}  // namespace rslm

@@ -1,0 +1,328 @@
+"""GPU path vs the float64 oracle, element by element, through the C ABI.
+
+Tolerances (the contract): codes bit-exact except groups decided within 1e-5
+of a decision boundary (at most 1e-4 of all groups); scale codes exact
+except where the exact value lies at a rounding tie; scores within 1e-4
+relative (floor 0.01 ||q|| max||x||, see lib_util.score_tol); top-k lists
+equal up to swaps of near-equal scores (lib_util.check_topk).
+"""
+
+import numpy as np
+import pytest
+
+from oracle import codec, constants as K, search
+from oracle.rotation import rotation_matrix, rotation_mode
+from paper_2608_30384_gb300 import workloads as W
+from tests.gpu_cases import Case, ue_near_tie
+from tests.lib_util import check_topk, ensure_library, score_tol
+
+torch = pytest.importorskip("torch")
+pytestmark = pytest.mark.gpu
+
+Wl = W.Workload
+CASES = {
+    # the small configuration, in full
+    "C1": W.WORKLOADS["C1"],
+    # reduced copies of the larger configurations: several tiles per partition and a ragged tail
+    "C2s": Wl("C2s", 30_000, 96, 64, 0.5, False, None, "true", 40, 2, 4, 8, 100, 10, seed=1),
+    "C3s": Wl("C3s", 12_000, 768, 24, 0.5, True, None, "mean", 12, 1, 4, 6, 100, 10, seed=2),
+    "C4s": Wl("C4s", 40_000, 128, 64, 0.5, False, 0.5, "mean", 40, 4, 0, 16, 10, 10, seed=3),
+    "C5s": Wl("C5s", 6_000, 1536, 12, 0.5, True, None, "mean", 6, 2, 4, 4, 200, 10, seed=4),
+    # zero padding of the last group (D not a multiple of g), odd group counts
+    "pad1": Wl("pad1", 5_000, 100, 8, 0.5, False, None, "true", 20, 1, 4, 3, 50, 5, seed=5),
+    "pad2": Wl("pad2", 5_000, 99, 8, 0.5, False, None, "true", 20, 2, 0, 3, 20, 20, seed=6),
+    # tiny dimensions: block size shrinks to 1, 2, 4 (Sec. 3.1.1)
+    "D1": Wl("D1", 2_000, 1, 4, 0.5, False, None, "true", 20, 4, 0, 2, 8, 8, seed=7),
+    "D5": Wl("D5", 2_000, 5, 4, 0.5, False, None, "true", 20, 2, 4, 2, 16, 4, seed=8),
+    "D300": Wl("D300", 4_000, 300, 8, 0.5, True, None, "mean", 10, 4, 0, 3, 30, 30, seed=9),
+}
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    ensure_library()
+
+
+@pytest.fixture(scope="module", params=list(CASES))
+def case(request):
+    return Case(CASES[request.param])
+
+
+@pytest.fixture(scope="module")
+def local_case():
+    return Case(Wl("loc", 6_000, 64, 8, 0.5, False, 0.5, "mean", 20, 4, 4, 3, 40, 10, seed=10),
+                global_scale=False)
+
+
+# ------------------------------------------------------------------ rotation
+@pytest.mark.parametrize("D", [1, 2, 3, 5, 64, 96, 100, 127, 128, 129, 200, 256, 300, 768, 1536, 2049])
+@pytest.mark.parametrize("bits", [1, 4])
+def test_query_rotation(D, bits):
+    from paper_2608_30384_gb300 import Index
+    C = torch.zeros((1, D), device="cuda")
+    ix = Index(C, bits)
+    q = np.random.default_rng(D).standard_normal((37, D)).astype(np.float32)
+    out = ix.rotate(torch.from_numpy(q).cuda()).cpu().numpy()
+    R = rotation_matrix(D, rotation_mode(bits, D))
+    ref = q.astype(np.float64) @ R.T
+    g = K.group_size(bits)
+    Dp = g * -(-D // g)
+    assert out.shape == (37, Dp)
+    assert np.all(out[:, D:] == 0)
+    err = np.abs(out[:, :D] - ref).max(1) / np.linalg.norm(q, axis=1)
+    assert err.max() < 2e-6
+
+
+# -------------------------------------------------------------------- encode
+def _check_stage(gpu_codes, gpu_L, gpu_G, enc, X, A, bits, global_scale, name):
+    ng = enc.codes.shape[1]
+    got = codec.unpack_nibbles(gpu_codes, ng)
+    mism = got != enc.codes
+    near = codec.near_threshold(enc.u, bits, 1e-5)
+    assert np.all(near[mism]), f"{name}: code mismatch away from a decision boundary"
+    assert mism.sum() <= max(1, 1e-4 * mism.size), f"{name}: {mism.sum()} mismatched codes"
+    ok = ~mism.any(1)
+    for gv, ov, ex, fmt in ((gpu_L, enc.L_u16, enc.L_exact, K.UE7M9), (gpu_G, enc.G_u16, enc.G_exact, K.UE4M12)):
+        bad = ok & (gv.astype(np.int64) != ov)
+        if bad.any():
+            tie = ue_near_tie(ex[bad], fmt)
+            assert np.all(tie) and np.all(np.abs(gv[bad].astype(np.int64) - ov[bad]) <= 1), \
+                f"{name}: {bad.sum()} scale codes differ away from rounding ties"
+    # rows with a boundary code flip: the GPU's scales must be those its codes imply
+    for r in np.nonzero(~ok)[0]:
+        Lu, Gu, Le, Ge = codec.scales_from_codes(X[r:r + 1], A[r:r + 1], bits, got[r:r + 1], global_scale)
+        assert abs(int(gpu_L[r]) - int(Lu[0])) <= (1 if ue_near_tie(Le, K.UE7M9)[0] else 0)
+        assert abs(int(gpu_G[r]) - int(Gu[0])) <= (1 if ue_near_tie(Ge, K.UE4M12)[0] else 0)
+    return ok
+
+
+def _encode_check(case):
+    ix = case.gpu_index()
+    w = case.w
+    c1, L1, G1 = (t.cpu().numpy() for t in ix.export_codes(1))
+    A1 = case.C[case.A].astype(np.float64)
+    ok = _check_stage(c1, L1, G1, case.oracle.stage1, case.X, A1, w.bits, case.global_scale, "stage 1")
+    if w.rescore_bits:
+        c2, L2, G2 = (t.cpu().numpy() for t in ix.export_codes(2))
+        st2 = case.oracle.stage2
+        sel = np.nonzero(ok)[0]
+        sub = codec.Encoded(st2.bits, st2.mode, st2.D, st2.g, st2.codes[sel], st2.L_u16[sel],
+                            st2.G_u16[sel], st2.Lhat[sel], st2.Ghat[sel], st2.uhat[sel], st2.u[sel],
+                            st2.recon[sel], st2.L_exact[sel], st2.G_exact[sel])
+        _check_stage(c2[sel], L2[sel], G2[sel], sub, case.X[sel], case.oracle.stage1.recon[sel],
+                     w.rescore_bits, case.global_scale, "stage 2")
+    return ix
+
+
+def test_encode_parity(case):
+    _encode_check(case)
+
+
+def test_encode_parity_local_scale(local_case):
+    _encode_check(local_case)
+
+
+def test_chunked_encode_matches_single_pass():
+    """Encoding in several chunks, out of order, gives the same index."""
+    case = Case(CASES["C4s"])
+    a = case.gpu_index()
+    b = case.gpu_index(encode=False)
+    X = torch.from_numpy(case.X).cuda()
+    for lo in (30_000, 0, 10_000, 20_000):
+        b.encode(X[lo:lo + 10_000], lo)
+    for which in (1,):
+        for u, v in zip(a.export_codes(which), b.export_codes(which)):
+            assert torch.equal(u, v)
+
+
+# ------------------------------------------------------------------- search
+def _oracle_stage1(case, i, probes, cs):
+    rows, s1 = search.stage1_scores(case.oracle, case.Q[i], probes, cs)
+    return dict(zip(case.oracle.ids[rows].tolist(), s1.tolist())), s1
+
+
+def _kth(values, k):
+    v = np.sort(np.asarray(values))[::-1]
+    return v[k - 1] if len(v) >= k else -np.inf
+
+
+def test_probe_parity(case):
+    ix = case.gpu_index(encode=False)
+    w = case.w
+    p, cs = (t.cpu().numpy() for t in ix.probe(torch.from_numpy(case.Q).cuda(), w.nprobe))
+    full = case.Q.astype(np.float64) @ case.C.astype(np.float64).T
+    cn = np.linalg.norm(case.C, axis=1).max()
+    for i in range(len(case.Q)):
+        tol = lambda s: 1e-5 * case.qnorm(i) * cn  # noqa: E731
+        probs = check_topk(p[i], cs[i], lambda j: full[i, j], _kth(full[i], w.nprobe), tol)
+        assert not probs, (i, probs[:3])
+
+
+def _scan_inputs(case):
+    probes, cs, _ = search.probe(case.Q, case.C, case.w.nprobe)
+    return probes, cs
+
+
+def test_scan_parity_on_oracle_codes(case):
+    """rslm_scan with the oracle's probes, on the oracle's imported codes."""
+    w = case.w
+    ix = case.gpu_index(encode=False)
+    case.import_oracle_codes(ix)
+    probes, cs = _scan_inputs(case)
+    qrot = ix.rotate(torch.from_numpy(case.Q).cuda())
+    ids, sc = ix.scan(qrot, torch.from_numpy(probes.astype(np.int32)).cuda(),
+                      torch.from_numpy(cs.astype(np.float32)).cuda(), w.k)
+    ix.sync()
+    ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
+    xm = case.xnorm_max()
+    for i in range(len(case.Q)):
+        ref, s1 = _oracle_stage1(case, i, probes[i], cs[i])
+        tol = lambda s: float(score_tol(s, case.qnorm(i), xm))  # noqa: E731
+        probs = check_topk(ids[i], sc[i], lambda j: ref[j], _kth(s1, w.k), tol, allowed_ids=ref)
+        assert not probs, (i, probs[:3])
+        assert (ids[i] >= 0).sum() == min(w.k, len(s1))
+
+
+def test_rescore_parity_on_oracle_codes(case):
+    w = case.w
+    if not w.rescore_bits:
+        pytest.skip("no rescoring codes")
+    ix = case.gpu_index(encode=False)
+    case.import_oracle_codes(ix)
+    res = search.search(case.oracle, case.Q, w.nprobe, w.k, w.k_final)
+    q2 = ix.rotate(torch.from_numpy(case.Q).cuda(), which=2)
+    ids, sc = ix.rescore(q2, torch.from_numpy(res["s1_ids"]).cuda(),
+                         torch.from_numpy(res["s1_scores"].astype(np.float32)).cuda(), w.k_final)
+    ix.sync()
+    ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
+    xm = case.xnorm_max()
+    for i in range(len(case.Q)):
+        _, _, s2 = search.rescore(case.oracle, case.Q[i], res["s1_ids"][i], res["s1_scores"][i], w.k)
+        cid = res["s1_ids"][i][res["s1_ids"][i] >= 0]
+        ref = dict(zip(cid.tolist(), s2.tolist()))
+        tol = lambda s: float(score_tol(s, case.qnorm(i), xm))  # noqa: E731
+        probs = check_topk(ids[i], sc[i], lambda j: ref[j], _kth(s2, w.k_final), tol, allowed_ids=ref)
+        assert not probs, (i, probs[:3])
+
+
+def _end_to_end(case, ix, code_ok=None):
+    w = case.w
+    Qt = torch.from_numpy(case.Q).cuda()
+    ids, sc = ix.search(Qt, w.nprobe, w.k, k_final=w.k_final)
+    gp, _ = ix.probe(Qt, w.nprobe)
+    ix.sync()
+    ids, sc, gp = ids.cpu().numpy(), sc.cpu().numpy(), gp.cpu().numpy()
+    oprobes, ocs = _scan_inputs(case)
+    xm = case.xnorm_max()
+    for i in range(len(case.Q)):
+        probes, cs = oprobes[i], ocs[i]
+        if set(gp[i].tolist()) != set(probes.tolist()):
+            # a near-tie at the nprobe boundary (validated by test_probe_parity): follow the GPU's set
+            probes = gp[i].astype(np.int64)
+            cs = case.Q[i].astype(np.float64) @ case.C[probes].astype(np.float64).T
+        ref1, s1 = _oracle_stage1(case, i, probes, cs)
+        tol = lambda s: float(score_tol(s, case.qnorm(i), xm))  # noqa: E731
+        if w.rescore_bits:
+            cid = np.array(list(ref1), dtype=np.int64)
+            cs1 = np.array([ref1[j] for j in cid])
+            _, _, s2 = search.rescore(case.oracle, case.Q[i], cid, cs1, len(cid))
+            ref = dict(zip(cid.tolist(), s2.tolist()))
+            surv, _ = search.take_top(cs1, cid, w.k)
+            kth = _kth([ref[j] for j in surv if j >= 0], w.k_final)
+        else:
+            ref, kth = ref1, _kth(s1, w.k_final)
+        gpu_score = dict(zip(ids[i].tolist(), sc[i].tolist()))
+        # rows whose GPU codes sit on the other side of a decision boundary score differently
+        score_of = lambda j: gpu_score[j] if (code_ok is not None and not code_ok[j]) else ref[j]  # noqa: E731
+        probs = check_topk(ids[i], sc[i], score_of, kth, tol, allowed_ids=ref)
+        assert not probs, (i, probs[:3])
+
+
+def test_search_end_to_end_on_oracle_codes(case):
+    ix = case.gpu_index(encode=False)
+    case.import_oracle_codes(ix)
+    _end_to_end(case, ix)
+
+
+def test_search_end_to_end_gpu_encoded(case):
+    """GPU encode + GPU search vs oracle encode + oracle search."""
+    ix = case.gpu_index()
+    c1, _, _ = ix.export_codes(1)
+    got = codec.unpack_nibbles(c1.cpu().numpy(), case.oracle.stage1.codes.shape[1])
+    code_ok = (got == case.oracle.stage1.codes).all(1)
+    if case.w.rescore_bits:
+        c2, _, _ = ix.export_codes(2)
+        got2 = codec.unpack_nibbles(c2.cpu().numpy(), case.oracle.stage2.codes.shape[1])
+        code_ok &= (got2 == case.oracle.stage2.codes).all(1)
+    _end_to_end(case, ix, code_ok)
+
+
+# --------------------------------------------------------------- edge cases
+def test_edge_cases():
+    from paper_2608_30384_gb300 import RslmError, rslm_scan
+    case = Case(Wl("edge", 700, 32, 6, 0.5, False, None, "true", 5, 4, 0, 6, 256, 256, seed=11))
+    A = case.A.copy()
+    A[A == 2] = 3  # partition 2 left empty
+    case.A = A
+    case.oracle = search.build_index(case.X, np.arange(700), A, case.C, 4, 0)
+    ix = case.gpu_index()
+    Q = torch.from_numpy(case.Q).cuda()
+    # nq = 0 is a no-op
+    e_ids = torch.empty((0, 4), dtype=torch.int64, device="cuda")
+    e_sc = torch.empty((0, 4), dtype=torch.float32, device="cuda")
+    ix.search(Q[:0], 2, 4, out=(e_ids, e_sc))
+    # nprobe = nlist, k = 256 > rows of the probed lists: tail is -1 / -inf
+    ids, sc = ix.search(Q, 6, 256)
+    ix.sync()
+    ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
+    assert np.all((ids >= 0).sum(1) == 256)  # 700 rows, k = 256
+    ids1, sc1 = ix.search(Q, 1, 256)
+    ix.sync()
+    n1 = (ids1.cpu().numpy() >= 0).sum(1)
+    probes, _ = ix.probe(Q, 1)
+    sizes = np.bincount(A, minlength=6)[probes.cpu().numpy()[:, 0]]
+    assert np.array_equal(n1, np.minimum(sizes, 256))
+    tail = ids1.cpu().numpy() < 0
+    assert np.all(np.isneginf(sc1.cpu().numpy()[tail]))
+    # k = 1
+    i1, _ = ix.search(Q, 3, 1)
+    i10, _ = ix.search(Q, 3, 10)
+    assert torch.equal(i1[:, 0], i10[:, 0])
+    # an out-of-range probe id sets the sticky device error, reported by rslm_sync
+    qrot = ix.rotate(Q)
+    bad = torch.full((Q.shape[0], 2), 1, dtype=torch.int32, device="cuda")
+    bad[:, 1] = 99
+    cs = torch.zeros((Q.shape[0], 2), device="cuda")
+    out_i = torch.empty((Q.shape[0], 4), dtype=torch.int64, device="cuda")
+    out_s = torch.empty((Q.shape[0], 4), dtype=torch.float32, device="cuda")
+    rslm_scan(ix.handle, qrot, bad, cs, 4, out_i, out_s)
+    with pytest.raises(RslmError) as ei:
+        ix.sync()
+    assert ei.value.status == 6
+    ix.sync()  # cleared
+    # argument errors are reported synchronously
+    with pytest.raises(RslmError) as ei:
+        ix.search(Q, 7, 4)
+    assert ei.value.status == 1
+    with pytest.raises(RslmError):
+        ix.search(Q, 2, 300)
+
+
+def test_state_errors():
+    from paper_2608_30384_gb300 import Index, RslmError
+    C = torch.zeros((4, 16), device="cuda")
+    ix = Index(C, 4)
+    with pytest.raises(RslmError) as ei:
+        ix.encode(torch.zeros((3, 16), device="cuda"), 0)
+    assert ei.value.status == 5
+    with pytest.raises(RslmError) as ei:
+        ix.reserve(torch.tensor([0, 1, 9], dtype=torch.int32, device="cuda"))
+    assert ei.value.status == 1
+    ix.reserve(torch.tensor([0, 1, 3], dtype=torch.int32, device="cuda"))
+    with pytest.raises(RslmError) as ei:
+        ix.reserve(torch.tensor([0, 1, 3], dtype=torch.int32, device="cuda"))
+    assert ei.value.status == 5
+    with pytest.raises(RslmError):
+        ix.encode(torch.zeros((3, 16), device="cuda"), 1)  # rows 1..3 exceed n = 3
