@@ -1,0 +1,431 @@
+#!/usr/bin/env python
+"""Benchmark of the RSLM IVF-probe search path on GB300.
+
+One step = the whole query path over one batch of synthetic queries with the
+index resident in HBM: probe (<q, centroid> GEMM + top-nprobe), query
+rotation, code scan with the norm-correction epilogue and per-query top-k,
+and (for configurations with rescoring codes) rotation + rescoring.
+
+Default workload: C4 -- N=1e7 d=128 log-normal-norm mixture, IVF8192,
+4-bit codes (680 MB index, larger than the 129 MB L2, so no flush is
+needed), 1e5 queries, nprobe=64, top-10.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--config C4] [--nq n]
+  python bench.py --impl reference ...   # the float64 CPU oracle arm
+
+Under torchrun every rank builds its own replica of the index and searches
+the full query batch (weak scaling, no data-path collective); rank 0 prints
+one JSON line with the max-over-ranks time.
+"""
+
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import math
+import os
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+from paper_2608_30384_gb300 import workloads as W  # noqa: E402
+
+METRIC = "candidates scored/s (IVF probe + RSLM code scan + top-k)"
+UNIT = "candidates/s"
+HBM_FALLBACK = 6800.0
+CLOCK_FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
+                "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
+                "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
+SCAN_SOURCES = ["paper_2608_30384_gb300/csrc/search.cu", "paper_2608_30384_gb300/csrc/device_common.cuh"]
+
+
+def parse_args():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=5)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gb300", choices=["gb300", "reference"])
+    ap.add_argument("--config", default="C4", choices=sorted(W.WORKLOADS))
+    ap.add_argument("--nq", type=int, default=None, help="override the query count")
+    ap.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU time of the oracle leg")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    return ap.parse_args()
+
+
+def workload_label(w: W.Workload) -> str:
+    return f"{w.name}: {w.description}"
+
+
+# ------------------------------------------------------------------ helpers
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return HBM_FALLBACK, "fallback"
+
+
+def scan_source_hash() -> str:
+    h = hashlib.sha256()
+    for rel in SCAN_SOURCES:
+        with open(os.path.join(ROOT, rel), "rb") as f:
+            h.update(f.read())
+    return h.hexdigest()[:16]
+
+
+def traffic_record(config: str):
+    """DRAM bytes per candidate of the scan kernel from a committed ncu summary.
+
+    Returns None when no capture exists or the kernel changed since.
+    """
+    p = os.path.join(ROOT, "profiles", "scan_kernel_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        d = json.load(f)
+    rec = d.get(config)
+    if not rec or rec.get("kernel_hash") != scan_source_hash():
+        return None
+    return rec
+
+
+def visible_gpu_index(local_rank: int) -> str:
+    vis = os.environ.get("CUDA_VISIBLE_DEVICES")
+    if vis:
+        parts = [p.strip() for p in vis.split(",") if p.strip()]
+        if local_rank < len(parts):
+            return parts[local_rank]
+    return str(local_rank)
+
+
+class ClockSampler:
+    """nvidia-smi clock / throttle samples every 200 ms during the timed region."""
+
+    def __init__(self, gpu: str):
+        self.gpu, self.proc, self.lines = gpu, None, []
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "--query-gpu=" + ",".join(CLOCK_FIELDS), "--format=csv,noheader,nounits",
+                 "-lms", "200", "-i", self.gpu], stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        time.sleep(0.25)
+        self.proc.terminate()
+        out, _ = self.proc.communicate(timeout=10)
+        sm, smax, reasons = [], [], set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.splitlines():
+            f = [x.strip() for x in line.split(",")]
+            if len(f) < len(CLOCK_FIELDS):
+                continue
+            try:
+                sm.append(float(f[1]))
+                smax.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[5:9]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": float(np.median(sm)) if sm else None, "sm_max_mhz": max(smax) if smax else None,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+def dist_setup(args):
+    ws = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    if ws != args.gpus:
+        raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE={ws}")
+    return ws, rank, local
+
+
+# --------------------------------------------------------- oracle (CPU) leg
+def oracle_sample(w: W.Workload, X, A, C, Q, n_queries: int):
+    """Oracle index over the rows of the partitions the sample queries probe."""
+    from oracle import search as osearch
+    probes, _, _ = osearch.probe(Q[:n_queries], C, w.nprobe)
+    parts = np.unique(probes)
+    rows = np.nonzero(np.isin(A, parts))[0]
+    index = osearch.build_index(X[rows], rows, A[rows], C, w.bits, w.rescore_bits)
+    sizes = np.bincount(A, minlength=w.P)
+    cand = int(sizes[probes].sum())
+    return index, cand, len(rows)
+
+
+def oracle_time(w, index, Q, n_queries, cand_per_pass, seconds, min_passes=1):
+    from oracle import search as osearch
+    t0 = time.perf_counter()
+    passes = 0
+    while passes < min_passes or time.perf_counter() - t0 < seconds:
+        osearch.search(index, Q[:n_queries], w.nprobe, w.k, w.k_final)
+        passes += 1
+    dt = time.perf_counter() - t0
+    return cand_per_pass * passes / dt, passes, dt
+
+
+def cpu_cores() -> int:
+    try:
+        return len(os.sched_getaffinity(0))
+    except AttributeError:
+        return os.cpu_count() or 1
+
+
+SAMPLE_QUERIES = {"C1": 100, "C2": 8, "C3": 4, "C4": 8, "C5": 1}
+
+
+def run_reference(args):
+    ws, rank, _ = dist_setup(args)
+    if rank != 0:
+        return 0
+    w = W.WORKLOADS[args.config]
+    if args.nq:
+        w = w.scaled(nq=args.nq)
+    X, A = W.database(w)
+    C = W.ivf_centroids(w, X, A)
+    nqs = min(SAMPLE_QUERIES[w.name], w.nq)
+    Q = W.queries(w, nqs)
+    index, cand, nrows = oracle_sample(w, X, A, C, Q, nqs)
+    for _ in range(args.warmup):
+        oracle_time(w, index, Q, nqs, cand, 0.0)
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        oracle_time(w, index, Q, nqs, cand, 0.0)
+    dt = time.perf_counter() - t0
+    value = cand * args.steps / dt
+    sample = (f"{nqs} of the {w.nq} queries of {w.name} per step ({cand} candidates), float64 oracle "
+              f"index over the {nrows} rows of their probed partitions")
+    line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic", "config": {"workload": workload_label(w), "nq_per_step": nqs},
+            "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+                             "sample": sample},
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+    return 0
+
+
+# ------------------------------------------------------------------- GPU arm
+def launches_per_step(w: W.Workload, nq: int) -> int:
+    """Kernels of librslm launched by one step (cuBLAS GEMMs not counted)."""
+    qc = max(1, min(nq, (64 << 20) // w.P))
+    n = math.ceil(nq / qc)  # probe selection, one per query chunk
+    n += 2                   # query rotation + scan
+    if w.rescore_bits:
+        n += 2               # second rotation + rescore
+    return n
+
+
+def run_gpu(args):
+    import torch
+    import torch.distributed as dist
+
+    from paper_2608_30384_gb300 import Index
+    from paper_2608_30384_gb300 import binding as B
+
+    ws, rank, local = dist_setup(args)
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    if ws > 1:
+        os.environ.setdefault("MASTER_ADDR", "127.0.0.1")
+        dist.init_process_group("nccl", device_id=dev)
+
+    w = W.WORKLOADS[args.config]
+    if args.nq:
+        w = w.scaled(nq=args.nq)
+    X, A = W.database(w)
+    C = W.ivf_centroids(w, X, A)
+    Q = W.queries(w)
+    nq = w.nq
+
+    # index build (not timed as part of the step)
+    ix = Index(torch.from_numpy(C).to(dev), w.bits, w.rescore_bits)
+    ix.reserve(torch.from_numpy(A).to(dev))
+    torch.cuda.synchronize()
+    t0 = time.perf_counter()
+    chunk = 1 << 20
+    for lo in range(0, w.N, chunk):
+        ix.encode(torch.from_numpy(X[lo:lo + chunk]).to(dev), lo)
+    ix.sync()
+    encode_s = time.perf_counter() - t0
+    desc = ix.desc
+
+    Qd = torch.from_numpy(Q).to(dev)
+    probes = torch.empty((nq, w.nprobe), dtype=torch.int32, device=dev)
+    cs = torch.empty((nq, w.nprobe), dtype=torch.float32, device=dev)
+    qrot = torch.empty((nq, desc["padded_dim"]), dtype=torch.float32, device=dev)
+    s1_ids = torch.empty((nq, w.k), dtype=torch.int64, device=dev)
+    s1_sc = torch.empty((nq, w.k), dtype=torch.float32, device=dev)
+    if w.rescore_bits:
+        qrot2 = torch.empty((nq, desc["rescore_padded_dim"]), dtype=torch.float32, device=dev)
+        f_ids = torch.empty((nq, w.k_final), dtype=torch.int64, device=dev)
+        f_sc = torch.empty((nq, w.k_final), dtype=torch.float32, device=dev)
+    h = ix.handle
+
+    def step(ev=None):
+        B.rslm_probe(h, Qd, w.nprobe, probes, cs)
+        if ev is not None:
+            ev[0].record()
+        B.rslm_rotate_queries(h, 1, Qd, qrot)
+        if ev is not None:
+            ev[1].record()
+        B.rslm_scan(h, qrot, probes, cs, w.k, s1_ids, s1_sc)
+        if ev is not None:
+            ev[2].record()
+        if w.rescore_bits:
+            B.rslm_rotate_queries(h, 2, Qd, qrot2)
+            B.rslm_rescore(h, qrot2, s1_ids, s1_sc, w.k_final, f_ids, f_sc)
+        if ev is not None:
+            ev[3].record()
+
+    for _ in range(args.warmup):
+        step()
+    ix.sync()
+    sizes = torch.bincount(torch.from_numpy(A).to(dev).long(), minlength=w.P)
+    cand_per_step = int(sizes[probes.long()].sum().item())
+    bytes_per_cand = desc["code_bytes"] + 4  # codes + UE7M9 + UE4M12 scales
+
+    E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
+    starts = [E() for _ in range(args.steps)]
+    evs = [[E() for _ in range(4)] for _ in range(args.steps)]
+    t_end = E()
+    if ws > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    sampler = ClockSampler(visible_gpu_index(local))
+    sampler.start()
+    time.sleep(0.3)
+    for i in range(args.steps):
+        starts[i].record()
+        step(evs[i])
+    t_end.record()
+    torch.cuda.synchronize()
+    clocks = sampler.stop()
+    if ws > 1:
+        dist.barrier()
+    total_ms = starts[0].elapsed_time(t_end)
+    probe_ms = sum(starts[i].elapsed_time(evs[i][0]) for i in range(args.steps)) / args.steps
+    rot_ms = sum(evs[i][0].elapsed_time(evs[i][1]) for i in range(args.steps)) / args.steps
+    scan_ms = sum(evs[i][1].elapsed_time(evs[i][2]) for i in range(args.steps)) / args.steps
+    resc_ms = sum(evs[i][2].elapsed_time(evs[i][3]) for i in range(args.steps)) / args.steps
+    ix.sync()
+    if ws > 1:
+        t = torch.tensor([total_ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        total_ms = float(t.item())
+    ms_per_step = total_ms / args.steps
+    value = cand_per_step * ws * args.steps / (total_ms / 1e3)
+
+    # end to end through the public one-call API with host buffers
+    e2e = None
+    if not args.no_e2e:
+        Qh = torch.from_numpy(Q).pin_memory()
+        Qd2 = torch.empty_like(Qd)
+        o_ids = torch.empty((nq, w.k_final), dtype=torch.int64, device=dev)
+        o_sc = torch.empty((nq, w.k_final), dtype=torch.float32, device=dev)
+        h_ids = torch.empty((nq, w.k_final), dtype=torch.int64).pin_memory()
+        h_sc = torch.empty((nq, w.k_final), dtype=torch.float32).pin_memory()
+
+        def e2e_step():
+            Qd2.copy_(Qh, non_blocking=True)
+            B.rslm_search(h, Qd2, w.nprobe, w.k, bool(w.rescore_bits), w.k_final, o_ids, o_sc)
+            h_ids.copy_(o_ids, non_blocking=True)
+            h_sc.copy_(o_sc, non_blocking=True)
+
+        for _ in range(max(1, min(args.warmup, 2))):
+            e2e_step()
+        torch.cuda.synchronize()
+        a, b = E(), E()
+        if ws > 1:
+            dist.barrier()
+        a.record()
+        for _ in range(args.steps):
+            e2e_step()
+        b.record()
+        torch.cuda.synchronize()
+        ems = a.elapsed_time(b)
+        if ws > 1:
+            t = torch.tensor([ems], device=dev)
+            dist.all_reduce(t, op=dist.ReduceOp.MAX)
+            ems = float(t.item())
+        ix.sync()
+        e2e = {"value": cand_per_step * ws * args.steps / (ems / 1e3), "unit": UNIT,
+               "h2d_bytes_per_step": int(Qh.numel() * 4),
+               "d2h_bytes_per_step": int(h_ids.numel() * 8 + h_sc.numel() * 4),
+               "ms_per_step": ems / args.steps}
+
+    peak, peak_kind = load_peaks()
+    scan_bytes = cand_per_step * bytes_per_cand
+    achieved = scan_bytes / (scan_ms / 1e3) / 1e9
+    trec = traffic_record(w.name)
+    roofline = {"bound": "hbm", "kernel": "scan_kernel", "achieved": achieved, "peak": peak,
+                "unit": "GB/s", "frac": achieved / peak, "peak_kind": peak_kind,
+                "traffic": (trec["dram_bytes_per_candidate"] * cand_per_step) if trec else None,
+                "algorithmic_bytes": scan_bytes}
+
+    cpu = None
+    if rank == 0 and ws == 1 and not args.no_cpu_baseline:
+        nqs = min(SAMPLE_QUERIES[w.name], nq)
+        index, cand, nrows = oracle_sample(w, X, A, C, Q, nqs)
+        cval, passes, dt = oracle_time(w, index, Q, nqs, cand, args.cpu_seconds)
+        cpu = {"value": cval, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
+               "sample": f"{nqs} of the {nq} queries of {w.name} ({cand} candidates per pass) x {passes} "
+                         f"passes = {dt:.1f} s, float64 oracle index over the {nrows} rows of their "
+                         f"probed partitions"}
+
+    if rank == 0:
+        line = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
+            "config": {"workload": workload_label(w), "nq": nq, "nprobe": w.nprobe, "k": w.k,
+                       "k_final": w.k_final, "score_bits": w.bits, "rescore_bits": w.rescore_bits,
+                       "l2": f"inputs larger than L2: {scan_bytes_index(desc) / 1e6:.0f} MB of codes "
+                             f"and scales vs 129 MB L2" if scan_bytes_index(desc) > 129e6 else
+                             "index fits in L2 (no flush: every step re-reads it)",
+                       "parallelism": f"replica x{ws}"},
+            "qps": nq * ws / (ms_per_step / 1e3),
+            "code_stream_gbps": scan_bytes * ws / (ms_per_step / 1e3) / 1e9,
+            "stage_ms": {"probe": probe_ms, "rotate": rot_ms, "scan": scan_ms, "rescore": resc_ms},
+            "candidates_per_step": cand_per_step,
+            "encode_rows_per_s": w.N / encode_s,
+            "roofline": roofline,
+            "cpu_baseline": cpu,
+            "e2e": e2e,
+            "gpu_launches": launches_per_step(w, nq) * args.steps,
+            "clocks": clocks,
+        }
+        print(json.dumps(line), flush=True)
+    if ws > 1:
+        dist.destroy_process_group()
+    return 0
+
+
+def scan_bytes_index(desc) -> int:
+    return int(desc["n_slots"]) * (int(desc["code_bytes"]) + 4)
+
+
+def main():
+    args = parse_args()
+    if args.impl == "reference":
+        return run_reference(args)
+    return run_gpu(args)
+
+
+if __name__ == "__main__":
+    sys.exit(main())

@@ -21,6 +21,8 @@ the true centers or the member means of the generated rows.
 from __future__ import annotations
 
 import math
+import os
+from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass, replace
 
 import numpy as np
@@ -83,19 +85,33 @@ def centers(w: Workload) -> np.ndarray:
     return _rng(w.seed, 0).standard_normal((w.P, w.D), dtype=np.float32)
 
 
-def _rows(w: Workload, ctr: np.ndarray, n: int, base: int, chunk: int):
+def _rows(w: Workload, ctr: np.ndarray, n: int, base: int, chunk: int, out: np.ndarray | None = None):
     comp = _rng(w.seed, base + 1, chunk).integers(0, w.P, size=n, dtype=np.int64)
-    y = ctr[comp] + np.float32(w.sigma) * _rng(w.seed, base + 2, chunk).standard_normal(
-        (n, w.D), dtype=np.float32)
-    if w.normalize or w.lognormal_sigma is not None:
-        nrm = np.sqrt(np.einsum("ij,ij->i", y.astype(np.float64), y.astype(np.float64)))
-        nrm = np.where(nrm > 0, nrm, 1.0)
-        scale = 1.0 / nrm
-        if w.lognormal_sigma is not None:
-            rho = _rng(w.seed, base + 3, chunk).lognormal(0.0, w.lognormal_sigma, size=n)
-            scale = scale * rho
-        y = (y.astype(np.float64) * scale[:, None]).astype(np.float32)
+    y = out if out is not None else np.empty((n, w.D), dtype=np.float32)
+    _rng(w.seed, base + 2, chunk).standard_normal((n, w.D), dtype=np.float32, out=y)
+    rho = None
+    if w.lognormal_sigma is not None:
+        rho = _rng(w.seed, base + 3, chunk).lognormal(0.0, w.lognormal_sigma, size=n)
+    step = max(1, (1 << 18) // w.D)  # small temporaries: about 1 MB per sub-block
+    for lo in range(0, n, step):
+        yb = y[lo:lo + step]
+        yb *= np.float32(w.sigma)
+        yb += ctr[comp[lo:lo + step]]
+        if w.normalize or rho is not None:
+            nrm = np.sqrt(np.einsum("ij,ij->i", yb, yb, dtype=np.float64))
+            scale = 1.0 / np.where(nrm > 0, nrm, 1.0)
+            if rho is not None:
+                scale = scale * rho[lo:lo + step]
+            yb *= scale.astype(np.float32)[:, None]
     return y, comp.astype(np.int32)
+
+
+def _workers() -> int:
+    try:
+        n = len(os.sched_getaffinity(0))
+    except AttributeError:
+        n = os.cpu_count() or 1
+    return max(1, min(16, n))
 
 
 def chunk_rows(w: Workload, chunk: int, ctr: np.ndarray | None = None):
@@ -125,28 +141,44 @@ def rows(w: Workload, ids, ctr: np.ndarray | None = None):
 
 
 def database(w: Workload):
-    """All N rows (float32) and their components (int32)."""
+    """All N rows (float32) and their components (int32), chunks generated in threads."""
     ctr = centers(w)
     X = np.empty((w.N, w.D), dtype=np.float32)
     A = np.empty(w.N, dtype=np.int32)
-    for c in range(n_chunks(w)):
-        Xc, Ac = chunk_rows(w, c, ctr)
-        X[c * CHUNK:c * CHUNK + len(Ac)] = Xc
-        A[c * CHUNK:c * CHUNK + len(Ac)] = Ac
+
+    def one(c):
+        lo = c * CHUNK
+        n = min(w.N, lo + CHUNK) - lo
+        _, a = _rows(w, ctr, n, 0, c, out=X[lo:lo + n])
+        A[lo:lo + n] = a
+
+    with ThreadPoolExecutor(_workers()) as ex:
+        list(ex.map(one, range(n_chunks(w))))
     return X, A
 
 
 def member_means(w: Workload, X: np.ndarray, A: np.ndarray, ctr: np.ndarray) -> np.ndarray:
-    """Per-component mean of the rows (float32); empty components keep the center."""
-    sums = np.zeros((w.P, w.D))
+    """Per-component mean of the rows (float32); empty components keep the center.
+
+    Each row block of 2^16 is summed by a sparse one-hot product (float32,
+    about 8 rows per partition); block sums are added in float64 in block
+    order so the result does not depend on thread scheduling.
+    """
+    from scipy import sparse
     cnt = np.bincount(A, minlength=w.P)
-    for lo in range(0, X.shape[0], CHUNK):
-        a = A[lo:lo + CHUNK]
-        o = np.argsort(a, kind="stable")
-        a_sorted = a[o]
-        starts = np.r_[0, np.nonzero(np.diff(a_sorted))[0] + 1]
-        part = np.add.reduceat(X[lo:lo + CHUNK][o].astype(np.float64), starts, axis=0)
-        sums[a_sorted[starts]] += part
+    block = 1 << 16
+    bounds = list(range(0, X.shape[0], block)) + [X.shape[0]]
+
+    def part(i):
+        lo, hi = bounds[i], bounds[i + 1]
+        m = sparse.csr_matrix((np.ones(hi - lo, dtype=np.float32), (A[lo:hi], np.arange(hi - lo))),
+                              shape=(w.P, hi - lo))
+        return m @ X[lo:hi]
+
+    sums = np.zeros((w.P, w.D))
+    with ThreadPoolExecutor(_workers()) as ex:
+        for p in ex.map(part, range(len(bounds) - 1)):
+            sums += p
     out = ctr.astype(np.float64).copy()
     nz = cnt > 0
     out[nz] = sums[nz] / cnt[nz, None]
