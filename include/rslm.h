@@ -135,6 +135,25 @@ rslm_status rslm_rotate_queries(const rslm_index* index, int32_t which, const fl
 rslm_status rslm_probe(const rslm_index* index, const float* queries, int64_t nq, int32_t nprobe,
                        int32_t* out_probes, float* out_cs, void* stream);
 
+/* rslm_probe that allocates no device memory.  The paper has no counterpart:
+ * this exists for callers that cannot allocate on the query path -- programs
+ * whose device memory is all owned by another allocator (a framework's
+ * caching allocator, a fixed budget handed out up front) and latency-critical
+ * serving loops that forbid cudaMalloc / cudaFree because those calls can
+ * synchronize the device.  Same arguments and results as rslm_probe; the
+ * <q, centroid> scores of a query chunk live in a fixed 16 MiB device array
+ * inside the library (held by every GPU that loads it, until exit) and are
+ * computed by the library's own kernel rather than cuBLAS.
+ * - The first call made with an index on a given device looks up that
+ *   array's address on the device (cudaGetSymbolAddress); make that first
+ *   call before any stream capture.
+ * - All calls on a device share the array.  Calls whose GPU work may overlap
+ *   (other streams, unordered host threads) race on it: serialise them.
+ * - nlist above 4,194,304 (one query's scores must fit) returns
+ *   RSLM_ERR_INVALID_ARG; larger nq is processed in chunks. */
+rslm_status rslm_probe_noalloc(const rslm_index* index, const float* queries, int64_t nq,
+                               int32_t nprobe, int32_t* out_probes, float* out_cs, void* stream);
+
 /* Scan (Sec. 5.5.1 step 3 with the scores of Sec. 3.5.1-3.5.2): every row j
  * of every probed partition p scores s_j = G_j (cs_p + L_j <R q, u^_j>),
  * and the top k per query are kept.

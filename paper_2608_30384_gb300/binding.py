@@ -31,6 +31,7 @@ SIGNATURES = {
     "rslm_encode": (ctypes.c_int, [_P, _P, _I64, _I64, _P]),
     "rslm_rotate_queries": (ctypes.c_int, [_P, _I32, _P, _I64, _P, _P]),
     "rslm_probe": (ctypes.c_int, [_P, _P, _I64, _I32, _P, _P, _P]),
+    "rslm_probe_noalloc": (ctypes.c_int, [_P, _P, _I64, _I32, _P, _P, _P]),
     "rslm_scan": (ctypes.c_int, [_P, _P, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
     "rslm_rescore": (ctypes.c_int, [_P, _P, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
     "rslm_search": (ctypes.c_int, [_P, _P, _I64, _I32, _I32, _I32, _I32, _P, _P, _P]),
@@ -165,6 +166,16 @@ def rslm_probe(index, queries, nprobe, out_probes, out_cs, stream=None):
     _check(lib().rslm_probe(_ptr(index), _dev(queries, torch.float32, "queries"), nq, nprobe,
                             _dev(out_probes, torch.int32, "out_probes", nq * nprobe),
                             _dev(out_cs, torch.float32, "out_cs", nq * nprobe), _stream(stream)))
+
+
+def rslm_probe_noalloc(index, queries, nprobe, out_probes, out_cs, stream=None):
+    """rslm_probe with its scratch in the library's fixed device array (no allocation)."""
+    import torch
+    nq = queries.shape[0]
+    _check(lib().rslm_probe_noalloc(_ptr(index), _dev(queries, torch.float32, "queries"), nq, nprobe,
+                                    _dev(out_probes, torch.int32, "out_probes", nq * nprobe),
+                                    _dev(out_cs, torch.float32, "out_cs", nq * nprobe),
+                                    _stream(stream)))
 
 
 def rslm_scan(index, qrot, probes, cs, k, out_ids, out_scores, stream=None):

@@ -118,6 +118,8 @@ rslm_status check_query_args(const rslm_index* ix, int64_t nq, int nprobe) {
 
 }  // namespace
 
+rslm_status rslm::set_last_error(rslm_status st, const std::string& msg) { return fail(st, msg); }
+
 extern "C" {
 
 rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids, int32_t score_bits,

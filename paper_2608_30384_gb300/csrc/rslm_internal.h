@@ -60,6 +60,9 @@ bool make_codec_spec(int bits, int D, bool interleaved, CodecSpec* out);
 double e_max(int D);
 uint32_t ue_encode_host(double v, int ebits, int mbits);
 
+// Record the calling thread's rslm_last_error() message and return `st`.
+rslm_status set_last_error(rslm_status st, const std::string& msg);
+
 }  // namespace rslm
 
 // Index state (host object; arrays are device pointers).
