@@ -4,7 +4,8 @@
 // The query, already rotated (Sec. 5.4), becomes a lookup table
 // T[group][code] = <q_group, codeword_code> in shared memory, so that the
 // dot product <R q, uhat> of a row is the sum of one table entry per 4-bit
-// code.  Warps stream 128-row tiles of the probed partitions; every lane
+// code; per code the work is one byte permute (its table address), one
+// shared-memory load and one add.  Warps stream 128-row tiles of the probed partitions; every lane
 // owns 4 rows of a tile and reads 16-byte chunks that are contiguous across
 // the warp (tile-interleaved layout).  The epilogue applies the scales,
 // s = G (cs + L dot) (Sec. 3.5.2), and feeds a per-warp top-k list; the
@@ -141,6 +142,12 @@ __device__ __forceinline__ void load_chunk(const uint8_t* p, uint32_t (&w)[CH / 
   }
 }
 
+__device__ __forceinline__ float lds_f32(uint32_t addr) {
+  float v;
+  asm("ld.shared.f32 %0, [%1];" : "=f"(v) : "r"(addr));
+  return v;
+}
+
 // Insert (s, p) into a warp's list sorted by (score desc, position asc).
 // Every lane calls with the same (s, p).
 __device__ __forceinline__ void warp_insert(float* sc, int* ps, int& cnt, int k, float s, int p,
@@ -187,21 +194,31 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   __shared__ int scratch[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, W = blockDim.x >> 5;
   const int64_t q = blockIdx.x;
-  float* lut = reinterpret_cast<float*>(ssm);
-  float* wsc = reinterpret_cast<float*>(ssm + a.lut_region);
+  // The table starts on a 256-byte boundary of the shared window (up to 255
+  // bytes of padding are reserved by the launcher).
+  const uint32_t ssm_addr = uint32_t(__cvta_generic_to_shared(ssm));
+  const uint32_t lut_pad = (256u - (ssm_addr & 255u)) & 255u;
+  float* lut = reinterpret_cast<float*>(ssm + lut_pad);
+  const uint32_t lut_block0 = (ssm_addr + lut_pad) >> 8;
+  float* wsc = reinterpret_cast<float*>(ssm + 256 + a.lut_region);
   int* wps = reinterpret_cast<int*>(wsc + W * a.k);
   int* wcnt = wps + W * a.k;
   int* pid = wcnt + W;
   int* tpref = pid + a.nprobe;
 
-  // Query lookup table: T[group][code] = <q_group, C[code]>.
+  // Query lookup table T[position][code] = <q_group, C[code]>, one entry per
+  // (4-bit code position of a row, code value).  Layout: the 8 positions of
+  // each 32-bit code word w go to two 256-byte blocks, even positions in
+  // block 2w and odd ones in block 2w + 1, position 2k (+1) at byte 64 k.  A
+  // code's shared-memory address is then (block << 8) | (64 k + 4 code):
+  // one byte permute per code builds it (see the scan loop).
   const float* qr = a.qrot + q * a.Dp;
   for (int e = tid; e < a.lut_groups * 16; e += blockDim.x) {
     const int grp = e >> 4, code = e & 15;
     float v = 0.0f;
     if (grp < a.ngroups)
       for (int j = 0; j < a.g; ++j) v = fmaf(qr[grp * a.g + j], a.cb[code * a.g + j], v);
-    lut[e] = v;
+    lut[(2 * (grp >> 3) + (grp & 1)) * 64 + ((grp & 7) >> 1) * 16 + code] = v;
   }
   // Probe list -> tiles to visit.
   int run = 0;
@@ -245,17 +262,27 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
     const uint8_t* tp = a.codes + slot0 * a.stride;
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     for (int c = 0; c < nch; ++c) {
-      const float* lc = lut + c * (2 * CH) * 16;
       uint32_t w[4][CH / 4];
 #pragma unroll
       for (int r = 0; r < 4; ++r)
         load_chunk<CH>(tp + (size_t(c) * kTile + r * 32 + lane) * CH, w[r]);
 #pragma unroll
-      for (int r = 0; r < 4; ++r)
+      for (int v = 0; v < CH / 4; ++v) {
+        // bits 8.. of the addresses of this word's even / odd positions
+        const uint32_t blk_even = (lut_block0 + 2u * uint32_t(c * (CH / 4) + v)) << 8;
+        const uint32_t blk_odd = blk_even + 256u;
 #pragma unroll
-        for (int v = 0; v < CH / 4; ++v)
+        for (int r = 0; r < 4; ++r) {
+          // byte k of ev (od) = 64 k + 4 * code of position 2k (2k + 1)
+          const uint32_t ev = ((w[r][v] << 2) & 0x3C3C3C3Cu) | 0xC0804000u;
+          const uint32_t od = ((w[r][v] >> 2) & 0x3C3C3C3Cu) | 0xC0804000u;
 #pragma unroll
-          for (int n = 0; n < 8; ++n) acc[r] += lc[(v * 8 + n) * 16 + ((w[r][v] >> (4 * n)) & 15u)];
+          for (int k = 0; k < 4; ++k) {
+            acc[r] += lds_f32(__byte_perm(ev, blk_even, 0x7650u + k));
+            acc[r] += lds_f32(__byte_perm(od, blk_odd, 0x7650u + k));
+          }
+        }
+      }
     }
 #pragma unroll
     for (int r = 0; r < 4; ++r) {
@@ -292,7 +319,8 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   int np2 = 1;
   while (np2 < tot) np2 <<= 1;
   float* mkey = lut;
-  int64_t* mid = reinterpret_cast<int64_t*>(ssm + ((size_t(np2) * 4 + 15) & ~size_t(15)));
+  int64_t* mid = reinterpret_cast<int64_t*>(reinterpret_cast<uint8_t*>(lut) +
+                                            ((size_t(np2) * 4 + 15) & ~size_t(15)));
   for (int e = tid; e < np2; e += blockDim.x) {
     float kv = -CUDART_INF_F;
     int64_t iv = LLONG_MAX;
@@ -442,7 +470,7 @@ cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, con
   size_t region = lut_bytes > merge_bytes ? lut_bytes : merge_bytes;
   region = (region + 15) & ~size_t(15);
   a.lut_region = int(region);
-  const size_t smem = region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
+  const size_t smem = 256 + region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
   switch (ix->cs1.chunk) {
     case 16: return launch_scan_ch<16>(a, nq, smem, s);
     case 8: return launch_scan_ch<8>(a, nq, smem, s);
