@@ -40,10 +40,16 @@ from paper_2608_30384_gb300 import workloads as W  # noqa: E402
 METRIC = "candidates scored/s (IVF probe + RSLM code scan + top-k)"
 UNIT = "candidates/s"
 HBM_FALLBACK = 6800.0
+TENSOR_FALLBACK = 1700.0  # sustained dense bf16 TFLOP/s (fallback figure)
+BATCH_MIN_QUERIES = 16    # rslm_search's rule: batched scan when nq*nprobe >= 16*nlist
 CLOCK_FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_event_reasons.active",
                 "clocks_event_reasons.hw_slowdown", "clocks_event_reasons.hw_thermal_slowdown",
                 "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
-SCAN_SOURCES = ["paper_2608_30384_gb300/csrc/search.cu", "paper_2608_30384_gb300/csrc/device_common.cuh"]
+SCAN_SOURCES = {
+    "scan_kernel": ["paper_2608_30384_gb300/csrc/search.cu", "paper_2608_30384_gb300/csrc/device_common.cuh"],
+    "batched_scan_kernel": ["paper_2608_30384_gb300/csrc/batched.cu",
+                            "paper_2608_30384_gb300/csrc/device_common.cuh"],
+}
 
 
 def parse_args():
@@ -57,6 +63,8 @@ def parse_args():
     ap.add_argument("--cpu-seconds", type=float, default=12.0, help="CPU time of the oracle leg")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--scan", default="auto", choices=["auto", "gemv", "batched"],
+                    help="scan form; auto = rslm_search's rule (batched when nq*nprobe >= 16*nlist)")
     return ap.parse_args()
 
 
@@ -66,24 +74,25 @@ def workload_label(w: W.Workload) -> str:
 
 # ------------------------------------------------------------------ helpers
 def load_peaks():
+    """(HBM GB/s, sustained dense bf16/fp16 TFLOP/s, 'measured' | 'fallback')."""
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
         with open(p) as f:
             d = json.load(f)
-        return float(d["hbm_gbs"]), "measured"
-    return HBM_FALLBACK, "fallback"
+        return float(d["hbm_gbs"]), float(d.get("bf16_tflops_sustained", d["bf16_tflops"])), "measured"
+    return HBM_FALLBACK, TENSOR_FALLBACK, "fallback"
 
 
-def scan_source_hash() -> str:
+def scan_source_hash(kernel: str) -> str:
     h = hashlib.sha256()
-    for rel in SCAN_SOURCES:
+    for rel in SCAN_SOURCES[kernel]:
         with open(os.path.join(ROOT, rel), "rb") as f:
             h.update(f.read())
     return h.hexdigest()[:16]
 
 
-def traffic_record(config: str):
-    """DRAM bytes per candidate of the scan kernel from a committed ncu summary.
+def traffic_record(config: str, kernel: str):
+    """DRAM bytes per candidate of a scan kernel from a committed ncu summary.
 
     Returns None when no capture exists or the kernel changed since.
     """
@@ -92,8 +101,8 @@ def traffic_record(config: str):
         return None
     with open(p) as f:
         d = json.load(f)
-    rec = d.get(config)
-    if not rec or rec.get("kernel_hash") != scan_source_hash():
+    rec = d.get(f"{config}/{kernel}") or (d.get(config) if kernel == "scan_kernel" else None)
+    if not rec or rec.get("kernel_hash") != scan_source_hash(kernel):
         return None
     return rec
 
@@ -221,11 +230,14 @@ def run_reference(args):
 
 
 # ------------------------------------------------------------------- GPU arm
-def launches_per_step(w: W.Workload, nq: int) -> int:
+def launches_per_step(w: W.Workload, nq: int, batched: bool) -> int:
     """Kernels of librslm launched by one step (cuBLAS GEMMs not counted)."""
     qc = max(1, min(nq, (64 << 20) // w.P))
     n = math.ceil(nq / qc)  # probe selection, one per query chunk
-    n += 2                   # query rotation + scan
+    n += 1                   # query rotation
+    # batched: count, list scan, scatter, query split, first-probe scan,
+    # threshold, tensor-core scan, finalize, overflow re-scan; else one scan
+    n += 9 if batched else 1
     if w.rescore_bits:
         n += 2               # second rotation + rescore
     return n
@@ -276,6 +288,9 @@ def run_gpu(args):
         f_ids = torch.empty((nq, w.k_final), dtype=torch.int64, device=dev)
         f_sc = torch.empty((nq, w.k_final), dtype=torch.float32, device=dev)
     h = ix.handle
+    batched = (args.scan == "batched" or
+               (args.scan == "auto" and nq * w.nprobe >= BATCH_MIN_QUERIES * w.P))
+    scan_fn = B.rslm_scan_batched if batched else B.rslm_scan
 
     def step(ev=None):
         B.rslm_probe(h, Qd, w.nprobe, probes, cs)
@@ -284,7 +299,7 @@ def run_gpu(args):
         B.rslm_rotate_queries(h, 1, Qd, qrot)
         if ev is not None:
             ev[1].record()
-        B.rslm_scan(h, qrot, probes, cs, w.k, s1_ids, s1_sc)
+        scan_fn(h, qrot, probes, cs, w.k, s1_ids, s1_sc)
         if ev is not None:
             ev[2].record()
         if w.rescore_bits:
@@ -310,12 +325,15 @@ def run_gpu(args):
     sampler = ClockSampler(visible_gpu_index(local))
     sampler.start()
     time.sleep(0.3)
+    B.rslm_profile_enable(h, True)
     for i in range(args.steps):
         starts[i].record()
         step(evs[i])
     t_end.record()
     torch.cuda.synchronize()
     clocks = sampler.stop()
+    kern_ms, kern_n, kern_name = B.rslm_profile_read(h)
+    B.rslm_profile_enable(h, False)
     if ws > 1:
         dist.barrier()
     total_ms = starts[0].elapsed_time(t_end)
@@ -369,14 +387,27 @@ def run_gpu(args):
                "d2h_bytes_per_step": int(h_ids.numel() * 8 + h_sc.numel() * 4),
                "ms_per_step": ems / args.steps}
 
-    peak, peak_kind = load_peaks()
+    hbm_peak, tensor_peak, peak_kind = load_peaks()
     scan_bytes = cand_per_step * bytes_per_cand
-    achieved = scan_bytes / (scan_ms / 1e3) / 1e9
-    trec = traffic_record(w.name)
-    roofline = {"bound": "hbm", "kernel": "scan_kernel", "achieved": achieved, "peak": peak,
-                "unit": "GB/s", "frac": achieved / peak, "peak_kind": peak_kind,
-                "traffic": (trec["dram_bytes_per_candidate"] * cand_per_step) if trec else None,
-                "algorithmic_bytes": scan_bytes}
+    kern_avg_s = kern_ms / max(1, kern_n) / 1e3
+    trec = traffic_record(w.name, kern_name)
+    traffic = (trec["dram_bytes_per_candidate"] * cand_per_step) if trec else None
+    if kern_name == "batched_scan_kernel":
+        # dense contraction: 2 D flops per candidate (the fp16 hi/lo split is
+        # counted once); one launch scores the whole step's candidates
+        flops = 2.0 * w.D * cand_per_step
+        achieved = flops / kern_avg_s / 1e12
+        roofline = {"bound": "tensor", "kernel": kern_name, "achieved": achieved,
+                    "peak": tensor_peak, "unit": "TFLOP/s", "frac": achieved / tensor_peak,
+                    "peak_kind": f"{peak_kind} sustained dense bf16 (fp16 runs at the same rate)",
+                    "traffic": traffic, "algorithmic_flops": flops,
+                    "kernel_ms": kern_avg_s * 1e3, "launches": kern_n}
+    else:
+        achieved = scan_bytes / kern_avg_s / 1e9
+        roofline = {"bound": "hbm", "kernel": kern_name, "achieved": achieved, "peak": hbm_peak,
+                    "unit": "GB/s", "frac": achieved / hbm_peak, "peak_kind": peak_kind,
+                    "traffic": traffic, "algorithmic_bytes": scan_bytes,
+                    "kernel_ms": kern_avg_s * 1e3, "launches": kern_n}
 
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
@@ -398,7 +429,9 @@ def run_gpu(args):
                        "l2": f"inputs larger than L2: {scan_bytes_index(desc) / 1e6:.0f} MB of codes "
                              f"and scales vs 129 MB L2" if scan_bytes_index(desc) > 129e6 else
                              "index fits in L2 (no flush: every step re-reads it)",
-                       "parallelism": f"replica x{ws}"},
+                       "parallelism": f"replica x{ws}",
+                       "scan": "batched (partition-major, tensor cores)" if batched else
+                               "single-query (shared-memory table)"},
             "qps": nq * ws / (ms_per_step / 1e3),
             "code_stream_gbps": scan_bytes * ws / (ms_per_step / 1e3) / 1e9,
             "stage_ms": {"probe": probe_ms, "rotate": rot_ms, "scan": scan_ms, "rescore": resc_ms},
@@ -407,7 +440,7 @@ def run_gpu(args):
             "roofline": roofline,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": launches_per_step(w, nq) * args.steps,
+            "gpu_launches": launches_per_step(w, nq, batched) * args.steps,
             "clocks": clocks,
         }
         print(json.dumps(line), flush=True)

@@ -165,6 +165,22 @@ rslm_status rslm_scan(const rslm_index* index, const float* qrot, int64_t nq, co
                       const float* cs, int32_t nprobe, int32_t k, int64_t* out_ids,
                       float* out_scores, void* stream);
 
+/* Same inputs, outputs and results as rslm_scan, computed partition-major for
+ * batches whose queries share partitions ("batched processing throughput" is
+ * the IVF advantage the paper names in Sec. 1.2): the probe lists are
+ * inverted per partition, each 128-row tile of codes is decoded once and
+ * multiplied with up to 128 of its queries on the tensor cores (fp16 codeword
+ * components, which are exact; queries split into fp16 hi + lo parts; fp32
+ * accumulation), and only candidates at or above a per-query lower bound of
+ * the k-th score (from a first pass over each query's first probed
+ * partition) are kept.  A query with more than 16 k + 1024 such candidates is
+ * re-scanned by the rslm_scan kernel.  Scores agree with rslm_scan within
+ * float32 rounding; temporary device memory comes from the stream-ordered
+ * allocator.  rslm_search picks this path when nq * nprobe >= 16 * nlist. */
+rslm_status rslm_scan_batched(const rslm_index* index, const float* qrot, int64_t nq,
+                              const int32_t* probes, const float* cs, int32_t nprobe, int32_t k,
+                              int64_t* out_ids, float* out_scores, void* stream);
+
 /* Rescore (Sec. 2.1, Sec. 5.2): each candidate j with first-stage score
  * s1_j = <q, a2_j> gets s2_j = G2_j (s1_j + L2_j <R2 q, u2^_j>) from its
  * 4-bit rescoring codes; the top k_final per query are returned.
@@ -211,6 +227,18 @@ rslm_status rslm_rotation_tables(int8_t* s1, int32_t* perm);
 
 /* E_max(D), the expected maximum of D iid |N(0,1)| (Sec. 3.2).  Needs no GPU. */
 rslm_status rslm_e_max(int32_t dim, double* out);
+
+/* Measurement support (no counterpart in the paper).  While enabled, every
+ * launch of the dominant scan kernel of rslm_scan / rslm_scan_batched /
+ * rslm_search on this index is bracketed by CUDA events recorded on the
+ * launching stream.  rslm_profile_enable(index, 1) starts recording (and
+ * clears earlier records), 0 stops.  rslm_profile_read waits for the recorded
+ * events, returns the summed kernel time in *total_ms and the number of
+ * launches in *launches (host pointers), writes the kernel's name into
+ * kernel[kernel_len] (host, may be NULL) and clears the records. */
+rslm_status rslm_profile_enable(rslm_index* index, int32_t on);
+rslm_status rslm_profile_read(rslm_index* index, double* total_ms, int64_t* launches, char* kernel,
+                              int32_t kernel_len);
 
 /* Wait for `stream`, then report and clear the index's sticky device error
  * flag (RSLM_ERR_DEVICE) or a pending CUDA error (RSLM_ERR_CUDA). */

@@ -33,6 +33,7 @@ SIGNATURES = {
     "rslm_probe": (ctypes.c_int, [_P, _P, _I64, _I32, _P, _P, _P]),
     "rslm_probe_noalloc": (ctypes.c_int, [_P, _P, _I64, _I32, _P, _P, _P]),
     "rslm_scan": (ctypes.c_int, [_P, _P, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
+    "rslm_scan_batched": (ctypes.c_int, [_P, _P, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
     "rslm_rescore": (ctypes.c_int, [_P, _P, _I64, _P, _P, _I32, _I32, _P, _P, _P]),
     "rslm_search": (ctypes.c_int, [_P, _P, _I64, _I32, _I32, _I32, _I32, _P, _P, _P]),
     "rslm_export_codes": (ctypes.c_int, [_P, _I32, _I64, _I64, _P, _P, _P, _P]),
@@ -40,6 +41,8 @@ SIGNATURES = {
     "rslm_codebook": (ctypes.c_int, [_I32, _P, _P, _P]),
     "rslm_rotation_tables": (ctypes.c_int, [_P, _P]),
     "rslm_e_max": (ctypes.c_int, [_I32, ctypes.POINTER(_D)]),
+    "rslm_profile_enable": (ctypes.c_int, [_P, _I32]),
+    "rslm_profile_read": (ctypes.c_int, [_P, ctypes.POINTER(_D), ctypes.POINTER(_I64), _P, _I32]),
     "rslm_sync": (ctypes.c_int, [_P, _P]),
     "rslm_last_error": (ctypes.c_char_p, []),
     "rslm_index_destroy": (None, [_P]),
@@ -187,6 +190,16 @@ def rslm_scan(index, qrot, probes, cs, k, out_ids, out_scores, stream=None):
                            _dev(out_scores, torch.float32, "out_scores", nq * k), _stream(stream)))
 
 
+def rslm_scan_batched(index, qrot, probes, cs, k, out_ids, out_scores, stream=None):
+    import torch
+    nq, nprobe = probes.shape
+    _check(lib().rslm_scan_batched(_ptr(index), _dev(qrot, torch.float32, "qrot"), nq,
+                                   _dev(probes, torch.int32, "probes"), _dev(cs, torch.float32, "cs"),
+                                   nprobe, k, _dev(out_ids, torch.int64, "out_ids", nq * k),
+                                   _dev(out_scores, torch.float32, "out_scores", nq * k),
+                                   _stream(stream)))
+
+
 def rslm_rescore(index, qrot2, cand_ids, cand_scores, k_final, out_ids, out_scores, stream=None):
     import torch
     nq, k = cand_ids.shape
@@ -244,6 +257,18 @@ def rslm_e_max(dim) -> float:
     v = ctypes.c_double()
     _check(lib().rslm_e_max(dim, ctypes.byref(v)))
     return v.value
+
+
+def rslm_profile_enable(index, on=True):
+    _check(lib().rslm_profile_enable(_ptr(index), int(bool(on))))
+
+
+def rslm_profile_read(index):
+    """(total kernel ms, launches, kernel name) recorded since enable / last read."""
+    ms, n = ctypes.c_double(), ctypes.c_int64()
+    name = ctypes.create_string_buffer(64)
+    _check(lib().rslm_profile_read(_ptr(index), ctypes.byref(ms), ctypes.byref(n), name, 64))
+    return ms.value, n.value, name.value.decode()
 
 
 def rslm_sync(index, stream=None):

@@ -120,6 +120,36 @@ rslm_status check_query_args(const rslm_index* ix, int64_t nq, int nprobe) {
 
 rslm_status rslm::set_last_error(rslm_status st, const std::string& msg) { return fail(st, msg); }
 
+cudaEvent_t rslm::prof_start(const rslm_index* ix, cudaStream_t s, const char* kernel) {
+  if (!ix->profile) return nullptr;
+  cudaEvent_t a = nullptr, b = nullptr;
+  if (cudaEventCreate(&a) != cudaSuccess) return nullptr;
+  if (cudaEventCreate(&b) != cudaSuccess) {
+    cudaEventDestroy(a);
+    return nullptr;
+  }
+  cudaEventRecord(a, s);
+  std::lock_guard<std::mutex> lock(ix->prof_mu);
+  ix->prof_events.emplace_back(a, b);
+  ix->prof_kernel = kernel;
+  return b;
+}
+
+void rslm::prof_stop(cudaEvent_t stop, cudaStream_t s) {
+  if (stop) cudaEventRecord(stop, s);
+}
+
+namespace {
+void prof_clear(const rslm_index* ix) {
+  std::lock_guard<std::mutex> lock(ix->prof_mu);
+  for (auto& e : ix->prof_events) {
+    cudaEventDestroy(e.first);
+    cudaEventDestroy(e.second);
+  }
+  ix->prof_events.clear();
+}
+}  // namespace
+
 extern "C" {
 
 rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids, int32_t score_bits,
@@ -173,6 +203,9 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
     delete ix;
     return fail(RSLM_ERR_CUDA, "cublasCreate failed");
   }
+  // FP32 GEMM with float32 accuracy, allowed to run as BF16x9 on the tensor
+  // cores when cuBLAS finds that faster.
+  cublasSetMathMode(h, CUBLAS_FP32_EMULATED_BF16X9_MATH);
   ix->cublas = h;
   *out = ix;
   return RSLM_OK;
@@ -269,6 +302,7 @@ rslm_status rslm_index_reserve(rslm_index* ix, const int32_t* assignment, int64_
   }
   ix->n_rows = n;
   ix->n_slots = n_slots;
+  ix->max_part_n = *std::max_element(pn.begin(), pn.end());
   return RSLM_OK;
 }
 
@@ -320,6 +354,21 @@ rslm_status rslm_scan(const rslm_index* ix, const float* qrot, int64_t nq, const
   return RSLM_OK;
 }
 
+rslm_status rslm_scan_batched(const rslm_index* ix, const float* qrot, int64_t nq,
+                              const int32_t* probes, const float* cs, int32_t nprobe, int32_t k,
+                              int64_t* out_ids, float* out_scores, void* stream) {
+  rslm_status st = check_query_args(ix, nq, nprobe);
+  if (st != RSLM_OK) return st;
+  if (!ix->slot_of_row) return fail(RSLM_ERR_STATE, "rslm_index_reserve has not been called");
+  RSLM_ARG(k >= 1 && k <= kMaxK, "k must be in [1, 256]");
+  RSLM_ARG(nq == 0 || (qrot && probes && cs && out_ids && out_scores), "NULL array");
+  DeviceGuard g(ix->device);
+  RSLM_CK(launch_scan_batched(ix, qrot, nq, probes, cs, nprobe, k, out_ids, out_scores,
+                              as_stream(stream)),
+          "batched scan");
+  return RSLM_OK;
+}
+
 rslm_status rslm_rescore(const rslm_index* ix, const float* qrot2, int64_t nq, const int64_t* cand_ids,
                          const float* cand_scores, int32_t k, int32_t k_final, int64_t* out_ids,
                          float* out_scores, void* stream) {
@@ -367,7 +416,13 @@ rslm_status rslm_search(const rslm_index* ix, const float* queries, int64_t nq, 
   if (st == RSLM_OK) st = run_probe(ix, queries, nq, nprobe, probes, cs, s);
   if (st == RSLM_OK) {
     e = launch_rotate_rows(ix->rot1, queries, nq, q1, ix->cs1.Dp, s);
-    if (e == cudaSuccess)
+    // Partition-major tensor-core scan once partitions are shared by enough
+    // queries (on average at least kBatchMinQueries per probed list).
+    const bool batched = nq * nprobe >= int64_t(kBatchMinQueries) * ix->nlist;
+    if (e == cudaSuccess && batched && (rs || k_final == k))
+      e = launch_scan_batched(ix, q1, nq, probes, cs, nprobe, k, rs ? s1i : out_ids,
+                              rs ? s1s : out_scores, s);
+    else if (e == cudaSuccess)
       e = launch_scan(ix, q1, nq, probes, cs, nprobe, k, rs ? k : k_final, rs ? s1i : out_ids,
                       rs ? s1s : out_scores, s);
     if (e == cudaSuccess && rs) e = launch_rotate_rows(ix->rot2, queries, nq, q2, ix->cs2.Dp, s);
@@ -444,6 +499,8 @@ rslm_status rslm_sync(const rslm_index* ix, void* stream) {
   RSLM_CK(cudaMemcpy(&h, ix->d_err, sizeof(int), cudaMemcpyDeviceToHost), "read device error flag");
   if (h != 0) {
     cudaMemset(ix->d_err, 0, sizeof(int));
+    if (h == kErrTimeout)
+      return fail(RSLM_ERR_TIMEOUT, "a bounded wait for the tensor-core pipeline expired");
     const char* what = h == kErrBadProbe ? "probe list holds a partition id outside [0, nlist)"
                        : h == kErrBadCandidate ? "candidate id outside [-1, n_rows)"
                                                : "device-side check failed";
@@ -454,9 +511,46 @@ rslm_status rslm_sync(const rslm_index* ix, void* stream) {
 
 const char* rslm_last_error(void) { return g_last_error.c_str(); }
 
+rslm_status rslm_profile_enable(rslm_index* ix, int32_t on) {
+  RSLM_ARG(ix, "index is NULL");
+  DeviceGuard g(ix->device);
+  prof_clear(ix);
+  ix->profile = on ? 1 : 0;
+  return RSLM_OK;
+}
+
+rslm_status rslm_profile_read(rslm_index* ix, double* total_ms, int64_t* launches, char* kernel,
+                              int32_t kernel_len) {
+  RSLM_ARG(ix && total_ms && launches, "NULL argument");
+  DeviceGuard g(ix->device);
+  double tot = 0.0;
+  int64_t n = 0;
+  std::string name;
+  {
+    std::lock_guard<std::mutex> lock(ix->prof_mu);
+    for (auto& e : ix->prof_events) {
+      RSLM_CK(cudaEventSynchronize(e.second), "profile event");
+      float ms = 0.0f;
+      RSLM_CK(cudaEventElapsedTime(&ms, e.first, e.second), "profile elapsed");
+      tot += ms;
+      ++n;
+    }
+    name = ix->prof_kernel;
+  }
+  prof_clear(ix);
+  *total_ms = tot;
+  *launches = n;
+  if (kernel && kernel_len > 0) {
+    std::strncpy(kernel, name.c_str(), size_t(kernel_len) - 1);
+    kernel[kernel_len - 1] = 0;
+  }
+  return RSLM_OK;
+}
+
 void rslm_index_destroy(rslm_index* ix) {
   if (!ix) return;
   DeviceGuard g(ix->device);
+  prof_clear(ix);
   free_all(ix);
   delete ix;
 }

@@ -1,0 +1,1113 @@
+// batched.cu -- partition-major scan for query batches that share partitions.
+//
+// When many queries probe the same partition (nq * nprobe / nlist large), the
+// per-row dot products <R q, uhat_j> of Sec. 3.5 form a dense contraction:
+// (rows of a partition x D) decoded codewords times (D x queries) rotated
+// queries.  This path
+//   1. inverts the probe lists into per-partition query lists,
+//   2. takes a per-query lower bound theta_q on the k-th best score from a
+//      one-partition pass of the single-query scan (the k-th best score of
+//      any subset of the candidates is <= the k-th best of all of them),
+//   3. for every (partition, tile of up to 128 of its queries) decodes the
+//      codes of 128-row tiles once into shared memory as fp16 (the codebook
+//      components are binary16-exact) and multiplies them on the tensor cores
+//      with the queries split into fp16 hi + lo parts (fp32 accumulation: the
+//      split keeps about 22 significant bits of the query), then applies
+//      s = G (cs + L dot) and appends only the candidates with s >= theta_q to
+//      a per-query buffer,
+//   4. takes the exact top-k of every buffer, ordered by (score desc, id asc);
+//      a query whose buffer overflowed is re-scanned by the single-query path.
+#include <cuda_fp16.h>
+#include <cuda_runtime.h>
+#include <math_constants.h>
+
+#include <climits>
+
+#include "device_common.cuh"
+#include "launch.h"
+
+namespace rslm {
+namespace {
+
+constexpr int kNQ = 128;    // queries per work item
+constexpr int kMR = 128;    // rows per tile
+constexpr int kKC = 128;    // dimensions per K chunk held in shared memory
+
+// ------------------------------------------------------ probe-list inversion
+// Pairs (query q, probe slot j < eff) of probe lists with rows `stride` long.
+__global__ void count_pairs_kernel(const int32_t* __restrict__ probes, int64_t nq, int stride, int eff,
+                                   int nlist, int* __restrict__ cnt, int* err) {
+  const int64_t npairs = nq * eff;
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < npairs;
+       i += int64_t(gridDim.x) * blockDim.x) {
+    const int p = probes[(i / eff) * stride + i % eff];
+    if (p >= 0 && p < nlist) atomicAdd(&cnt[p], 1);
+    else set_device_error(err, kErrBadProbe);
+  }
+}
+
+// Single block: off[p] = exclusive prefix of cnt; items[p] = prefix of
+// ceil(cnt / kNQ); off[nlist], items[nlist] = totals.
+__global__ void scan_lists_kernel(const int* __restrict__ cnt, int nlist, int* __restrict__ off,
+                                  int* __restrict__ items) {
+  __shared__ int scratch[32];
+  int run_o = 0, run_i = 0;
+  for (int base = 0; base < nlist; base += blockDim.x) {
+    const int p = base + threadIdx.x;
+    const int c = p < nlist ? cnt[p] : 0;
+    int tot_o, tot_i;
+    const int eo = block_exclusive_scan(c, scratch, &tot_o);
+    const int ei = block_exclusive_scan((c + kNQ - 1) / kNQ, scratch, &tot_i);
+    if (p < nlist) {
+      off[p] = run_o + eo;
+      items[p] = run_i + ei;
+    }
+    run_o += tot_o;
+    run_i += tot_i;
+  }
+  if (threadIdx.x == 0) {
+    off[nlist] = run_o;
+    items[nlist] = run_i;
+  }
+}
+
+__global__ void scatter_pairs_kernel(const int32_t* __restrict__ probes, const float* __restrict__ cs,
+                                     int64_t nq, int stride, int eff, int nlist,
+                                     const int* __restrict__ off, int* __restrict__ fill,
+                                     int32_t* __restrict__ lq, float* __restrict__ lcs) {
+  const int64_t npairs = nq * eff;
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < npairs;
+       i += int64_t(gridDim.x) * blockDim.x) {
+    const int64_t src = (i / eff) * stride + i % eff;
+    const int p = probes[src];
+    if (p < 0 || p >= nlist) continue;
+    const int at = off[p] + atomicAdd(&fill[p], 1);
+    lq[at] = int32_t(i / eff);
+    lcs[at] = cs[src];
+  }
+}
+
+// --------------------------------------------------------- query operands
+// q * 2^s (s puts max |q| in [1024, 2048)) split into fp16 hi + lo;
+// inv = 2^-s.  Dimensions Dp..Dp16 are zero.
+__global__ void split_queries_kernel(const float* __restrict__ qrot, int64_t nq, int Dp, int Dp16,
+                                     __half* __restrict__ qhi, __half* __restrict__ qlo,
+                                     float* __restrict__ qinv) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, W = blockDim.x >> 5;
+  for (int64_t q = int64_t(blockIdx.x) * W + warp; q < nq; q += int64_t(gridDim.x) * W) {
+    const float* src = qrot + q * Dp;
+    float m = 0.0f;
+    for (int d = lane; d < Dp; d += 32) m = fmaxf(m, fabsf(src[d]));
+#pragma unroll
+    for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
+    int e = 0;
+    if (m > 0.0f) frexpf(m, &e);  // m in [2^(e-1), 2^e)
+    const int s = 11 - e;
+    const float sc = ldexpf(1.0f, s);
+    for (int d = lane; d < Dp16; d += 32) {
+      const float v = d < Dp ? src[d] * sc : 0.0f;
+      const __half h = __float2half_rn(v);
+      qhi[q * Dp16 + d] = h;
+      qlo[q * Dp16 + d] = __float2half_rn(v - __half2float(h));
+    }
+    if (lane == 0) qinv[q] = ldexpf(1.0f, -s);
+  }
+}
+
+// Radix select, by one block, of the k-th largest order key among n scores
+// (n > k).  Returns the key; every thread gets it.
+__device__ uint32_t block_kth_key(const float* s, int n, int k, uint32_t* hist, uint32_t* sh) {
+  const int tid = threadIdx.x;
+  uint32_t prefix = 0, mask = 0, rem = uint32_t(k);
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0;
+    __syncthreads();
+    for (int base = 0; base < n; base += blockDim.x) {
+      const int i = base + tid;
+      const uint32_t kk = i < n ? float_order_key(s[i]) : 0u;
+      warp_hist_add(hist, (kk >> shift) & 255u, i < n && (kk & mask) == prefix);
+    }
+    __syncthreads();
+    if (tid == 0) {
+      uint32_t cum = 0;
+      int b = 255;
+      for (; b > 0; --b) {
+        if (cum + hist[b] >= rem) break;
+        cum += hist[b];
+      }
+      sh[0] = rem - cum;
+      sh[1] = prefix | (uint32_t(b) << shift);
+    }
+    __syncthreads();
+    rem = sh[0];
+    prefix = sh[1];
+    mask |= 255u << shift;
+    __syncthreads();
+  }
+  return prefix;
+}
+
+// theta_q = k-th best score of the query's first probed partition (all of its
+// candidates are in the buffer), lowered by a relative margin of 1e-6; -inf
+// when that partition has fewer than k rows.
+__global__ void theta_kernel(const float* __restrict__ buf_s, const int* __restrict__ cnt, int cap,
+                             int k, float* __restrict__ theta) {
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t sh[2];
+  const int64_t q = blockIdx.x;
+  const int n = min(cnt[q], cap);
+  float t = -CUDART_INF_F;
+  if (n >= k) {
+    const float* s = buf_s + q * cap;
+    if (n == k) {
+      // smallest of the n scores
+      float m = CUDART_INF_F;
+      for (int i = threadIdx.x; i < n; i += blockDim.x) m = fminf(m, s[i]);
+      for (int o = 16; o; o >>= 1) m = fminf(m, __shfl_xor_sync(kFull, m, o));
+      if ((threadIdx.x & 31) == 0) hist[threadIdx.x >> 5] = __float_as_uint(m);
+      __syncthreads();
+      if (threadIdx.x == 0) {
+        for (int w = 0; w < int(blockDim.x >> 5); ++w) m = fminf(m, __uint_as_float(hist[w]));
+        hist[255] = __float_as_uint(m);
+      }
+      __syncthreads();
+      t = __uint_as_float(hist[255]);
+    } else {
+      t = float_from_order_key(block_kth_key(s, n, k, hist, sh));
+    }
+    t = t - 1e-6f * fabsf(t) - 1e-30f;
+  }
+  if (threadIdx.x == 0) theta[q] = t;
+}
+
+// ------------------------------------------------- tcgen05 / mbarrier helpers
+// Shared-memory matrix descriptor of a K-major operand without swizzle: core
+// matrices of 8 rows x 16 bytes stored as 128 contiguous bytes; `lbo` = byte
+// distance between core matrices adjacent along K, `sbo` = between 8-row
+// groups adjacent along M (or N).  Bits 46-47 hold the descriptor version (1).
+__device__ __forceinline__ uint64_t smem_desc(uint32_t saddr, uint32_t lbo, uint32_t sbo) {
+  return uint64_t((saddr >> 4) & 0x3FFFu) | (uint64_t((lbo >> 4) & 0x3FFFu) << 16) |
+         (uint64_t((sbo >> 4) & 0x3FFFu) << 32) | (uint64_t(1) << 46);
+}
+
+// Instruction descriptor of tcgen05.mma kind::f16: D f32 (bits 4-5 = 1),
+// A and B f16 (formats 0), both K-major, N >> 3 at bits 17-22, M >> 4 at
+// bits 24-28.
+__host__ __device__ constexpr uint32_t f16_idesc(int M, int N) {
+  return (1u << 4) | (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
+}
+
+__device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
+                                         uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], %1, %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "l"(adesc), "l"(bdesc), "r"(idesc), "r"(accumulate));
+}
+
+__device__ __forceinline__ void umma_commit(uint32_t mbar) {
+  asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(mbar)
+               : "memory");
+}
+
+__device__ __forceinline__ void fence_after_sync() {
+  asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_before_sync() {
+  asm volatile("tcgen05.fence::before_thread_sync;" ::: "memory");
+}
+__device__ __forceinline__ void fence_proxy_async() {
+  asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
+}
+
+// Bounded wait for the mbarrier phase `parity` to complete.
+__device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t parity) {
+  for (int i = 0; i < (1 << 22); ++i) {
+    uint32_t ok;
+    asm volatile(
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        " selp.u32 %0, 1, 0, p;\n}\n"
+        : "=r"(ok)
+        : "r"(mbar), "r"(parity)
+        : "memory");
+    if (ok) return true;
+  }
+  return false;
+}
+
+// 1-D bulk copy global -> shared on the async proxy, completing `bytes` of
+// transaction count on `mbar` (one arrival with the expected byte count).
+__device__ __forceinline__ void tma_load_1d(uint32_t dst, const void* src, uint32_t bytes,
+                                            uint32_t mbar) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mbar), "r"(bytes)
+               : "memory");
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(mbar)
+      : "memory");
+}
+
+// 32 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
+  uint32_t r[32];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x32.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31}, [%32];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15]), "=r"(r[16]), "=r"(r[17]), "=r"(r[18]), "=r"(r[19]), "=r"(r[20]),
+        "=r"(r[21]), "=r"(r[22]), "=r"(r[23]), "=r"(r[24]), "=r"(r[25]), "=r"(r[26]), "=r"(r[27]),
+        "=r"(r[28]), "=r"(r[29]), "=r"(r[30]), "=r"(r[31])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+struct BatchArgs {
+  const uint8_t* codes;
+  const uint32_t* scales;
+  const int64_t* part_off;
+  const int32_t* part_n;
+  int nlist;
+  int stride, chunk, g, Dp16, nkc;
+  uint32_t cbbits[64];  // codebook components as binary16 bits, K x g
+  const int* off;       // [nlist + 1] per-partition query list offsets
+  const int* items;     // [nlist + 1] per-partition work-item offsets
+  const int32_t* lq;
+  const float* lcs;
+  const __half* qhi;
+  const __half* qlo;
+  const float* qinv;
+  const float* theta;  // nullptr: keep every candidate
+  float* buf_s;
+  int32_t* buf_p;
+  int* cnt;
+  int cap;
+  int* work;
+  int* err;
+};
+
+constexpr int kSBO = (kKC / 8) * 128;  // bytes between 8-row groups of an operand tile
+constexpr int kTileBytes = kMR * kKC * 2;
+constexpr uint32_t kTmemCols = 128;
+// Codes of one K chunk of a tile: kKC / g positions of 4 bits per row.
+__host__ __device__ constexpr int slab_bytes(int g) { return kMR * kKC / (2 * g); }
+
+// Shared offset of element (row, k) of a K-major operand tile (core
+// matrices of 8 rows x 8 halves, K-adjacent ones 128 bytes apart).
+__device__ __forceinline__ uint32_t tile_off(int row, int k8) {
+  return uint32_t((row >> 3) * kSBO + k8 * 128 + (row & 7) * 16);
+}
+
+// One CTA of 8 warps works on (partition, query tile) items taken from a
+// global counter.  Per 128-row tile of the partition: all threads decode the
+// codes into the A operand (fp16) and, for the first tile or when D needs
+// several K chunks, copy the queries' hi / lo parts into two B operands;
+// thread 0 issues the tcgen05.mma chain into a 128 x 128 fp32 TMEM
+// accumulator (rows x queries) and commits it to an mbarrier; then every
+// thread reads its row of the accumulator (warps w and w + 4 share a lane
+// quadrant and split the 128 columns) and applies the epilogue.
+// Per-query epilogue parameters of a work item.
+struct QParam {
+  float inv;  // 2^-s of the query's hi / lo split
+  float cs;   // <q, c_p>
+  float th;   // theta_q (+inf for padding columns)
+  int q;      // query index (-1 for padding columns)
+};
+
+// Decoded halves of the two codes of one byte: 2 G halves.
+template <int G> struct DecT;
+template <> struct DecT<1> { using T = uint32_t; };
+template <> struct DecT<2> { using T = uint2; };
+template <> struct DecT<4> { using T = uint4; };
+
+template <int G>
+__global__ void __launch_bounds__(256, 2) batched_scan_kernel(const __grid_constant__ BatchArgs a) {
+  using Dec = typename DecT<G>::T;
+  extern __shared__ __align__(16) uint8_t bsm[];
+  uint8_t* As = bsm;
+  uint8_t* Bh = As + kTileBytes;
+  uint8_t* Bl = Bh + kTileBytes;
+  uint8_t* slab = Bl + kTileBytes;  // codes of the current (tile, K chunk), copied by TMA
+  QParam* qp = reinterpret_cast<QParam*>(slab + slab_bytes(G));
+  Dec* dec = reinterpret_cast<Dec*>(qp + kNQ);  // byte -> its two codes' 2 G halves
+  __shared__ __align__(8) uint64_t mbar_storage;
+  __shared__ __align__(8) uint64_t tma_mbar_storage;
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ int s_item;
+  __shared__ int s_fail;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  constexpr int g = G;
+
+  // byte -> the 2 g halves of its two codes (low nibble first)
+  for (int b = tid; b < 256; b += blockDim.x) {
+    uint32_t h[8] = {0, 0, 0, 0, 0, 0, 0, 0};
+#pragma unroll
+    for (int j = 0; j < g; ++j) {
+      h[j] = a.cbbits[(b & 15) * g + j];
+      h[g + j] = a.cbbits[(b >> 4) * g + j];
+    }
+    const uint32_t w0 = h[0] | (h[1] << 16), w1 = h[2] | (h[3] << 16);
+    const uint32_t w2 = h[4] | (h[5] << 16), w3 = h[6] | (h[7] << 16);
+    if constexpr (G == 1) dec[b] = w0;
+    else if constexpr (G == 2) dec[b] = make_uint2(w0, w1);
+    else dec[b] = make_uint4(w0, w1, w2, w3);
+  }
+  const uint32_t mbar = uint32_t(__cvta_generic_to_shared(&mbar_storage));
+  const uint32_t tmbar = uint32_t(__cvta_generic_to_shared(&tma_mbar_storage));
+  const uint32_t slab_addr = uint32_t(__cvta_generic_to_shared(slab));
+  if (tid == 0) {
+    s_fail = 0;
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar) : "memory");
+    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(tmbar) : "memory");
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    const uint32_t dst = uint32_t(__cvta_generic_to_shared(&tmem_base_sh));
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst),
+                 "r"(kTmemCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = tmem_base_sh;
+  const uint32_t as_addr = uint32_t(__cvta_generic_to_shared(As));
+  const uint32_t bh_addr = uint32_t(__cvta_generic_to_shared(Bh));
+  const uint32_t bl_addr = uint32_t(__cvta_generic_to_shared(Bl));
+  constexpr uint32_t idesc = f16_idesc(kMR, kNQ);
+  const int n_items = a.items[a.nlist];
+  const int quad = warp & 3;          // TMEM lane quadrant of this warp
+  const int colh = (warp >> 2) * 64;  // the 64 accumulator columns this warp reads
+  const int row_t = quad * 32 + lane; // this thread's row of the tile
+  uint32_t phase = 0, tphase = 0;
+  const int CH = a.chunk;
+  // Chunks [c0, c1) of the tile-interleaved layout hold K chunk kc of a tile.
+  auto slab_range = [&](int kc, int& c0, int& c1) {
+    const int k0 = kc * kKC;
+    const int klen = min(kKC, a.Dp16 - k0);
+    const int b0 = k0 / (2 * g), b1 = b0 + (klen + 2 * g - 1) / (2 * g);
+    c0 = b0 / CH;
+    c1 = min((b1 + CH - 1) / CH, a.stride / CH);
+  };
+
+  for (;;) {
+    __syncthreads();
+    if (tid == 0) s_item = s_fail ? n_items : atomicAdd(a.work, 1);
+    __syncthreads();
+    const int item = s_item;
+    if (item >= n_items) break;
+    int lo = 0, hi = a.nlist - 1;  // partition p: items[p] <= item < items[p + 1]
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.items[mid] <= item) lo = mid;
+      else hi = mid - 1;
+    }
+    const int p = lo;
+    const int q0 = a.off[p] + (item - a.items[p]) * kNQ;
+    const int nqt = min(kNQ, a.off[p + 1] - q0);
+    for (int j = tid; j < kNQ; j += blockDim.x) {
+      const bool v = j < nqt;
+      const int q = v ? a.lq[q0 + j] : -1;
+      QParam pr;
+      pr.q = q;
+      pr.cs = v ? a.lcs[q0 + j] : 0.0f;
+      pr.th = v ? (a.theta ? a.theta[q] : -CUDART_INF_F) : CUDART_INF_F;
+      pr.inv = v ? a.qinv[q] : 0.0f;
+      qp[j] = pr;
+    }
+    __syncthreads();
+    const int nrows = a.part_n[p];
+    const int64_t slot0 = a.part_off[p];
+    const int ntiles = (nrows + kMR - 1) / kMR;
+    // TMA of the codes of (tile t, K chunk kc) into the slab.
+    auto issue_slab = [&](int t, int kc) {
+      int c0, c1;
+      slab_range(kc, c0, c1);
+      const uint8_t* src = a.codes + (slot0 + int64_t(t) * kMR) * a.stride + size_t(c0) * kMR * CH;
+      tma_load_1d(slab_addr, src, uint32_t((c1 - c0) * kMR * CH), tmbar);
+    };
+    if (tid == 0 && ntiles > 0) issue_slab(0, 0);
+    for (int t = 0; t < ntiles; ++t) {
+      const int nvalid = min(kMR, nrows - t * kMR);
+      for (int kc = 0; kc < a.nkc; ++kc) {
+        const int k0 = kc * kKC;
+        const int klen = min(kKC, a.Dp16 - k0);
+        if (t == 0 || a.nkc > 1) {
+          const int k8n = klen / 8;
+          for (int e = tid; e < kNQ * k8n; e += blockDim.x) {
+            const int j = e / k8n, k8 = e - j * k8n;
+            uint4 h = make_uint4(0, 0, 0, 0), l = make_uint4(0, 0, 0, 0);
+            if (j < nqt) {
+              const int64_t src = int64_t(qp[j].q) * a.Dp16 + k0 + k8 * 8;
+              h = *reinterpret_cast<const uint4*>(a.qhi + src);
+              l = *reinterpret_cast<const uint4*>(a.qlo + src);
+            }
+            *reinterpret_cast<uint4*>(Bh + tile_off(j, k8)) = h;
+            *reinterpret_cast<uint4*>(Bl + tile_off(j, k8)) = l;
+          }
+        }
+        // Decode: one 32-bit code word (8 codes, 8 g dimensions) per unit,
+        // read from the slab once its TMA has landed.
+        if (!mbar_wait(tmbar, tphase)) {
+          if (lane == 0) {
+            set_device_error(a.err, kErrTimeout);
+            atomicExch(&s_fail, 1);
+          }
+        }
+        tphase ^= 1u;
+        int c0, c1;
+        slab_range(kc, c0, c1);
+        const int w0 = k0 / (8 * g);                 // first code word of the chunk
+        const int nw = (klen + 8 * g - 1) / (8 * g);  // code words covering it
+        const int k8end = klen / 8;
+        for (int e = tid; e < kMR * nw; e += blockDim.x) {
+          const int r = e % kMR, wi = e / kMR;
+          const int b = 4 * (w0 + wi);
+          const int c = b / CH;
+          uint32_t word = 0;
+          if (c < c1)
+            word = *reinterpret_cast<const uint32_t*>(slab + ((c - c0) * kMR + r) * CH + (b % CH));
+          const int k8base = wi * g;  // k8 groups of this word: g of them
+#pragma unroll
+          for (int bb = 0; bb < 4; ++bb) {
+            // byte bb covers 2 g halves: k8 group k8base + (2 g bb) / 8 at half offset (2 g bb) % 8
+            const int hoff = 2 * g * bb;
+            if (k8base + hoff / 8 >= k8end) break;  // beyond this chunk's dimensions
+            *reinterpret_cast<Dec*>(As + tile_off(r, k8base + hoff / 8) + (hoff % 8) * 2) =
+                dec[(word >> (8 * bb)) & 255u];
+          }
+        }
+        fence_proxy_async();
+        fence_before_sync();
+        __syncthreads();
+        if (tid == 0) {
+          fence_after_sync();
+          for (int ks = 0; ks < klen / 16; ++ks) {
+            const uint64_t ad = smem_desc(as_addr + ks * 256, 128, kSBO);
+            umma_f16(tmem, ad, smem_desc(bh_addr + ks * 256, 128, kSBO), idesc,
+                     (kc > 0 || ks > 0) ? 1u : 0u);
+            umma_f16(tmem, ad, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
+          }
+          umma_commit(mbar);
+          // every thread has finished reading the slab: fetch the next unit's codes
+          if (kc + 1 < a.nkc) issue_slab(t, kc + 1);
+          else if (t + 1 < ntiles) issue_slab(t + 1, 0);
+        }
+        if (!mbar_wait(mbar, phase)) {
+          if (lane == 0) {
+            set_device_error(a.err, kErrTimeout);
+            atomicExch(&s_fail, 1);
+          }
+        }
+        phase ^= 1u;
+        fence_after_sync();
+      }
+      // Epilogue: this thread's row, 64 query columns.
+      float L = 0.0f, Gs = 0.0f;
+      if (row_t < nvalid) {
+        const uint32_t sc = a.scales[slot0 + int64_t(t) * kMR + row_t];
+        L = ue7m9_to_f32(sc & 0xffffu);
+        Gs = ue4m12_to_f32(sc >> 16);
+      }
+      const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row_t);
+#pragma unroll
+      for (int half = 0; half < 2; ++half) {
+        float v[32];
+        tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + uint32_t(colh + half * 32), v);
+        if (row_t < nvalid) {
+#pragma unroll
+          for (int i = 0; i < 32; ++i) {
+            const int col = colh + half * 32 + i;
+            const QParam pr = qp[col];
+            const float s = Gs * fmaf(L, v[i] * pr.inv, pr.cs);
+            if (s >= pr.th && col < nqt) {
+              const int q = pr.q;
+              const int at = atomicAdd(&a.cnt[q], 1);
+              if (at < a.cap) {
+                a.buf_s[int64_t(q) * a.cap + at] = s;
+                a.buf_p[int64_t(q) * a.cap + at] = pos;
+              }
+            }
+          }
+        }
+      }
+      fence_before_sync();
+      __syncthreads();
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {
+    fence_after_sync();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------------ pipelined kernel (D <= 128)
+// The same computation for a single K chunk (padded D <= 128), with the
+// stages overlapped across the 128-row tiles of an item:
+//   warps 0-7  decode: thread = (row, half of the row's columns); wait for
+//              the tile's codes (TMA), decode them into registers and store
+//              them into the A operand buffer of that tile in TMEM
+//              (tcgen05.st; lane = row, two halves per 32-bit column);
+//   warp 16    lane 0 issues the TMA copies (two tiles ahead) and the MMAs
+//              (A from TMEM, B hi / lo from shared memory) into one of two
+//              TMEM accumulators;
+//   warps 8-15 epilogue: thread = (row, half of the 128 query columns); read
+//              its accumulator part, apply s = G (cs + L dot) and append
+//              candidates >= theta_q.
+// A warp reaches only its TMEM lane quadrant (warp index mod 4), so every
+// role spans the four quadrants twice.
+// A and the accumulator are double-buffered (TMEM columns: acc 0-127 and
+// 128-255, A 256-319 and 320-383).  mbarriers: slab_full (TMA landed),
+// a_full (8 decoder warps wrote A), mma_done (the MMAs of a tile finished:
+// A free, accumulator ready), acc_empty (8 epilogue warps read it).  Every
+// wait is bounded; a timeout sets the error flag and stops the item loop.
+constexpr int kPipeThreads = 17 * 32;  // 8 decoder, 8 epilogue, 1 producer warps
+constexpr int kProducerWarp = 16;
+constexpr uint32_t kPipeCols = 512;
+__device__ __forceinline__ uint32_t acc_col(uint32_t b) { return b * 128u; }       // accumulators
+__device__ __forceinline__ uint32_t a_col(uint32_t b) { return 256u + b * 64u; }   // A operands
+
+__device__ __forceinline__ void mbar_init(uint32_t mbar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(mbar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void mbar_arrive(uint32_t mbar) {
+  asm volatile("mbarrier.arrive.shared::cta.b64 _, [%0];" ::"r"(mbar) : "memory");
+}
+
+__device__ __forceinline__ void umma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, uint64_t bdesc,
+                                            uint32_t idesc, uint32_t accumulate) {
+  asm volatile(
+      "{\n .reg .pred p;\n setp.ne.b32 p, %4, 0;\n"
+      " tcgen05.mma.cta_group::1.kind::f16 [%0], [%1], %2, %3, p;\n}\n" ::"r"(d_tmem),
+      "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate));
+}
+
+// 64 consecutive 32-bit columns of this thread's TMEM lane <- v.
+__device__ __forceinline__ void tmem_st64(uint32_t taddr, const uint32_t (&v)[64]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x64.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,"
+      "%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,"
+      "%61,%62,%63,%64};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+      "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]),
+      "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]),
+      "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31]),
+      "r"(v[32]), "r"(v[33]), "r"(v[34]), "r"(v[35]), "r"(v[36]), "r"(v[37]), "r"(v[38]), "r"(v[39]),
+      "r"(v[40]), "r"(v[41]), "r"(v[42]), "r"(v[43]), "r"(v[44]), "r"(v[45]), "r"(v[46]), "r"(v[47]),
+      "r"(v[48]), "r"(v[49]), "r"(v[50]), "r"(v[51]), "r"(v[52]), "r"(v[53]), "r"(v[54]), "r"(v[55]),
+      "r"(v[56]), "r"(v[57]), "r"(v[58]), "r"(v[59]), "r"(v[60]), "r"(v[61]), "r"(v[62]), "r"(v[63])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+// 32 consecutive 32-bit columns of this thread's TMEM lane <- v.
+__device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
+  asm volatile(
+      "tcgen05.st.sync.aligned.32x32b.x32.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32};" ::"r"(taddr),
+      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
+      "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]),
+      "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]),
+      "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31])
+      : "memory");
+  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
+}
+
+template <int G>
+__global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
+  extern __shared__ __align__(16) uint8_t psm[];
+  uint8_t* Bh = psm;
+  uint8_t* Bl = Bh + kTileBytes;
+  uint8_t* slab0 = Bl + kTileBytes;                  // two slabs of slab_bytes(G)
+  QParam* qp = reinterpret_cast<QParam*>(slab0 + 2 * slab_bytes(G));
+  // decode tables: G = 1: byte -> 2 halves; G = 2: code -> 2 halves; G = 4: code -> 4 halves
+  uint32_t* t32 = reinterpret_cast<uint32_t*>(qp + kNQ);
+  __shared__ __align__(8) uint64_t bars[8];  // slab_full[2], a_full[2], mma_done[2], acc_empty[2]
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ int s_item;
+  __shared__ int s_fail;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int CH = a.chunk;
+
+  if (G == 1) {
+    for (int b = tid; b < 256; b += blockDim.x) t32[b] = a.cbbits[b & 15] | (a.cbbits[b >> 4] << 16);
+  } else if (G == 2) {
+    for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[2 * c] | (a.cbbits[2 * c + 1] << 16);
+  } else {
+    for (int c = tid; c < 16; c += blockDim.x) {
+      t32[2 * c] = a.cbbits[4 * c] | (a.cbbits[4 * c + 1] << 16);
+      t32[2 * c + 1] = a.cbbits[4 * c + 2] | (a.cbbits[4 * c + 3] << 16);
+    }
+  }
+  const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
+  auto slab_full = [&](int b) { return bar0 + 8u * uint32_t(b); };
+  auto a_full = [&](int b) { return bar0 + 8u * uint32_t(2 + b); };
+  auto mma_done = [&](int b) { return bar0 + 8u * uint32_t(4 + b); };
+  auto acc_empty = [&](int b) { return bar0 + 8u * uint32_t(6 + b); };
+  if (tid == 0) {
+    s_fail = 0;
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(slab_full(b), 1);
+      mbar_init(a_full(b), 8);
+      mbar_init(mma_done(b), 1);
+      mbar_init(acc_empty(b), 8);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    const uint32_t dst = uint32_t(__cvta_generic_to_shared(&tmem_base_sh));
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst),
+                 "r"(kPipeCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = tmem_base_sh;
+  const uint32_t bh_addr = uint32_t(__cvta_generic_to_shared(Bh));
+  const uint32_t bl_addr = uint32_t(__cvta_generic_to_shared(Bl));
+  const uint32_t slab_addr0 = uint32_t(__cvta_generic_to_shared(slab0));
+  constexpr uint32_t idesc = f16_idesc(kMR, kNQ);
+  const int n_items = a.items[a.nlist];
+  const int klen = a.Dp16;                   // single K chunk
+  const int nbytes = (klen + 2 * G - 1) / (2 * G);
+  int c1 = min((nbytes + CH - 1) / CH, a.stride / CH);  // code chunks of a row used
+  const uint32_t slab_len = uint32_t(c1 * kMR * CH);
+  uint32_t gt = 0;  // tiles this CTA has processed (buffer = gt & 1, use = gt >> 1)
+  auto fail = [&]() {
+    set_device_error(a.err, kErrTimeout);
+    atomicExch(&s_fail, 1);
+  };
+
+  for (;;) {
+    __syncthreads();
+    if (tid == 0) s_item = s_fail ? n_items : atomicAdd(a.work, 1);
+    __syncthreads();
+    const int item = s_item;
+    if (item >= n_items) break;
+    int lo = 0, hi = a.nlist - 1;
+    while (lo < hi) {
+      const int mid = (lo + hi + 1) >> 1;
+      if (a.items[mid] <= item) lo = mid;
+      else hi = mid - 1;
+    }
+    const int p = lo;
+    const int q0 = a.off[p] + (item - a.items[p]) * kNQ;
+    const int nqt = min(kNQ, a.off[p + 1] - q0);
+    for (int j = tid; j < kNQ; j += blockDim.x) {
+      const bool v = j < nqt;
+      const int q = v ? a.lq[q0 + j] : -1;
+      QParam pr;
+      pr.q = q;
+      pr.cs = v ? a.lcs[q0 + j] : 0.0f;
+      pr.th = v ? (a.theta ? a.theta[q] : -CUDART_INF_F) : CUDART_INF_F;
+      pr.inv = v ? a.qinv[q] : 0.0f;
+      qp[j] = pr;
+    }
+    __syncthreads();
+    // B operands (hi / lo parts of the item's queries); the previous item's
+    // MMAs have all completed (its epilogue waited for them).
+    {
+      const int k8n = klen / 8;
+      for (int e = tid; e < kNQ * k8n; e += blockDim.x) {
+        const int j = e / k8n, k8 = e - j * k8n;
+        uint4 h = make_uint4(0, 0, 0, 0), l = make_uint4(0, 0, 0, 0);
+        if (j < nqt) {
+          const int64_t src = int64_t(qp[j].q) * a.Dp16 + k8 * 8;
+          h = *reinterpret_cast<const uint4*>(a.qhi + src);
+          l = *reinterpret_cast<const uint4*>(a.qlo + src);
+        }
+        *reinterpret_cast<uint4*>(Bh + tile_off(j, k8)) = h;
+        *reinterpret_cast<uint4*>(Bl + tile_off(j, k8)) = l;
+      }
+    }
+    fence_proxy_async();
+    __syncthreads();
+    const int nrows = a.part_n[p];
+    const int64_t slot0 = a.part_off[p];
+    const int ntiles = (nrows + kMR - 1) / kMR;
+    const uint8_t* codes0 = a.codes + slot0 * a.stride;
+
+    if (warp == kProducerWarp) {
+      // ---------------- producer: TMA two tiles ahead, MMAs
+      if (lane == 0) {
+        for (int t = 0; t < min(ntiles, 2); ++t)
+          tma_load_1d(slab_addr0 + uint32_t(((gt + t) & 1) * slab_bytes(G)),
+                      codes0 + size_t(t) * kMR * a.stride, slab_len, slab_full((gt + t) & 1));
+        for (int t = 0; t < ntiles; ++t) {
+          const uint32_t g2 = gt + t, b = g2 & 1, u = g2 >> 1;
+          if (!mbar_wait(a_full(b), u & 1)) fail();
+          if (u > 0 && !mbar_wait(acc_empty(b), (u - 1) & 1)) fail();
+          fence_after_sync();
+          for (int ks = 0; ks < klen / 16; ++ks) {
+            const uint32_t at = tmem + a_col(b) + uint32_t(ks * 8);
+            umma_f16_ts(tmem + acc_col(b), at, smem_desc(bh_addr + ks * 256, 128, kSBO), idesc,
+                        ks > 0 ? 1u : 0u);
+            umma_f16_ts(tmem + acc_col(b), at, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
+          }
+          umma_commit(mma_done(b));
+          // decode of tile t is done (a_full), so its slab is free for tile t + 2
+          if (t + 2 < ntiles)
+            tma_load_1d(slab_addr0 + b * uint32_t(slab_bytes(G)), codes0 + size_t(t + 2) * kMR * a.stride,
+                        slab_len, slab_full(b));
+        }
+      }
+      __syncwarp();
+    } else if (warp < 8) {
+      // ---------------- decoders: thread = row r of the tile, column half dh
+      const int r = (warp & 3) * 32 + lane;
+      const int dh = warp >> 2;
+      for (int t = 0; t < ntiles; ++t) {
+        const uint32_t g2 = gt + t, b = g2 & 1, u = g2 >> 1;
+        if (!mbar_wait(slab_full(b), u & 1)) fail();
+        const uint8_t* sl = slab0 + b * slab_bytes(G);
+        uint32_t av[32];
+        // word w (bytes 4w .. 4w + 3) of row r in the slab
+        auto word_at = [&](int w) -> uint32_t {
+          const int byte = 4 * w;
+          const int c = byte / CH;
+          if (c >= c1) return 0u;
+          return *reinterpret_cast<const uint32_t*>(sl + (c * kMR + r) * CH + (byte % CH));
+        };
+        // 32 columns = 64 halves = 64 / G codes = 32 / G bytes = 8 / G words
+        if constexpr (G == 1) {
+#pragma unroll
+          for (int w = 0; w < 8; ++w) {
+            const uint32_t wd = word_at(dh * 8 + w);
+#pragma unroll
+            for (int bb = 0; bb < 4; ++bb) av[4 * w + bb] = t32[(wd >> (8 * bb)) & 255u];
+          }
+        } else if constexpr (G == 2) {
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            const uint32_t wd = word_at(dh * 4 + w);
+#pragma unroll
+            for (int n = 0; n < 8; ++n) av[8 * w + n] = t32[(wd >> (4 * n)) & 15u];
+          }
+        } else {
+#pragma unroll
+          for (int w = 0; w < 2; ++w) {
+            const uint32_t wd = word_at(dh * 2 + w);
+#pragma unroll
+            for (int n = 0; n < 8; ++n) {
+              const uint32_t c = (wd >> (4 * n)) & 15u;
+              av[16 * w + 2 * n] = t32[2 * c];
+              av[16 * w + 2 * n + 1] = t32[2 * c + 1];
+            }
+          }
+        }
+        // A buffer b is free once the MMAs of tile g2 - 2 have completed
+        if (u > 0 && !mbar_wait(mma_done(b), (u - 1) & 1)) fail();
+        fence_after_sync();
+        tmem_st32(tmem + (uint32_t((warp & 3) * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
+        fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(a_full(b));
+      }
+    } else {
+      // ---------------- epilogue: thread = row of quadrant warp % 4, columns eh * 64 ..
+      const int quad = warp & 3;
+      const int eh = (warp - 8) >> 2;
+      const int row = quad * 32 + lane;
+      for (int t = 0; t < ntiles; ++t) {
+        const uint32_t g2 = gt + t, b = g2 & 1, u = g2 >> 1;
+        const int nvalid = min(kMR, nrows - t * kMR);
+        const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row);
+        float L = 0.0f, Gs = 0.0f;
+        if (row < nvalid) {
+          const uint32_t sc = a.scales[pos];
+          L = ue7m9_to_f32(sc & 0xffffu);
+          Gs = ue4m12_to_f32(sc >> 16);
+        }
+        if (!mbar_wait(mma_done(b), u & 1)) fail();
+        fence_after_sync();
+#pragma unroll 1
+        for (int part = 0; part < 2; ++part) {
+          float v[32];
+          const int cbase = eh * 64 + part * 32;
+          tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(b) + uint32_t(cbase), v);
+          if (part == 1) {
+            fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(acc_empty(b));
+          }
+          if (row < nvalid) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) {
+              const int col = cbase + i;
+              const QParam pr = qp[col];
+              const float sv = Gs * fmaf(L, v[i] * pr.inv, pr.cs);
+              if (sv >= pr.th && col < nqt) {
+                const int at = atomicAdd(&a.cnt[pr.q], 1);
+                if (at < a.cap) {
+                  a.buf_s[int64_t(pr.q) * a.cap + at] = sv;
+                  a.buf_p[int64_t(pr.q) * a.cap + at] = pos;
+                }
+              }
+            }
+          }
+        }
+      }
+    }
+    gt += uint32_t(ntiles);
+  }
+  __syncthreads();
+  if (warp == 0) {
+    fence_after_sync();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kPipeCols)
+                 : "memory");
+  }
+}
+
+// ---------------------------------------------------------------- finalize
+// Exact top-k of a query's buffer by (score desc, id asc).  A buffer that
+// overflowed marks the query for the single-query re-scan.
+__global__ void finalize_kernel(const float* __restrict__ buf_s, const int32_t* __restrict__ buf_p,
+                                const int* __restrict__ cnt, int cap, const int64_t* __restrict__ ids,
+                                int k, int* __restrict__ overflow, int64_t* __restrict__ out_ids,
+                                float* __restrict__ out_scores) {
+  extern __shared__ __align__(16) uint8_t fsm[];
+  __shared__ uint32_t hist[256];
+  __shared__ uint32_t sh_prefix[2];
+  __shared__ uint32_t sh_n;
+  const int64_t q = blockIdx.x;
+  const int tid = threadIdx.x;
+  const int n = cnt[q];
+  if (n > cap) {
+    if (tid == 0) overflow[q] = 1;
+    return;
+  }
+  if (tid == 0) overflow[q] = 0;
+  int p2 = 1;
+  while (p2 < k + 64) p2 <<= 1;
+  float* key = reinterpret_cast<float*>(fsm);
+  int64_t* idv = reinterpret_cast<int64_t*>(fsm + size_t(p2) * 4);
+  const float* s = buf_s + q * cap;
+  const int32_t* pp = buf_p + q * cap;
+  // Threshold T: the k-th largest order key (everything kept when n <= k).
+  uint32_t T = 0;
+  if (n > k) {
+    T = block_kth_key(s, n, k, hist, sh_prefix);
+  }
+  if (tid == 0) sh_n = 0;
+  __syncthreads();
+  for (int i = tid; i < n; i += blockDim.x) {
+    if (float_order_key(s[i]) >= T) {
+      const uint32_t at = atomicAdd(&sh_n, 1u);
+      if (at < uint32_t(p2)) {
+        key[at] = s[i];
+        idv[at] = ids[pp[i]];
+      }
+    }
+  }
+  __syncthreads();
+  const int m = min(int(sh_n), p2);
+  for (int i = m + tid; i < p2; i += blockDim.x) {
+    key[i] = -CUDART_INF_F;
+    idv[i] = LLONG_MAX;
+  }
+  block_bitonic_sort(key, idv, p2);
+  for (int i = tid; i < k; i += blockDim.x) {
+    const bool ok = i < m && idv[i] != LLONG_MAX;
+    out_ids[q * k + i] = ok ? idv[i] : -1;
+    out_scores[q * k + i] = ok ? key[i] : -CUDART_INF_F;
+  }
+}
+
+int blocks_for(int64_t n, int per, int maxb) {
+  int64_t b = (n + per - 1) / per;
+  if (b < 1) b = 1;
+  return int(b < maxb ? b : maxb);
+}
+
+}  // namespace
+
+namespace {
+
+// Per-partition query lists of the probe pairs (q, j < eff).
+struct Lists {
+  int* cnt;
+  int* fill;
+  int* off;
+  int* items;
+  int32_t* lq;
+  float* lcs;
+};
+
+cudaError_t build_lists(const rslm_index* ix, const int32_t* probes, const float* cs, int64_t nq,
+                        int stride, int eff, const Lists& L, cudaStream_t s) {
+  const int nlist = ix->nlist;
+  const int64_t npairs = nq * eff;
+  cudaError_t e = cudaMemsetAsync(L.cnt, 0, size_t(nlist) * 4, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(L.fill, 0, size_t(nlist) * 4, s);
+  if (e != cudaSuccess) return e;
+  count_pairs_kernel<<<blocks_for(npairs, 256, 152 * 8), 256, 0, s>>>(probes, nq, stride, eff, nlist,
+                                                                      L.cnt, ix->d_err);
+  scan_lists_kernel<<<1, 1024, 0, s>>>(L.cnt, nlist, L.off, L.items);
+  scatter_pairs_kernel<<<blocks_for(npairs, 256, 152 * 8), 256, 0, s>>>(
+      probes, cs, nq, stride, eff, nlist, L.off, L.fill, L.lq, L.lcs);
+  return cudaGetLastError();
+}
+
+cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi, const __half* qlo,
+                        const float* qinv, int Dp16, const float* theta, float* bs, int32_t* bp, int* bc,
+                        int cap, int* work, bool profile, cudaStream_t s) {
+  const CodecSpec& c1 = ix->cs1;
+  BatchArgs b;
+  b.codes = ix->codes1;
+  b.scales = ix->scales1;
+  b.part_off = ix->part_off;
+  b.part_n = ix->part_n;
+  b.nlist = ix->nlist;
+  b.stride = c1.stride;
+  b.chunk = c1.chunk;
+  b.g = c1.g;
+  b.Dp16 = Dp16;
+  b.nkc = (Dp16 + kKC - 1) / kKC;
+  for (int i = 0; i < 64; ++i) b.cbbits[i] = __half_as_ushort(__float2half_rn(c1.cbf[i]));
+  b.off = L.off;
+  b.items = L.items;
+  b.lq = L.lq;
+  b.lcs = L.lcs;
+  b.qhi = qhi;
+  b.qlo = qlo;
+  b.qinv = qinv;
+  b.theta = theta;
+  b.buf_s = bs;
+  b.buf_p = bp;
+  b.cnt = bc;
+  b.cap = cap;
+  b.work = work;
+  b.err = ix->d_err;
+  cudaError_t e = cudaMemsetAsync(work, 0, 4, s);
+  if (e != cudaSuccess) return e;
+  const int g = c1.g;
+  const size_t dec_bytes = size_t(256) * 2 * g * 2;  // 2 g halves per byte value
+  const size_t smem = size_t(3) * kTileBytes + slab_bytes(g) + size_t(kNQ) * sizeof(QParam) + dec_bytes;
+  int sms = 152;
+  int dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  if (b.nkc == 1) {
+    // padded D <= 128: the pipelined, warp-specialized kernel (one CTA per SM)
+    const size_t psmem = size_t(2) * kTileBytes + 2 * size_t(slab_bytes(g)) +
+                         size_t(kNQ) * sizeof(QParam) + 256 * 4;
+    auto pk = g == 1 ? batched_pipe_kernel<1> : (g == 2 ? batched_pipe_kernel<2> : batched_pipe_kernel<4>);
+    e = cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(psmem));
+    if (e != cudaSuccess) return e;
+    cudaEvent_t stop = profile ? prof_start(ix, s, "batched_scan_kernel") : nullptr;
+    pk<<<sms, kPipeThreads, psmem, s>>>(b);
+    prof_stop(stop, s);
+    return cudaGetLastError();
+  }
+  auto kern = c1.g == 1 ? batched_scan_kernel<1> : (c1.g == 2 ? batched_scan_kernel<2> : batched_scan_kernel<4>);
+  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  cudaEvent_t stop = profile ? prof_start(ix, s, "batched_scan_kernel") : nullptr;
+  kern<<<sms * 2, 256, smem, s>>>(b);
+  prof_stop(stop, s);
+  return cudaGetLastError();
+}
+
+}  // namespace
+
+cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t nq,
+                                const int32_t* probes, const float* cs, int nprobe, int k,
+                                int64_t* out_ids, float* out_scores, cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  const CodecSpec& c1 = ix->cs1;
+  const int Dp16 = (c1.Dp + 15) / 16 * 16;
+  const int nlist = ix->nlist;
+  const int cap = 16 * k + 1024;                       // per-query candidate buffer
+  const int capA = ix->max_part_n > 0 ? ix->max_part_n : 1;  // first pass: a whole partition
+  const int64_t npairs = nq * nprobe;
+  size_t bytes = 0;
+  auto take = [&](size_t n) {
+    size_t at = bytes;
+    bytes += (n + 255) / 256 * 256;
+    return at;
+  };
+  size_t oL[2][6];
+  for (int l = 0; l < 2; ++l) {
+    const int64_t np = l ? npairs : nq;
+    oL[l][0] = take(size_t(nlist) * 4);
+    oL[l][1] = take(size_t(nlist) * 4);
+    oL[l][2] = take(size_t(nlist + 1) * 4);
+    oL[l][3] = take(size_t(nlist + 1) * 4);
+    oL[l][4] = take(size_t(np) * 4);
+    oL[l][5] = take(size_t(np) * 4);
+  }
+  const size_t o_qhi = take(size_t(nq) * Dp16 * 2), o_qlo = take(size_t(nq) * Dp16 * 2),
+               o_qinv = take(size_t(nq) * 4), o_theta = take(size_t(nq) * 4),
+               o_as = take(size_t(nq) * capA * 4), o_ap = take(size_t(nq) * capA * 4),
+               o_ac = take(size_t(nq) * 4), o_bs = take(size_t(nq) * cap * 4),
+               o_bp = take(size_t(nq) * cap * 4), o_bc = take(size_t(nq) * 4),
+               o_ovf = take(size_t(nq) * 4), o_work = take(4);
+  uint8_t* ws = nullptr;
+  cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, s);
+  if (e != cudaSuccess) return e;
+  Lists L[2];
+  for (int l = 0; l < 2; ++l)
+    L[l] = Lists{reinterpret_cast<int*>(ws + oL[l][0]), reinterpret_cast<int*>(ws + oL[l][1]),
+                 reinterpret_cast<int*>(ws + oL[l][2]), reinterpret_cast<int*>(ws + oL[l][3]),
+                 reinterpret_cast<int32_t*>(ws + oL[l][4]), reinterpret_cast<float*>(ws + oL[l][5])};
+  __half* qhi = reinterpret_cast<__half*>(ws + o_qhi);
+  __half* qlo = reinterpret_cast<__half*>(ws + o_qlo);
+  float* qinv = reinterpret_cast<float*>(ws + o_qinv);
+  float* theta = reinterpret_cast<float*>(ws + o_theta);
+  float* as = reinterpret_cast<float*>(ws + o_as);
+  int32_t* ap = reinterpret_cast<int32_t*>(ws + o_ap);
+  int* ac = reinterpret_cast<int*>(ws + o_ac);
+  float* bs = reinterpret_cast<float*>(ws + o_bs);
+  int32_t* bp = reinterpret_cast<int32_t*>(ws + o_bp);
+  int* bc = reinterpret_cast<int*>(ws + o_bc);
+  int* ovf = reinterpret_cast<int*>(ws + o_ovf);
+  int* work = reinterpret_cast<int*>(ws + o_work);
+
+  // lists: L[0] the first probe of every query, L[1] all probe pairs
+  e = build_lists(ix, probes, cs, nq, nprobe, 1, L[0], s);
+  if (e == cudaSuccess) e = build_lists(ix, probes, cs, nq, nprobe, nprobe, L[1], s);
+  if (e == cudaSuccess) {
+    split_queries_kernel<<<blocks_for(nq, 8, 152 * 32), 256, 0, s>>>(qrot, nq, c1.Dp, Dp16, qhi, qlo,
+                                                                      qinv);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) e = cudaMemsetAsync(ac, 0, size_t(nq) * 4, s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(bc, 0, size_t(nq) * 4, s);
+  // Pass 1: every candidate of each query's first probed partition; its
+  // exact k-th best score bounds the query's k-th best score from below.
+  if (e == cudaSuccess)
+    e = run_batched(ix, L[0], qhi, qlo, qinv, Dp16, nullptr, as, ap, ac, capA, work, false, s);
+  if (e == cudaSuccess) {
+    theta_kernel<<<unsigned(nq), 256, 0, s>>>(as, ac, capA, k, theta);
+    e = cudaGetLastError();
+  }
+  // Pass 2: all probed partitions, keeping candidates >= theta.
+  if (e == cudaSuccess)
+    e = run_batched(ix, L[1], qhi, qlo, qinv, Dp16, theta, bs, bp, bc, cap, work, true, s);
+  if (e == cudaSuccess) {
+    int p2 = 1;
+    while (p2 < k + 64) p2 <<= 1;
+    const size_t smem = size_t(p2) * 12;
+    e = cudaFuncSetAttribute(finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    if (e == cudaSuccess) {
+      finalize_kernel<<<unsigned(nq), 256, smem, s>>>(bs, bp, bc, cap, ix->ids, k, ovf, out_ids, out_scores);
+      e = cudaGetLastError();
+    }
+  }
+  // Queries whose buffer overflowed: exact single-query scan of all probes.
+  if (e == cudaSuccess)
+    e = launch_scan_strided(ix, qrot, nq, probes, nprobe, cs, nprobe, k, k, out_ids, out_scores, ovf, s);
+  cudaError_t f = cudaFreeAsync(ws, s);
+  return e != cudaSuccess ? e : f;
+}
+
+}  // namespace rslm

@@ -226,6 +226,16 @@ __device__ __forceinline__ float float_from_order_key(uint32_t k) {
   return __uint_as_float((k & 0x80000000u) ? (k & 0x7fffffffu) : ~k);
 }
 
+// hist[bin] += 1 for this lane's bin when `active`; lanes of a warp with
+// the same bin are combined into one shared-memory atomic (radix-select
+// histograms are dominated by a few bins, which would serialise).
+__device__ __forceinline__ void warp_hist_add(uint32_t* hist, uint32_t bin, bool active) {
+  const unsigned act = __ballot_sync(kFull, active);
+  if (!active) return;
+  const unsigned peers = __match_any_sync(act, bin);
+  if ((threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], uint32_t(__popc(peers)));
+}
+
 __device__ __forceinline__ void set_device_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
 }

@@ -21,6 +21,16 @@ cudaError_t launch_select_topn(const float* S, int64_t rows, int n, int kk, int3
 cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, const int32_t* probes,
                         const float* cs, int nprobe, int k, int out_k, int64_t* out_ids,
                         float* out_scores, cudaStream_t s);
+// Single-query scan of the first `nprobe` entries of probe lists whose rows
+// are `probe_stride` long; queries with only_if[q] == 0 are skipped.
+cudaError_t launch_scan_strided(const rslm_index* ix, const float* qrot, int64_t nq,
+                                const int32_t* probes, int probe_stride, const float* cs, int nprobe,
+                                int k, int out_k, int64_t* out_ids, float* out_scores,
+                                const int* only_if, cudaStream_t s);
+// Partition-major scan on the tensor cores (batched.cu); output as launch_scan.
+cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t nq,
+                                const int32_t* probes, const float* cs, int nprobe, int k,
+                                int64_t* out_ids, float* out_scores, cudaStream_t s);
 cudaError_t launch_rescore(const rslm_index* ix, const float* qrot2, int64_t nq,
                            const int64_t* cand_ids, const float* cand_scores, int k, int k_final,
                            int64_t* out_ids, float* out_scores, cudaStream_t s);

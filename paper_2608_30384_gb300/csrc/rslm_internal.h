@@ -4,7 +4,10 @@
 #include <cuda_runtime.h>
 #include <stdint.h>
 
+#include <mutex>
 #include <string>
+#include <utility>
+#include <vector>
 
 #include "rslm.h"
 
@@ -14,6 +17,7 @@ constexpr int kTile = 128;      // rows per layout tile (partitions start on til
 constexpr int kMaxDim = 4096;
 constexpr int kMaxK = 256;
 constexpr int kMaxNprobe = 4096;
+constexpr int kBatchMinQueries = 16;  // rslm_search: batched scan above this queries/partition
 
 // Device error codes written to the index's sticky flag.
 enum DeviceError : int {
@@ -21,6 +25,7 @@ enum DeviceError : int {
   kErrBadProbe = 1,      // partition id out of range in a probe list
   kErrBadCandidate = 2,  // candidate id out of range in rescoring
   kErrBadAssignment = 3,
+  kErrTimeout = 4,       // a bounded wait on the tensor-core pipeline gave up
 };
 
 // Block-wise cascaded FWHT rotation (Sec. 3.1.1-3.1.3).
@@ -63,6 +68,12 @@ uint32_t ue_encode_host(double v, int ebits, int mbits);
 // Record the calling thread's rslm_last_error() message and return `st`.
 rslm_status set_last_error(rslm_status st, const std::string& msg);
 
+// Timing of the dominant scan kernel (rslm_profile_enable / rslm_profile_read):
+// prof_start records a start event on `s` and returns the stop event to record
+// after the launch (nullptr when profiling is off).
+cudaEvent_t prof_start(const rslm_index* ix, cudaStream_t s, const char* kernel);
+void prof_stop(cudaEvent_t stop, cudaStream_t s);
+
 }  // namespace rslm
 
 // Index state (host object; arrays are device pointers).
@@ -74,6 +85,7 @@ struct rslm_index {
   rslm::CodecSpec cs1{}, cs2{};
   float* centroids = nullptr;   // [nlist * D]
   int64_t n_rows = 0, n_slots = 0;
+  int32_t max_part_n = 0;       // rows of the largest partition
   int64_t* part_off = nullptr;  // [nlist + 1] first slot of each partition
   int32_t* part_n = nullptr;    // [nlist] rows in each partition
   int32_t* assign = nullptr;    // [n_rows]
@@ -86,4 +98,9 @@ struct rslm_index {
   int* d_err = nullptr;         // sticky device error flag
   void* cublas = nullptr;       // cublasHandle_t
   int64_t device_bytes = 0;
+  // profiling of the dominant scan kernel
+  mutable std::mutex prof_mu;
+  mutable std::vector<std::pair<cudaEvent_t, cudaEvent_t>> prof_events;
+  mutable std::string prof_kernel;
+  int profile = 0;
 };

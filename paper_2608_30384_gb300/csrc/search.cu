@@ -22,6 +22,9 @@ namespace rslm {
 namespace {
 
 // ------------------------------------------------------------ probe select
+// Top-kk of one row of S per block.  STAGED: the row's order keys are first
+// copied to shared memory so the radix passes read it from there.
+template <bool STAGED>
 __global__ void select_topn_kernel(const float* __restrict__ S, int n, int kk,
                                    int32_t* __restrict__ out_idx, float* __restrict__ out_val) {
   extern __shared__ uint32_t xsm[];
@@ -32,8 +35,14 @@ __global__ void select_topn_kernel(const float* __restrict__ S, int n, int kk,
   while (p2 < kk) p2 <<= 1;
   uint32_t* skey = xsm;
   int32_t* sidx = reinterpret_cast<int32_t*>(xsm + p2);
+  uint32_t* rowk = xsm + 2 * p2;
   const float* s = S + int64_t(blockIdx.x) * n;
   const int tid = threadIdx.x;
+  if (STAGED) {
+    for (int i = tid; i < n; i += blockDim.x) rowk[i] = float_order_key(s[i]);
+    __syncthreads();
+  }
+  auto key_at = [&](int i) { return STAGED ? rowk[i] : float_order_key(s[i]); };
 
   // Radix select of the kk-th largest order key, 8 bits at a time.
   uint32_t prefix = 0, mask = 0, rem = uint32_t(kk);
@@ -41,9 +50,10 @@ __global__ void select_topn_kernel(const float* __restrict__ S, int n, int kk,
     const int shift = 24 - 8 * pass;
     for (int i = tid; i < 256; i += blockDim.x) hist[i] = 0;
     __syncthreads();
-    for (int i = tid; i < n; i += blockDim.x) {
-      const uint32_t key = float_order_key(s[i]);
-      if ((key & mask) == prefix) atomicAdd(&hist[(key >> shift) & 255u], 1u);
+    for (int base = 0; base < n; base += blockDim.x) {
+      const int i = base + tid;
+      const uint32_t key = i < n ? key_at(i) : 0u;
+      warp_hist_add(hist, (key >> shift) & 255u, i < n && (key & mask) == prefix);
     }
     __syncthreads();
     if (tid == 0) {
@@ -68,7 +78,7 @@ __global__ void select_topn_kernel(const float* __restrict__ S, int n, int kk,
   if (tid == 0) sh_gt = 0;
   __syncthreads();
   for (int i = tid; i < n; i += blockDim.x) {
-    const uint32_t key = float_order_key(s[i]);
+    const uint32_t key = key_at(i);
     if (key > T) {
       const uint32_t slot = atomicAdd(&sh_gt, 1u);
       skey[slot] = key;
@@ -79,7 +89,7 @@ __global__ void select_topn_kernel(const float* __restrict__ S, int n, int kk,
   int taken = 0;
   for (int base = 0; base < n && taken < int(rem); base += blockDim.x) {
     const int i = base + tid;
-    const int e = (i < n && float_order_key(s[i]) == T) ? 1 : 0;
+    const int e = (i < n && key_at(i) == T) ? 1 : 0;
     int tot;
     const int ex = block_exclusive_scan(e, scratch, &tot);
     if (e && taken + ex < int(rem)) {
@@ -105,7 +115,9 @@ struct ScanArgs {
   int Dp;
   const int32_t* probes;
   const float* cs;
-  int nprobe;
+  int nprobe;        // probes scanned per query (the first nprobe of each list)
+  int probe_stride;  // row stride of probes / cs
+  const int* only_if;  // optional: scan query q only if only_if[q] != 0
   int k;
   int out_k;
   const uint8_t* codes;
@@ -194,6 +206,7 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   __shared__ int scratch[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, W = blockDim.x >> 5;
   const int64_t q = blockIdx.x;
+  if (a.only_if && a.only_if[q] == 0) return;
   // The table starts on a 256-byte boundary of the shared window (up to 255
   // bytes of padding are reserved by the launcher).
   const uint32_t ssm_addr = uint32_t(__cvta_generic_to_shared(ssm));
@@ -226,7 +239,7 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
     const int j = base + tid;
     int nt = 0;
     if (j < a.nprobe) {
-      const int p = a.probes[q * a.nprobe + j];
+      const int p = a.probes[q * a.probe_stride + j];
       if (p < 0 || p >= a.nlist) {
         set_device_error(a.err, kErrBadProbe);
         pid[j] = -1;
@@ -258,7 +271,7 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
     const int t = it - tpref[j];
     const int64_t slot0 = a.part_off[p] + int64_t(t) * kTile;
     const int nvalid = min(kTile, a.part_n[p] - t * kTile);
-    const float csj = a.cs[q * a.nprobe + j];
+    const float csj = a.cs[q * a.probe_stride + j];
     const uint8_t* tp = a.codes + slot0 * a.stride;
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     for (int c = 0; c < nch; ++c) {
@@ -413,11 +426,14 @@ __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ Re
 }
 
 template <int CH>
-cudaError_t launch_scan_ch(const ScanArgs& a, int64_t nq, size_t smem, cudaStream_t s) {
+cudaError_t launch_scan_ch(const rslm_index* ix, const ScanArgs& a, int64_t nq, size_t smem,
+                           cudaStream_t s) {
   cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        int(smem));
   if (e != cudaSuccess) return e;
+  cudaEvent_t stop = a.only_if == nullptr && a.nprobe > 1 ? prof_start(ix, s, "scan_kernel") : nullptr;
   scan_kernel<CH><<<unsigned(nq), 256, smem, s>>>(a);
+  prof_stop(stop, s);
   return cudaGetLastError();
 }
 
@@ -428,17 +444,34 @@ cudaError_t launch_select_topn(const float* S, int64_t rows, int n, int kk, int3
   if (rows == 0) return cudaSuccess;
   int p2 = 1;
   while (p2 < kk) p2 <<= 1;
-  const size_t smem = size_t(p2) * 8;
-  cudaError_t e = cudaFuncSetAttribute(select_topn_kernel,
-                                       cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
-  if (e != cudaSuccess) return e;
-  select_topn_kernel<<<unsigned(rows), 256, smem, s>>>(S, n, kk, out_idx, out_val);
+  const size_t base = size_t(p2) * 8;
+  const size_t staged = base + size_t(n) * 4;
+  cudaError_t e;
+  if (staged <= size_t(160) * 1024) {
+    e = cudaFuncSetAttribute(select_topn_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(staged));
+    if (e != cudaSuccess) return e;
+    select_topn_kernel<true><<<unsigned(rows), 256, staged, s>>>(S, n, kk, out_idx, out_val);
+  } else {
+    e = cudaFuncSetAttribute(select_topn_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             int(base));
+    if (e != cudaSuccess) return e;
+    select_topn_kernel<false><<<unsigned(rows), 256, base, s>>>(S, n, kk, out_idx, out_val);
+  }
   return cudaGetLastError();
 }
 
 cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, const int32_t* probes,
                         const float* cs, int nprobe, int k, int out_k, int64_t* out_ids,
                         float* out_scores, cudaStream_t s) {
+  return launch_scan_strided(ix, qrot, nq, probes, nprobe, cs, nprobe, k, out_k, out_ids, out_scores,
+                             nullptr, s);
+}
+
+cudaError_t launch_scan_strided(const rslm_index* ix, const float* qrot, int64_t nq,
+                                const int32_t* probes, int probe_stride, const float* cs, int nprobe,
+                                int k, int out_k, int64_t* out_ids, float* out_scores,
+                                const int* only_if, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   ScanArgs a;
   a.qrot = qrot;
@@ -446,6 +479,8 @@ cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, con
   a.probes = probes;
   a.cs = cs;
   a.nprobe = nprobe;
+  a.probe_stride = probe_stride;
+  a.only_if = only_if;
   a.k = k;
   a.out_k = out_k;
   a.codes = ix->codes1;
@@ -472,9 +507,9 @@ cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, con
   a.lut_region = int(region);
   const size_t smem = 256 + region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
   switch (ix->cs1.chunk) {
-    case 16: return launch_scan_ch<16>(a, nq, smem, s);
-    case 8: return launch_scan_ch<8>(a, nq, smem, s);
-    default: return launch_scan_ch<4>(a, nq, smem, s);
+    case 16: return launch_scan_ch<16>(ix, a, nq, smem, s);
+    case 8: return launch_scan_ch<8>(ix, a, nq, smem, s);
+    default: return launch_scan_ch<4>(ix, a, nq, smem, s);
   }
 }
 

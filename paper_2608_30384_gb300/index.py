@@ -66,6 +66,14 @@ class Index:
         B.rslm_scan(self.handle, qrot, probes, cs, k, ids, sc, stream)
         return ids, sc
 
+    def scan_batched(self, qrot, probes, cs, k: int, stream=None):
+        import torch
+        nq = probes.shape[0]
+        ids = torch.empty((nq, k), dtype=torch.int64, device=probes.device)
+        sc = torch.empty((nq, k), dtype=torch.float32, device=probes.device)
+        B.rslm_scan_batched(self.handle, qrot, probes, cs, k, ids, sc, stream)
+        return ids, sc
+
     def rescore(self, qrot2, cand_ids, cand_scores, k_final: int, stream=None):
         import torch
         nq = cand_ids.shape[0]

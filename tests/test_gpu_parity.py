@@ -185,6 +185,38 @@ def test_scan_parity_on_oracle_codes(case):
         assert (ids[i] >= 0).sum() == min(w.k, len(s1))
 
 
+def _scan_parity(case, batched: bool):
+    w = case.w
+    ix = case.gpu_index(encode=False)
+    case.import_oracle_codes(ix)
+    probes, cs = _scan_inputs(case)
+    qrot = ix.rotate(torch.from_numpy(case.Q).cuda())
+    fn = ix.scan_batched if batched else ix.scan
+    ids, sc = fn(qrot, torch.from_numpy(probes.astype(np.int32)).cuda(),
+                 torch.from_numpy(cs.astype(np.float32)).cuda(), w.k)
+    ix.sync()
+    ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
+    xm = case.xnorm_max()
+    for i in range(len(case.Q)):
+        ref, s1 = _oracle_stage1(case, i, probes[i], cs[i])
+        tol = lambda s: float(score_tol(s, case.qnorm(i), xm))  # noqa: E731
+        probs = check_topk(ids[i], sc[i], lambda j: ref[j], _kth(s1, w.k), tol, allowed_ids=ref)
+        assert not probs, (i, probs[:3])
+        assert (ids[i] >= 0).sum() == min(w.k, len(s1))
+
+
+def test_batched_scan_parity_on_oracle_codes(case):
+    """rslm_scan_batched (tensor cores, partition-major) with the oracle's probes."""
+    _scan_parity(case, batched=True)
+
+
+def test_batched_scan_overflow_fallback():
+    """Partitions smaller than k give no threshold: every candidate is kept,
+    the per-query buffer overflows and the single-query kernel re-scans."""
+    _scan_parity(Case(Wl("ovf", 20_000, 64, 256, 0.5, False, None, "true", 24, 4, 0, 128, 100, 100,
+                         seed=12)), batched=True)
+
+
 def test_rescore_parity_on_oracle_codes(case):
     w = case.w
     if not w.rescore_bits:
