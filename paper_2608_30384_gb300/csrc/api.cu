@@ -76,12 +76,14 @@ rslm_status run_probe(const rslm_index* ix, const float* queries, int64_t nq, in
                       int32_t* out_probes, float* out_cs, cudaStream_t s) {
   if (nq == 0) return RSLM_OK;
   const int64_t budget = int64_t(64) << 20;  // floats in the score chunk (256 MB)
-  int64_t qc = budget / ix->nlist;
+  const int64_t ld = (int64_t(ix->nlist) + 3) & ~int64_t(3);  // row stride, 16-byte multiple
+  int64_t qc = budget / ld;
   if (qc < 1) qc = 1;
   if (qc > nq) qc = nq;
   float* S = nullptr;
-  RSLM_CK(cudaMallocAsync(reinterpret_cast<void**>(&S), size_t(qc) * ix->nlist * sizeof(float), s),
+  RSLM_CK(cudaMallocAsync(reinterpret_cast<void**>(&S), size_t(qc) * (ld + 1) * sizeof(float), s),
           "cudaMallocAsync(probe scores)");
+  int* flags = reinterpret_cast<int*>(S + size_t(qc) * ld);  // one int per query row
   rslm_status st = RSLM_OK;
   {
     std::lock_guard<std::mutex> lock(g_cublas_mutex);
@@ -93,13 +95,13 @@ rslm_status run_probe(const rslm_index* ix, const float* queries, int64_t nq, in
       // Row-major S[n x nlist] = Q[n x D] C^T, i.e. column-major S^T = C^T^T Q^T.
       cublasStatus_t cb = cublasSgemm(h, CUBLAS_OP_T, CUBLAS_OP_N, ix->nlist, int(n), ix->D, &one,
                                       ix->centroids, ix->D, queries + q0 * ix->D, ix->D, &zero, S,
-                                      ix->nlist);
+                                      int(ld));
       if (cb != CUBLAS_STATUS_SUCCESS) {
         st = fail(RSLM_ERR_CUDA, "cublasSgemm failed with status " + std::to_string(int(cb)));
         break;
       }
-      cudaError_t e = launch_select_topn(S, n, ix->nlist, nprobe, out_probes + q0 * nprobe,
-                                         out_cs + q0 * nprobe, s);
+      cudaError_t e = launch_select_topn(S, n, ld, ix->nlist, nprobe, out_probes + q0 * nprobe,
+                                         out_cs + q0 * nprobe, flags, s);
       if (e != cudaSuccess) st = cuda_fail(e, "select_topn launch");
     }
   }

@@ -627,9 +627,14 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   uint8_t* Bh = psm;
   uint8_t* Bl = Bh + kTileBytes;
   uint8_t* slab0 = Bl + kTileBytes;                  // two slabs of slab_bytes(G)
-  QParam* qp = reinterpret_cast<QParam*>(slab0 + 2 * slab_bytes(G));
+  // per query column: (cs, theta) scaled by the query's 2^s (exact), so the
+  // epilogue tests G (cs' + L acc) >= theta' without the 2^-s multiply;
+  // padding columns have theta' = +inf
+  float2* qct = reinterpret_cast<float2*>(slab0 + 2 * slab_bytes(G));
+  float* qinv_s = reinterpret_cast<float*>(qct + kNQ);
+  int* qid_s = reinterpret_cast<int*>(qinv_s + kNQ);
   // decode tables: G = 1: byte -> 2 halves; G = 2: code -> 2 halves; G = 4: code -> 4 halves
-  uint32_t* t32 = reinterpret_cast<uint32_t*>(qp + kNQ);
+  uint32_t* t32 = reinterpret_cast<uint32_t*>(qid_s + kNQ);
   __shared__ __align__(8) uint64_t bars[8];  // slab_full[2], a_full[2], mma_done[2], acc_empty[2]
   __shared__ uint32_t tmem_base_sh;
   __shared__ int s_item;
@@ -638,7 +643,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   const int CH = a.chunk;
 
   if (G == 1) {
-    for (int b = tid; b < 256; b += blockDim.x) t32[b] = a.cbbits[b & 15] | (a.cbbits[b >> 4] << 16);
+    for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[c];  // one half per code
   } else if (G == 2) {
     for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[2 * c] | (a.cbbits[2 * c + 1] << 16);
   } else {
@@ -706,28 +711,43 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
     for (int j = tid; j < kNQ; j += blockDim.x) {
       const bool v = j < nqt;
       const int q = v ? a.lq[q0 + j] : -1;
-      QParam pr;
-      pr.q = q;
-      pr.cs = v ? a.lcs[q0 + j] : 0.0f;
-      pr.th = v ? (a.theta ? a.theta[q] : -CUDART_INF_F) : CUDART_INF_F;
-      pr.inv = v ? a.qinv[q] : 0.0f;
-      qp[j] = pr;
+      const float inv = v ? a.qinv[q] : 1.0f;
+      const float cs = v ? a.lcs[q0 + j] : 0.0f;
+      const float th = v ? (a.theta ? a.theta[q] : -CUDART_INF_F) : CUDART_INF_F;
+      qct[j] = make_float2(cs / inv, th / inv);  // exact: inv is a power of two
+      qinv_s[j] = inv;
+      qid_s[j] = q;
     }
     __syncthreads();
     // B operands (hi / lo parts of the item's queries); the previous item's
     // MMAs have all completed (its epilogue waited for them).
     {
+      // 4 vectors per thread per round, all loads issued before the stores
       const int k8n = klen / 8;
-      for (int e = tid; e < kNQ * k8n; e += blockDim.x) {
-        const int j = e / k8n, k8 = e - j * k8n;
-        uint4 h = make_uint4(0, 0, 0, 0), l = make_uint4(0, 0, 0, 0);
-        if (j < nqt) {
-          const int64_t src = int64_t(qp[j].q) * a.Dp16 + k8 * 8;
-          h = *reinterpret_cast<const uint4*>(a.qhi + src);
-          l = *reinterpret_cast<const uint4*>(a.qlo + src);
+      const int total = kNQ * k8n;
+      for (int e0 = tid; e0 < total; e0 += 4 * blockDim.x) {
+        uint4 h[4], l[4];
+#pragma unroll
+        for (int u2 = 0; u2 < 4; ++u2) {
+          const int e = e0 + u2 * blockDim.x;
+          const int j = e / k8n, k8 = e - j * k8n;
+          h[u2] = make_uint4(0, 0, 0, 0);
+          l[u2] = make_uint4(0, 0, 0, 0);
+          if (e < total && j < nqt) {
+            const int64_t src = int64_t(qid_s[j]) * a.Dp16 + k8 * 8;
+            h[u2] = __ldg(reinterpret_cast<const uint4*>(a.qhi + src));
+            l[u2] = __ldg(reinterpret_cast<const uint4*>(a.qlo + src));
+          }
         }
-        *reinterpret_cast<uint4*>(Bh + tile_off(j, k8)) = h;
-        *reinterpret_cast<uint4*>(Bl + tile_off(j, k8)) = l;
+#pragma unroll
+        for (int u2 = 0; u2 < 4; ++u2) {
+          const int e = e0 + u2 * blockDim.x;
+          if (e < total) {
+            const int j = e / k8n, k8 = e - j * k8n;
+            *reinterpret_cast<uint4*>(Bh + tile_off(j, k8)) = h[u2];
+            *reinterpret_cast<uint4*>(Bl + tile_off(j, k8)) = l[u2];
+          }
+        }
       }
     }
     fence_proxy_async();
@@ -780,11 +800,14 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         };
         // 32 columns = 64 halves = 64 / G codes = 32 / G bytes = 8 / G words
         if constexpr (G == 1) {
+          // 16-entry table (distinct banks: conflict-free); two codes -> one
+          // 32-bit column (low half = even position)
 #pragma unroll
           for (int w = 0; w < 8; ++w) {
             const uint32_t wd = word_at(dh * 8 + w);
 #pragma unroll
-            for (int bb = 0; bb < 4; ++bb) av[4 * w + bb] = t32[(wd >> (8 * bb)) & 255u];
+            for (int bb = 0; bb < 4; ++bb)
+              av[4 * w + bb] = __byte_perm(t32[(wd >> (8 * bb)) & 15u], t32[(wd >> (8 * bb + 4)) & 15u], 0x5410);
           }
         } else if constexpr (G == 2) {
 #pragma unroll
@@ -841,17 +864,27 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
             if (lane == 0) mbar_arrive(acc_empty(b));
           }
           if (row < nvalid) {
+            // test pass without stores (so the table reads pipeline), then
+            // the rare appends
+            uint32_t hit = 0;
 #pragma unroll
             for (int i = 0; i < 32; ++i) {
+              const float2 ct = qct[cbase + i];
+              v[i] = Gs * fmaf(L, v[i], ct.x);  // the score times 2^s
+              hit |= (v[i] >= ct.y ? 1u : 0u) << i;
+            }
+            while (hit) {
+              const int i = __ffs(hit) - 1;
+              hit &= hit - 1;
+              float sv = 0.0f;
+#pragma unroll
+              for (int kk = 0; kk < 32; ++kk) sv = kk == i ? v[kk] : sv;
               const int col = cbase + i;
-              const QParam pr = qp[col];
-              const float sv = Gs * fmaf(L, v[i] * pr.inv, pr.cs);
-              if (sv >= pr.th && col < nqt) {
-                const int at = atomicAdd(&a.cnt[pr.q], 1);
-                if (at < a.cap) {
-                  a.buf_s[int64_t(pr.q) * a.cap + at] = sv;
-                  a.buf_p[int64_t(pr.q) * a.cap + at] = pos;
-                }
+              const int q = qid_s[col];
+              const int at = atomicAdd(&a.cnt[q], 1);
+              if (at < a.cap) {
+                a.buf_s[int64_t(q) * a.cap + at] = sv * qinv_s[col];
+                a.buf_p[int64_t(q) * a.cap + at] = pos;
               }
             }
           }
@@ -998,8 +1031,7 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (b.nkc == 1) {
     // padded D <= 128: the pipelined, warp-specialized kernel (one CTA per SM)
-    const size_t psmem = size_t(2) * kTileBytes + 2 * size_t(slab_bytes(g)) +
-                         size_t(kNQ) * sizeof(QParam) + 256 * 4;
+    const size_t psmem = size_t(2) * kTileBytes + 2 * size_t(slab_bytes(g)) + size_t(kNQ) * 16 + 256 * 4;
     auto pk = g == 1 ? batched_pipe_kernel<1> : (g == 2 ? batched_pipe_kernel<2> : batched_pipe_kernel<4>);
     e = cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(psmem));
     if (e != cudaSuccess) return e;

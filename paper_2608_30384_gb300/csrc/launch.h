@@ -15,9 +15,12 @@ cudaError_t launch_encode(const rslm_index* ix, const float* x, int64_t row_begi
 cudaError_t launch_export_import(const rslm_index* ix, int which, int64_t row_begin, int64_t rows,
                                  uint8_t* codes, uint16_t* lscale, uint16_t* gscale, bool import,
                                  cudaStream_t s);
-// Top-kk of every row of S [rows * n] by (value desc, column asc).
-cudaError_t launch_select_topn(const float* S, int64_t rows, int n, int kk, int32_t* out_idx,
-                               float* out_val, cudaStream_t s);
+// Top-kk of the first n entries of every row of S (row stride ld) by
+// (value desc, column asc).  flags: optional device scratch of `rows` ints
+// enabling the warp-per-row kernel (used when ld % 4 == 0 and S is 16-byte
+// aligned).
+cudaError_t launch_select_topn(const float* S, int64_t rows, int64_t ld, int n, int kk,
+                               int32_t* out_idx, float* out_val, int* flags, cudaStream_t s);
 cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, const int32_t* probes,
                         const float* cs, int nprobe, int k, int out_k, int64_t* out_ids,
                         float* out_scores, cudaStream_t s);

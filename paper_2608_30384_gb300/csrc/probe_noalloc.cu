@@ -137,7 +137,8 @@ extern "C" rslm_status rslm_probe_noalloc(const rslm_index* ix, const float* que
     probe_scores_kernel<<<grid, 256, 0, s>>>(queries + q0 * ix->D, n, ix->centroids, ix->nlist, ix->D, S);
     e = cudaGetLastError();
     if (e == cudaSuccess)
-      e = launch_select_topn(S, n, ix->nlist, nprobe, out_probes + q0 * nprobe, out_cs + q0 * nprobe, s);
+      e = launch_select_topn(S, n, ix->nlist, ix->nlist, nprobe, out_probes + q0 * nprobe,
+                             out_cs + q0 * nprobe, nullptr, s);
     if (e != cudaSuccess)
       st = set_last_error(RSLM_ERR_CUDA, std::string("probe_noalloc launch: ") + cudaGetErrorString(e));
   }

@@ -25,24 +25,91 @@ namespace {
 // Top-kk of one row of S per block.  STAGED: the row's order keys are first
 // copied to shared memory so the radix passes read it from there.
 template <bool STAGED>
-__global__ void select_topn_kernel(const float* __restrict__ S, int n, int kk,
-                                   int32_t* __restrict__ out_idx, float* __restrict__ out_val) {
+__global__ void select_topn_kernel(const float* __restrict__ S, int64_t ld, int n, int kk,
+                                   int32_t* __restrict__ out_idx, float* __restrict__ out_val,
+                                   const int* __restrict__ only_if) {
+  if (only_if && only_if[blockIdx.x] == 0) return;
   extern __shared__ uint32_t xsm[];
   __shared__ uint32_t hist[256];
   __shared__ int scratch[32];
   __shared__ uint32_t sh_prefix, sh_rem, sh_gt;
   int p2 = 1;
   while (p2 < kk) p2 <<= 1;
+  const int sbuf = p2 >= 1024 ? p2 : 1024;  // candidate buffer entries
   uint32_t* skey = xsm;
-  int32_t* sidx = reinterpret_cast<int32_t*>(xsm + p2);
-  uint32_t* rowk = xsm + 2 * p2;
-  const float* s = S + int64_t(blockIdx.x) * n;
+  int32_t* sidx = reinterpret_cast<int32_t*>(xsm + sbuf);
+  uint32_t* rowk = xsm + 2 * sbuf;
+  const float* s = S + int64_t(blockIdx.x) * ld;
   const int tid = threadIdx.x;
   if (STAGED) {
     for (int i = tid; i < n; i += blockDim.x) rowk[i] = float_order_key(s[i]);
     __syncthreads();
   }
   auto key_at = [&](int i) { return STAGED ? rowk[i] : float_order_key(s[i]); };
+
+  // Fast path.  Split the row into kk groups; the smallest of the kk group
+  // maxima is at most the kk-th largest key (the maxima are kk distinct
+  // elements), so every element of the top kk is >= it.  Collect those
+  // elements (usually a few times kk) and sort them.
+  {
+    __shared__ uint32_t gmax_sh[kMaxNprobe];
+    __shared__ uint32_t sh_bound, sh_cnt;
+    const int gs = (n + kk - 1) / kk;  // group size
+    for (int g = tid; g < kk; g += blockDim.x) gmax_sh[g] = 0u;
+    if (tid == 0) {
+      sh_bound = 0xffffffffu;
+      sh_cnt = 0;
+    }
+    __syncthreads();
+    for (int base = 0; base < n; base += blockDim.x) {
+      const int i = base + tid;
+      const uint32_t key = i < n ? key_at(i) : 0u;
+      const int g = (i < n ? i : n - 1) / gs;
+      // lanes of a warp mostly share a group: reduce them first
+      const unsigned same = __match_any_sync(kFull, g);
+      const uint32_t m = __reduce_max_sync(same, key);
+      if ((tid & 31) == __ffs(same) - 1) atomicMax(&gmax_sh[g], m);
+    }
+    __syncthreads();
+    const int ng = (n + gs - 1) / gs;  // groups that hold elements
+    for (int g = tid; g < ng; g += blockDim.x) atomicMin(&sh_bound, gmax_sh[g]);
+    __syncthreads();
+    // fewer than kk non-empty groups: no bound, every element is a candidate
+    const uint32_t bound = ng >= kk ? sh_bound : 0u;
+    const int cap = p2 >= 1024 ? p2 : 1024;  // candidates that fit skey / sidx
+    for (int base = 0; base < n; base += blockDim.x) {
+      const int i = base + tid;
+      const bool c = i < n && key_at(i) >= bound;
+      const unsigned bal = __ballot_sync(kFull, c);
+      uint32_t at0 = 0;
+      if ((tid & 31) == 0 && bal) at0 = atomicAdd(&sh_cnt, uint32_t(__popc(bal)));
+      at0 = __shfl_sync(kFull, at0, 0);
+      if (c) {
+        const uint32_t at = at0 + uint32_t(__popc(bal & ((1u << (tid & 31)) - 1)));
+        if (at < uint32_t(cap)) {
+          skey[at] = key_at(i);
+          sidx[at] = i;
+        }
+      }
+    }
+    __syncthreads();
+    const int m = int(sh_cnt);
+    if (m <= cap) {
+      int q2 = 1;
+      while (q2 < m) q2 <<= 1;
+      for (int i = m + tid; i < q2; i += blockDim.x) {
+        skey[i] = 0;
+        sidx[i] = INT_MAX;
+      }
+      block_bitonic_sort(skey, sidx, q2);
+      for (int i = tid; i < kk; i += blockDim.x) {
+        out_idx[int64_t(blockIdx.x) * kk + i] = sidx[i];
+        out_val[int64_t(blockIdx.x) * kk + i] = float_from_order_key(skey[i]);
+      }
+      return;
+    }
+    __syncthreads();
+  }
 
   // Radix select of the kk-th largest order key, 8 bits at a time.
   uint32_t prefix = 0, mask = 0, rem = uint32_t(kk);
@@ -106,6 +173,115 @@ __global__ void select_topn_kernel(const float* __restrict__ S, int n, int kk,
   for (int i = tid; i < kk; i += blockDim.x) {
     out_idx[int64_t(blockIdx.x) * kk + i] = sidx[i];
     out_val[int64_t(blockIdx.x) * kk + i] = float_from_order_key(skey[i]);
+  }
+}
+
+// Warp-per-row top-kk (kk <= 256) of rows with a stride ld % 4 == 0.  Each
+// lane reads two float4 per 256-element step, so element i belongs to one of
+// 256 interleaved groups (i mod 256).  The kk-th largest of the 256 group
+// maxima is at most the kk-th largest key (kk groups, each with a distinct
+// element at or above it), so the top kk are among the elements >= that
+// bound -- usually about kk, for scores in random order.  They are compacted
+// into a per-warp buffer of kSelCap entries and sorted by the warp; a row
+// with more sets need_cta[row] for select_topn_kernel.
+constexpr int kSelCap = 512;
+constexpr int kSelWarps = 8;
+
+__device__ __forceinline__ void keys_at(const float* s, int j, int n, uint32_t (&k)[8], int lane) {
+  // Elements 4 (lane + 32 h) + c + 256 j for h = 0, 1 and c = 0..3.
+#pragma unroll
+  for (int h = 0; h < 2; ++h) {
+    const int i0 = j * 256 + 4 * (lane + 32 * h);
+    float4 v = make_float4(0.f, 0.f, 0.f, 0.f);
+    if (i0 < n) v = __ldg(reinterpret_cast<const float4*>(s + i0));
+    k[4 * h + 0] = i0 + 0 < n ? float_order_key(v.x) : 0u;
+    k[4 * h + 1] = i0 + 1 < n ? float_order_key(v.y) : 0u;
+    k[4 * h + 2] = i0 + 2 < n ? float_order_key(v.z) : 0u;
+    k[4 * h + 3] = i0 + 3 < n ? float_order_key(v.w) : 0u;
+  }
+}
+
+__global__ void __launch_bounds__(kSelWarps * 32) select_warp_kernel(
+    const float* __restrict__ S, int64_t rows, int64_t ld, int n, int kk, int32_t* __restrict__ out_idx,
+    float* __restrict__ out_val, int* __restrict__ need_cta) {
+  __shared__ uint32_t ckey[kSelWarps][kSelCap];
+  __shared__ int32_t cidx[kSelWarps][kSelCap];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t row = int64_t(blockIdx.x) * kSelWarps + w;
+  if (row >= rows) return;
+  const float* s = S + row * ld;
+  const int steps = (n + 255) / 256;
+  uint32_t gm[8];
+#pragma unroll
+  for (int c = 0; c < 8; ++c) gm[c] = 0u;
+  for (int j = 0; j < steps; ++j) {
+    uint32_t k[8];
+    keys_at(s, j, n, k, lane);
+#pragma unroll
+    for (int c = 0; c < 8; ++c) gm[c] = max(gm[c], k[c]);
+  }
+  // Bound = kk-th largest of the 256 group maxima (empty groups hold 0),
+  // found bit by bit: the largest t with #{gm >= t} >= kk.
+  uint32_t bound = 0u;
+  for (int bit = 31; bit >= 0; --bit) {
+    const uint32_t t = bound | (1u << bit);
+    int c0 = 0;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) c0 += gm[c] >= t ? 1 : 0;
+    if (int(__reduce_add_sync(kFull, uint32_t(c0))) >= kk) bound = t;
+  }
+  const unsigned lt = (1u << lane) - 1u;
+  int cnt = 0;
+  for (int j = 0; j < steps; ++j) {
+    uint32_t k[8];
+    keys_at(s, j, n, k, lane);
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const int i = j * 256 + 4 * (lane + 32 * (c >> 2)) + (c & 3);
+      const bool hit = i < n && k[c] >= bound;
+      const unsigned bal = __ballot_sync(kFull, hit);
+      const int at = cnt + __popc(bal & lt);
+      if (hit && at < kSelCap) {
+        ckey[w][at] = k[c];
+        cidx[w][at] = i;
+      }
+      cnt += __popc(bal);
+    }
+  }
+  if (cnt > kSelCap) {
+    if (lane == 0) need_cta[row] = 1;
+    return;
+  }
+  if (lane == 0) need_cta[row] = 0;
+  int p2 = 1;
+  while (p2 < cnt) p2 <<= 1;
+  for (int i = cnt + lane; i < p2; i += 32) {
+    ckey[w][i] = 0u;
+    cidx[w][i] = INT_MAX;
+  }
+  __syncwarp();
+  for (int size = 2; size <= p2; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = lane; i < (p2 >> 1); i += 32) {
+        const int lo = 2 * i - (i & (stride - 1));
+        const int hi = lo + stride;
+        const bool asc = (lo & size) == 0;
+        const uint32_t klo = ckey[w][lo], khi = ckey[w][hi];
+        const int32_t ilo = cidx[w][lo], ihi = cidx[w][hi];
+        const bool swap = asc ? better(khi, ihi, klo, ilo) : better(klo, ilo, khi, ihi);
+        if (swap) {
+          ckey[w][lo] = khi;
+          ckey[w][hi] = klo;
+          cidx[w][lo] = ihi;
+          cidx[w][hi] = ilo;
+        }
+      }
+      __syncwarp();
+    }
+  }
+  for (int i = lane; i < kk; i += 32) {
+    out_idx[row * kk + i] = cidx[w][i];
+    out_val[row * kk + i] = float_from_order_key(ckey[w][i]);
   }
 }
 
@@ -439,24 +615,32 @@ cudaError_t launch_scan_ch(const rslm_index* ix, const ScanArgs& a, int64_t nq, 
 
 }  // namespace
 
-cudaError_t launch_select_topn(const float* S, int64_t rows, int n, int kk, int32_t* out_idx,
-                               float* out_val, cudaStream_t s) {
+cudaError_t launch_select_topn(const float* S, int64_t rows, int64_t ld, int n, int kk,
+                               int32_t* out_idx, float* out_val, int* flags, cudaStream_t s) {
   if (rows == 0) return cudaSuccess;
   int p2 = 1;
   while (p2 < kk) p2 <<= 1;
-  const size_t base = size_t(p2) * 8;
-  const size_t staged = base + size_t(n) * 4;
+  const int* only_if = nullptr;
   cudaError_t e;
+  if (kk <= 256 && flags && ld % 4 == 0 && (reinterpret_cast<uintptr_t>(S) & 15) == 0) {
+    select_warp_kernel<<<unsigned((rows + kSelWarps - 1) / kSelWarps), kSelWarps * 32, 0, s>>>(
+        S, rows, ld, n, kk, out_idx, out_val, flags);
+    e = cudaGetLastError();
+    if (e != cudaSuccess) return e;
+    only_if = flags;  // rows whose candidates overflowed the warp buffer
+  }
+  const size_t base = size_t(p2 >= 1024 ? p2 : 1024) * 8;
+  const size_t staged = base + size_t(n) * 4;
   if (staged <= size_t(160) * 1024) {
     e = cudaFuncSetAttribute(select_topn_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              int(staged));
     if (e != cudaSuccess) return e;
-    select_topn_kernel<true><<<unsigned(rows), 256, staged, s>>>(S, n, kk, out_idx, out_val);
+    select_topn_kernel<true><<<unsigned(rows), 256, staged, s>>>(S, ld, n, kk, out_idx, out_val, only_if);
   } else {
     e = cudaFuncSetAttribute(select_topn_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              int(base));
     if (e != cudaSuccess) return e;
-    select_topn_kernel<false><<<unsigned(rows), 256, base, s>>>(S, n, kk, out_idx, out_val);
+    select_topn_kernel<false><<<unsigned(rows), 256, base, s>>>(S, ld, n, kk, out_idx, out_val, only_if);
   }
   return cudaGetLastError();
 }

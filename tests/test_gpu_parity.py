@@ -160,6 +160,41 @@ def test_probe_parity(case):
         assert not probs, (i, probs[:3])
 
 
+@pytest.mark.parametrize("nlist,nprobe,layout", [
+    (1001, 1, "random"), (1001, 64, "random"), (8192, 64, "random"), (8192, 256, "random"),
+    (777, 200, "random"), (4099, 300, "random"), (3000, 64, "sorted"), (2048, 100, "tied"),
+    (513, 513, "random"), (6, 5, "random"),
+])
+def test_probe_selection_paths(nlist, nprobe, layout):
+    """Top-nprobe of <q, c> on layouts that steer the selection kernels: random
+    order (the warp kernel's bound leaves about nprobe candidates), scores
+    sorted along the centroid index, all centroids equal (every element ties
+    at the bound, so rows go to the block kernel), nprobe above 256 (block
+    kernel only), and nlist not a multiple of 4."""
+    rng = np.random.default_rng(nlist * 7 + nprobe)
+    D, nq = 32, 70
+    Q = rng.standard_normal((nq, D)).astype(np.float32)
+    if layout == "tied":
+        C = np.repeat(rng.standard_normal((1, D)), nlist, axis=0).astype(np.float32)
+    else:
+        C = rng.standard_normal((nlist, D)).astype(np.float32)
+    if layout == "sorted":
+        # same direction, decreasing norm: <q, c_j> is monotone in j for every q
+        C = (np.linspace(2.0, 1.0, nlist)[:, None] * C[:1]).astype(np.float32)
+    from paper_2608_30384_gb300 import Index
+    ix = Index(torch.from_numpy(C).cuda(), 4)
+    p, cs = (t.cpu().numpy() for t in ix.probe(torch.from_numpy(Q).cuda(), nprobe))
+    full = Q.astype(np.float64) @ C.astype(np.float64).T
+    cn = np.linalg.norm(C, axis=1).max()
+    for i in range(nq):
+        tol = lambda s: 1e-5 * np.linalg.norm(Q[i]) * cn  # noqa: E731
+        probs = check_topk(p[i], cs[i], lambda j: full[i, j], _kth(full[i], nprobe), tol)
+        assert not probs, (i, probs[:3])
+        if layout == "tied":
+            # equal scores are ordered by centroid index
+            np.testing.assert_array_equal(p[i], np.arange(nprobe))
+
+
 def _scan_inputs(case):
     probes, cs, _ = search.probe(case.Q, case.C, case.w.nprobe)
     return probes, cs
