@@ -151,11 +151,14 @@ __device__ uint32_t block_kth_key(const float* s, int n, int k, uint32_t* hist, 
 // theta_q = k-th best score of the query's first probed partition (all of its
 // candidates are in the buffer), lowered by a relative margin of 1e-6; -inf
 // when that partition has fewer than k rows.
+__device__ __forceinline__ float theta_from(float t) { return t - 1e-6f * fabsf(t) - 1e-30f; }
+
 __global__ void theta_kernel(const float* __restrict__ buf_s, const int* __restrict__ cnt, int cap,
-                             int k, float* __restrict__ theta) {
+                             int k, float* __restrict__ theta, const int* __restrict__ only_if) {
   __shared__ uint32_t hist[256];
   __shared__ uint32_t sh[2];
   const int64_t q = blockIdx.x;
+  if (only_if && only_if[q] == 0) return;
   const int n = min(cnt[q], cap);
   float t = -CUDART_INF_F;
   if (n >= k) {
@@ -176,9 +179,80 @@ __global__ void theta_kernel(const float* __restrict__ buf_s, const int* __restr
     } else {
       t = float_from_order_key(block_kth_key(s, n, k, hist, sh));
     }
-    t = t - 1e-6f * fabsf(t) - 1e-30f;
+    t = theta_from(t);
   }
   if (threadIdx.x == 0) theta[q] = t;
+}
+
+// The same theta_q by one warp per query.  Bound: the k-th largest of the
+// maxima of 256 interleaved groups (element i in group i mod 256) is at most
+// the k-th largest score; the scores at or above it (usually about k) are
+// compacted into shared memory and their k-th largest found bit by bit.  A
+// query with more than kThetaCap of them sets need_block[q] for theta_kernel.
+constexpr int kThetaCap = 512;
+__global__ void __launch_bounds__(256) theta_warp_kernel(const float* __restrict__ buf_s,
+                                                         const int* __restrict__ cnt, int64_t nq, int cap,
+                                                         int k, float* __restrict__ theta,
+                                                         int* __restrict__ need_block) {
+  __shared__ uint32_t ck[8][kThetaCap];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t q = int64_t(blockIdx.x) * 8 + w;
+  if (q >= nq) return;
+  const int n = min(cnt[q], cap);
+  if (n < k) {
+    if (lane == 0) {
+      theta[q] = -CUDART_INF_F;
+      need_block[q] = 0;
+    }
+    return;
+  }
+  const float* s = buf_s + q * cap;
+  uint32_t gm[8];
+#pragma unroll
+  for (int c = 0; c < 8; ++c) gm[c] = 0u;
+  for (int base = 0; base < n; base += 256) {
+#pragma unroll
+    for (int c = 0; c < 8; ++c) {
+      const int i = base + 32 * c + lane;
+      if (i < n) gm[c] = max(gm[c], float_order_key(s[i]));
+    }
+  }
+  // the largest t with #{gm >= t} >= k
+  uint32_t bound = 0u;
+  for (int bit = 31; bit >= 0; --bit) {
+    const uint32_t t = bound | (1u << bit);
+    int c0 = 0;
+#pragma unroll
+    for (int c = 0; c < 8; ++c) c0 += gm[c] >= t ? 1 : 0;
+    if (int(__reduce_add_sync(kFull, uint32_t(c0))) >= k) bound = t;
+  }
+  const unsigned lt = (1u << lane) - 1u;
+  int m = 0;
+  for (int base = 0; base < n; base += 32) {
+    const int i = base + lane;
+    const uint32_t key = i < n ? float_order_key(s[i]) : 0u;
+    const bool hit = i < n && key >= bound;
+    const unsigned bal = __ballot_sync(kFull, hit);
+    const int at = m + __popc(bal & lt);
+    if (hit && at < kThetaCap) ck[w][at] = key;
+    m += __popc(bal);
+  }
+  if (m > kThetaCap) {
+    if (lane == 0) need_block[q] = 1;
+    return;
+  }
+  __syncwarp();
+  uint32_t res = 0u;
+  for (int bit = 31; bit >= 0; --bit) {
+    const uint32_t t = res | (1u << bit);
+    int c0 = 0;
+    for (int e = lane; e < m; e += 32) c0 += ck[w][e] >= t ? 1 : 0;
+    if (int(__reduce_add_sync(kFull, uint32_t(c0))) >= k) res = t;
+  }
+  if (lane == 0) {
+    theta[q] = theta_from(float_from_order_key(res));
+    need_block[q] = 0;
+  }
 }
 
 // ------------------------------------------------- tcgen05 / mbarrier helpers
@@ -549,30 +623,58 @@ __global__ void __launch_bounds__(256, 2) batched_scan_kernel(const __grid_const
 }
 
 // ------------------------------------------------ pipelined kernel (D <= 128)
-// The same computation for a single K chunk (padded D <= 128), with the
-// stages overlapped across the 128-row tiles of an item:
-//   warps 0-7  decode: thread = (row, half of the row's columns); wait for
-//              the tile's codes (TMA), decode them into registers and store
-//              them into the A operand buffer of that tile in TMEM
+// The same computation for a single K chunk (padded D <= 128), as one
+// persistent CTA per SM whose warps each take one stage, overlapped across
+// the 128-row tiles of an item and across items:
+//   warps 18-19 load: fetch the next item (partition, up to 128 of its
+//              queries) and stage its per-query epilogue constants and its B
+//              operands (the queries' fp16 hi / lo parts in the no-swizzle
+//              K-major layout) into one of two item slots while the other
+//              slot's item computes;
+//   warp 17    lane 0 streams each tile's codes (one contiguous slab of the
+//              tile-interleaved layout) by TMA into a ring of kSlabs buffers;
+//   warps 0-7  decode: thread = (row, half of the row's columns); take the
+//              tile's codes from the slab, decode them through a 16-entry
+//              table and store them into one of two A operands in TMEM
 //              (tcgen05.st; lane = row, two halves per 32-bit column);
-//   warp 16    lane 0 issues the TMA copies (two tiles ahead) and the MMAs
-//              (A from TMEM, B hi / lo from shared memory) into one of two
-//              TMEM accumulators;
-//   warps 8-15 epilogue: thread = (row, half of the 128 query columns); read
-//              its accumulator part, apply s = G (cs + L dot) and append
-//              candidates >= theta_q.
-// A warp reaches only its TMEM lane quadrant (warp index mod 4), so every
-// role spans the four quadrants twice.
-// A and the accumulator are double-buffered (TMEM columns: acc 0-127 and
-// 128-255, A 256-319 and 320-383).  mbarriers: slab_full (TMA landed),
-// a_full (8 decoder warps wrote A), mma_done (the MMAs of a tile finished:
-// A free, accumulator ready), acc_empty (8 epilogue warps read it).  Every
-// wait is bounded; a timeout sets the error flag and stops the item loop.
-constexpr int kPipeThreads = 17 * 32;  // 8 decoder, 8 epilogue, 1 producer warps
-constexpr int kProducerWarp = 16;
+//   warp 16    lane 0 issues the MMAs (A from TMEM, B hi / lo from the item
+//              slot, N = the item's query count rounded up to 16) into one
+//              of two TMEM accumulators;
+//   warps 8-15 epilogue: thread = (row, half of the query columns); read its
+//              accumulator part, apply s = G (cs + L dot) and append the
+//              candidates with s >= theta_q.
+// A warp reaches only its TMEM lane quadrant (warp index mod 4), so the
+// decode and epilogue roles span the four quadrants twice.  TMEM columns:
+// accumulators 0-127 and 128-255, A operands 256-319 and 320-383.
+// mbarriers: item_full (loader -> all roles), item_empty (epilogue ->
+// loader), slab_full (TMA landed), slab_empty (decoders read it), a_full
+// (decoders wrote A), mma_done (the tile's MMAs finished: A free,
+// accumulator ready), acc_empty (epilogue read the accumulator).  Every wait
+// is bounded; a timeout sets the error flag and every role leaves its loop.
+constexpr int kPipeThreads = 20 * 32;
+constexpr int kMmaWarp = 16, kTmaWarp = 17, kLoadWarp0 = 18;
+constexpr int kLoadThreads = 64;
+constexpr int kSlabs = 4;
 constexpr uint32_t kPipeCols = 512;
 __device__ __forceinline__ uint32_t acc_col(uint32_t b) { return b * 128u; }       // accumulators
 __device__ __forceinline__ uint32_t a_col(uint32_t b) { return 256u + b * 64u; }   // A operands
+
+// One work item as staged by the loader.
+struct ItemDesc {
+  int64_t slot0;  // first row slot of the partition
+  int p;          // partition; -1: no more items
+  int q0;         // first entry of the item in the partition's query list
+  int nqt;        // queries of the item (<= kNQ)
+  int nrows;      // rows of the partition
+};
+// Item slot layout: B hi, B lo, (cs, theta) scaled by 2^s, 2^-s, query ids,
+// descriptor.
+constexpr int kOffBl = kTileBytes, kOffQct = 2 * kTileBytes, kOffQinv = kOffQct + kNQ * 8,
+              kOffQid = kOffQinv + kNQ * 4, kOffDesc = kOffQid + kNQ * 4,
+              kSlotBytes = (kOffDesc + int(sizeof(ItemDesc)) + 127) / 128 * 128;
+__host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
+  return size_t(2) * kSlotBytes + size_t(kSlabs) * slab_bytes(g) + 32 * 4;
+}
 
 __device__ __forceinline__ void mbar_init(uint32_t mbar, uint32_t count) {
   asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(mbar), "r"(count) : "memory");
@@ -589,25 +691,6 @@ __device__ __forceinline__ void umma_f16_ts(uint32_t d_tmem, uint32_t a_tmem, ui
       "r"(a_tmem), "l"(bdesc), "r"(idesc), "r"(accumulate));
 }
 
-// 64 consecutive 32-bit columns of this thread's TMEM lane <- v.
-__device__ __forceinline__ void tmem_st64(uint32_t taddr, const uint32_t (&v)[64]) {
-  asm volatile(
-      "tcgen05.st.sync.aligned.32x32b.x64.b32 [%0], {%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
-      "%15,%16,%17,%18,%19,%20,%21,%22,%23,%24,%25,%26,%27,%28,%29,%30,%31,%32,%33,%34,%35,%36,%37,"
-      "%38,%39,%40,%41,%42,%43,%44,%45,%46,%47,%48,%49,%50,%51,%52,%53,%54,%55,%56,%57,%58,%59,%60,"
-      "%61,%62,%63,%64};" ::"r"(taddr),
-      "r"(v[0]), "r"(v[1]), "r"(v[2]), "r"(v[3]), "r"(v[4]), "r"(v[5]), "r"(v[6]), "r"(v[7]),
-      "r"(v[8]), "r"(v[9]), "r"(v[10]), "r"(v[11]), "r"(v[12]), "r"(v[13]), "r"(v[14]), "r"(v[15]),
-      "r"(v[16]), "r"(v[17]), "r"(v[18]), "r"(v[19]), "r"(v[20]), "r"(v[21]), "r"(v[22]), "r"(v[23]),
-      "r"(v[24]), "r"(v[25]), "r"(v[26]), "r"(v[27]), "r"(v[28]), "r"(v[29]), "r"(v[30]), "r"(v[31]),
-      "r"(v[32]), "r"(v[33]), "r"(v[34]), "r"(v[35]), "r"(v[36]), "r"(v[37]), "r"(v[38]), "r"(v[39]),
-      "r"(v[40]), "r"(v[41]), "r"(v[42]), "r"(v[43]), "r"(v[44]), "r"(v[45]), "r"(v[46]), "r"(v[47]),
-      "r"(v[48]), "r"(v[49]), "r"(v[50]), "r"(v[51]), "r"(v[52]), "r"(v[53]), "r"(v[54]), "r"(v[55]),
-      "r"(v[56]), "r"(v[57]), "r"(v[58]), "r"(v[59]), "r"(v[60]), "r"(v[61]), "r"(v[62]), "r"(v[63])
-      : "memory");
-  asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
-}
-
 // 32 consecutive 32-bit columns of this thread's TMEM lane <- v.
 __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32]) {
   asm volatile(
@@ -621,29 +704,20 @@ __device__ __forceinline__ void tmem_st32(uint32_t taddr, const uint32_t (&v)[32
   asm volatile("tcgen05.wait::st.sync.aligned;" ::: "memory");
 }
 
-template <int G>
+template <int G, bool DENSE>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
-  extern __shared__ __align__(16) uint8_t psm[];
-  uint8_t* Bh = psm;
-  uint8_t* Bl = Bh + kTileBytes;
-  uint8_t* slab0 = Bl + kTileBytes;                  // two slabs of slab_bytes(G)
-  // per query column: (cs, theta) scaled by the query's 2^s (exact), so the
-  // epilogue tests G (cs' + L acc) >= theta' without the 2^-s multiply;
-  // padding columns have theta' = +inf
-  float2* qct = reinterpret_cast<float2*>(slab0 + 2 * slab_bytes(G));
-  float* qinv_s = reinterpret_cast<float*>(qct + kNQ);
-  int* qid_s = reinterpret_cast<int*>(qinv_s + kNQ);
-  // decode tables: G = 1: byte -> 2 halves; G = 2: code -> 2 halves; G = 4: code -> 4 halves
-  uint32_t* t32 = reinterpret_cast<uint32_t*>(qid_s + kNQ);
-  __shared__ __align__(8) uint64_t bars[8];  // slab_full[2], a_full[2], mma_done[2], acc_empty[2]
+  extern __shared__ __align__(128) uint8_t psm[];
+  uint8_t* slab0 = psm + 2 * kSlotBytes;
+  // decode table: G = 1: code -> 1 half; G = 2: code -> 2 halves; G = 4: code -> 4 halves
+  uint32_t* t32 = reinterpret_cast<uint32_t*>(slab0 + kSlabs * slab_bytes(G));
+  __shared__ __align__(8) uint64_t bars[18];
   __shared__ uint32_t tmem_base_sh;
-  __shared__ int s_item;
   __shared__ int s_fail;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int CH = a.chunk;
 
   if (G == 1) {
-    for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[c];  // one half per code
+    for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[c];
   } else if (G == 2) {
     for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[2 * c] | (a.cbbits[2 * c + 1] << 16);
   } else {
@@ -653,17 +727,25 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
     }
   }
   const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
-  auto slab_full = [&](int b) { return bar0 + 8u * uint32_t(b); };
-  auto a_full = [&](int b) { return bar0 + 8u * uint32_t(2 + b); };
-  auto mma_done = [&](int b) { return bar0 + 8u * uint32_t(4 + b); };
-  auto acc_empty = [&](int b) { return bar0 + 8u * uint32_t(6 + b); };
+  auto item_full = [&](uint32_t s) { return bar0 + 8u * s; };
+  auto item_empty = [&](uint32_t s) { return bar0 + 8u * (2 + s); };
+  auto slab_full = [&](uint32_t b) { return bar0 + 8u * (4 + b); };
+  auto slab_empty = [&](uint32_t b) { return bar0 + 8u * (8 + b); };
+  auto a_full = [&](uint32_t b) { return bar0 + 8u * (12 + b); };
+  auto mma_done = [&](uint32_t b) { return bar0 + 8u * (14 + b); };
+  auto acc_empty = [&](uint32_t b) { return bar0 + 8u * (16 + b); };
   if (tid == 0) {
     s_fail = 0;
-    for (int b = 0; b < 2; ++b) {
-      mbar_init(slab_full(b), 1);
+    for (uint32_t b = 0; b < 2; ++b) {
+      mbar_init(item_full(b), kLoadThreads);
+      mbar_init(item_empty(b), 8);
       mbar_init(a_full(b), 8);
       mbar_init(mma_done(b), 1);
       mbar_init(acc_empty(b), 8);
+    }
+    for (uint32_t b = 0; b < kSlabs; ++b) {
+      mbar_init(slab_full(b), 1);
+      mbar_init(slab_empty(b), 8);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -678,95 +760,160 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = tmem_base_sh;
-  const uint32_t bh_addr = uint32_t(__cvta_generic_to_shared(Bh));
-  const uint32_t bl_addr = uint32_t(__cvta_generic_to_shared(Bl));
+  const uint32_t psm_addr = uint32_t(__cvta_generic_to_shared(psm));
   const uint32_t slab_addr0 = uint32_t(__cvta_generic_to_shared(slab0));
-  constexpr uint32_t idesc = f16_idesc(kMR, kNQ);
   const int n_items = a.items[a.nlist];
-  const int klen = a.Dp16;                   // single K chunk
+  const int klen = a.Dp16;  // single K chunk
   const int nbytes = (klen + 2 * G - 1) / (2 * G);
-  int c1 = min((nbytes + CH - 1) / CH, a.stride / CH);  // code chunks of a row used
+  const int c1 = min((nbytes + CH - 1) / CH, a.stride / CH);  // code chunks of a row used
   const uint32_t slab_len = uint32_t(c1 * kMR * CH);
-  uint32_t gt = 0;  // tiles this CTA has processed (buffer = gt & 1, use = gt >> 1)
+  auto slot = [&](uint32_t s) { return psm + s * kSlotBytes; };
+  auto desc = [&](uint32_t s) { return reinterpret_cast<const volatile ItemDesc*>(slot(s) + kOffDesc); };
+  auto failed = [&]() { return *reinterpret_cast<volatile int*>(&s_fail) != 0; };
   auto fail = [&]() {
     set_device_error(a.err, kErrTimeout);
     atomicExch(&s_fail, 1);
   };
 
-  for (;;) {
-    __syncthreads();
-    if (tid == 0) s_item = s_fail ? n_items : atomicAdd(a.work, 1);
-    __syncthreads();
-    const int item = s_item;
-    if (item >= n_items) break;
-    int lo = 0, hi = a.nlist - 1;
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (a.items[mid] <= item) lo = mid;
-      else hi = mid - 1;
-    }
-    const int p = lo;
-    const int q0 = a.off[p] + (item - a.items[p]) * kNQ;
-    const int nqt = min(kNQ, a.off[p + 1] - q0);
-    for (int j = tid; j < kNQ; j += blockDim.x) {
-      const bool v = j < nqt;
-      const int q = v ? a.lq[q0 + j] : -1;
-      const float inv = v ? a.qinv[q] : 1.0f;
-      const float cs = v ? a.lcs[q0 + j] : 0.0f;
-      const float th = v ? (a.theta ? a.theta[q] : -CUDART_INF_F) : CUDART_INF_F;
-      qct[j] = make_float2(cs / inv, th / inv);  // exact: inv is a power of two
-      qinv_s[j] = inv;
-      qid_s[j] = q;
-    }
-    __syncthreads();
-    // B operands (hi / lo parts of the item's queries); the previous item's
-    // MMAs have all completed (its epilogue waited for them).
-    {
-      // 4 vectors per thread per round, all loads issued before the stores
-      const int k8n = klen / 8;
-      const int total = kNQ * k8n;
-      for (int e0 = tid; e0 < total; e0 += 4 * blockDim.x) {
-        uint4 h[4], l[4];
-#pragma unroll
-        for (int u2 = 0; u2 < 4; ++u2) {
-          const int e = e0 + u2 * blockDim.x;
-          const int j = e / k8n, k8 = e - j * k8n;
-          h[u2] = make_uint4(0, 0, 0, 0);
-          l[u2] = make_uint4(0, 0, 0, 0);
-          if (e < total && j < nqt) {
-            const int64_t src = int64_t(qid_s[j]) * a.Dp16 + k8 * 8;
-            h[u2] = __ldg(reinterpret_cast<const uint4*>(a.qhi + src));
-            l[u2] = __ldg(reinterpret_cast<const uint4*>(a.qlo + src));
+  if (warp >= kLoadWarp0) {
+    // ---------------- loader: one item per slot use
+    const int lt = tid - kLoadWarp0 * 32;
+    const int k8n = klen / 8;
+    for (uint32_t seq = 0;; ++seq) {
+      const uint32_t s = seq & 1, use = seq >> 1;
+      bool ok = !(use > 0 && !mbar_wait(item_empty(s), (use - 1) & 1));
+      if (!ok) fail();
+      uint8_t* sb = slot(s);
+      ItemDesc* d = reinterpret_cast<ItemDesc*>(sb + kOffDesc);
+      if (lt == 0) {
+        const int item = (ok && !failed()) ? atomicAdd(a.work, 1) : n_items;
+        if (item < n_items) {
+          int lo = 0, hi = a.nlist - 1;
+          while (lo < hi) {
+            const int mid = (lo + hi + 1) >> 1;
+            if (a.items[mid] <= item) lo = mid;
+            else hi = mid - 1;
           }
-        }
-#pragma unroll
-        for (int u2 = 0; u2 < 4; ++u2) {
-          const int e = e0 + u2 * blockDim.x;
-          if (e < total) {
-            const int j = e / k8n, k8 = e - j * k8n;
-            *reinterpret_cast<uint4*>(Bh + tile_off(j, k8)) = h[u2];
-            *reinterpret_cast<uint4*>(Bl + tile_off(j, k8)) = l[u2];
-          }
+          d->p = lo;
+          d->q0 = a.off[lo] + (item - a.items[lo]) * kNQ;
+          d->nqt = min(kNQ, a.off[lo + 1] - d->q0);
+          d->nrows = a.part_n[lo];
+          d->slot0 = a.part_off[lo];
+        } else {
+          d->p = -1;
         }
       }
+      asm volatile("bar.sync 1, %0;" ::"n"(kLoadThreads) : "memory");
+      const int p = d->p, q0 = d->q0, nqt = d->nqt;
+      if (p >= 0) {
+        float2* qct = reinterpret_cast<float2*>(sb + kOffQct);
+        float* qinv = reinterpret_cast<float*>(sb + kOffQinv);
+        int* qid = reinterpret_cast<int*>(sb + kOffQid);
+        int qs[kNQ / kLoadThreads];
+#pragma unroll
+        for (int u = 0; u < kNQ / kLoadThreads; ++u) {
+          const int j = lt + u * kLoadThreads;
+          qs[u] = j < nqt ? __ldg(a.lq + q0 + j) : -1;
+        }
+#pragma unroll
+        for (int u = 0; u < kNQ / kLoadThreads; ++u) {
+          const int j = lt + u * kLoadThreads;
+          const bool v = qs[u] >= 0;
+          const float inv = v ? __ldg(a.qinv + qs[u]) : 1.0f;
+          const float cs = v ? __ldg(a.lcs + q0 + j) : 0.0f;
+          const float th = v ? (a.theta ? __ldg(a.theta + qs[u]) : -CUDART_INF_F) : CUDART_INF_F;
+          qct[j] = make_float2(cs / inv, -th / inv);  // exact: inv is a power of two
+          qinv[j] = inv;
+          qid[j] = qs[u];
+        }
+        // B rows: lane = query row, so each 16-byte store of a warp fills
+        // four whole 128-byte core-matrix rows (no bank conflicts)
+#pragma unroll
+        for (int u = 0; u < kNQ / kLoadThreads; ++u) {
+          const int j = lt + u * kLoadThreads;
+          const int64_t base = int64_t(qs[u] >= 0 ? qs[u] : 0) * a.Dp16;
+          for (int k0 = 0; k0 < k8n; k0 += 8) {
+            uint4 hv[8], lv[8];
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              hv[e] = make_uint4(0, 0, 0, 0);
+              lv[e] = make_uint4(0, 0, 0, 0);
+              if (qs[u] >= 0 && k0 + e < k8n) {
+                hv[e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + (k0 + e) * 8));
+                lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
+              }
+            }
+#pragma unroll
+            for (int e = 0; e < 8; ++e) {
+              if (k0 + e < k8n) {
+                *reinterpret_cast<uint4*>(sb + tile_off(j, k0 + e)) = hv[e];
+                *reinterpret_cast<uint4*>(sb + kOffBl + tile_off(j, k0 + e)) = lv[e];
+              }
+            }
+          }
+        }
+        fence_proxy_async();  // B is read by the tensor cores (async proxy)
+      }
+      mbar_arrive(item_full(s));
+      if (p < 0) break;
     }
-    fence_proxy_async();
-    __syncthreads();
-    const int nrows = a.part_n[p];
-    const int64_t slot0 = a.part_off[p];
-    const int ntiles = (nrows + kMR - 1) / kMR;
-    const uint8_t* codes0 = a.codes + slot0 * a.stride;
-
-    if (warp == kProducerWarp) {
-      // ---------------- producer: TMA two tiles ahead, MMAs
-      if (lane == 0) {
-        for (int t = 0; t < min(ntiles, 2); ++t)
-          tma_load_1d(slab_addr0 + uint32_t(((gt + t) & 1) * slab_bytes(G)),
-                      codes0 + size_t(t) * kMR * a.stride, slab_len, slab_full((gt + t) & 1));
-        for (int t = 0; t < ntiles; ++t) {
-          const uint32_t g2 = gt + t, b = g2 & 1, u = g2 >> 1;
-          if (!mbar_wait(a_full(b), u & 1)) fail();
-          if (u > 0 && !mbar_wait(acc_empty(b), (u - 1) & 1)) fail();
+  } else if (warp == kTmaWarp) {
+    // ---------------- TMA: the code slab of every tile, kSlabs ahead
+    if (lane == 0) {
+      uint32_t gt = 0;
+      bool ok = true;
+      for (uint32_t seq = 0; ok; ++seq) {
+        const uint32_t s = seq & 1;
+        if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+          fail();
+          break;
+        }
+        const int p = desc(s)->p;
+        if (p < 0 || failed()) break;
+        const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
+        const uint8_t* codes0 = a.codes + desc(s)->slot0 * a.stride;
+        for (int t = 0; t < ntiles; ++t, ++gt) {
+          const uint32_t sb = gt % kSlabs, u = gt / kSlabs;
+          if (u > 0 && !mbar_wait(slab_empty(sb), (u - 1) & 1)) {
+            fail();
+            ok = false;
+            break;
+          }
+          tma_load_1d(slab_addr0 + sb * uint32_t(slab_bytes(G)), codes0 + size_t(t) * kMR * a.stride,
+                      slab_len, slab_full(sb));
+        }
+      }
+      // no copy may still be landing when the CTA exits
+      for (uint32_t sb = 0; sb < kSlabs && sb < gt; ++sb) {
+        const uint32_t last = (gt - 1 - sb) / kSlabs;  // last use of buffer sb
+        mbar_wait(slab_full(sb), last & 1);
+      }
+    }
+    __syncwarp();
+  } else if (warp == kMmaWarp) {
+    // ---------------- MMA issue
+    if (lane == 0) {
+      uint32_t gt = 0;
+      bool ok = true;
+      for (uint32_t seq = 0; ok; ++seq) {
+        const uint32_t s = seq & 1;
+        if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+          fail();
+          break;
+        }
+        const int p = desc(s)->p;
+        if (p < 0 || failed()) break;
+        const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
+        const int nqt = desc(s)->nqt;
+        const uint32_t idesc = f16_idesc(kMR, max(16, (nqt + 15) & ~15));
+        const uint32_t bh_addr = psm_addr + s * kSlotBytes, bl_addr = bh_addr + kOffBl;
+        for (int t = 0; t < ntiles; ++t, ++gt) {
+          const uint32_t b = gt & 1, u = gt >> 1;
+          if (!mbar_wait(a_full(b), u & 1) || (u > 0 && !mbar_wait(acc_empty(b), (u - 1) & 1))) {
+            fail();
+            ok = false;
+            break;
+          }
           fence_after_sync();
           for (int ks = 0; ks < klen / 16; ++ks) {
             const uint32_t at = tmem + a_col(b) + uint32_t(ks * 8);
@@ -775,123 +922,223 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
             umma_f16_ts(tmem + acc_col(b), at, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
           }
           umma_commit(mma_done(b));
-          // decode of tile t is done (a_full), so its slab is free for tile t + 2
-          if (t + 2 < ntiles)
-            tma_load_1d(slab_addr0 + b * uint32_t(slab_bytes(G)), codes0 + size_t(t + 2) * kMR * a.stride,
-                        slab_len, slab_full(b));
         }
       }
-      __syncwarp();
-    } else if (warp < 8) {
-      // ---------------- decoders: thread = row r of the tile, column half dh
-      const int r = (warp & 3) * 32 + lane;
-      const int dh = warp >> 2;
-      for (int t = 0; t < ntiles; ++t) {
-        const uint32_t g2 = gt + t, b = g2 & 1, u = g2 >> 1;
-        if (!mbar_wait(slab_full(b), u & 1)) fail();
-        const uint8_t* sl = slab0 + b * slab_bytes(G);
-        uint32_t av[32];
-        // word w (bytes 4w .. 4w + 3) of row r in the slab
-        auto word_at = [&](int w) -> uint32_t {
-          const int byte = 4 * w;
-          const int c = byte / CH;
-          if (c >= c1) return 0u;
-          return *reinterpret_cast<const uint32_t*>(sl + (c * kMR + r) * CH + (byte % CH));
-        };
-        // 32 columns = 64 halves = 64 / G codes = 32 / G bytes = 8 / G words
-        if constexpr (G == 1) {
-          // 16-entry table (distinct banks: conflict-free); two codes -> one
-          // 32-bit column (low half = even position)
+      // no MMA may still be running when TMEM is freed
+      if (gt > 0) mbar_wait(mma_done((gt - 1) & 1), ((gt - 1) >> 1) & 1);
+    }
+    __syncwarp();
+  } else if (warp < 8) {
+    // ---------------- decoders: thread = row r of the tile, column half dh
+    const int r = (warp & 3) * 32 + lane;
+    const int dh = warp >> 2;
+    uint32_t gt = 0;
+    bool ok = true;
+    for (uint32_t seq = 0; ok; ++seq) {
+      const uint32_t s = seq & 1;
+      if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+        fail();
+        break;
+      }
+      const int p = desc(s)->p;
+      if (p < 0 || failed()) break;
+      const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
+      for (int t = 0; t < ntiles; ++t, ++gt) {
+        const uint32_t sb = gt % kSlabs, us = gt / kSlabs;
+        if (!mbar_wait(slab_full(sb), us & 1)) {
+          fail();
+          ok = false;
+          break;
+        }
+        // the 32 / G bytes = 8 / G words of row r this thread decodes
+        constexpr int NW = 8 / G;
+        uint32_t wd[NW];
+        {
+          const uint8_t* sl = slab0 + sb * slab_bytes(G);
+          const int byte0 = dh * 4 * NW;
+          if (CH == 16) {
+            // whole 16-byte chunks (G = 1: two, G = 2: one) or half of one (G = 4)
+            if constexpr (NW >= 4) {
 #pragma unroll
-          for (int w = 0; w < 8; ++w) {
-            const uint32_t wd = word_at(dh * 8 + w);
+              for (int v = 0; v < NW / 4; ++v) {
+                const int c = byte0 / 16 + v;
+                uint4 x = make_uint4(0, 0, 0, 0);
+                if (c < c1) x = *reinterpret_cast<const uint4*>(sl + (c * kMR + r) * 16);
+                wd[4 * v] = x.x;
+                wd[4 * v + 1] = x.y;
+                wd[4 * v + 2] = x.z;
+                wd[4 * v + 3] = x.w;
+              }
+            } else {
+              const int c = byte0 / 16;
+              uint2 x = make_uint2(0, 0);
+              if (c < c1) x = *reinterpret_cast<const uint2*>(sl + (c * kMR + r) * 16 + byte0 % 16);
+              wd[0] = x.x;
+              wd[1] = x.y;
+            }
+          } else {
 #pragma unroll
-            for (int bb = 0; bb < 4; ++bb)
-              av[4 * w + bb] = __byte_perm(t32[(wd >> (8 * bb)) & 15u], t32[(wd >> (8 * bb + 4)) & 15u], 0x5410);
-          }
-        } else if constexpr (G == 2) {
-#pragma unroll
-          for (int w = 0; w < 4; ++w) {
-            const uint32_t wd = word_at(dh * 4 + w);
-#pragma unroll
-            for (int n = 0; n < 8; ++n) av[8 * w + n] = t32[(wd >> (4 * n)) & 15u];
-          }
-        } else {
-#pragma unroll
-          for (int w = 0; w < 2; ++w) {
-            const uint32_t wd = word_at(dh * 2 + w);
-#pragma unroll
-            for (int n = 0; n < 8; ++n) {
-              const uint32_t c = (wd >> (4 * n)) & 15u;
-              av[16 * w + 2 * n] = t32[2 * c];
-              av[16 * w + 2 * n + 1] = t32[2 * c + 1];
+            for (int w = 0; w < NW; ++w) {
+              const int byte = byte0 + 4 * w;
+              const int c = byte / CH;
+              wd[w] = c < c1 ? *reinterpret_cast<const uint32_t*>(sl + (c * kMR + r) * CH + (byte % CH))
+                             : 0u;
             }
           }
         }
-        // A buffer b is free once the MMAs of tile g2 - 2 have completed
-        if (u > 0 && !mbar_wait(mma_done(b), (u - 1) & 1)) fail();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(slab_empty(sb));
+        // 32 columns = 64 halves = 64 / G codes
+        uint32_t av[32];
+        if constexpr (G == 1) {
+          // two codes -> one 32-bit column (low half = even position)
+#pragma unroll
+          for (int w = 0; w < 8; ++w)
+#pragma unroll
+            for (int bb = 0; bb < 4; ++bb)
+              av[4 * w + bb] =
+                  __byte_perm(t32[(wd[w] >> (8 * bb)) & 15u], t32[(wd[w] >> (8 * bb + 4)) & 15u], 0x5410);
+        } else if constexpr (G == 2) {
+#pragma unroll
+          for (int w = 0; w < 4; ++w)
+#pragma unroll
+            for (int n = 0; n < 8; ++n) av[8 * w + n] = t32[(wd[w] >> (4 * n)) & 15u];
+        } else {
+#pragma unroll
+          for (int w = 0; w < 2; ++w)
+#pragma unroll
+            for (int n = 0; n < 8; ++n) {
+              const uint32_t c = (wd[w] >> (4 * n)) & 15u;
+              av[16 * w + 2 * n] = t32[2 * c];
+              av[16 * w + 2 * n + 1] = t32[2 * c + 1];
+            }
+        }
+        // A buffer b is free once the MMAs of tile gt - 2 have completed
+        const uint32_t b = gt & 1, u = gt >> 1;
+        if (u > 0 && !mbar_wait(mma_done(b), (u - 1) & 1)) {
+          fail();
+          ok = false;
+          break;
+        }
         fence_after_sync();
         tmem_st32(tmem + (uint32_t((warp & 3) * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
         fence_before_sync();
         __syncwarp();
         if (lane == 0) mbar_arrive(a_full(b));
       }
-    } else {
-      // ---------------- epilogue: thread = row of quadrant warp % 4, columns eh * 64 ..
-      const int quad = warp & 3;
-      const int eh = (warp - 8) >> 2;
-      const int row = quad * 32 + lane;
-      for (int t = 0; t < ntiles; ++t) {
-        const uint32_t g2 = gt + t, b = g2 & 1, u = g2 >> 1;
+    }
+  } else {
+    // ---------------- epilogue: thread = row of quadrant warp % 4, columns eh * 64 ..
+    const int quad = warp & 3;
+    const int eh = (warp - 8) >> 2;
+    const int row = quad * 32 + lane;
+    uint32_t gt = 0;
+    bool ok = true;
+    for (uint32_t seq = 0; ok; ++seq) {
+      const uint32_t s = seq & 1;
+      if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+        fail();
+        break;
+      }
+      const int p = desc(s)->p;
+      if (p < 0 || failed()) break;
+      const int nrows = desc(s)->nrows, nqt = desc(s)->nqt;
+      const int64_t slot0 = desc(s)->slot0;
+      const int ntiles = (nrows + kMR - 1) / kMR;
+      const float2* qct = reinterpret_cast<const float2*>(slot(s) + kOffQct);
+      const float* qinv_s = reinterpret_cast<const float*>(slot(s) + kOffQinv);
+      const int* qid_s = reinterpret_cast<const int*>(slot(s) + kOffQid);
+      // column parts of 32 this warp reads: [eh * 64, eh * 64 + 32 * nparts)
+      const int nparts = min(2, max(0, (nqt - eh * 64 + 31) / 32));
+      for (int t = 0; t < ntiles; ++t, ++gt) {
+        const uint32_t b = gt & 1, u = gt >> 1;
         const int nvalid = min(kMR, nrows - t * kMR);
         const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row);
         float L = 0.0f, Gs = 0.0f;
         if (row < nvalid) {
-          const uint32_t sc = a.scales[pos];
+          const uint32_t sc = __ldg(a.scales + pos);
           L = ue7m9_to_f32(sc & 0xffffu);
           Gs = ue4m12_to_f32(sc >> 16);
         }
-        if (!mbar_wait(mma_done(b), u & 1)) fail();
+        if (!mbar_wait(mma_done(b), u & 1)) {
+          fail();
+          ok = false;
+          break;
+        }
         fence_after_sync();
+        if (nparts == 0) {
+          fence_before_sync();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(acc_empty(b));
+        }
 #pragma unroll 1
-        for (int part = 0; part < 2; ++part) {
+        for (int part = 0; part < nparts; ++part) {
           float v[32];
           const int cbase = eh * 64 + part * 32;
           tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(b) + uint32_t(cbase), v);
-          if (part == 1) {
+          if (part == nparts - 1) {
             fence_before_sync();
             __syncwarp();
             if (lane == 0) mbar_arrive(acc_empty(b));
           }
           if (row < nvalid) {
-            // test pass without stores (so the table reads pipeline), then
-            // the rare appends
-            uint32_t hit = 0;
+            // (cs', -theta') of columns 2i, 2i + 1 in one float4
+            const float4* q4 = reinterpret_cast<const float4*>(qct + cbase);
+            if constexpr (DENSE) {
+              // first pass: every score, at its row of the query's buffer
+              float* dst = a.buf_s + int64_t(t) * kMR + row;
 #pragma unroll
-            for (int i = 0; i < 32; ++i) {
-              const float2 ct = qct[cbase + i];
-              v[i] = Gs * fmaf(L, v[i], ct.x);  // the score times 2^s
-              hit |= (v[i] >= ct.y ? 1u : 0u) << i;
-            }
-            while (hit) {
-              const int i = __ffs(hit) - 1;
-              hit &= hit - 1;
-              float sv = 0.0f;
+              for (int i = 0; i < 32; ++i) {
+                const float4 c = q4[i / 2];
+                const int col = cbase + i;
+                if (col < nqt) {
+                  const float sc = Gs * fmaf(L, v[i], (i & 1) ? c.z : c.x);
+                  dst[int64_t(qid_s[col]) * a.cap] = sc * qinv_s[col];
+                  if (t == 0 && row == 0) a.cnt[qid_s[col]] = nrows;
+                }
+              }
+            } else {
+              // G (cs' + L acc) - theta' >= 0 decides; its maximum over the
+              // 32 columns rules out most rows at once
+              float m = -CUDART_INF_F;
 #pragma unroll
-              for (int kk = 0; kk < 32; ++kk) sv = kk == i ? v[kk] : sv;
-              const int col = cbase + i;
-              const int q = qid_s[col];
-              const int at = atomicAdd(&a.cnt[q], 1);
-              if (at < a.cap) {
-                a.buf_s[int64_t(q) * a.cap + at] = sv * qinv_s[col];
-                a.buf_p[int64_t(q) * a.cap + at] = pos;
+              for (int i = 0; i < 32; i += 2) {
+                const float4 c = q4[i / 2];
+                m = fmaxf(m, fmaf(Gs, fmaf(L, v[i], c.x), c.y));
+                m = fmaxf(m, fmaf(Gs, fmaf(L, v[i + 1], c.z), c.w));
+              }
+              if (m >= 0.0f) {
+                uint32_t hit = 0;
+#pragma unroll
+                for (int i = 0; i < 32; i += 2) {
+                  const float4 c = q4[i / 2];
+                  hit |= (fmaf(Gs, fmaf(L, v[i], c.x), c.y) >= 0.0f ? 1u : 0u) << i;
+                  hit |= (fmaf(Gs, fmaf(L, v[i + 1], c.z), c.w) >= 0.0f ? 2u : 0u) << i;
+                }
+                while (hit) {
+                  const int i = __ffs(hit) - 1;
+                  hit &= hit - 1;
+                  float acc = 0.0f;
+#pragma unroll
+                  for (int kk = 0; kk < 32; ++kk) acc = kk == i ? v[kk] : acc;
+                  const int col = cbase + i;
+                  const int q = qid_s[col];
+                  if (q < 0) continue;
+                  const float sc = Gs * fmaf(L, acc, qct[col].x);  // the score times 2^s
+                  const int at = atomicAdd(&a.cnt[q], 1);
+                  if (at < a.cap) {
+                    a.buf_s[int64_t(q) * a.cap + at] = sc * qinv_s[col];
+                    a.buf_p[int64_t(q) * a.cap + at] = pos;
+                  }
+                }
               }
             }
           }
         }
       }
+      __syncwarp();
+      if (ok && lane == 0) mbar_arrive(item_empty(s));
     }
-    gt += uint32_t(ntiles);
   }
   __syncthreads();
   if (warp == 0) {
@@ -1031,8 +1278,11 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   if (b.nkc == 1) {
     // padded D <= 128: the pipelined, warp-specialized kernel (one CTA per SM)
-    const size_t psmem = size_t(2) * kTileBytes + 2 * size_t(slab_bytes(g)) + size_t(kNQ) * 16 + 256 * 4;
-    auto pk = g == 1 ? batched_pipe_kernel<1> : (g == 2 ? batched_pipe_kernel<2> : batched_pipe_kernel<4>);
+    const size_t psmem = pipe_smem_bytes(g);
+    auto pk = theta ? (g == 1 ? batched_pipe_kernel<1, false>
+                              : (g == 2 ? batched_pipe_kernel<2, false> : batched_pipe_kernel<4, false>))
+                    : (g == 1 ? batched_pipe_kernel<1, true>
+                              : (g == 2 ? batched_pipe_kernel<2, true> : batched_pipe_kernel<4, true>));
     e = cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(psmem));
     if (e != cudaSuccess) return e;
     cudaEvent_t stop = profile ? prof_start(ix, s, "batched_scan_kernel") : nullptr;
@@ -1119,7 +1369,8 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   if (e == cudaSuccess)
     e = run_batched(ix, L[0], qhi, qlo, qinv, Dp16, nullptr, as, ap, ac, capA, work, false, s);
   if (e == cudaSuccess) {
-    theta_kernel<<<unsigned(nq), 256, 0, s>>>(as, ac, capA, k, theta);
+    theta_warp_kernel<<<unsigned((nq + 7) / 8), 256, 0, s>>>(as, ac, nq, capA, k, theta, ovf);
+    theta_kernel<<<unsigned(nq), 256, 0, s>>>(as, ac, capA, k, theta, ovf);
     e = cudaGetLastError();
   }
   // Pass 2: all probed partitions, keeping candidates >= theta.
