@@ -295,19 +295,51 @@ __device__ __forceinline__ void fence_proxy_async() {
   asm volatile("fence.proxy.async.shared::cta;" ::: "memory");
 }
 
-// Bounded wait for the mbarrier phase `parity` to complete.
+__device__ __forceinline__ uint64_t global_ns() {
+  uint64_t t;
+  asm volatile("mov.u64 %0, %%globaltimer;" : "=l"(t));
+  return t;
+}
+
+// Bounded wait for the mbarrier phase `parity` to complete: each try_wait
+// may suspend the thread until the phase completes (up to the hint), so
+// waiting warps do not take issue slots; after 2 s of wall time it gives up.
 __device__ __forceinline__ bool mbar_wait(uint32_t mbar, uint32_t parity) {
-  for (int i = 0; i < (1 << 22); ++i) {
+  constexpr uint64_t kLimitNs = 2000000000ull;
+  uint64_t t0 = 0;
+  for (int i = 0;; ++i) {
     uint32_t ok;
     asm volatile(
-        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n"
+        "{\n .reg .pred p;\n mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n"
         " selp.u32 %0, 1, 0, p;\n}\n"
         : "=r"(ok)
-        : "r"(mbar), "r"(parity)
+        : "r"(mbar), "r"(parity), "r"(10000000u)
         : "memory");
     if (ok) return true;
+    const uint64_t now = global_ns();
+    if (i == 0) t0 = now;
+    else if (now - t0 > kLimitNs) return false;
   }
-  return false;
+}
+
+// Packed fp32 pairs: d = a * b + c elementwise (each rounded once, as fmaf).
+__device__ __forceinline__ uint64_t f2pack(float lo, float hi) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(r) : "f"(lo), "f"(hi));
+  return r;
+}
+__device__ __forceinline__ void f2unpack(uint64_t v, float& lo, float& hi) {
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(v));
+}
+__device__ __forceinline__ uint64_t fma2(uint64_t a, uint64_t b, uint64_t c) {
+  uint64_t d;
+  asm("fma.rn.f32x2 %0, %1, %2, %3;" : "=l"(d) : "l"(a), "l"(b), "l"(c));
+  return d;
+}
+__device__ __forceinline__ float fmax3(float a, float b, float c) {
+  float d;
+  asm("max.f32 %0, %1, %2, %3;" : "=f"(d) : "f"(a), "f"(b), "f"(c));
+  return d;
 }
 
 // 1-D bulk copy global -> shared on the async proxy, completing `bytes` of
@@ -316,6 +348,20 @@ __device__ __forceinline__ void tma_load_1d(uint32_t dst, const void* src, uint3
                                             uint32_t mbar) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mbar), "r"(bytes)
                : "memory");
+  asm volatile(
+      "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
+          dst),
+      "l"(src), "r"(bytes), "r"(mbar)
+      : "memory");
+}
+
+// One arrival on `mbar` that also expects `bytes` of transaction count.
+__device__ __forceinline__ void mbar_arrive_expect(uint32_t mbar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(mbar), "r"(bytes)
+               : "memory");
+}
+// 1-D bulk copy global -> shared completing its bytes on `mbar` (no arrival).
+__device__ __forceinline__ void bulk_copy_1d(uint32_t dst, const void* src, uint32_t bytes, uint32_t mbar) {
   asm volatile(
       "cp.async.bulk.shared::cluster.global.mbarrier::complete_tx::bytes [%0], [%1], %2, [%3];" ::"r"(
           dst),
@@ -338,6 +384,21 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, float (&v)[32]) {
   asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
 #pragma unroll
   for (int i = 0; i < 32; ++i) v[i] = __uint_as_float(r[i]);
+}
+
+// 16 consecutive fp32 columns of this thread's TMEM lane.
+__device__ __forceinline__ void tmem_ld16(uint32_t taddr, float (&v)[16]) {
+  uint32_t r[16];
+  asm volatile(
+      "tcgen05.ld.sync.aligned.32x32b.x16.b32 {%0,%1,%2,%3,%4,%5,%6,%7,%8,%9,%10,%11,%12,%13,%14,"
+      "%15}, [%16];"
+      : "=r"(r[0]), "=r"(r[1]), "=r"(r[2]), "=r"(r[3]), "=r"(r[4]), "=r"(r[5]), "=r"(r[6]),
+        "=r"(r[7]), "=r"(r[8]), "=r"(r[9]), "=r"(r[10]), "=r"(r[11]), "=r"(r[12]), "=r"(r[13]),
+        "=r"(r[14]), "=r"(r[15])
+      : "r"(taddr));
+  asm volatile("tcgen05.wait::ld.sync.aligned;" ::: "memory");
+#pragma unroll
+  for (int i = 0; i < 16; ++i) v[i] = __uint_as_float(r[i]);
 }
 
 struct BatchArgs {
@@ -651,9 +712,10 @@ __global__ void __launch_bounds__(256, 2) batched_scan_kernel(const __grid_const
 // (decoders wrote A), mma_done (the tile's MMAs finished: A free,
 // accumulator ready), acc_empty (epilogue read the accumulator).  Every wait
 // is bounded; a timeout sets the error flag and every role leaves its loop.
-constexpr int kPipeThreads = 20 * 32;
-constexpr int kMmaWarp = 16, kTmaWarp = 17, kLoadWarp0 = 18;
+constexpr int kDecWarps = 4, kEpiWarps = 16;  // decoders: warps 0-3, epilogue: warps 4-19
+constexpr int kMmaWarp = 20, kTmaWarp = 21, kLoadWarp0 = 22;
 constexpr int kLoadThreads = 64;
+constexpr int kPipeThreads = (kLoadWarp0 * 32) + kLoadThreads;
 constexpr int kSlabs = 4;
 constexpr uint32_t kPipeCols = 512;
 __device__ __forceinline__ uint32_t acc_col(uint32_t b) { return b * 128u; }       // accumulators
@@ -672,8 +734,14 @@ struct ItemDesc {
 constexpr int kOffBl = kTileBytes, kOffQct = 2 * kTileBytes, kOffQinv = kOffQct + kNQ * 8,
               kOffQid = kOffQinv + kNQ * 4, kOffDesc = kOffQid + kNQ * 4,
               kSlotBytes = (kOffDesc + int(sizeof(ItemDesc)) + 127) / 128 * 128;
+constexpr int kScaleBytes = kMR * 4;  // a tile's (L | G << 16) words
+// 4-bit codes decode a whole byte (two codes -> two halves) through a
+// 256-entry table held once per lane (entry (byte, lane) at word byte * 32 +
+// lane), so the 32 lookups of a warp always fall into 32 distinct banks.
+constexpr int kByteTableBytes = 256 * 32 * 4;
 __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
-  return size_t(2) * kSlotBytes + size_t(kSlabs) * slab_bytes(g) + 32 * 4;
+  return size_t(2) * kSlotBytes + size_t(kSlabs) * (slab_bytes(g) + kScaleBytes) + 32 * 4 +
+         (g == 1 ? kByteTableBytes : 0);
 }
 
 __device__ __forceinline__ void mbar_init(uint32_t mbar, uint32_t count) {
@@ -708,16 +776,22 @@ template <int G, bool DENSE>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
   extern __shared__ __align__(128) uint8_t psm[];
   uint8_t* slab0 = psm + 2 * kSlotBytes;
+  // the scales of the tile in slab buffer b: scl0 + b * kMR
+  uint32_t* scl0 = reinterpret_cast<uint32_t*>(slab0 + kSlabs * slab_bytes(G));
   // decode table: G = 1: code -> 1 half; G = 2: code -> 2 halves; G = 4: code -> 4 halves
-  uint32_t* t32 = reinterpret_cast<uint32_t*>(slab0 + kSlabs * slab_bytes(G));
-  __shared__ __align__(8) uint64_t bars[18];
+  uint32_t* t32 = scl0 + kSlabs * kMR;
+  __shared__ __align__(8) uint64_t bars[18 + kSlabs];
   __shared__ uint32_t tmem_base_sh;
   __shared__ int s_fail;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int CH = a.chunk;
 
+  uint32_t* t256 = t32 + 32;  // G = 1 only
   if (G == 1) {
-    for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[c];
+    for (int e = tid; e < 256 * 32; e += blockDim.x) {
+      const uint32_t byte = uint32_t(e) >> 5;  // low nibble -> low half (even position)
+      t256[e] = a.cbbits[byte & 15u] | (a.cbbits[byte >> 4] << 16);
+    }
   } else if (G == 2) {
     for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[2 * c] | (a.cbbits[2 * c + 1] << 16);
   } else {
@@ -734,18 +808,20 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   auto a_full = [&](uint32_t b) { return bar0 + 8u * (12 + b); };
   auto mma_done = [&](uint32_t b) { return bar0 + 8u * (14 + b); };
   auto acc_empty = [&](uint32_t b) { return bar0 + 8u * (16 + b); };
+  auto scale_empty = [&](uint32_t b) { return bar0 + 8u * (18 + b); };
   if (tid == 0) {
     s_fail = 0;
     for (uint32_t b = 0; b < 2; ++b) {
       mbar_init(item_full(b), kLoadThreads);
-      mbar_init(item_empty(b), 8);
-      mbar_init(a_full(b), 8);
+      mbar_init(item_empty(b), kEpiWarps);
+      mbar_init(a_full(b), kDecWarps);
       mbar_init(mma_done(b), 1);
-      mbar_init(acc_empty(b), 8);
+      mbar_init(acc_empty(b), kEpiWarps);
     }
     for (uint32_t b = 0; b < kSlabs; ++b) {
       mbar_init(slab_full(b), 1);
-      mbar_init(slab_empty(b), 8);
+      mbar_init(slab_empty(b), kDecWarps);
+      mbar_init(scale_empty(b), kEpiWarps);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -762,6 +838,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   const uint32_t tmem = tmem_base_sh;
   const uint32_t psm_addr = uint32_t(__cvta_generic_to_shared(psm));
   const uint32_t slab_addr0 = uint32_t(__cvta_generic_to_shared(slab0));
+  const uint32_t scl_addr0 = uint32_t(__cvta_generic_to_shared(scl0));
   const int n_items = a.items[a.nlist];
   const int klen = a.Dp16;  // single K chunk
   const int nbytes = (klen + 2 * G - 1) / (2 * G);
@@ -806,7 +883,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       asm volatile("bar.sync 1, %0;" ::"n"(kLoadThreads) : "memory");
       const int p = d->p, q0 = d->q0, nqt = d->nqt;
       if (p >= 0) {
-        float2* qct = reinterpret_cast<float2*>(sb + kOffQct);
+        float* qpair = reinterpret_cast<float*>(sb + kOffQct);
         float* qinv = reinterpret_cast<float*>(sb + kOffQinv);
         int* qid = reinterpret_cast<int*>(sb + kOffQid);
         int qs[kNQ / kLoadThreads];
@@ -822,7 +899,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           const float inv = v ? __ldg(a.qinv + qs[u]) : 1.0f;
           const float cs = v ? __ldg(a.lcs + q0 + j) : 0.0f;
           const float th = v ? (a.theta ? __ldg(a.theta + qs[u]) : -CUDART_INF_F) : CUDART_INF_F;
-          qct[j] = make_float2(cs / inv, -th / inv);  // exact: inv is a power of two
+          // (cs', cs'', -theta', -theta'') of the column pair: exact, inv is a power of two
+          qpair[(j >> 1) * 4 + (j & 1)] = cs / inv;
+          qpair[(j >> 1) * 4 + 2 + (j & 1)] = -th / inv;
           qinv[j] = inv;
           qid[j] = qs[u];
         }
@@ -832,10 +911,10 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         for (int u = 0; u < kNQ / kLoadThreads; ++u) {
           const int j = lt + u * kLoadThreads;
           const int64_t base = int64_t(qs[u] >= 0 ? qs[u] : 0) * a.Dp16;
-          for (int k0 = 0; k0 < k8n; k0 += 8) {
-            uint4 hv[8], lv[8];
+          for (int k0 = 0; k0 < k8n; k0 += 4) {
+            uint4 hv[4], lv[4];
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
+            for (int e = 0; e < 4; ++e) {
               hv[e] = make_uint4(0, 0, 0, 0);
               lv[e] = make_uint4(0, 0, 0, 0);
               if (qs[u] >= 0 && k0 + e < k8n) {
@@ -844,7 +923,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
               }
             }
 #pragma unroll
-            for (int e = 0; e < 8; ++e) {
+            for (int e = 0; e < 4; ++e) {
               if (k0 + e < k8n) {
                 *reinterpret_cast<uint4*>(sb + tile_off(j, k0 + e)) = hv[e];
                 *reinterpret_cast<uint4*>(sb + kOffBl + tile_off(j, k0 + e)) = lv[e];
@@ -858,7 +937,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       if (p < 0) break;
     }
   } else if (warp == kTmaWarp) {
-    // ---------------- TMA: the code slab of every tile, kSlabs ahead
+    // ---------------- TMA: the code slab and the scales of every tile, kSlabs ahead
     if (lane == 0) {
       uint32_t gt = 0;
       bool ok = true;
@@ -871,16 +950,20 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         const int p = desc(s)->p;
         if (p < 0 || failed()) break;
         const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
-        const uint8_t* codes0 = a.codes + desc(s)->slot0 * a.stride;
+        const int64_t slot0 = desc(s)->slot0;  // a multiple of kMR: scale blocks are 512-byte aligned
+        const uint8_t* codes0 = a.codes + slot0 * a.stride;
         for (int t = 0; t < ntiles; ++t, ++gt) {
           const uint32_t sb = gt % kSlabs, u = gt / kSlabs;
-          if (u > 0 && !mbar_wait(slab_empty(sb), (u - 1) & 1)) {
+          if (u > 0 && (!mbar_wait(slab_empty(sb), (u - 1) & 1) || !mbar_wait(scale_empty(sb), (u - 1) & 1))) {
             fail();
             ok = false;
             break;
           }
-          tma_load_1d(slab_addr0 + sb * uint32_t(slab_bytes(G)), codes0 + size_t(t) * kMR * a.stride,
-                      slab_len, slab_full(sb));
+          mbar_arrive_expect(slab_full(sb), slab_len + kScaleBytes);
+          bulk_copy_1d(slab_addr0 + sb * uint32_t(slab_bytes(G)), codes0 + size_t(t) * kMR * a.stride,
+                       slab_len, slab_full(sb));
+          bulk_copy_1d(scl_addr0 + sb * uint32_t(kScaleBytes), a.scales + slot0 + int64_t(t) * kMR,
+                       kScaleBytes, slab_full(sb));
         }
       }
       // no copy may still be landing when the CTA exits
@@ -928,10 +1011,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       if (gt > 0) mbar_wait(mma_done((gt - 1) & 1), ((gt - 1) >> 1) & 1);
     }
     __syncwarp();
-  } else if (warp < 8) {
-    // ---------------- decoders: thread = row r of the tile, column half dh
-    const int r = (warp & 3) * 32 + lane;
-    const int dh = warp >> 2;
+  } else if (warp < kDecWarps) {
+    // ---------------- decoders: thread = row r of the tile (both column halves)
+    const int r = warp * 32 + lane;
     uint32_t gt = 0;
     bool ok = true;
     for (uint32_t seq = 0; ok; ++seq) {
@@ -950,36 +1032,26 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           ok = false;
           break;
         }
-        // the 32 / G bytes = 8 / G words of row r this thread decodes
+        // the 64 / G bytes = 16 / G words of row r (half dh: words dh * NW ..)
         constexpr int NW = 8 / G;
-        uint32_t wd[NW];
+        uint32_t wd[2 * NW];
         {
           const uint8_t* sl = slab0 + sb * slab_bytes(G);
-          const int byte0 = dh * 4 * NW;
           if (CH == 16) {
-            // whole 16-byte chunks (G = 1: two, G = 2: one) or half of one (G = 4)
-            if constexpr (NW >= 4) {
+            // whole 16-byte chunks (G = 1: four, G = 2: two, G = 4: one)
 #pragma unroll
-              for (int v = 0; v < NW / 4; ++v) {
-                const int c = byte0 / 16 + v;
-                uint4 x = make_uint4(0, 0, 0, 0);
-                if (c < c1) x = *reinterpret_cast<const uint4*>(sl + (c * kMR + r) * 16);
-                wd[4 * v] = x.x;
-                wd[4 * v + 1] = x.y;
-                wd[4 * v + 2] = x.z;
-                wd[4 * v + 3] = x.w;
-              }
-            } else {
-              const int c = byte0 / 16;
-              uint2 x = make_uint2(0, 0);
-              if (c < c1) x = *reinterpret_cast<const uint2*>(sl + (c * kMR + r) * 16 + byte0 % 16);
-              wd[0] = x.x;
-              wd[1] = x.y;
+            for (int v = 0; v < (2 * NW) / 4; ++v) {
+              uint4 x = make_uint4(0, 0, 0, 0);
+              if (v < c1) x = *reinterpret_cast<const uint4*>(sl + (v * kMR + r) * 16);
+              wd[4 * v] = x.x;
+              wd[4 * v + 1] = x.y;
+              wd[4 * v + 2] = x.z;
+              wd[4 * v + 3] = x.w;
             }
           } else {
 #pragma unroll
-            for (int w = 0; w < NW; ++w) {
-              const int byte = byte0 + 4 * w;
+            for (int w = 0; w < 2 * NW; ++w) {
+              const int byte = 4 * w;
               const int c = byte / CH;
               wd[w] = c < c1 ? *reinterpret_cast<const uint32_t*>(sl + (c * kMR + r) * CH + (byte % CH))
                              : 0u;
@@ -988,31 +1060,6 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         }
         __syncwarp();
         if (lane == 0) mbar_arrive(slab_empty(sb));
-        // 32 columns = 64 halves = 64 / G codes
-        uint32_t av[32];
-        if constexpr (G == 1) {
-          // two codes -> one 32-bit column (low half = even position)
-#pragma unroll
-          for (int w = 0; w < 8; ++w)
-#pragma unroll
-            for (int bb = 0; bb < 4; ++bb)
-              av[4 * w + bb] =
-                  __byte_perm(t32[(wd[w] >> (8 * bb)) & 15u], t32[(wd[w] >> (8 * bb + 4)) & 15u], 0x5410);
-        } else if constexpr (G == 2) {
-#pragma unroll
-          for (int w = 0; w < 4; ++w)
-#pragma unroll
-            for (int n = 0; n < 8; ++n) av[8 * w + n] = t32[(wd[w] >> (4 * n)) & 15u];
-        } else {
-#pragma unroll
-          for (int w = 0; w < 2; ++w)
-#pragma unroll
-            for (int n = 0; n < 8; ++n) {
-              const uint32_t c = (wd[w] >> (4 * n)) & 15u;
-              av[16 * w + 2 * n] = t32[2 * c];
-              av[16 * w + 2 * n + 1] = t32[2 * c + 1];
-            }
-        }
         // A buffer b is free once the MMAs of tile gt - 2 have completed
         const uint32_t b = gt & 1, u = gt >> 1;
         if (u > 0 && !mbar_wait(mma_done(b), (u - 1) & 1)) {
@@ -1021,16 +1068,43 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           break;
         }
         fence_after_sync();
-        tmem_st32(tmem + (uint32_t((warp & 3) * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
+#pragma unroll
+        for (int dh = 0; dh < 2; ++dh) {
+          // 32 columns = 64 halves = 64 / G codes
+          uint32_t av[32];
+          if constexpr (G == 1) {
+            // one byte (two codes) -> one 32-bit column (low half = even position)
+            const uint32_t* tl = t256 + lane;
+#pragma unroll
+            for (int w = 0; w < 8; ++w)
+#pragma unroll
+              for (int bb = 0; bb < 4; ++bb) av[4 * w + bb] = tl[((wd[8 * dh + w] >> (8 * bb)) & 255u) << 5];
+          } else if constexpr (G == 2) {
+#pragma unroll
+            for (int w = 0; w < 4; ++w)
+#pragma unroll
+              for (int n = 0; n < 8; ++n) av[8 * w + n] = t32[(wd[4 * dh + w] >> (4 * n)) & 15u];
+          } else {
+#pragma unroll
+            for (int w = 0; w < 2; ++w)
+#pragma unroll
+              for (int n = 0; n < 8; ++n) {
+                const uint32_t c = (wd[2 * dh + w] >> (4 * n)) & 15u;
+                av[16 * w + 2 * n] = t32[2 * c];
+                av[16 * w + 2 * n + 1] = t32[2 * c + 1];
+              }
+          }
+          tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
+        }
         fence_before_sync();
         __syncwarp();
         if (lane == 0) mbar_arrive(a_full(b));
       }
     }
   } else {
-    // ---------------- epilogue: thread = row of quadrant warp % 4, columns eh * 64 ..
+    // ---------------- epilogue: thread = row of quadrant warp % 4, columns eh * 32 ..
     const int quad = warp & 3;
-    const int eh = (warp - 8) >> 2;
+    const int eh = (warp - kDecWarps) >> 2;
     const int row = quad * 32 + lane;
     uint32_t gt = 0;
     bool ok = true;
@@ -1045,18 +1119,29 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       const int nrows = desc(s)->nrows, nqt = desc(s)->nqt;
       const int64_t slot0 = desc(s)->slot0;
       const int ntiles = (nrows + kMR - 1) / kMR;
-      const float2* qct = reinterpret_cast<const float2*>(slot(s) + kOffQct);
+      const float* qpair = reinterpret_cast<const float*>(slot(s) + kOffQct);
       const float* qinv_s = reinterpret_cast<const float*>(slot(s) + kOffQinv);
       const int* qid_s = reinterpret_cast<const int*>(slot(s) + kOffQid);
-      // column parts of 32 this warp reads: [eh * 64, eh * 64 + 32 * nparts)
-      const int nparts = min(2, max(0, (nqt - eh * 64 + 31) / 32));
+      // this warp's 32 columns [eh * 32, eh * 32 + 32) hold queries when eh * 32 < nqt;
+      // they are processed in parts of kPart
+      constexpr int kPart = 16;
+      const bool active = eh * 32 < nqt;
       for (int t = 0; t < ntiles; ++t, ++gt) {
         const uint32_t b = gt & 1, u = gt >> 1;
         const int nvalid = min(kMR, nrows - t * kMR);
         const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row);
+        // the tile's scales arrived with its codes (slab buffer sb)
+        const uint32_t sb = gt % kSlabs;
+        if (!mbar_wait(slab_full(sb), (gt / kSlabs) & 1)) {
+          fail();
+          ok = false;
+          break;
+        }
+        const uint32_t sc = scl0[sb * kMR + row];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(scale_empty(sb));
         float L = 0.0f, Gs = 0.0f;
         if (row < nvalid) {
-          const uint32_t sc = __ldg(a.scales + pos);
           L = ue7m9_to_f32(sc & 0xffffu);
           Gs = ue4m12_to_f32(sc >> 16);
         }
@@ -1066,65 +1151,67 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           break;
         }
         fence_after_sync();
-        if (nparts == 0) {
-          fence_before_sync();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(acc_empty(b));
-        }
-#pragma unroll 1
-        for (int part = 0; part < nparts; ++part) {
-          float v[32];
-          const int cbase = eh * 64 + part * 32;
-          tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(b) + uint32_t(cbase), v);
-          if (part == nparts - 1) {
-            fence_before_sync();
-            __syncwarp();
-            if (lane == 0) mbar_arrive(acc_empty(b));
-          }
+        float vall[32];
+        if (active) tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(b) + uint32_t(eh * 32), vall);
+        // the accumulator is in registers: release it to the next tile's MMAs
+        fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty(b));
+        if (active) {
+#pragma unroll
+        for (int part = 0; part < 32 / kPart; ++part) {
+          float v[kPart];
+#pragma unroll
+          for (int i = 0; i < kPart; ++i) v[i] = vall[part * kPart + i];
+          const int cbase = eh * 32 + part * kPart;
           if (row < nvalid) {
-            // (cs', -theta') of columns 2i, 2i + 1 in one float4
-            const float4* q4 = reinterpret_cast<const float4*>(qct + cbase);
+            // (cs', cs'', -theta', -theta'') of columns cbase + 2i, + 2i + 1
+            const float4* q4 = reinterpret_cast<const float4*>(qpair + 2 * cbase);
             if constexpr (DENSE) {
               // first pass: every score, at its row of the query's buffer
               float* dst = a.buf_s + int64_t(t) * kMR + row;
 #pragma unroll
-              for (int i = 0; i < 32; ++i) {
+              for (int i = 0; i < kPart; ++i) {
                 const float4 c = q4[i / 2];
                 const int col = cbase + i;
                 if (col < nqt) {
-                  const float sc = Gs * fmaf(L, v[i], (i & 1) ? c.z : c.x);
+                  const float sc = Gs * fmaf(L, v[i], (i & 1) ? c.y : c.x);
                   dst[int64_t(qid_s[col]) * a.cap] = sc * qinv_s[col];
                   if (t == 0 && row == 0) a.cnt[qid_s[col]] = nrows;
                 }
               }
             } else {
               // G (cs' + L acc) - theta' >= 0 decides; its maximum over the
-              // 32 columns rules out most rows at once
+              // part's columns rules out most rows at once
+              const uint64_t L2 = f2pack(L, L), G2 = f2pack(Gs, Gs);
               float m = -CUDART_INF_F;
 #pragma unroll
-              for (int i = 0; i < 32; i += 2) {
+              for (int i = 0; i < kPart; i += 2) {
                 const float4 c = q4[i / 2];
-                m = fmaxf(m, fmaf(Gs, fmaf(L, v[i], c.x), c.y));
-                m = fmaxf(m, fmaf(Gs, fmaf(L, v[i + 1], c.z), c.w));
+                const uint64_t y2 = fma2(G2, fma2(L2, f2pack(v[i], v[i + 1]), f2pack(c.x, c.y)),
+                                         f2pack(c.z, c.w));
+                float y0, y1;
+                f2unpack(y2, y0, y1);
+                m = fmax3(m, y0, y1);
               }
               if (m >= 0.0f) {
                 uint32_t hit = 0;
 #pragma unroll
-                for (int i = 0; i < 32; i += 2) {
+                for (int i = 0; i < kPart; i += 2) {
                   const float4 c = q4[i / 2];
-                  hit |= (fmaf(Gs, fmaf(L, v[i], c.x), c.y) >= 0.0f ? 1u : 0u) << i;
-                  hit |= (fmaf(Gs, fmaf(L, v[i + 1], c.z), c.w) >= 0.0f ? 2u : 0u) << i;
+                  hit |= (fmaf(Gs, fmaf(L, v[i], c.x), c.z) >= 0.0f ? 1u : 0u) << i;
+                  hit |= (fmaf(Gs, fmaf(L, v[i + 1], c.y), c.w) >= 0.0f ? 2u : 0u) << i;
                 }
                 while (hit) {
                   const int i = __ffs(hit) - 1;
                   hit &= hit - 1;
                   float acc = 0.0f;
 #pragma unroll
-                  for (int kk = 0; kk < 32; ++kk) acc = kk == i ? v[kk] : acc;
+                  for (int kk = 0; kk < kPart; ++kk) acc = kk == i ? v[kk] : acc;
                   const int col = cbase + i;
                   const int q = qid_s[col];
                   if (q < 0) continue;
-                  const float sc = Gs * fmaf(L, acc, qct[col].x);  // the score times 2^s
+                  const float sc = Gs * fmaf(L, acc, qpair[(col >> 1) * 4 + (col & 1)]);  // score x 2^s
                   const int at = atomicAdd(&a.cnt[q], 1);
                   if (at < a.cap) {
                     a.buf_s[int64_t(q) * a.cap + at] = sc * qinv_s[col];
@@ -1134,6 +1221,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
               }
             }
           }
+        }
         }
       }
       __syncwarp();
@@ -1154,12 +1242,13 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
 __global__ void finalize_kernel(const float* __restrict__ buf_s, const int32_t* __restrict__ buf_p,
                                 const int* __restrict__ cnt, int cap, const int64_t* __restrict__ ids,
                                 int k, int* __restrict__ overflow, int64_t* __restrict__ out_ids,
-                                float* __restrict__ out_scores) {
+                                float* __restrict__ out_scores, const int* __restrict__ only_if) {
   extern __shared__ __align__(16) uint8_t fsm[];
   __shared__ uint32_t hist[256];
   __shared__ uint32_t sh_prefix[2];
   __shared__ uint32_t sh_n;
   const int64_t q = blockIdx.x;
+  if (only_if && only_if[q] == 0) return;
   const int tid = threadIdx.x;
   const int n = cnt[q];
   if (n > cap) {
@@ -1200,6 +1289,67 @@ __global__ void finalize_kernel(const float* __restrict__ buf_s, const int32_t* 
     const bool ok = i < m && idv[i] != LLONG_MAX;
     out_ids[q * k + i] = ok ? idv[i] : -1;
     out_scores[q * k + i] = ok ? key[i] : -CUDART_INF_F;
+  }
+}
+
+// The same result by one warp per query for buffers of at most kFinCap
+// candidates: sort them in shared memory by (score desc, id asc).  A buffer
+// with more sets need_block[q] for finalize_kernel.
+constexpr int kFinCap = 512;
+constexpr int kFinWarps = 4;
+__global__ void __launch_bounds__(kFinWarps * 32) finalize_warp_kernel(
+    const float* __restrict__ buf_s, const int32_t* __restrict__ buf_p, const int* __restrict__ cnt,
+    int64_t nq, int cap, const int64_t* __restrict__ ids, int k, int* __restrict__ overflow,
+    int* __restrict__ need_block, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+  __shared__ uint32_t fk[kFinWarps][kFinCap];
+  __shared__ int64_t fi[kFinWarps][kFinCap];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t q = int64_t(blockIdx.x) * kFinWarps + w;
+  if (q >= nq) return;
+  const int n = cnt[q];
+  if (n > cap || n > kFinCap) {
+    if (lane == 0) {
+      overflow[q] = n > cap ? 1 : 0;
+      need_block[q] = n > cap ? 0 : 1;
+    }
+    return;
+  }
+  int p2 = 1;
+  while (p2 < n || p2 < k) p2 <<= 1;
+  const float* s = buf_s + q * cap;
+  const int32_t* pp = buf_p + q * cap;
+  for (int i = lane; i < p2; i += 32) {
+    fk[w][i] = i < n ? float_order_key(s[i]) : 0u;
+    fi[w][i] = i < n ? ids[pp[i]] : LLONG_MAX;
+  }
+  __syncwarp();
+  for (int size = 2; size <= p2; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = lane; i < (p2 >> 1); i += 32) {
+        const int lo = 2 * i - (i & (stride - 1));
+        const int hi = lo + stride;
+        const bool asc = (lo & size) == 0;
+        const uint32_t klo = fk[w][lo], khi = fk[w][hi];
+        const int64_t ilo = fi[w][lo], ihi = fi[w][hi];
+        const bool swap = asc ? better(khi, ihi, klo, ilo) : better(klo, ilo, khi, ihi);
+        if (swap) {
+          fk[w][lo] = khi;
+          fk[w][hi] = klo;
+          fi[w][lo] = ihi;
+          fi[w][hi] = ilo;
+        }
+      }
+      __syncwarp();
+    }
+  }
+  for (int i = lane; i < k; i += 32) {
+    const bool ok = i < n && fi[w][i] != LLONG_MAX;
+    out_ids[q * k + i] = ok ? fi[w][i] : -1;
+    out_scores[q * k + i] = ok ? float_from_order_key(fk[w][i]) : -CUDART_INF_F;
+  }
+  if (lane == 0) {
+    overflow[q] = 0;
+    need_block[q] = 0;
   }
 }
 
@@ -1382,7 +1532,11 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
     const size_t smem = size_t(p2) * 12;
     e = cudaFuncSetAttribute(finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     if (e == cudaSuccess) {
-      finalize_kernel<<<unsigned(nq), 256, smem, s>>>(bs, bp, bc, cap, ix->ids, k, ovf, out_ids, out_scores);
+      // ac (the first pass's counts) is free again: it holds the hand-over flags
+      finalize_warp_kernel<<<unsigned((nq + kFinWarps - 1) / kFinWarps), kFinWarps * 32, 0, s>>>(
+          bs, bp, bc, nq, cap, ix->ids, k, ovf, ac, out_ids, out_scores);
+      finalize_kernel<<<unsigned(nq), 256, smem, s>>>(bs, bp, bc, cap, ix->ids, k, ovf, out_ids, out_scores,
+                                                      ac);
       e = cudaGetLastError();
     }
   }
