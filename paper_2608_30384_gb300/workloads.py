@@ -106,7 +106,7 @@ def _rows(w: Workload, ctr: np.ndarray, n: int, base: int, chunk: int, out: np.n
     return y, comp.astype(np.int32)
 
 
-def _workers() -> int:
+def workers() -> int:
     try:
         n = len(os.sched_getaffinity(0))
     except AttributeError:
@@ -152,7 +152,7 @@ def database(w: Workload):
         _, a = _rows(w, ctr, n, 0, c, out=X[lo:lo + n])
         A[lo:lo + n] = a
 
-    with ThreadPoolExecutor(_workers()) as ex:
+    with ThreadPoolExecutor(workers()) as ex:
         list(ex.map(one, range(n_chunks(w))))
     return X, A
 
@@ -176,9 +176,43 @@ def member_means(w: Workload, X: np.ndarray, A: np.ndarray, ctr: np.ndarray) -> 
         return m @ X[lo:hi]
 
     sums = np.zeros((w.P, w.D))
-    with ThreadPoolExecutor(_workers()) as ex:
+    with ThreadPoolExecutor(workers()) as ex:
         for p in ex.map(part, range(len(bounds) - 1)):
             sums += p
+    out = ctr.astype(np.float64).copy()
+    nz = cnt > 0
+    out[nz] = sums[nz] / cnt[nz, None]
+    return out.astype(np.float32)
+
+
+def assignment(w: Workload) -> np.ndarray:
+    """Component (= IVF partition) of every row, without generating the rows."""
+    A = np.empty(w.N, dtype=np.int32)
+    for c in range(n_chunks(w)):
+        lo = c * CHUNK
+        n = min(w.N, lo + CHUNK) - lo
+        A[lo:lo + n] = _rng(w.seed, 1, c).integers(0, w.P, size=n, dtype=np.int64)
+    return A
+
+
+def member_means_streamed(w: Workload, ctr: np.ndarray | None = None) -> np.ndarray:
+    """``member_means`` computed chunk by chunk (same blocks, same order, same
+    result) without holding the N x D database in memory."""
+    from scipy import sparse
+    ctr = centers(w) if ctr is None else ctr
+
+    def part(c):
+        X, A = chunk_rows(w, c, ctr)
+        m = sparse.csr_matrix((np.ones(A.size, dtype=np.float32), (A, np.arange(A.size))),
+                              shape=(w.P, A.size))
+        return m @ X, np.bincount(A, minlength=w.P)
+
+    sums = np.zeros((w.P, w.D))
+    cnt = np.zeros(w.P, dtype=np.int64)
+    with ThreadPoolExecutor(workers()) as ex:
+        for ps, pc in ex.map(part, range(n_chunks(w))):
+            sums += ps
+            cnt += pc
     out = ctr.astype(np.float64).copy()
     nz = cnt > 0
     out[nz] = sums[nz] / cnt[nz, None]
@@ -191,7 +225,7 @@ def ivf_centroids(w: Workload, X: np.ndarray | None = None, A: np.ndarray | None
     if w.centroids == "true":
         return ctr
     if X is None:
-        X, A = database(w)
+        return member_means_streamed(w, ctr)
     return member_means(w, X, A, ctr)
 
 

@@ -64,3 +64,30 @@ class Case:
 
     def xnorm_max(self):
         return float(np.linalg.norm(self.X.astype(np.float64), axis=1).max())
+
+
+def check_stage(gpu_codes, gpu_L, gpu_G, enc, X, A, bits, global_scale, name):
+    """Encode parity of one stage (tolerance rules in test_gpu_parity's header):
+    codes bit-exact except near a decision boundary (at most 1e-4 of them),
+    scale codes exact except at rounding ties, and on rows with a boundary
+    flip the scales the GPU's own codes imply.  Returns the rows without a
+    code flip."""
+    ng = enc.codes.shape[1]
+    got = codec.unpack_nibbles(gpu_codes, ng)
+    mism = got != enc.codes
+    near = codec.near_threshold(enc.u, bits, 1e-5)
+    assert np.all(near[mism]), f"{name}: code mismatch away from a decision boundary"
+    assert mism.sum() <= max(1, 1e-4 * mism.size), f"{name}: {mism.sum()} mismatched codes"
+    ok = ~mism.any(1)
+    for gv, ov, ex, fmt in ((gpu_L, enc.L_u16, enc.L_exact, K.UE7M9), (gpu_G, enc.G_u16, enc.G_exact, K.UE4M12)):
+        bad = ok & (gv.astype(np.int64) != ov)
+        if bad.any():
+            tie = ue_near_tie(ex[bad], fmt)
+            assert np.all(tie) and np.all(np.abs(gv[bad].astype(np.int64) - ov[bad]) <= 1), \
+                f"{name}: {bad.sum()} scale codes differ away from rounding ties"
+    # rows with a boundary code flip: the GPU's scales must be those its codes imply
+    for r in np.nonzero(~ok)[0]:
+        Lu, Gu, Le, Ge = codec.scales_from_codes(X[r:r + 1], A[r:r + 1], bits, got[r:r + 1], global_scale)
+        assert abs(int(gpu_L[r]) - int(Lu[0])) <= (1 if ue_near_tie(Le, K.UE7M9)[0] else 0)
+        assert abs(int(gpu_G[r]) - int(Gu[0])) <= (1 if ue_near_tie(Ge, K.UE4M12)[0] else 0)
+    return ok

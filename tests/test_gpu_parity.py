@@ -13,7 +13,7 @@ import pytest
 from oracle import codec, constants as K, search
 from oracle.rotation import rotation_matrix, rotation_mode
 from paper_2608_30384_gb300 import workloads as W
-from tests.gpu_cases import Case, ue_near_tie
+from tests.gpu_cases import Case, check_stage
 from tests.lib_util import check_topk, ensure_library, score_tol
 
 torch = pytest.importorskip("torch")
@@ -76,34 +76,12 @@ def test_query_rotation(D, bits):
 
 
 # -------------------------------------------------------------------- encode
-def _check_stage(gpu_codes, gpu_L, gpu_G, enc, X, A, bits, global_scale, name):
-    ng = enc.codes.shape[1]
-    got = codec.unpack_nibbles(gpu_codes, ng)
-    mism = got != enc.codes
-    near = codec.near_threshold(enc.u, bits, 1e-5)
-    assert np.all(near[mism]), f"{name}: code mismatch away from a decision boundary"
-    assert mism.sum() <= max(1, 1e-4 * mism.size), f"{name}: {mism.sum()} mismatched codes"
-    ok = ~mism.any(1)
-    for gv, ov, ex, fmt in ((gpu_L, enc.L_u16, enc.L_exact, K.UE7M9), (gpu_G, enc.G_u16, enc.G_exact, K.UE4M12)):
-        bad = ok & (gv.astype(np.int64) != ov)
-        if bad.any():
-            tie = ue_near_tie(ex[bad], fmt)
-            assert np.all(tie) and np.all(np.abs(gv[bad].astype(np.int64) - ov[bad]) <= 1), \
-                f"{name}: {bad.sum()} scale codes differ away from rounding ties"
-    # rows with a boundary code flip: the GPU's scales must be those its codes imply
-    for r in np.nonzero(~ok)[0]:
-        Lu, Gu, Le, Ge = codec.scales_from_codes(X[r:r + 1], A[r:r + 1], bits, got[r:r + 1], global_scale)
-        assert abs(int(gpu_L[r]) - int(Lu[0])) <= (1 if ue_near_tie(Le, K.UE7M9)[0] else 0)
-        assert abs(int(gpu_G[r]) - int(Gu[0])) <= (1 if ue_near_tie(Ge, K.UE4M12)[0] else 0)
-    return ok
-
-
 def _encode_check(case):
     ix = case.gpu_index()
     w = case.w
     c1, L1, G1 = (t.cpu().numpy() for t in ix.export_codes(1))
     A1 = case.C[case.A].astype(np.float64)
-    ok = _check_stage(c1, L1, G1, case.oracle.stage1, case.X, A1, w.bits, case.global_scale, "stage 1")
+    ok = check_stage(c1, L1, G1, case.oracle.stage1, case.X, A1, w.bits, case.global_scale, "stage 1")
     if w.rescore_bits:
         c2, L2, G2 = (t.cpu().numpy() for t in ix.export_codes(2))
         st2 = case.oracle.stage2
@@ -111,7 +89,7 @@ def _encode_check(case):
         sub = codec.Encoded(st2.bits, st2.mode, st2.D, st2.g, st2.codes[sel], st2.L_u16[sel],
                             st2.G_u16[sel], st2.Lhat[sel], st2.Ghat[sel], st2.uhat[sel], st2.u[sel],
                             st2.recon[sel], st2.L_exact[sel], st2.G_exact[sel])
-        _check_stage(c2[sel], L2[sel], G2[sel], sub, case.X[sel], case.oracle.stage1.recon[sel],
+        check_stage(c2[sel], L2[sel], G2[sel], sub, case.X[sel], case.oracle.stage1.recon[sel],
                      w.rescore_bits, case.global_scale, "stage 2")
     return ix
 
