@@ -20,7 +20,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "librslm.so")
 
-SOURCES = ["api.cu", "codec.cu", "search.cu", "batched.cu", "probe_noalloc.cu", "tables.cpp"]
+SOURCES = ["api.cu", "codec.cu", "search.cu", "batched.cu", "probe_noalloc.cu", "probe.cu", "tables.cpp"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

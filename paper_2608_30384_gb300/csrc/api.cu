@@ -64,7 +64,8 @@ cudaError_t dev_alloc(rslm_index* ix, T** p, size_t count) {
 
 void free_all(rslm_index* ix) {
   void* ptrs[] = {ix->centroids, ix->part_off, ix->part_n, ix->assign, ix->slot_of_row, ix->ids,
-                  ix->codes1,    ix->scales1,  ix->codes2, ix->scales2, ix->d_err};
+                  ix->codes1,    ix->scales1,  ix->codes2, ix->scales2, ix->d_err,   ix->ctiles,
+                  ix->cmeta,     ix->crows};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (ix->cublas) cublasDestroy(reinterpret_cast<cublasHandle_t>(ix->cublas));
@@ -75,6 +76,10 @@ void free_all(rslm_index* ix) {
 rslm_status run_probe(const rslm_index* ix, const float* queries, int64_t nq, int nprobe,
                       int32_t* out_probes, float* out_cs, cudaStream_t s) {
   if (nq == 0) return RSLM_OK;
+  if (probe_fused_supported(ix, nprobe)) {
+    RSLM_CK(launch_probe_fused(ix, queries, nq, nprobe, out_probes, out_cs, s), "fused probe launch");
+    return RSLM_OK;
+  }
   const int64_t budget = int64_t(64) << 20;  // floats in the score chunk (256 MB)
   const int64_t ld = (int64_t(ix->nlist) + 3) & ~int64_t(3);  // row stride, 16-byte multiple
   int64_t qc = budget / ld;
@@ -193,6 +198,7 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
     e = cudaMemcpyAsync(ix->centroids, centroids, size_t(nlist) * dim * sizeof(float),
                         cudaMemcpyDeviceToDevice, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(ix->d_err, 0, sizeof(int), s);
+  if (e == cudaSuccess) e = probe_prepare(ix, s);
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) {
     free_all(ix);

@@ -138,19 +138,23 @@ def test_probe_parity(case):
         assert not probs, (i, probs[:3])
 
 
-@pytest.mark.parametrize("nlist,nprobe,layout", [
-    (1001, 1, "random"), (1001, 64, "random"), (8192, 64, "random"), (8192, 256, "random"),
-    (777, 200, "random"), (4099, 300, "random"), (3000, 64, "sorted"), (2048, 100, "tied"),
-    (513, 513, "random"), (6, 5, "random"),
+@pytest.mark.parametrize("nlist,nprobe,layout,D", [
+    (1001, 1, "random", 32), (1001, 64, "random", 32), (8192, 64, "random", 32),
+    (8192, 256, "random", 32), (777, 200, "random", 32), (4099, 300, "random", 32),
+    (3000, 64, "sorted", 32), (2048, 100, "tied", 32), (513, 513, "random", 32), (6, 5, "random", 32),
+    # tensor-core probe (D <= 128, nlist >= 32 nprobe): ragged nlist and D, sorted
+    # scores, ties everywhere (list overflow: every centroid is rescored)
+    (8192, 64, "random", 128), (1000, 31, "random", 100), (4100, 128, "sorted", 96),
+    (4096, 64, "tied", 128), (2500, 77, "random", 5), (300, 9, "random", 128),
 ])
-def test_probe_selection_paths(nlist, nprobe, layout):
+def test_probe_selection_paths(nlist, nprobe, layout, D):
     """Top-nprobe of <q, c> on layouts that steer the selection kernels: random
     order (the warp kernel's bound leaves about nprobe candidates), scores
     sorted along the centroid index, all centroids equal (every element ties
     at the bound, so rows go to the block kernel), nprobe above 256 (block
     kernel only), and nlist not a multiple of 4."""
-    rng = np.random.default_rng(nlist * 7 + nprobe)
-    D, nq = 32, 70
+    rng = np.random.default_rng(nlist * 7 + nprobe + D)
+    nq = 300
     Q = rng.standard_normal((nq, D)).astype(np.float32)
     if layout == "tied":
         C = np.repeat(rng.standard_normal((1, D)), nlist, axis=0).astype(np.float32)
