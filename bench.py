@@ -48,7 +48,8 @@ CLOCK_FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_eve
 SCAN_SOURCES = {
     "scan_kernel": ["paper_2608_30384_gb300/csrc/search.cu", "paper_2608_30384_gb300/csrc/device_common.cuh"],
     "batched_scan_kernel": ["paper_2608_30384_gb300/csrc/batched.cu",
-                            "paper_2608_30384_gb300/csrc/device_common.cuh"],
+                            "paper_2608_30384_gb300/csrc/device_common.cuh",
+                            "paper_2608_30384_gb300/csrc/tcgen05.cuh"],
 }
 
 

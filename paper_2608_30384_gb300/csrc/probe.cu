@@ -185,7 +185,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int TB = tile_bytes(a.Kp);
   uint8_t* A0 = sm;                 // two query tiles
-  uint8_t* B0 = sm + 2 * TB;        // kPStages centroid tiles
+  uint8_t* B0 = sm + 2 * TB;        // kPStages centroid tiles, then the value stage
   const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
   const uint32_t a_full = bar0;
   auto b_full = [&](uint32_t s) { return bar0 + 8u * (1 + s); };
@@ -284,7 +284,9 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
 #pragma unroll
     for (int j = 0; j < 8; ++j) top[j] = -CUDART_INF_F;
     float bound = CUDART_INF_F, thr = CUDART_INF_F;
-    int n = 0;
+    int n = 0, in_group = 0;  // chunks of the current bound group seen
+    // this thread's row of the value stage: value i of a chunk at word i * kPThreads + tid
+    float* stage = reinterpret_cast<float*>(sm + (2 + kPStages) * size_t(TB)) + tid;
     int32_t* out = a.cand + (valid ? q : 0) * int64_t(a.cap);
     float* outv = a.cval + (valid ? q : 0) * int64_t(a.cap);
     for (int gt = 0; gt < ngt; ++gt) {
@@ -319,7 +321,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
               x = fminf(top[j], x);
               top[j] = hi;
             }
-            if ((gc + 1) % a.mch == 0) {
+            if (++in_group == a.mch) {
               // at least jth centroids of this group reach top[jth - 1]
               float tj = top[0];
 #pragma unroll
@@ -327,6 +329,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
               bound = fminf(bound, tj);
 #pragma unroll
               for (int j = 0; j < 8; ++j) top[j] = -CUDART_INF_F;
+              in_group = 0;
             }
           }
         } else if (mx >= thr && valid) {
@@ -337,15 +340,16 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
           for (int i = 0; i < 32; ++i) hit |= (v[i] >= thr ? 1u : 0u) << i;
           const int nreal = max(0, min(32, a.nlist - col0));  // columns beyond nlist are padding
           hit &= nreal == 32 ? ~0u : ((1u << nreal) - 1u);
+          if (hit) {
+#pragma unroll
+            for (int i = 0; i < 32; ++i) stage[i * kPThreads] = v[i];
+          }
           while (hit) {
             const int i = __ffs(hit) - 1;
             hit &= hit - 1;
-            float x = v[0];
-#pragma unroll
-            for (int j = 1; j < 32; ++j) x = i == j ? v[j] : x;
             if (n < a.cap) {
               out[n] = col0 + i;
-              outv[n] = x;
+              outv[n] = stage[i * kPThreads];
             }
             ++n;
           }
@@ -621,7 +625,8 @@ cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64
     a.cnt = reinterpret_cast<int*>(ws + o_cnt);
     a.err = ix->d_err;
     // at least 116 KB, so one CTA per SM: each CTA holds all 512 TMEM columns
-    const size_t smem = std::max(size_t(2 + kPStages) * tile_bytes(Kp), size_t(116) * 1024);
+    const size_t smem = std::max(size_t(2 + kPStages) * tile_bytes(Kp) + size_t(32) * kPThreads * 4,
+                                 size_t(116) * 1024);
     e = cudaFuncSetAttribute(probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     if (e == cudaSuccess) {
       probe_kernel<<<unsigned(nblk), kPThreads, smem, s>>>(a);
