@@ -732,32 +732,21 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           qinv[j] = inv;
           qid[j] = qs[u];
         }
-        // B rows: lane = query row, so each 16-byte store of a warp fills
-        // four whole 128-byte core-matrix rows (no bank conflicts)
+        // B rows by 16-byte asynchronous copies straight into their
+        // core-matrix positions, all in flight at once (lane = query row, so a
+        // warp's copies fill whole 128-byte rows); padding columns get zeros
+        const uint32_t sb_addr = uint32_t(__cvta_generic_to_shared(sb));
 #pragma unroll
         for (int u = 0; u < kNQ / kLoadThreads; ++u) {
           const int j = lt + u * kLoadThreads;
-          const int64_t base = int64_t(qs[u] >= 0 ? qs[u] : 0) * a.Dp16;
-          for (int k0 = 0; k0 < k8n; k0 += 4) {
-            uint4 hv[4], lv[4];
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              hv[e] = make_uint4(0, 0, 0, 0);
-              lv[e] = make_uint4(0, 0, 0, 0);
-              if (qs[u] >= 0 && k0 + e < k8n) {
-                hv[e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + (k0 + e) * 8));
-                lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
-              }
-            }
-#pragma unroll
-            for (int e = 0; e < 4; ++e) {
-              if (k0 + e < k8n) {
-                *reinterpret_cast<uint4*>(sb + tile_off(j, k0 + e)) = hv[e];
-                *reinterpret_cast<uint4*>(sb + kOffBl + tile_off(j, k0 + e)) = lv[e];
-              }
-            }
+          const bool v = qs[u] >= 0;
+          const int64_t base = int64_t(v ? qs[u] : 0) * a.Dp16;
+          for (int k8 = 0; k8 < k8n; ++k8) {
+            cp_async16(sb_addr + tile_off(j, k8), a.qhi + base + k8 * 8, v ? 16u : 0u);
+            cp_async16(sb_addr + uint32_t(kOffBl) + tile_off(j, k8), a.qlo + base + k8 * 8, v ? 16u : 0u);
           }
         }
+        cp_async_wait_all();
         fence_proxy_async();  // B is read by the tensor cores (async proxy)
       }
       mbar_arrive(item_full(s));
