@@ -233,16 +233,20 @@ def run_reference(args):
 # ------------------------------------------------------------------- GPU arm
 def launches_per_step(w: W.Workload, nq: int, batched: bool) -> int:
     """Kernels of librslm launched by one step (cuBLAS GEMMs not counted)."""
-    ld = (w.P + 3) // 4 * 4
-    qc = max(1, min(nq, (64 << 20) // ld))
-    # probe selection per query chunk: the warp-per-query kernel, then the
-    # block kernel for the rows it hands over (nprobe <= 256)
-    n = math.ceil(nq / qc) * (2 if w.nprobe <= 256 else 1)
+    if (w.D + 15) // 16 * 16 <= 128 and w.P >= 32 * w.nprobe and w.nprobe <= 256:
+        n = 3                # tensor-core probe: query operands, two-pass probe, exact selection
+    else:
+        ld = (w.P + 3) // 4 * 4
+        qc = max(1, min(nq, (64 << 20) // ld))
+        # per query chunk: the warp-per-query selection, then the block
+        # kernel for the rows it hands over (nprobe <= 256)
+        n = math.ceil(nq / qc) * (2 if w.nprobe <= 256 else 1)
     n += 1                   # query rotation
-    # batched: two probe-list inversions (count, list scan, scatter), query
-    # split, first-probe pass, threshold (warp kernel + block fallback),
-    # tensor-core scan, finalize, overflow re-scan; else one scan
-    n += 6 + 1 + 1 + 2 + 1 + 1 + 1 if batched else 1
+    # batched: two probe-list inversions (count, list scan, item table,
+    # scatter), query split, first-probe pass, threshold (warp kernel + block
+    # fallback), tensor-core scan, finalize (warp kernel + block fallback),
+    # overflow re-scan; else one scan
+    n += 8 + 1 + 1 + 2 + 1 + 2 + 1 if batched else 1
     if w.rescore_bits:
         n += 2               # second rotation + rescore
     return n

@@ -72,6 +72,12 @@ __global__ void scan_lists_kernel(const int* __restrict__ cnt, int nlist, int* _
   }
 }
 
+// item_p[i] = the partition of work item i (items[p] <= i < items[p + 1]).
+__global__ void item_part_kernel(const int* __restrict__ items, int nlist, int* __restrict__ item_p) {
+  for (int p = blockIdx.x * blockDim.x + threadIdx.x; p < nlist; p += gridDim.x * blockDim.x)
+    for (int i = items[p]; i < items[p + 1]; ++i) item_p[i] = p;
+}
+
 __global__ void scatter_pairs_kernel(const int32_t* __restrict__ probes, const float* __restrict__ cs,
                                      int64_t nq, int stride, int eff, int nlist,
                                      const int* __restrict__ off, int* __restrict__ fill,
@@ -266,6 +272,7 @@ struct BatchArgs {
   uint32_t cbbits[64];  // codebook components as binary16 bits, K x g
   const int* off;       // [nlist + 1] per-partition query list offsets
   const int* items;     // [nlist + 1] per-partition work-item offsets
+  const int* item_p;    // [items[nlist]] partition of each work item
   const int32_t* lq;
   const float* lcs;
   const __half* qhi;
@@ -391,13 +398,7 @@ __global__ void __launch_bounds__(256, 2) batched_scan_kernel(const __grid_const
     __syncthreads();
     const int item = s_item;
     if (item >= n_items) break;
-    int lo = 0, hi = a.nlist - 1;  // partition p: items[p] <= item < items[p + 1]
-    while (lo < hi) {
-      const int mid = (lo + hi + 1) >> 1;
-      if (a.items[mid] <= item) lo = mid;
-      else hi = mid - 1;
-    }
-    const int p = lo;
+    const int p = a.item_p[item];
     const int q0 = a.off[p] + (item - a.items[p]) * kNQ;
     const int nqt = min(kNQ, a.off[p + 1] - q0);
     for (int j = tid; j < kNQ; j += blockDim.x) {
@@ -548,7 +549,8 @@ __global__ void __launch_bounds__(256, 2) batched_scan_kernel(const __grid_const
 //              K-major layout) into one of two item slots while the other
 //              slot's item computes;
 //   warp 17    lane 0 streams each tile's codes (one contiguous slab of the
-//              tile-interleaved layout) by TMA into a ring of kSlabs buffers;
+//              tile-interleaved layout) and its scales by TMA into rings
+//              of kSlabs and kScaleStages buffers;
 //   warps 0-7  decode: thread = (row, half of the row's columns); take the
 //              tile's codes from the slab, decode them through a 16-entry
 //              table and store them into one of two A operands in TMEM
@@ -560,21 +562,27 @@ __global__ void __launch_bounds__(256, 2) batched_scan_kernel(const __grid_const
 //              accumulator part, apply s = G (cs + L dot) and append the
 //              candidates with s >= theta_q.
 // A warp reaches only its TMEM lane quadrant (warp index mod 4), so the
-// decode and epilogue roles span the four quadrants twice.  TMEM columns:
-// accumulators 0-127 and 128-255, A operands 256-319 and 320-383.
+// decode and epilogue roles span the four quadrants.  TMEM columns: three
+// accumulators 0-127, 128-255, 256-383 (a tcgen05.ld issued while the
+// tensor core is busy takes ~1.6k cycles, so the epilogue gets two tiles of
+// MMA time per accumulator), A operands 384-447 and 448-511.
 // mbarriers: item_full (loader -> all roles), item_empty (epilogue ->
-// loader), slab_full (TMA landed), slab_empty (decoders read it), a_full
-// (decoders wrote A), mma_done (the tile's MMAs finished: A free,
-// accumulator ready), acc_empty (epilogue read the accumulator).  Every wait
+// loader), slab_full / scale_full (TMA landed), slab_empty (decoders read
+// the codes), scale_empty (epilogue read the scales), a_full
+// (decoders wrote A), a_free (the MMAs reading an A buffer finished),
+// acc_full (a tile's MMAs finished), acc_empty (epilogue read the
+// accumulator).  Every wait
 // is bounded; a timeout sets the error flag and every role leaves its loop.
 constexpr int kDecWarps = 4, kEpiWarps = 16;  // decoders: warps 0-3, epilogue: warps 4-19
 constexpr int kMmaWarp = 20, kTmaWarp = 21, kLoadWarp0 = 22;
 constexpr int kLoadThreads = 64;
 constexpr int kPipeThreads = (kLoadWarp0 * 32) + kLoadThreads;
-constexpr int kSlabs = 4;
+constexpr int kSlabs = 6;        // code slabs in flight (released by the decoders)
+constexpr int kScaleStages = 8;  // tile scales in flight (released by the epilogue, which lags)
 constexpr uint32_t kPipeCols = 512;
+constexpr uint32_t kAccBufs = 3;  // accumulators in flight (a TMEM load under MMA load is slow)
 __device__ __forceinline__ uint32_t acc_col(uint32_t b) { return b * 128u; }       // accumulators
-__device__ __forceinline__ uint32_t a_col(uint32_t b) { return 256u + b * 64u; }   // A operands
+__device__ __forceinline__ uint32_t a_col(uint32_t b) { return 384u + b * 64u; }   // A operands
 
 // One work item as staged by the loader.
 struct ItemDesc {
@@ -595,7 +603,7 @@ constexpr int kScaleBytes = kMR * 4;  // a tile's (L | G << 16) words
 // lane), so the 32 lookups of a warp always fall into 32 distinct banks.
 constexpr int kByteTableBytes = 256 * 32 * 4;
 __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
-  return size_t(2) * kSlotBytes + size_t(kSlabs) * (slab_bytes(g) + kScaleBytes) + 32 * 4 +
+  return size_t(2) * kSlotBytes + size_t(kSlabs) * slab_bytes(g) + size_t(kScaleStages) * kScaleBytes + 32 * 4 +
          (g == 1 ? kByteTableBytes : 0);
 }
 
@@ -603,11 +611,11 @@ template <int G, bool DENSE>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
   extern __shared__ __align__(128) uint8_t psm[];
   uint8_t* slab0 = psm + 2 * kSlotBytes;
-  // the scales of the tile in slab buffer b: scl0 + b * kMR
+  // the scales of the tile in scale stage b: scl0 + b * kMR
   uint32_t* scl0 = reinterpret_cast<uint32_t*>(slab0 + kSlabs * slab_bytes(G));
   // decode table: G = 1: code -> 1 half; G = 2: code -> 2 halves; G = 4: code -> 4 halves
-  uint32_t* t32 = scl0 + kSlabs * kMR;
-  __shared__ __align__(8) uint64_t bars[18 + kSlabs];
+  uint32_t* t32 = scl0 + kScaleStages * kMR;
+  __shared__ __align__(8) uint64_t bars[8 + 2 * kSlabs + 2 * kAccBufs + 2 * kScaleStages];
   __shared__ uint32_t tmem_base_sh;
   __shared__ int s_fail;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -628,27 +636,40 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
     }
   }
   const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
+  // mbarrier layout: item_full[2], item_empty[2], a_full[2], a_free[2],
+  // slab_full / slab_empty[kSlabs], acc_full / acc_empty[kAccBufs],
+  // scale_full / scale_empty[kScaleStages]
   auto item_full = [&](uint32_t s) { return bar0 + 8u * s; };
   auto item_empty = [&](uint32_t s) { return bar0 + 8u * (2 + s); };
-  auto slab_full = [&](uint32_t b) { return bar0 + 8u * (4 + b); };
-  auto slab_empty = [&](uint32_t b) { return bar0 + 8u * (8 + b); };
-  auto a_full = [&](uint32_t b) { return bar0 + 8u * (12 + b); };
-  auto mma_done = [&](uint32_t b) { return bar0 + 8u * (14 + b); };
-  auto acc_empty = [&](uint32_t b) { return bar0 + 8u * (16 + b); };
-  auto scale_empty = [&](uint32_t b) { return bar0 + 8u * (18 + b); };
+  auto a_full = [&](uint32_t b) { return bar0 + 8u * (4 + b); };
+  auto a_free = [&](uint32_t b) { return bar0 + 8u * (6 + b); };  // A buffer b read by its MMAs
+  auto slab_full = [&](uint32_t b) { return bar0 + 8u * (8 + b); };
+  auto slab_empty = [&](uint32_t b) { return bar0 + 8u * (8 + kSlabs + b); };
+  auto acc_full = [&](uint32_t b) { return bar0 + 8u * (8 + 2 * kSlabs + b); };
+  auto acc_empty = [&](uint32_t b) { return bar0 + 8u * (8 + 2 * kSlabs + kAccBufs + b); };
+  auto scale_full = [&](uint32_t b) { return bar0 + 8u * (8 + 2 * kSlabs + 2 * kAccBufs + b); };
+  auto scale_empty = [&](uint32_t b) {
+    return bar0 + 8u * (8 + 2 * kSlabs + 2 * kAccBufs + kScaleStages + b);
+  };
   if (tid == 0) {
     s_fail = 0;
     for (uint32_t b = 0; b < 2; ++b) {
       mbar_init(item_full(b), kLoadThreads);
       mbar_init(item_empty(b), kEpiWarps);
       mbar_init(a_full(b), kDecWarps);
-      mbar_init(mma_done(b), 1);
-      mbar_init(acc_empty(b), kEpiWarps);
+      mbar_init(a_free(b), 1);
     }
     for (uint32_t b = 0; b < kSlabs; ++b) {
       mbar_init(slab_full(b), 1);
       mbar_init(slab_empty(b), kDecWarps);
+    }
+    for (uint32_t b = 0; b < kScaleStages; ++b) {
+      mbar_init(scale_full(b), 1);
       mbar_init(scale_empty(b), kEpiWarps);
+    }
+    for (uint32_t b = 0; b < kAccBufs; ++b) {
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_empty(b), kEpiWarps);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -692,12 +713,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       if (lt == 0) {
         const int item = (ok && !failed()) ? atomicAdd(a.work, 1) : n_items;
         if (item < n_items) {
-          int lo = 0, hi = a.nlist - 1;
-          while (lo < hi) {
-            const int mid = (lo + hi + 1) >> 1;
-            if (a.items[mid] <= item) lo = mid;
-            else hi = mid - 1;
-          }
+          const int lo = a.item_p[item];
           d->p = lo;
           d->q0 = a.off[lo] + (item - a.items[lo]) * kNQ;
           d->nqt = min(kNQ, a.off[lo + 1] - d->q0);
@@ -770,22 +786,29 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         const uint8_t* codes0 = a.codes + slot0 * a.stride;
         for (int t = 0; t < ntiles; ++t, ++gt) {
           const uint32_t sb = gt % kSlabs, u = gt / kSlabs;
-          if (u > 0 && (!mbar_wait(slab_empty(sb), (u - 1) & 1) || !mbar_wait(scale_empty(sb), (u - 1) & 1))) {
+          const uint32_t ss = gt % kScaleStages, us = gt / kScaleStages;
+          if ((u > 0 && !mbar_wait(slab_empty(sb), (u - 1) & 1)) ||
+              (us > 0 && !mbar_wait(scale_empty(ss), (us - 1) & 1))) {
             fail();
             ok = false;
             break;
           }
-          mbar_arrive_expect(slab_full(sb), slab_len + kScaleBytes);
+          mbar_arrive_expect(slab_full(sb), slab_len);
           bulk_copy_1d(slab_addr0 + sb * uint32_t(slab_bytes(G)), codes0 + size_t(t) * kMR * a.stride,
                        slab_len, slab_full(sb));
-          bulk_copy_1d(scl_addr0 + sb * uint32_t(kScaleBytes), a.scales + slot0 + int64_t(t) * kMR,
-                       kScaleBytes, slab_full(sb));
+          mbar_arrive_expect(scale_full(ss), kScaleBytes);
+          bulk_copy_1d(scl_addr0 + ss * uint32_t(kScaleBytes), a.scales + slot0 + int64_t(t) * kMR,
+                       kScaleBytes, scale_full(ss));
         }
       }
       // no copy may still be landing when the CTA exits
       for (uint32_t sb = 0; sb < kSlabs && sb < gt; ++sb) {
         const uint32_t last = (gt - 1 - sb) / kSlabs;  // last use of buffer sb
         mbar_wait(slab_full(sb), last & 1);
+      }
+      for (uint32_t ss = 0; ss < kScaleStages && ss < gt; ++ss) {
+        const uint32_t last = (gt - 1 - ss) / kScaleStages;
+        mbar_wait(scale_full(ss), last & 1);
       }
     }
     __syncwarp();
@@ -807,8 +830,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         const uint32_t idesc = f16_idesc(kMR, max(16, (nqt + 15) & ~15));
         const uint32_t bh_addr = psm_addr + s * kSlotBytes, bl_addr = bh_addr + kOffBl;
         for (int t = 0; t < ntiles; ++t, ++gt) {
-          const uint32_t b = gt & 1, u = gt >> 1;
-          if (!mbar_wait(a_full(b), u & 1) || (u > 0 && !mbar_wait(acc_empty(b), (u - 1) & 1))) {
+          const uint32_t b = gt & 1, u = gt >> 1;             // A buffer
+          const uint32_t c = gt % kAccBufs, uc = gt / kAccBufs;  // accumulator
+          if (!mbar_wait(a_full(b), u & 1) || (uc > 0 && !mbar_wait(acc_empty(c), (uc - 1) & 1))) {
             fail();
             ok = false;
             break;
@@ -816,15 +840,16 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           fence_after_sync();
           for (int ks = 0; ks < klen / 16; ++ks) {
             const uint32_t at = tmem + a_col(b) + uint32_t(ks * 8);
-            umma_f16_ts(tmem + acc_col(b), at, smem_desc(bh_addr + ks * 256, 128, kSBO), idesc,
+            umma_f16_ts(tmem + acc_col(c), at, smem_desc(bh_addr + ks * 256, 128, kSBO), idesc,
                         ks > 0 ? 1u : 0u);
-            umma_f16_ts(tmem + acc_col(b), at, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
+            umma_f16_ts(tmem + acc_col(c), at, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
           }
-          umma_commit(mma_done(b));
+          umma_commit(a_free(b));
+          umma_commit(acc_full(c));
         }
       }
       // no MMA may still be running when TMEM is freed
-      if (gt > 0) mbar_wait(mma_done((gt - 1) & 1), ((gt - 1) >> 1) & 1);
+      if (gt > 0) mbar_wait(acc_full((gt - 1) % kAccBufs), ((gt - 1) / kAccBufs) & 1);
     }
     __syncwarp();
   } else if (warp < kDecWarps) {
@@ -878,7 +903,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         if (lane == 0) mbar_arrive(slab_empty(sb));
         // A buffer b is free once the MMAs of tile gt - 2 have completed
         const uint32_t b = gt & 1, u = gt >> 1;
-        if (u > 0 && !mbar_wait(mma_done(b), (u - 1) & 1)) {
+        if (u > 0 && !mbar_wait(a_free(b), (u - 1) & 1)) {
           fail();
           ok = false;
           break;
@@ -943,25 +968,25 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       constexpr int kPart = 16;
       const bool active = eh * 32 < nqt;
       for (int t = 0; t < ntiles; ++t, ++gt) {
-        const uint32_t b = gt & 1, u = gt >> 1;
+        const uint32_t b = gt % kAccBufs, u = gt / kAccBufs;  // accumulator
         const int nvalid = min(kMR, nrows - t * kMR);
         const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row);
-        // the tile's scales arrived with its codes (slab buffer sb)
-        const uint32_t sb = gt % kSlabs;
-        if (!mbar_wait(slab_full(sb), (gt / kSlabs) & 1)) {
+        // the tile's scales (scale stage ss)
+        const uint32_t ss = gt % kScaleStages;
+        if (!mbar_wait(scale_full(ss), (gt / kScaleStages) & 1)) {
           fail();
           ok = false;
           break;
         }
-        const uint32_t sc = scl0[sb * kMR + row];
+        const uint32_t sc = scl0[ss * kMR + row];
         __syncwarp();
-        if (lane == 0) mbar_arrive(scale_empty(sb));
+        if (lane == 0) mbar_arrive(scale_empty(ss));
         float L = 0.0f, Gs = 0.0f;
         if (row < nvalid) {
           L = ue7m9_to_f32(sc & 0xffffu);
           Gs = ue4m12_to_f32(sc >> 16);
         }
-        if (!mbar_wait(mma_done(b), u & 1)) {
+        if (!mbar_wait(acc_full(b), u & 1)) {
           fail();
           ok = false;
           break;
@@ -1187,6 +1212,7 @@ struct Lists {
   int* items;
   int32_t* lq;
   float* lcs;
+  int* item_p;
 };
 
 cudaError_t build_lists(const rslm_index* ix, const int32_t* probes, const float* cs, int64_t nq,
@@ -1199,6 +1225,7 @@ cudaError_t build_lists(const rslm_index* ix, const int32_t* probes, const float
   count_pairs_kernel<<<blocks_for(npairs, 256, 152 * 8), 256, 0, s>>>(probes, nq, stride, eff, nlist,
                                                                       L.cnt, ix->d_err);
   scan_lists_kernel<<<1, 1024, 0, s>>>(L.cnt, nlist, L.off, L.items);
+  item_part_kernel<<<blocks_for(nlist, 256, 152 * 4), 256, 0, s>>>(L.items, nlist, L.item_p);
   scatter_pairs_kernel<<<blocks_for(npairs, 256, 152 * 8), 256, 0, s>>>(
       probes, cs, nq, stride, eff, nlist, L.off, L.fill, L.lq, L.lcs);
   return cudaGetLastError();
@@ -1222,6 +1249,7 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   for (int i = 0; i < 64; ++i) b.cbbits[i] = __half_as_ushort(__float2half_rn(c1.cbf[i]));
   b.off = L.off;
   b.items = L.items;
+  b.item_p = L.item_p;
   b.lq = L.lq;
   b.lcs = L.lcs;
   b.qhi = qhi;
@@ -1283,7 +1311,7 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
     bytes += (n + 255) / 256 * 256;
     return at;
   };
-  size_t oL[2][6];
+  size_t oL[2][7];
   for (int l = 0; l < 2; ++l) {
     const int64_t np = l ? npairs : nq;
     oL[l][0] = take(size_t(nlist) * 4);
@@ -1292,6 +1320,7 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
     oL[l][3] = take(size_t(nlist + 1) * 4);
     oL[l][4] = take(size_t(np) * 4);
     oL[l][5] = take(size_t(np) * 4);
+    oL[l][6] = take(size_t(np / kNQ + nlist + 1) * 4);  // at most sum of ceil(cnt / kNQ) items
   }
   const size_t o_qhi = take(size_t(nq) * Dp16 * 2), o_qlo = take(size_t(nq) * Dp16 * 2),
                o_qinv = take(size_t(nq) * 4), o_theta = take(size_t(nq) * 4),
@@ -1306,7 +1335,8 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   for (int l = 0; l < 2; ++l)
     L[l] = Lists{reinterpret_cast<int*>(ws + oL[l][0]), reinterpret_cast<int*>(ws + oL[l][1]),
                  reinterpret_cast<int*>(ws + oL[l][2]), reinterpret_cast<int*>(ws + oL[l][3]),
-                 reinterpret_cast<int32_t*>(ws + oL[l][4]), reinterpret_cast<float*>(ws + oL[l][5])};
+                 reinterpret_cast<int32_t*>(ws + oL[l][4]), reinterpret_cast<float*>(ws + oL[l][5]),
+                 reinterpret_cast<int*>(ws + oL[l][6])};
   __half* qhi = reinterpret_cast<__half*>(ws + o_qhi);
   __half* qlo = reinterpret_cast<__half*>(ws + o_qlo);
   float* qinv = reinterpret_cast<float*>(ws + o_qinv);

@@ -299,15 +299,18 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
       const bool pass1 = gt < a.ntiles;
       const int t = pass1 ? gt : gt - a.ntiles;
       if (gt == a.ntiles) thr = bound - (valid ? a.delta2[q] : 0.0f);
-#pragma unroll 1
+      // the tile's 128 columns in one load (a TMEM load issued while the
+      // tensor core is busy has a long latency), then release the accumulator
+      float vt[kPRows];
+      tmem_ld128(tmem + lane_base + acc_col(m, b), vt);
+      fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty(b));
+#pragma unroll
       for (int c = 0; c < kPRows / 32; ++c) {
         float v[32];
-        tmem_ld32(tmem + lane_base + acc_col(m, b) + uint32_t(c * 32), v);
-        if (c == kPRows / 32 - 1) {
-          fence_before_sync();
-          __syncwarp();
-          if (lane == 0) mbar_arrive(acc_empty(b));
-        }
+#pragma unroll
+        for (int i = 0; i < 32; ++i) v[i] = vt[c * 32 + i];
         float mx = -CUDART_INF_F;
 #pragma unroll
         for (int i = 0; i < 32; i += 2) mx = fmax3(mx, v[i], v[i + 1]);
