@@ -127,17 +127,33 @@ def n_chunks(w: Workload) -> int:
 
 
 def rows(w: Workload, ids, ctr: np.ndarray | None = None):
-    """Rows with the given ids (regenerating only the chunks they live in)."""
+    """Rows with the given ids (regenerating only the chunks they live in, in threads)."""
     ids = np.asarray(ids, dtype=np.int64)
     ctr = centers(w) if ctr is None else ctr
     X = np.zeros((ids.size, w.D), dtype=np.float32)
     A = np.zeros(ids.size, dtype=np.int32)
-    for c in np.unique(ids // CHUNK):
+
+    def one(c):
         sel = np.nonzero(ids // CHUNK == c)[0]
         Xc, Ac = chunk_rows(w, int(c), ctr)
         X[sel] = Xc[ids[sel] - c * CHUNK]
         A[sel] = Ac[ids[sel] - c * CHUNK]
+
+    with ThreadPoolExecutor(workers()) as ex:
+        list(ex.map(one, np.unique(ids // CHUNK).tolist()))
     return X, A
+
+
+def row_blocks(w: Workload, block: int, ctr: np.ndarray | None = None):
+    """Yield (first row, rows) for consecutive blocks of `block` rows (a
+    multiple of the generation chunk), each generated in threads."""
+    assert block % CHUNK == 0
+    ctr = centers(w) if ctr is None else ctr
+    per = block // CHUNK
+    with ThreadPoolExecutor(workers()) as ex:
+        for c0 in range(0, n_chunks(w), per):
+            parts = list(ex.map(lambda c: chunk_rows(w, c, ctr)[0], range(c0, min(n_chunks(w), c0 + per))))
+            yield c0 * CHUNK, np.concatenate(parts)
 
 
 def database(w: Workload):

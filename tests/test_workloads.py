@@ -47,3 +47,10 @@ def test_queries_are_a_prefix_of_the_query_stream():
     Q = W.queries(SMALL)
     assert Q.shape == (SMALL.nq, SMALL.D)
     assert np.array_equal(W.queries(SMALL, 3), Q[:3])
+
+
+def test_row_blocks_cover_the_database_in_order():
+    X, _ = W.database(SMALL)
+    got = list(W.row_blocks(SMALL, 2 * W.CHUNK))
+    assert [lo for lo, _ in got] == [0, 2 * W.CHUNK]
+    assert np.array_equal(np.concatenate([b for _, b in got]), X)
