@@ -289,7 +289,6 @@ struct BatchArgs {
 
 constexpr int kSBO = (kKC / 8) * 128;  // bytes between 8-row groups of an operand tile
 constexpr int kTileBytes = kMR * kKC * 2;
-constexpr uint32_t kTmemCols = 128;
 // Codes of one K chunk of a tile: kKC / g positions of 4 bits per row.
 __host__ __device__ constexpr int slab_bytes(int g) { return kMR * kKC / (2 * g); }
 
@@ -297,246 +296,6 @@ __host__ __device__ constexpr int slab_bytes(int g) { return kMR * kKC / (2 * g)
 // matrices of 8 rows x 8 halves, K-adjacent ones 128 bytes apart).
 __device__ __forceinline__ uint32_t tile_off(int row, int k8) {
   return uint32_t((row >> 3) * kSBO + k8 * 128 + (row & 7) * 16);
-}
-
-// One CTA of 8 warps works on (partition, query tile) items taken from a
-// global counter.  Per 128-row tile of the partition: all threads decode the
-// codes into the A operand (fp16) and, for the first tile or when D needs
-// several K chunks, copy the queries' hi / lo parts into two B operands;
-// thread 0 issues the tcgen05.mma chain into a 128 x 128 fp32 TMEM
-// accumulator (rows x queries) and commits it to an mbarrier; then every
-// thread reads its row of the accumulator (warps w and w + 4 share a lane
-// quadrant and split the 128 columns) and applies the epilogue.
-// Per-query epilogue parameters of a work item.
-struct QParam {
-  float inv;  // 2^-s of the query's hi / lo split
-  float cs;   // <q, c_p>
-  float th;   // theta_q (+inf for padding columns)
-  int q;      // query index (-1 for padding columns)
-};
-
-// Decoded halves of the two codes of one byte: 2 G halves.
-template <int G> struct DecT;
-template <> struct DecT<1> { using T = uint32_t; };
-template <> struct DecT<2> { using T = uint2; };
-template <> struct DecT<4> { using T = uint4; };
-
-template <int G>
-__global__ void __launch_bounds__(256, 2) batched_scan_kernel(const __grid_constant__ BatchArgs a) {
-  using Dec = typename DecT<G>::T;
-  extern __shared__ __align__(16) uint8_t bsm[];
-  uint8_t* As = bsm;
-  uint8_t* Bh = As + kTileBytes;
-  uint8_t* Bl = Bh + kTileBytes;
-  uint8_t* slab = Bl + kTileBytes;  // codes of the current (tile, K chunk), copied by TMA
-  QParam* qp = reinterpret_cast<QParam*>(slab + slab_bytes(G));
-  Dec* dec = reinterpret_cast<Dec*>(qp + kNQ);  // byte -> its two codes' 2 G halves
-  __shared__ __align__(8) uint64_t mbar_storage;
-  __shared__ __align__(8) uint64_t tma_mbar_storage;
-  __shared__ uint32_t tmem_base_sh;
-  __shared__ int s_item;
-  __shared__ int s_fail;
-  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-  constexpr int g = G;
-
-  // byte -> the 2 g halves of its two codes (low nibble first)
-  for (int b = tid; b < 256; b += blockDim.x) {
-    uint32_t h[8] = {0, 0, 0, 0, 0, 0, 0, 0};
-#pragma unroll
-    for (int j = 0; j < g; ++j) {
-      h[j] = a.cbbits[(b & 15) * g + j];
-      h[g + j] = a.cbbits[(b >> 4) * g + j];
-    }
-    const uint32_t w0 = h[0] | (h[1] << 16), w1 = h[2] | (h[3] << 16);
-    const uint32_t w2 = h[4] | (h[5] << 16), w3 = h[6] | (h[7] << 16);
-    if constexpr (G == 1) dec[b] = w0;
-    else if constexpr (G == 2) dec[b] = make_uint2(w0, w1);
-    else dec[b] = make_uint4(w0, w1, w2, w3);
-  }
-  const uint32_t mbar = uint32_t(__cvta_generic_to_shared(&mbar_storage));
-  const uint32_t tmbar = uint32_t(__cvta_generic_to_shared(&tma_mbar_storage));
-  const uint32_t slab_addr = uint32_t(__cvta_generic_to_shared(slab));
-  if (tid == 0) {
-    s_fail = 0;
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(mbar) : "memory");
-    asm volatile("mbarrier.init.shared::cta.b64 [%0], 1;" ::"r"(tmbar) : "memory");
-    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
-  }
-  if (warp == 0) {
-    const uint32_t dst = uint32_t(__cvta_generic_to_shared(&tmem_base_sh));
-    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst),
-                 "r"(kTmemCols)
-                 : "memory");
-    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
-  }
-  fence_before_sync();
-  __syncthreads();
-  fence_after_sync();
-  const uint32_t tmem = tmem_base_sh;
-  const uint32_t as_addr = uint32_t(__cvta_generic_to_shared(As));
-  const uint32_t bh_addr = uint32_t(__cvta_generic_to_shared(Bh));
-  const uint32_t bl_addr = uint32_t(__cvta_generic_to_shared(Bl));
-  constexpr uint32_t idesc = f16_idesc(kMR, kNQ);
-  const int n_items = a.items[a.nlist];
-  const int quad = warp & 3;          // TMEM lane quadrant of this warp
-  const int colh = (warp >> 2) * 64;  // the 64 accumulator columns this warp reads
-  const int row_t = quad * 32 + lane; // this thread's row of the tile
-  uint32_t phase = 0, tphase = 0;
-  const int CH = a.chunk;
-  // Chunks [c0, c1) of the tile-interleaved layout hold K chunk kc of a tile.
-  auto slab_range = [&](int kc, int& c0, int& c1) {
-    const int k0 = kc * kKC;
-    const int klen = min(kKC, a.Dp16 - k0);
-    const int b0 = k0 / (2 * g), b1 = b0 + (klen + 2 * g - 1) / (2 * g);
-    c0 = b0 / CH;
-    c1 = min((b1 + CH - 1) / CH, a.stride / CH);
-  };
-
-  for (;;) {
-    __syncthreads();
-    if (tid == 0) s_item = s_fail ? n_items : atomicAdd(a.work, 1);
-    __syncthreads();
-    const int item = s_item;
-    if (item >= n_items) break;
-    const int p = a.item_p[item];
-    const int q0 = a.off[p] + (item - a.items[p]) * kNQ;
-    const int nqt = min(kNQ, a.off[p + 1] - q0);
-    for (int j = tid; j < kNQ; j += blockDim.x) {
-      const bool v = j < nqt;
-      const int q = v ? a.lq[q0 + j] : -1;
-      QParam pr;
-      pr.q = q;
-      pr.cs = v ? a.lcs[q0 + j] : 0.0f;
-      pr.th = v ? (a.theta ? a.theta[q] : -CUDART_INF_F) : CUDART_INF_F;
-      pr.inv = v ? a.qinv[q] : 0.0f;
-      qp[j] = pr;
-    }
-    __syncthreads();
-    const int nrows = a.part_n[p];
-    const int64_t slot0 = a.part_off[p];
-    const int ntiles = (nrows + kMR - 1) / kMR;
-    // TMA of the codes of (tile t, K chunk kc) into the slab.
-    auto issue_slab = [&](int t, int kc) {
-      int c0, c1;
-      slab_range(kc, c0, c1);
-      const uint8_t* src = a.codes + (slot0 + int64_t(t) * kMR) * a.stride + size_t(c0) * kMR * CH;
-      tma_load_1d(slab_addr, src, uint32_t((c1 - c0) * kMR * CH), tmbar);
-    };
-    if (tid == 0 && ntiles > 0) issue_slab(0, 0);
-    for (int t = 0; t < ntiles; ++t) {
-      const int nvalid = min(kMR, nrows - t * kMR);
-      for (int kc = 0; kc < a.nkc; ++kc) {
-        const int k0 = kc * kKC;
-        const int klen = min(kKC, a.Dp16 - k0);
-        if (t == 0 || a.nkc > 1) {
-          const int k8n = klen / 8;
-          for (int e = tid; e < kNQ * k8n; e += blockDim.x) {
-            const int j = e / k8n, k8 = e - j * k8n;
-            uint4 h = make_uint4(0, 0, 0, 0), l = make_uint4(0, 0, 0, 0);
-            if (j < nqt) {
-              const int64_t src = int64_t(qp[j].q) * a.Dp16 + k0 + k8 * 8;
-              h = *reinterpret_cast<const uint4*>(a.qhi + src);
-              l = *reinterpret_cast<const uint4*>(a.qlo + src);
-            }
-            *reinterpret_cast<uint4*>(Bh + tile_off(j, k8)) = h;
-            *reinterpret_cast<uint4*>(Bl + tile_off(j, k8)) = l;
-          }
-        }
-        // Decode: one 32-bit code word (8 codes, 8 g dimensions) per unit,
-        // read from the slab once its TMA has landed.
-        if (!mbar_wait(tmbar, tphase)) {
-          if (lane == 0) {
-            set_device_error(a.err, kErrTimeout);
-            atomicExch(&s_fail, 1);
-          }
-        }
-        tphase ^= 1u;
-        int c0, c1;
-        slab_range(kc, c0, c1);
-        const int w0 = k0 / (8 * g);                 // first code word of the chunk
-        const int nw = (klen + 8 * g - 1) / (8 * g);  // code words covering it
-        const int k8end = klen / 8;
-        for (int e = tid; e < kMR * nw; e += blockDim.x) {
-          const int r = e % kMR, wi = e / kMR;
-          const int b = 4 * (w0 + wi);
-          const int c = b / CH;
-          uint32_t word = 0;
-          if (c < c1)
-            word = *reinterpret_cast<const uint32_t*>(slab + ((c - c0) * kMR + r) * CH + (b % CH));
-          const int k8base = wi * g;  // k8 groups of this word: g of them
-#pragma unroll
-          for (int bb = 0; bb < 4; ++bb) {
-            // byte bb covers 2 g halves: k8 group k8base + (2 g bb) / 8 at half offset (2 g bb) % 8
-            const int hoff = 2 * g * bb;
-            if (k8base + hoff / 8 >= k8end) break;  // beyond this chunk's dimensions
-            *reinterpret_cast<Dec*>(As + tile_off(r, k8base + hoff / 8) + (hoff % 8) * 2) =
-                dec[(word >> (8 * bb)) & 255u];
-          }
-        }
-        fence_proxy_async();
-        fence_before_sync();
-        __syncthreads();
-        if (tid == 0) {
-          fence_after_sync();
-          for (int ks = 0; ks < klen / 16; ++ks) {
-            const uint64_t ad = smem_desc(as_addr + ks * 256, 128, kSBO);
-            umma_f16(tmem, ad, smem_desc(bh_addr + ks * 256, 128, kSBO), idesc,
-                     (kc > 0 || ks > 0) ? 1u : 0u);
-            umma_f16(tmem, ad, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
-          }
-          umma_commit(mbar);
-          // every thread has finished reading the slab: fetch the next unit's codes
-          if (kc + 1 < a.nkc) issue_slab(t, kc + 1);
-          else if (t + 1 < ntiles) issue_slab(t + 1, 0);
-        }
-        if (!mbar_wait(mbar, phase)) {
-          if (lane == 0) {
-            set_device_error(a.err, kErrTimeout);
-            atomicExch(&s_fail, 1);
-          }
-        }
-        phase ^= 1u;
-        fence_after_sync();
-      }
-      // Epilogue: this thread's row, 64 query columns.
-      float L = 0.0f, Gs = 0.0f;
-      if (row_t < nvalid) {
-        const uint32_t sc = a.scales[slot0 + int64_t(t) * kMR + row_t];
-        L = ue7m9_to_f32(sc & 0xffffu);
-        Gs = ue4m12_to_f32(sc >> 16);
-      }
-      const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row_t);
-#pragma unroll
-      for (int half = 0; half < 2; ++half) {
-        float v[32];
-        tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + uint32_t(colh + half * 32), v);
-        if (row_t < nvalid) {
-#pragma unroll
-          for (int i = 0; i < 32; ++i) {
-            const int col = colh + half * 32 + i;
-            const QParam pr = qp[col];
-            const float s = Gs * fmaf(L, v[i] * pr.inv, pr.cs);
-            if (s >= pr.th && col < nqt) {
-              const int q = pr.q;
-              const int at = atomicAdd(&a.cnt[q], 1);
-              if (at < a.cap) {
-                a.buf_s[int64_t(q) * a.cap + at] = s;
-                a.buf_p[int64_t(q) * a.cap + at] = pos;
-              }
-            }
-          }
-        }
-      }
-      fence_before_sync();
-      __syncthreads();
-    }
-  }
-  __syncthreads();
-  if (warp == 0) {
-    fence_after_sync();
-    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
-                 : "memory");
-  }
 }
 
 // ------------------------------------------------ pipelined kernel (D <= 128)
@@ -605,6 +364,106 @@ constexpr int kByteTableBytes = 256 * 32 * 4;
 __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
   return size_t(2) * kSlotBytes + size_t(kSlabs) * slab_bytes(g) + size_t(kScaleStages) * kScaleBytes + 32 * 4 +
          (g == 1 ? kByteTableBytes : 0);
+}
+
+// Half dh (32 columns = 64 halves = 64 / G codes) of a row's A operand from
+// the row's code words wd (G = 1: 16 words; byte -> column through the
+// per-lane table t256; G = 2, 4: nibble -> halves through t32).
+template <int G>
+__device__ __forceinline__ void decode_half(const uint32_t* wd, int dh, const uint32_t* t256,
+                                            const uint32_t* t32, int lane, uint32_t (&av)[32]) {
+  if constexpr (G == 1) {
+    // one byte (two codes) -> one 32-bit column (low half = even position)
+    const uint32_t* tl = t256 + lane;
+#pragma unroll
+    for (int w = 0; w < 8; ++w)
+#pragma unroll
+      for (int bb = 0; bb < 4; ++bb) av[4 * w + bb] = tl[((wd[8 * dh + w] >> (8 * bb)) & 255u) << 5];
+  } else if constexpr (G == 2) {
+#pragma unroll
+    for (int w = 0; w < 4; ++w)
+#pragma unroll
+      for (int n = 0; n < 8; ++n) av[8 * w + n] = t32[(wd[4 * dh + w] >> (4 * n)) & 15u];
+  } else {
+#pragma unroll
+    for (int w = 0; w < 2; ++w)
+#pragma unroll
+      for (int n = 0; n < 8; ++n) {
+        const uint32_t c = (wd[2 * dh + w] >> (4 * n)) & 15u;
+        av[16 * w + 2 * n] = t32[2 * c];
+        av[16 * w + 2 * n + 1] = t32[2 * c + 1];
+      }
+  }
+}
+
+// Epilogue of one row (thread) over the warp's 32 query columns of a tile:
+// DENSE stores every score at the row's place in the query's buffer;
+// otherwise G (cs' + L acc) - theta' >= 0 decides and the hits are appended.
+template <bool DENSE>
+__device__ __forceinline__ void epilogue_row(const BatchArgs& a, const float (&vall)[32], float L, float Gs,
+                                             int row, int t, int nrows, int nqt, int eh, int32_t pos,
+                                             const float* qpair, const float* qinv_s, const int* qid_s) {
+  constexpr int kPart = 16;
+#pragma unroll
+  for (int part = 0; part < 32 / kPart; ++part) {
+    float v[kPart];
+#pragma unroll
+    for (int i = 0; i < kPart; ++i) v[i] = vall[part * kPart + i];
+    const int cbase = eh * 32 + part * kPart;
+    // (cs', cs'', -theta', -theta'') of columns cbase + 2i, + 2i + 1
+    const float4* q4 = reinterpret_cast<const float4*>(qpair + 2 * cbase);
+    if constexpr (DENSE) {
+      // first pass: every score, at its row of the query's buffer
+      float* dst = a.buf_s + int64_t(t) * kMR + row;
+#pragma unroll
+      for (int i = 0; i < kPart; ++i) {
+        const float4 c = q4[i / 2];
+        const int col = cbase + i;
+        if (col < nqt) {
+          const float sc = Gs * fmaf(L, v[i], (i & 1) ? c.y : c.x);
+          dst[int64_t(qid_s[col]) * a.cap] = sc * qinv_s[col];
+          if (t == 0 && row == 0) a.cnt[qid_s[col]] = nrows;
+        }
+      }
+    } else {
+      // its maximum over the part's columns rules out most rows at once
+      const uint64_t L2 = f2pack(L, L), G2 = f2pack(Gs, Gs);
+      float m = -CUDART_INF_F;
+#pragma unroll
+      for (int i = 0; i < kPart; i += 2) {
+        const float4 c = q4[i / 2];
+        const uint64_t y2 = fma2(G2, fma2(L2, f2pack(v[i], v[i + 1]), f2pack(c.x, c.y)), f2pack(c.z, c.w));
+        float y0, y1;
+        f2unpack(y2, y0, y1);
+        m = fmax3(m, y0, y1);
+      }
+      if (m >= 0.0f) {
+        uint32_t hit = 0;
+#pragma unroll
+        for (int i = 0; i < kPart; i += 2) {
+          const float4 c = q4[i / 2];
+          hit |= (fmaf(Gs, fmaf(L, v[i], c.x), c.z) >= 0.0f ? 1u : 0u) << i;
+          hit |= (fmaf(Gs, fmaf(L, v[i + 1], c.y), c.w) >= 0.0f ? 2u : 0u) << i;
+        }
+        while (hit) {
+          const int i = __ffs(hit) - 1;
+          hit &= hit - 1;
+          float acc = 0.0f;
+#pragma unroll
+          for (int kk = 0; kk < kPart; ++kk) acc = kk == i ? v[kk] : acc;
+          const int col = cbase + i;
+          const int q = qid_s[col];
+          if (q < 0) continue;
+          const float sc = Gs * fmaf(L, acc, qpair[(col >> 1) * 4 + (col & 1)]);  // score x 2^s
+          const int at = atomicAdd(&a.cnt[q], 1);
+          if (at < a.cap) {
+            a.buf_s[int64_t(q) * a.cap + at] = sc * qinv_s[col];
+            a.buf_p[int64_t(q) * a.cap + at] = pos;
+          }
+        }
+      }
+    }
+  }
 }
 
 template <int G, bool DENSE>
@@ -748,21 +607,35 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           qinv[j] = inv;
           qid[j] = qs[u];
         }
-        // B rows by 16-byte asynchronous copies straight into their
-        // core-matrix positions, all in flight at once (lane = query row, so a
-        // warp's copies fill whole 128-byte rows); padding columns get zeros
-        const uint32_t sb_addr = uint32_t(__cvta_generic_to_shared(sb));
+        // B rows: loads in batches of four 16-byte pieces, then shared stores
+        // (lane = query row, so a warp's stores fill whole 128-byte
+        // core-matrix rows); padding columns get zeros.  Plain stores plus
+        // the proxy fence below: cp.async copies did not become reliably
+        // visible to the tensor cores through the same fence.
 #pragma unroll
         for (int u = 0; u < kNQ / kLoadThreads; ++u) {
           const int j = lt + u * kLoadThreads;
           const bool v = qs[u] >= 0;
           const int64_t base = int64_t(v ? qs[u] : 0) * a.Dp16;
-          for (int k8 = 0; k8 < k8n; ++k8) {
-            cp_async16(sb_addr + tile_off(j, k8), a.qhi + base + k8 * 8, v ? 16u : 0u);
-            cp_async16(sb_addr + uint32_t(kOffBl) + tile_off(j, k8), a.qlo + base + k8 * 8, v ? 16u : 0u);
+          for (int k0 = 0; k0 < k8n; k0 += 4) {
+            uint4 hv[4], lv[4];
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+              hv[e] = make_uint4(0, 0, 0, 0);
+              lv[e] = make_uint4(0, 0, 0, 0);
+              if (v && k0 + e < k8n) {
+                hv[e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + (k0 + e) * 8));
+                lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
+              }
+            }
+#pragma unroll
+            for (int e = 0; e < 4; ++e)
+              if (k0 + e < k8n) {
+                *reinterpret_cast<uint4*>(sb + tile_off(j, k0 + e)) = hv[e];
+                *reinterpret_cast<uint4*>(sb + kOffBl + tile_off(j, k0 + e)) = lv[e];
+              }
           }
         }
-        cp_async_wait_all();
         fence_proxy_async();  // B is read by the tensor cores (async proxy)
       }
       mbar_arrive(item_full(s));
@@ -911,30 +784,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         fence_after_sync();
 #pragma unroll
         for (int dh = 0; dh < 2; ++dh) {
-          // 32 columns = 64 halves = 64 / G codes
           uint32_t av[32];
-          if constexpr (G == 1) {
-            // one byte (two codes) -> one 32-bit column (low half = even position)
-            const uint32_t* tl = t256 + lane;
-#pragma unroll
-            for (int w = 0; w < 8; ++w)
-#pragma unroll
-              for (int bb = 0; bb < 4; ++bb) av[4 * w + bb] = tl[((wd[8 * dh + w] >> (8 * bb)) & 255u) << 5];
-          } else if constexpr (G == 2) {
-#pragma unroll
-            for (int w = 0; w < 4; ++w)
-#pragma unroll
-              for (int n = 0; n < 8; ++n) av[8 * w + n] = t32[(wd[4 * dh + w] >> (4 * n)) & 15u];
-          } else {
-#pragma unroll
-            for (int w = 0; w < 2; ++w)
-#pragma unroll
-              for (int n = 0; n < 8; ++n) {
-                const uint32_t c = (wd[2 * dh + w] >> (4 * n)) & 15u;
-                av[16 * w + 2 * n] = t32[2 * c];
-                av[16 * w + 2 * n + 1] = t32[2 * c + 1];
-              }
-          }
+          decode_half<G>(wd, dh, t256, t32, lane, av);
           tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
         }
         fence_before_sync();
@@ -963,9 +814,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       const float* qpair = reinterpret_cast<const float*>(slot(s) + kOffQct);
       const float* qinv_s = reinterpret_cast<const float*>(slot(s) + kOffQinv);
       const int* qid_s = reinterpret_cast<const int*>(slot(s) + kOffQid);
-      // this warp's 32 columns [eh * 32, eh * 32 + 32) hold queries when eh * 32 < nqt;
-      // they are processed in parts of kPart
-      constexpr int kPart = 16;
+      // this warp's 32 columns [eh * 32, eh * 32 + 32) hold queries when eh * 32 < nqt
       const bool active = eh * 32 < nqt;
       for (int t = 0; t < ntiles; ++t, ++gt) {
         const uint32_t b = gt % kAccBufs, u = gt / kAccBufs;  // accumulator
@@ -998,72 +847,460 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         fence_before_sync();
         __syncwarp();
         if (lane == 0) mbar_arrive(acc_empty(b));
-        if (active) {
+        if (active && row < nvalid)
+          epilogue_row<DENSE>(a, vall, L, Gs, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s);
+      }
+      __syncwarp();
+      if (ok && lane == 0) mbar_arrive(item_empty(s));
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {
+    fence_after_sync();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kPipeCols)
+                 : "memory");
+  }
+}
+
+// ------------------------------------------- pipelined kernel, D > 128
+// The same roles for several K chunks of 128 dims.  The query operands of
+// a whole item no longer fit in shared memory, so the rows are taken in
+// groups of kKR tiles (one TMEM accumulator each) and, per group, the K
+// chunks in order: the loader streams each chunk's B operands (the item's
+// queries, hi / lo, dims [128 kc, 128 kc + 128)) through a ring of two
+// stages, each used by the kKR tiles of the group; the TMA warp brings the
+// (tile, chunk) code slabs (a chunk's interleaved code bytes are contiguous)
+// and each tile's scales; the MMAs of a tile accumulate over its chunks.
+// Sequence per item: for group g, for chunk kc, for tile r of the group.
+constexpr int kKR = 3;                                   // tiles per group = accumulators
+constexpr int kBStageBytes = 2 * kTileBytes;             // B hi + lo of one K chunk
+constexpr int kKSlot = (kNQ * 16 + int(sizeof(ItemDesc)) + 127) / 128 * 128;  // constants + desc
+constexpr int kKOffQinv = kNQ * 8, kKOffQid = kNQ * 12, kKOffDesc = kNQ * 16;
+__host__ __device__ constexpr size_t kpipe_smem_bytes(int g) {
+  return size_t(2) * kBStageBytes + size_t(2) * kKSlot + size_t(kSlabs) * slab_bytes(g) +
+         size_t(kScaleStages) * kScaleBytes + 32 * 4 + (g == 1 ? kByteTableBytes : 0);
+}
+
+template <int G, bool DENSE>
+__global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __grid_constant__ BatchArgs a) {
+  extern __shared__ __align__(128) uint8_t psm[];
+  uint8_t* bst0 = psm;                               // B ring
+  uint8_t* islot0 = psm + 2 * kBStageBytes;          // item constants + descriptor
+  uint8_t* slab0 = islot0 + 2 * kKSlot;
+  uint32_t* scl0 = reinterpret_cast<uint32_t*>(slab0 + kSlabs * slab_bytes(G));
+  uint32_t* t32 = scl0 + kScaleStages * kMR;
+  uint32_t* t256 = t32 + 32;  // G = 1 only
+  __shared__ __align__(8) uint64_t bars[12 + 2 * kSlabs + 2 * kKR + 2 * kScaleStages];
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ int s_fail;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int CH = a.chunk;
+  if (G == 1) {
+    for (int e = tid; e < 256 * 32; e += blockDim.x) {
+      const uint32_t byte = uint32_t(e) >> 5;
+      t256[e] = a.cbbits[byte & 15u] | (a.cbbits[byte >> 4] << 16);
+    }
+  } else if (G == 2) {
+    for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[2 * c] | (a.cbbits[2 * c + 1] << 16);
+  } else {
+    for (int c = tid; c < 16; c += blockDim.x) {
+      t32[2 * c] = a.cbbits[4 * c] | (a.cbbits[4 * c + 1] << 16);
+      t32[2 * c + 1] = a.cbbits[4 * c + 2] | (a.cbbits[4 * c + 3] << 16);
+    }
+  }
+  const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
+  // mbarriers: item_full[2], item_empty[2], b_full[2], b_empty[2], a_full[2],
+  // a_free[2], slab_full / slab_empty[kSlabs], acc_full / acc_empty[kKR],
+  // scale_full / scale_empty[kScaleStages]
+  auto item_full = [&](uint32_t s) { return bar0 + 8u * s; };
+  auto item_empty = [&](uint32_t s) { return bar0 + 8u * (2 + s); };
+  auto b_full = [&](uint32_t s) { return bar0 + 8u * (4 + s); };
+  auto b_empty = [&](uint32_t s) { return bar0 + 8u * (6 + s); };
+  auto a_full = [&](uint32_t b) { return bar0 + 8u * (8 + b); };
+  auto a_free = [&](uint32_t b) { return bar0 + 8u * (10 + b); };
+  auto slab_full = [&](uint32_t b) { return bar0 + 8u * (12 + b); };
+  auto slab_empty = [&](uint32_t b) { return bar0 + 8u * (12 + kSlabs + b); };
+  auto acc_full = [&](uint32_t b) { return bar0 + 8u * (12 + 2 * kSlabs + b); };
+  auto acc_empty = [&](uint32_t b) { return bar0 + 8u * (12 + 2 * kSlabs + kKR + b); };
+  auto scale_full = [&](uint32_t b) { return bar0 + 8u * (12 + 2 * kSlabs + 2 * kKR + b); };
+  auto scale_empty = [&](uint32_t b) { return bar0 + 8u * (12 + 2 * kSlabs + 2 * kKR + kScaleStages + b); };
+  if (tid == 0) {
+    s_fail = 0;
+    for (uint32_t b = 0; b < 2; ++b) {
+      mbar_init(item_full(b), kLoadThreads);
+      mbar_init(item_empty(b), kEpiWarps);
+      mbar_init(b_full(b), kLoadThreads);
+      mbar_init(b_empty(b), 1);
+      mbar_init(a_full(b), kDecWarps);
+      mbar_init(a_free(b), 1);
+    }
+    for (uint32_t b = 0; b < kSlabs; ++b) {
+      mbar_init(slab_full(b), 1);
+      mbar_init(slab_empty(b), kDecWarps);
+    }
+    for (uint32_t b = 0; b < kKR; ++b) {
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_empty(b), kEpiWarps);
+    }
+    for (uint32_t b = 0; b < kScaleStages; ++b) {
+      mbar_init(scale_full(b), 1);
+      mbar_init(scale_empty(b), kEpiWarps);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  if (warp == 0) {
+    const uint32_t dst = uint32_t(__cvta_generic_to_shared(&tmem_base_sh));
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst),
+                 "r"(kPipeCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = tmem_base_sh;
+  const uint32_t bst_addr0 = uint32_t(__cvta_generic_to_shared(bst0));
+  const uint32_t slab_addr0 = uint32_t(__cvta_generic_to_shared(slab0));
+  const uint32_t scl_addr0 = uint32_t(__cvta_generic_to_shared(scl0));
+  const int n_items = a.items[a.nlist];
+  const int nkc = a.nkc;
+  // bytes of a full K chunk of a row; its code chunks [kc * cpk, kc * cpk + cpk)
+  const int kc_bytes = kKC / (2 * G);
+  const int cpk = kc_bytes / CH;
+  const int nchunks_row = a.stride / CH;
+  auto klen_of = [&](int kc) { return min(kKC, a.Dp16 - kc * kKC); };
+  auto slot = [&](uint32_t s) { return islot0 + s * kKSlot; };
+  auto desc = [&](uint32_t s) { return reinterpret_cast<const volatile ItemDesc*>(slot(s) + kKOffDesc); };
+  auto failed = [&]() { return *reinterpret_cast<volatile int*>(&s_fail) != 0; };
+  auto fail = [&]() {
+    set_device_error(a.err, kErrTimeout);
+    atomicExch(&s_fail, 1);
+  };
+
+  if (warp >= kLoadWarp0) {
+    // ---------------- loader: the item's constants, then its B chunks (group, chunk)
+    const int lt = tid - kLoadWarp0 * 32;
+    uint32_t bseq = 0;
+    bool ok = true;
+    for (uint32_t seq = 0; ok; ++seq) {
+      const uint32_t s = seq & 1, use = seq >> 1;
+      if (use > 0 && !mbar_wait(item_empty(s), (use - 1) & 1)) {
+        fail();
+        ok = false;
+      }
+      uint8_t* sb = slot(s);
+      ItemDesc* d = reinterpret_cast<ItemDesc*>(sb + kKOffDesc);
+      if (lt == 0) {
+        const int item = (ok && !failed()) ? atomicAdd(a.work, 1) : n_items;
+        if (item < n_items) {
+          const int lo = a.item_p[item];
+          d->p = lo;
+          d->q0 = a.off[lo] + (item - a.items[lo]) * kNQ;
+          d->nqt = min(kNQ, a.off[lo + 1] - d->q0);
+          d->nrows = a.part_n[lo];
+          d->slot0 = a.part_off[lo];
+        } else {
+          d->p = -1;
+        }
+      }
+      asm volatile("bar.sync 1, %0;" ::"n"(kLoadThreads) : "memory");
+      const int p = d->p, q0 = d->q0, nqt = d->nqt, nrows = d->nrows;
+      int qs[kNQ / kLoadThreads];
+      if (p >= 0) {
+        float* qpair = reinterpret_cast<float*>(sb);
+        float* qinv = reinterpret_cast<float*>(sb + kKOffQinv);
+        int* qid = reinterpret_cast<int*>(sb + kKOffQid);
 #pragma unroll
-        for (int part = 0; part < 32 / kPart; ++part) {
-          float v[kPart];
+        for (int u = 0; u < kNQ / kLoadThreads; ++u) {
+          const int j = lt + u * kLoadThreads;
+          qs[u] = j < nqt ? __ldg(a.lq + q0 + j) : -1;
+        }
 #pragma unroll
-          for (int i = 0; i < kPart; ++i) v[i] = vall[part * kPart + i];
-          const int cbase = eh * 32 + part * kPart;
-          if (row < nvalid) {
-            // (cs', cs'', -theta', -theta'') of columns cbase + 2i, + 2i + 1
-            const float4* q4 = reinterpret_cast<const float4*>(qpair + 2 * cbase);
-            if constexpr (DENSE) {
-              // first pass: every score, at its row of the query's buffer
-              float* dst = a.buf_s + int64_t(t) * kMR + row;
+        for (int u = 0; u < kNQ / kLoadThreads; ++u) {
+          const int j = lt + u * kLoadThreads;
+          const bool v = qs[u] >= 0;
+          const float inv = v ? __ldg(a.qinv + qs[u]) : 1.0f;
+          const float cs = v ? __ldg(a.lcs + q0 + j) : 0.0f;
+          const float th = v ? (a.theta ? __ldg(a.theta + qs[u]) : -CUDART_INF_F) : CUDART_INF_F;
+          qpair[(j >> 1) * 4 + (j & 1)] = cs / inv;  // exact: inv is a power of two
+          qpair[(j >> 1) * 4 + 2 + (j & 1)] = -th / inv;
+          qinv[j] = inv;
+          qid[j] = qs[u];
+        }
+      }
+      mbar_arrive(item_full(s));
+      if (p < 0) break;
+      // B chunks, one per (group, chunk), through the two-stage ring
+      const int ntiles = (nrows + kMR - 1) / kMR;
+      const int ngroups = (ntiles + kKR - 1) / kKR;
+      for (int g = 0; g < ngroups && ok; ++g) {
+        for (int kc = 0; kc < nkc; ++kc, ++bseq) {
+          const uint32_t bs = bseq & 1, bu = bseq >> 1;
+          if (bu > 0 && !mbar_wait(b_empty(bs), (bu - 1) & 1)) {
+            fail();
+            ok = false;
+            break;
+          }
+          uint8_t* dst = bst0 + bs * kBStageBytes;
+          const int k8n = klen_of(kc) / 8;
+          // loads in batches of four 16-byte pieces, then shared stores (lane =
+          // query row: a warp's stores fill whole 128-byte rows); see the
+          // single-chunk kernel on why not cp.async
 #pragma unroll
-              for (int i = 0; i < kPart; ++i) {
-                const float4 c = q4[i / 2];
-                const int col = cbase + i;
-                if (col < nqt) {
-                  const float sc = Gs * fmaf(L, v[i], (i & 1) ? c.y : c.x);
-                  dst[int64_t(qid_s[col]) * a.cap] = sc * qinv_s[col];
-                  if (t == 0 && row == 0) a.cnt[qid_s[col]] = nrows;
+          for (int u = 0; u < kNQ / kLoadThreads; ++u) {
+            const int j = lt + u * kLoadThreads;
+            const bool v = qs[u] >= 0;
+            const int64_t base = int64_t(v ? qs[u] : 0) * a.Dp16 + kc * kKC;
+            for (int k0 = 0; k0 < k8n; k0 += 4) {
+              uint4 hv[4], lv[4];
+#pragma unroll
+              for (int e = 0; e < 4; ++e) {
+                hv[e] = make_uint4(0, 0, 0, 0);
+                lv[e] = make_uint4(0, 0, 0, 0);
+                if (v && k0 + e < k8n) {
+                  hv[e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + (k0 + e) * 8));
+                  lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
                 }
               }
-            } else {
-              // G (cs' + L acc) - theta' >= 0 decides; its maximum over the
-              // part's columns rules out most rows at once
-              const uint64_t L2 = f2pack(L, L), G2 = f2pack(Gs, Gs);
-              float m = -CUDART_INF_F;
 #pragma unroll
-              for (int i = 0; i < kPart; i += 2) {
-                const float4 c = q4[i / 2];
-                const uint64_t y2 = fma2(G2, fma2(L2, f2pack(v[i], v[i + 1]), f2pack(c.x, c.y)),
-                                         f2pack(c.z, c.w));
-                float y0, y1;
-                f2unpack(y2, y0, y1);
-                m = fmax3(m, y0, y1);
+              for (int e = 0; e < 4; ++e)
+                if (k0 + e < k8n) {
+                  *reinterpret_cast<uint4*>(dst + tile_off(j, k0 + e)) = hv[e];
+                  *reinterpret_cast<uint4*>(dst + kTileBytes + tile_off(j, k0 + e)) = lv[e];
+                }
+            }
+          }
+          fence_proxy_async();  // B is read by the tensor cores (async proxy)
+          mbar_arrive(b_full(bs));
+        }
+      }
+    }
+  } else if (warp == kTmaWarp) {
+    // ---------------- TMA: (tile, chunk) code slabs in the group order, and each tile's scales
+    if (lane == 0) {
+      uint32_t sseq = 0, cseq = 0;
+      bool ok = true;
+      for (uint32_t seq = 0; ok; ++seq) {
+        const uint32_t s = seq & 1;
+        if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+          fail();
+          break;
+        }
+        const int p = desc(s)->p;
+        if (p < 0 || failed()) break;
+        const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
+        const int64_t slot0 = desc(s)->slot0;  // a multiple of kMR: scale blocks are 512-byte aligned
+        const uint8_t* codes0 = a.codes + slot0 * a.stride;
+        for (int g0 = 0; g0 < ntiles && ok; g0 += kKR) {
+          const int R = min(kKR, ntiles - g0);
+          for (int kc = 0; kc < nkc && ok; ++kc) {
+            const int c_lo = kc * cpk, c_n = min(cpk, nchunks_row - c_lo);
+            for (int r = 0; r < R; ++r, ++sseq) {
+              const int t = g0 + r;
+              const uint32_t sb = sseq % kSlabs, u = sseq / kSlabs;
+              if (u > 0 && !mbar_wait(slab_empty(sb), (u - 1) & 1)) {
+                fail();
+                ok = false;
+                break;
               }
-              if (m >= 0.0f) {
-                uint32_t hit = 0;
-#pragma unroll
-                for (int i = 0; i < kPart; i += 2) {
-                  const float4 c = q4[i / 2];
-                  hit |= (fmaf(Gs, fmaf(L, v[i], c.x), c.z) >= 0.0f ? 1u : 0u) << i;
-                  hit |= (fmaf(Gs, fmaf(L, v[i + 1], c.y), c.w) >= 0.0f ? 2u : 0u) << i;
+              const uint32_t len = uint32_t(c_n * kMR * CH);
+              mbar_arrive_expect(slab_full(sb), len);
+              bulk_copy_1d(slab_addr0 + sb * uint32_t(slab_bytes(G)),
+                           codes0 + size_t(t) * kMR * a.stride + size_t(c_lo) * kMR * CH, len, slab_full(sb));
+              if (kc == 0) {
+                const uint32_t ss = cseq % kScaleStages, us = cseq / kScaleStages;
+                ++cseq;
+                if (us > 0 && !mbar_wait(scale_empty(ss), (us - 1) & 1)) {
+                  fail();
+                  ok = false;
+                  break;
                 }
-                while (hit) {
-                  const int i = __ffs(hit) - 1;
-                  hit &= hit - 1;
-                  float acc = 0.0f;
-#pragma unroll
-                  for (int kk = 0; kk < kPart; ++kk) acc = kk == i ? v[kk] : acc;
-                  const int col = cbase + i;
-                  const int q = qid_s[col];
-                  if (q < 0) continue;
-                  const float sc = Gs * fmaf(L, acc, qpair[(col >> 1) * 4 + (col & 1)]);  // score x 2^s
-                  const int at = atomicAdd(&a.cnt[q], 1);
-                  if (at < a.cap) {
-                    a.buf_s[int64_t(q) * a.cap + at] = sc * qinv_s[col];
-                    a.buf_p[int64_t(q) * a.cap + at] = pos;
-                  }
-                }
+                mbar_arrive_expect(scale_full(ss), kScaleBytes);
+                bulk_copy_1d(scl_addr0 + ss * uint32_t(kScaleBytes), a.scales + slot0 + int64_t(t) * kMR,
+                             kScaleBytes, scale_full(ss));
               }
             }
           }
         }
+      }
+      // no copy may still be landing when the CTA exits
+      for (uint32_t sb = 0; sb < kSlabs && sb < sseq; ++sb) mbar_wait(slab_full(sb), ((sseq - 1 - sb) / kSlabs) & 1);
+      for (uint32_t ss = 0; ss < kScaleStages && ss < cseq; ++ss)
+        mbar_wait(scale_full(ss), ((cseq - 1 - ss) / kScaleStages) & 1);
+    }
+    __syncwarp();
+  } else if (warp == kMmaWarp) {
+    // ---------------- MMA issue: per group, per chunk, per tile
+    if (lane == 0) {
+      uint32_t bseq = 0, aseq = 0, accu[kKR] = {0, 0, 0}, last_acc = 0;
+      bool ok = true, any = false;
+      for (uint32_t seq = 0; ok; ++seq) {
+        const uint32_t s = seq & 1;
+        if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+          fail();
+          break;
         }
+        const int p = desc(s)->p;
+        if (p < 0 || failed()) break;
+        const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
+        const int nqt = desc(s)->nqt;
+        const uint32_t idesc = f16_idesc(kMR, max(16, (nqt + 15) & ~15));
+        for (int g0 = 0; g0 < ntiles && ok; g0 += kKR) {
+          const int R = min(kKR, ntiles - g0);
+          for (int kc = 0; kc < nkc && ok; ++kc, ++bseq) {
+            const uint32_t bs = bseq & 1;
+            if (!mbar_wait(b_full(bs), (bseq >> 1) & 1)) {
+              fail();
+              ok = false;
+              break;
+            }
+            const uint32_t bh = bst_addr0 + bs * uint32_t(kBStageBytes), bl = bh + uint32_t(kTileBytes);
+            const int nks = klen_of(kc) / 16;
+            for (int r = 0; r < R; ++r, ++aseq) {
+              const uint32_t ab = aseq & 1;
+              if (!mbar_wait(a_full(ab), (aseq >> 1) & 1) ||
+                  (kc == 0 && accu[r] > 0 && !mbar_wait(acc_empty(r), (accu[r] - 1) & 1))) {
+                fail();
+                ok = false;
+                break;
+              }
+              fence_after_sync();
+              for (int ks = 0; ks < nks; ++ks) {
+                const uint32_t at = tmem + a_col(ab) + uint32_t(ks * 8);
+                umma_f16_ts(tmem + acc_col(r), at, smem_desc(bh + ks * 256, 128, kSBO), idesc,
+                            (kc > 0 || ks > 0) ? 1u : 0u);
+                umma_f16_ts(tmem + acc_col(r), at, smem_desc(bl + ks * 256, 128, kSBO), idesc, 1u);
+              }
+              umma_commit(a_free(ab));
+            }
+            if (!ok) break;
+            umma_commit(b_empty(bs));
+          }
+          if (!ok) break;
+          for (int r = 0; r < R; ++r) {
+            umma_commit(acc_full(r));
+            ++accu[r];
+            last_acc = r;
+            any = true;
+          }
+        }
+      }
+      // no MMA may still be running when TMEM is freed
+      if (any) mbar_wait(acc_full(last_acc), (accu[last_acc] - 1) & 1);
+    }
+    __syncwarp();
+  } else if (warp < kDecWarps) {
+    // ---------------- decoders: thread = row r of the tile, one (tile, chunk) at a time
+    const int row = warp * 32 + lane;
+    uint32_t sseq = 0, aseq = 0;
+    bool ok = true;
+    for (uint32_t seq = 0; ok; ++seq) {
+      const uint32_t s = seq & 1;
+      if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+        fail();
+        break;
+      }
+      const int p = desc(s)->p;
+      if (p < 0 || failed()) break;
+      const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
+      for (int g0 = 0; g0 < ntiles && ok; g0 += kKR) {
+        const int R = min(kKR, ntiles - g0);
+        for (int kc = 0; kc < nkc && ok; ++kc) {
+          const int c_n = min(cpk, nchunks_row - kc * cpk);  // code chunks of this K chunk
+          for (int r = 0; r < R; ++r, ++sseq, ++aseq) {
+            const uint32_t sb = sseq % kSlabs;
+            if (!mbar_wait(slab_full(sb), (sseq / kSlabs) & 1)) {
+              fail();
+              ok = false;
+              break;
+            }
+            constexpr int NW = 8 / G;
+            uint32_t wd[2 * NW];
+            {
+              const uint8_t* sl = slab0 + sb * slab_bytes(G);
+#pragma unroll
+              for (int w = 0; w < 2 * NW; ++w) {
+                const int byte = 4 * w;
+                const int c = byte / CH;
+                wd[w] = c < c_n ? *reinterpret_cast<const uint32_t*>(sl + (c * kMR + row) * CH + (byte % CH)) : 0u;
+              }
+            }
+            __syncwarp();
+            if (lane == 0) mbar_arrive(slab_empty(sb));
+            const uint32_t ab = aseq & 1, au = aseq >> 1;
+            if (au > 0 && !mbar_wait(a_free(ab), (au - 1) & 1)) {
+              fail();
+              ok = false;
+              break;
+            }
+            fence_after_sync();
+#pragma unroll
+            for (int dh = 0; dh < 2; ++dh) {
+              uint32_t av[32];
+              decode_half<G>(wd, dh, t256, t32, lane, av);
+              tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(ab) + uint32_t(dh * 32), av);
+            }
+            fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(a_full(ab));
+          }
+        }
+      }
+    }
+  } else {
+    // ---------------- epilogue: thread = row of quadrant warp % 4, columns eh * 32 ..
+    const int quad = warp & 3;
+    const int eh = (warp - kDecWarps) >> 2;
+    const int row = quad * 32 + lane;
+    uint32_t cseq = 0, accu[kKR] = {0, 0, 0};
+    bool ok = true;
+    for (uint32_t seq = 0; ok; ++seq) {
+      const uint32_t s = seq & 1;
+      if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+        fail();
+        break;
+      }
+      const int p = desc(s)->p;
+      if (p < 0 || failed()) break;
+      const int nrows = desc(s)->nrows, nqt = desc(s)->nqt;
+      const int64_t slot0 = desc(s)->slot0;
+      const int ntiles = (nrows + kMR - 1) / kMR;
+      const float* qpair = reinterpret_cast<const float*>(slot(s));
+      const float* qinv_s = reinterpret_cast<const float*>(slot(s) + kKOffQinv);
+      const int* qid_s = reinterpret_cast<const int*>(slot(s) + kKOffQid);
+      const bool active = eh * 32 < nqt;
+      for (int t = 0; t < ntiles && ok; ++t, ++cseq) {
+        const int r = t % kKR;
+        const int nvalid = min(kMR, nrows - t * kMR);
+        const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row);
+        const uint32_t ss = cseq % kScaleStages;
+        if (!mbar_wait(scale_full(ss), (cseq / kScaleStages) & 1)) {
+          fail();
+          ok = false;
+          break;
+        }
+        const uint32_t sc = scl0[ss * kMR + row];
+        __syncwarp();
+        if (lane == 0) mbar_arrive(scale_empty(ss));
+        float L = 0.0f, Gs = 0.0f;
+        if (row < nvalid) {
+          L = ue7m9_to_f32(sc & 0xffffu);
+          Gs = ue4m12_to_f32(sc >> 16);
+        }
+        if (!mbar_wait(acc_full(r), accu[r] & 1)) {
+          fail();
+          ok = false;
+          break;
+        }
+        ++accu[r];
+        fence_after_sync();
+        float vall[32];
+        if (active) tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(r) + uint32_t(eh * 32), vall);
+        fence_before_sync();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(acc_empty(r));
+        if (active && row < nvalid)
+          epilogue_row<DENSE>(a, vall, L, Gs, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s);
       }
       __syncwarp();
       if (ok && lane == 0) mbar_arrive(item_empty(s));
@@ -1265,30 +1502,29 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   cudaError_t e = cudaMemsetAsync(work, 0, 4, s);
   if (e != cudaSuccess) return e;
   const int g = c1.g;
-  const size_t dec_bytes = size_t(256) * 2 * g * 2;  // 2 g halves per byte value
-  const size_t smem = size_t(3) * kTileBytes + slab_bytes(g) + size_t(kNQ) * sizeof(QParam) + dec_bytes;
   int sms = 152;
   int dev = 0;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  if (b.nkc == 1) {
-    // padded D <= 128: the pipelined, warp-specialized kernel (one CTA per SM)
-    const size_t psmem = pipe_smem_bytes(g);
-    auto pk = theta ? (g == 1 ? batched_pipe_kernel<1, false>
-                              : (g == 2 ? batched_pipe_kernel<2, false> : batched_pipe_kernel<4, false>))
-                    : (g == 1 ? batched_pipe_kernel<1, true>
-                              : (g == 2 ? batched_pipe_kernel<2, true> : batched_pipe_kernel<4, true>));
-    e = cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(psmem));
-    if (e != cudaSuccess) return e;
-    cudaEvent_t stop = profile ? prof_start(ix, s, "batched_scan_kernel") : nullptr;
-    pk<<<sms, kPipeThreads, psmem, s>>>(b);
-    prof_stop(stop, s);
-    return cudaGetLastError();
-  }
-  auto kern = c1.g == 1 ? batched_scan_kernel<1> : (c1.g == 2 ? batched_scan_kernel<2> : batched_scan_kernel<4>);
-  e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  // padded D <= 128: the whole K range per item (B once per item);
+  // otherwise K chunks of 128 with B streamed per group of tiles
+  const bool one = b.nkc == 1;
+  const size_t smem = one ? pipe_smem_bytes(g) : kpipe_smem_bytes(g);
+  using K = void (*)(BatchArgs);
+  K pk;
+  if (one)
+    pk = theta ? (g == 1 ? batched_pipe_kernel<1, false>
+                         : (g == 2 ? batched_pipe_kernel<2, false> : batched_pipe_kernel<4, false>))
+               : (g == 1 ? batched_pipe_kernel<1, true>
+                         : (g == 2 ? batched_pipe_kernel<2, true> : batched_pipe_kernel<4, true>));
+  else
+    pk = theta ? (g == 1 ? batched_kpipe_kernel<1, false>
+                         : (g == 2 ? batched_kpipe_kernel<2, false> : batched_kpipe_kernel<4, false>))
+               : (g == 1 ? batched_kpipe_kernel<1, true>
+                         : (g == 2 ? batched_kpipe_kernel<2, true> : batched_kpipe_kernel<4, true>));
+  e = cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
   cudaEvent_t stop = profile ? prof_start(ix, s, "batched_scan_kernel") : nullptr;
-  kern<<<sms * 2, 256, smem, s>>>(b);
+  pk<<<sms, kPipeThreads, smem, s>>>(b);
   prof_stop(stop, s);
   return cudaGetLastError();
 }

@@ -234,11 +234,13 @@ def test_batched_scan_overflow_fallback():
                          seed=12)), batched=True)
 
 
-@pytest.mark.parametrize("bits,D", [(4, 128), (2, 96), (1, 128)])
+@pytest.mark.parametrize("bits,D", [(4, 128), (2, 96), (1, 128), (4, 256), (1, 768), (2, 300),
+                                    (1, 256), (2, 768), (4, 768), (1, 384)])
 def test_batched_scan_many_queries_per_partition(bits, D):
     """About 225 queries per partition: two work items per partition (N = 128
-    and a partial N), about 20 row tiles each, so the pipelined kernel's
-    slot, slab and accumulator rings wrap many times."""
+    and a partial N), about 20 row tiles each, so the pipelined kernels'
+    slot, slab and accumulator rings wrap many times; D > 128 runs several
+    K chunks (D = 300: a partial last chunk)."""
     _scan_parity(Case(Wl(f"mq{bits}", 20_000, D, 8, 0.5, False, 0.5, "mean", 600, bits, 0, 3, 10, 10,
                          seed=13 + bits)), batched=True)
 
