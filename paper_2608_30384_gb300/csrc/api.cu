@@ -180,6 +180,16 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
   }
   rslm_index* ix = new rslm_index();
   cudaGetDevice(&ix->device);
+  {
+    // Search calls take their scratch from the device's stream-ordered pool;
+    // keep freed blocks cached in the pool across synchronizations instead
+    // of returning them to the driver (this process only).
+    cudaMemPool_t pool;
+    if (cudaDeviceGetDefaultMemPool(&pool, ix->device) == cudaSuccess) {
+      uint64_t keep = ~uint64_t(0);
+      cudaMemPoolSetAttribute(pool, cudaMemPoolAttrReleaseThreshold, &keep);
+    }
+  }
   ix->D = dim;
   ix->nlist = nlist;
   ix->bits = score_bits;
