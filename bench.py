@@ -252,7 +252,8 @@ def run_reference(args):
 def launches_per_step(w: W.Workload, nq: int, batched: bool) -> int:
     """Kernels of librslm launched by one step (cuBLAS GEMMs not counted)."""
     if (w.D + 15) // 16 * 16 <= 128 and w.P >= 32 * w.nprobe and w.nprobe <= 256:
-        n = 3                # tensor-core probe: query operands, two-pass probe, exact selection
+        n = 4                # tensor-core probe: query operands, two-pass probe, list selection,
+                             # exact fallback for overflowed lists
     else:
         ld = (w.P + 3) // 4 * 4
         qc = max(1, min(nq, (64 << 20) // ld))

@@ -4,23 +4,30 @@
 //
 // For padded D <= 128 and nlist >= 32 nprobe:
 //   1. queries and centroids are scaled by powers of two (max |q| and max |c|
-//      into [1024, 2048)) and rounded to fp16 ("hi"); a = <q_hi, c_hi> is
-//      within delta = 2^-9 ||q|| max ||c|| of <q, c> (each fp16 rounding is
-//      relative 2^-11, Cauchy-Schwarz bounds the sum, fp32 accumulation adds
-//      far less);
-//   2. probe_kernel, per CTA of 256 queries, streams all centroid tiles
-//      through tcgen05.mma twice.  Pass 1: the columns are split into
+//      into [1024, 2048)) and split into fp16 parts, x = x_hi + x_lo + e with
+//      x_hi = fp16(x) and x_lo = fp16(x - x_hi).
+//        a1 = <q_hi, c_hi> is within delta1 = 2^-9 ||q|| max ||c|| of <q, c>
+//          (each fp16 rounding is relative 2^-11, Cauchy-Schwarz bounds the
+//          sum, fp32 accumulation adds far less);
+//        a3 = <q_hi, c_hi> + <q_lo, c_hi> + <q_hi, c_lo> is within
+//          delta3 = 2^-14 ||q|| max ||c||: the dropped parts (<q_lo, c_lo>,
+//          the fp16 rounding of the lo parts) are below 2^-20, and the
+//          tensor core's fp32 accumulation of 3 x 128 products stays below
+//          about 384 x 2^-23 of sum |q_i c_i| <= ||q|| ||c||;
+//   2. probe_kernel, per CTA of 256 queries, streams the centroid tiles
+//      through tcgen05.mma twice.  Pass 1 (a1): the columns are split into
 //      ceil(nprobe / j) disjoint groups of whole 32-column chunks, and each
-//      group contributes the j-th largest of its chunk maxima of a (j <= 8),
-//      which j distinct centroids of the group reach; the smallest
-//      contribution is therefore reached by at least nprobe centroids, and
-//      B = that value - delta is at most the nprobe-th largest true score.
-//      Pass 2 appends every centroid with a >= B - delta (which includes
-//      every centroid whose true score is >= B), with its a, to the query's
-//      list in increasing index order;
-//   3. probe_finish_kernel computes the exact fp32 <q, c> of the listed
-//      centroids (all centroids when a list overflowed) and takes the top
-//      nprobe by (score desc, p asc).
+//      group contributes the j-th largest of its chunk maxima of a1 (j in
+//      {1, 2, 4, 8}, a template parameter), which j distinct centroids of
+//      the group reach; the smallest
+//      contribution B1 is therefore reached by at least nprobe centroids, so
+//      the nprobe-th largest <q, c> is at least B1 - delta1.  Pass 2 (a3)
+//      appends every centroid with a3 >= B1 - delta1 - delta3, which includes
+//      every centroid of the exact top nprobe, with a3, to the query's list;
+//   3. probe_select_kernel takes the top nprobe of each list by
+//      (a3 desc, p asc) and returns <q, c> = a3 / (2^sq 2^sC).  A list that
+//      overflowed its capacity (many centroids tied at the bound) goes to
+//      probe_exact_kernel, which scores every centroid in fp32.
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <math_constants.h>
@@ -41,6 +48,7 @@ constexpr int kPStages = 3;       // centroid tiles in flight
 constexpr int kPThreads = 10 * 32;  // warps 0-7 epilogue, 8 TMA, 9 MMA
 constexpr int kPEpiWarps = 8;
 constexpr uint32_t kPCols = 512;  // TMEM: (M block, buffer) accumulators of 128 columns
+constexpr int kListCap = 1024;    // listed centroids per query before the exact fallback
 
 __host__ __device__ constexpr int tile_bytes(int Kp) { return kPRows * Kp * 2; }
 
@@ -57,6 +65,12 @@ __device__ __forceinline__ int pow2_exp_for(float m) {
   return 11 - e;                // m * 2^s in [1024, 2048)
 }
 
+// x = hi + lo with hi = fp16(x), lo = fp16(x - hi) (x - hi is exact in fp32).
+__device__ __forceinline__ void split_half(float x, __half& hi, __half& lo) {
+  hi = __float2half_rn(x);
+  lo = __float2half_rn(x - __half2float(hi));
+}
+
 // meta[0] = max |c|, meta[1] = max ||c||^2 over the centroids (one block).
 __global__ void centroid_stats_kernel(const float* __restrict__ C, int64_t n, int D, float* __restrict__ meta) {
   __shared__ float sa[32], sb[32];
@@ -70,10 +84,8 @@ __global__ void centroid_stats_kernel(const float* __restrict__ C, int64_t n, in
     }
     nm = fmaxf(nm, s2);
   }
-  am = fmaxf(am, __shfl_xor_sync(kFull, am, 16));
-  nm = fmaxf(nm, __shfl_xor_sync(kFull, nm, 16));
 #pragma unroll
-  for (int o = 8; o; o >>= 1) {
+  for (int o = 16; o; o >>= 1) {
     am = fmaxf(am, __shfl_xor_sync(kFull, am, o));
     nm = fmaxf(nm, __shfl_xor_sync(kFull, nm, o));
   }
@@ -92,9 +104,9 @@ __global__ void centroid_stats_kernel(const float* __restrict__ C, int64_t n, in
   }
 }
 
-// Centroid operand: c * 2^sC rounded to fp16, one tile per 128 centroids
-// (rows beyond nlist and dims beyond D are zero).  meta[2] = 2^sC,
-// meta[3] = max ||c|| * 2^sC.
+// Centroid operand tiles: c * 2^sC split into fp16 hi (tiles 0 .. ntiles-1)
+// and lo (tiles ntiles .. 2 ntiles-1), 128 centroids per tile (rows beyond
+// nlist and dims beyond D are zero).  meta[2] = 2^sC, meta[3] = max ||c|| 2^sC.
 __global__ void centroid_tiles_kernel(const float* __restrict__ C, int nlist, int D, int Kp,
                                       float* __restrict__ meta, uint8_t* __restrict__ tiles) {
   const int s = pow2_exp_for(meta[0]);
@@ -110,26 +122,28 @@ __global__ void centroid_tiles_kernel(const float* __restrict__ C, int nlist, in
        i += int64_t(gridDim.x) * blockDim.x) {
     const int k8 = int(i % k8n);
     const int64_t p = i / k8n;
-    __align__(16) __half h[8];
+    __align__(16) __half h[8], l[8];
 #pragma unroll
     for (int j = 0; j < 8; ++j) {
       const int d = k8 * 8 + j;
-      const float v = (p < nlist && d < D) ? C[p * D + d] * sc : 0.0f;
-      h[j] = __float2half_rn(v);
+      split_half((p < nlist && d < D) ? C[p * D + d] * sc : 0.0f, h[j], l[j]);
     }
     const int64_t t = p / kPRows;
     const int r = int(p % kPRows);
-    *reinterpret_cast<uint4*>(tiles + t * tile_bytes(Kp) + ptile_off(r, k8 * 8, Kp)) =
-        *reinterpret_cast<const uint4*>(h);
+    const uint32_t off = ptile_off(r, k8 * 8, Kp);
+    *reinterpret_cast<uint4*>(tiles + t * tile_bytes(Kp) + off) = *reinterpret_cast<const uint4*>(h);
+    *reinterpret_cast<uint4*>(tiles + (ntiles + t) * tile_bytes(Kp) + off) = *reinterpret_cast<const uint4*>(l);
   }
 }
 
-// Query operand tiles (q * 2^sq in fp16, 128 queries per tile, nqb tiles,
-// queries beyond nq zero) and 2 delta per query in the scaled units of
-// <q_hi, c_hi>: 2 * 2^-9 ||q|| 2^sq * max ||c|| 2^sC.
+// Query operand tiles, four per CTA of 256 queries: hi of M block 0 and 1,
+// then lo of M block 0 and 1 (q * 2^sq split like the centroids; queries
+// beyond nq are zero).  Per query: dthr = (delta1 + delta3) in the scaled
+// units of a1 and a3, with a 1.001 margin for its own rounding, and
+// qinv = 1 / (2^sq 2^sC), which maps a3 back to <q, c>.
 __global__ void query_tiles_kernel(const float* __restrict__ Q, int64_t nq, int64_t nqp, int D, int Kp,
                                    const float* __restrict__ meta, uint8_t* __restrict__ tiles,
-                                   float* __restrict__ delta2) {
+                                   float* __restrict__ dthr, float* __restrict__ qinv) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, W = blockDim.x >> 5;
   for (int64_t q = int64_t(blockIdx.x) * W + warp; q < nqp; q += int64_t(gridDim.x) * W) {
     float m = 0.0f, s2 = 0.0f;
@@ -145,47 +159,81 @@ __global__ void query_tiles_kernel(const float* __restrict__ Q, int64_t nq, int6
       m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
       s2 += __shfl_xor_sync(kFull, s2, o);
     }
-    const float sc = ldexpf(1.0f, pow2_exp_for(m));
-    const int64_t t = q / kPRows;
-    const int r = int(q % kPRows);
+    const int sq = pow2_exp_for(m);
+    const float sc = ldexpf(1.0f, sq);
+    const int64_t cta = q / kPQ;
+    const int mb = int((q / kPRows) % 2), r = int(q % kPRows);
+    uint8_t* hi_tile = tiles + (cta * 4 + mb) * tile_bytes(Kp);
+    uint8_t* lo_tile = tiles + (cta * 4 + 2 + mb) * tile_bytes(Kp);
     for (int k8 = lane; k8 < Kp / 8; k8 += 32) {
-      __align__(16) __half h[8];
+      __align__(16) __half h[8], l[8];
 #pragma unroll
       for (int j = 0; j < 8; ++j) {
         const int d = k8 * 8 + j;
-        h[j] = __float2half_rn((q < nq && d < D) ? Q[q * D + d] * sc : 0.0f);
+        split_half((q < nq && d < D) ? Q[q * D + d] * sc : 0.0f, h[j], l[j]);
       }
-      *reinterpret_cast<uint4*>(tiles + t * tile_bytes(Kp) + ptile_off(r, k8 * 8, Kp)) =
-          *reinterpret_cast<const uint4*>(h);
+      const uint32_t off = ptile_off(r, k8 * 8, Kp);
+      *reinterpret_cast<uint4*>(hi_tile + off) = *reinterpret_cast<const uint4*>(h);
+      *reinterpret_cast<uint4*>(lo_tile + off) = *reinterpret_cast<const uint4*>(l);
     }
-    if (lane == 0 && q < nq) delta2[q] = 2.0f * ldexpf(1.0f, -9) * sqrtf(s2) * sc * meta[3] * 1.001f;
+    if (lane == 0 && q < nq) {
+      dthr[q] = (ldexpf(1.0f, -9) + ldexpf(1.0f, -14)) * sqrtf(s2) * sc * meta[3] * 1.001f;
+      qinv[q] = ldexpf(1.0f, -sq) / meta[2];
+    }
   }
+}
+
+// Largest of 32 values by a depth-4 tree of 3-input maxima.
+__device__ __forceinline__ float max32(const float* v) {
+  float a[11];
+#pragma unroll
+  for (int j = 0; j < 10; ++j) a[j] = fmax3(v[3 * j], v[3 * j + 1], v[3 * j + 2]);
+  a[10] = fmaxf(v[30], v[31]);
+  return fmax3(fmax3(a[0], a[1], a[2]), fmax3(a[3], a[4], a[5]), fmax3(a[6], a[7], fmax3(a[8], a[9], a[10])));
+}
+
+// v[i] for a lane-varying i in [0, 32) without leaving registers: a select
+// tree on the bits of i.
+__device__ __forceinline__ float pick32(const float* v, int i) {
+  float a[16], b[8], c[4];
+#pragma unroll
+  for (int j = 0; j < 16; ++j) a[j] = (i & 1) ? v[2 * j + 1] : v[2 * j];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) b[j] = (i & 2) ? a[2 * j + 1] : a[2 * j];
+#pragma unroll
+  for (int j = 0; j < 4; ++j) c[j] = (i & 4) ? b[2 * j + 1] : b[2 * j];
+  const float d0 = (i & 8) ? c[1] : c[0], d1 = (i & 8) ? c[3] : c[2];
+  return (i & 16) ? d1 : d0;
+}
+
+// List entry: larger key = better (a3 desc, then p asc); keys are unique.
+__device__ __forceinline__ uint64_t list_key(float a, int p) {
+  return (uint64_t(float_order_key(a)) << 32) | uint64_t(~uint32_t(p));
 }
 
 struct ProbeArgs {
   const uint8_t* qtiles;
   const uint8_t* ctiles;
-  const float* delta2;
+  const float* dthr;
   int64_t nq;
   // bound groups: ngr groups of mch consecutive 32-column chunks; a group
-  // contributes its jth-largest chunk maximum (jth <= 8, jth * ngr >= nprobe)
-  int nlist, Kp, ntiles, nprobe, mch, ngr, jth;
+  // contributes its JTH-largest chunk maximum (JTH * ngr >= nprobe)
+  int nlist, Kp, ntiles, nprobe, mch, ngr;
   int cap;
-  int32_t* cand;  // [nq * cap] listed centroids
-  float* cval;    // [nq * cap] their a = <q_hi, c_hi>
-  int* cnt;       // [nq]
+  uint64_t* keys;  // [nq * cap] list_key of the listed centroids
+  int* cnt;        // [nq]
   int* err;
 };
 
+template <int JTH>
 __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_constant__ ProbeArgs a) {
   extern __shared__ __align__(128) uint8_t sm[];
   __shared__ __align__(8) uint64_t bars[1 + 2 * kPStages + 4];
   __shared__ uint32_t tmem_base_sh;
-  __shared__ int s_fail;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int TB = tile_bytes(a.Kp);
-  uint8_t* A0 = sm;                 // two query tiles
-  uint8_t* B0 = sm + 2 * TB;        // kPStages centroid tiles, then the value stage
+  uint8_t* A0 = sm;            // query tiles: hi M0, hi M1, lo M0, lo M1
+  uint8_t* B0 = sm + 4 * TB;   // kPStages centroid tiles
   const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
   const uint32_t a_full = bar0;
   auto b_full = [&](uint32_t s) { return bar0 + 8u * (1 + s); };
@@ -193,7 +241,6 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
   auto mma_done = [&](uint32_t b) { return bar0 + 8u * (1 + 2 * kPStages + b); };
   auto acc_empty = [&](uint32_t b) { return bar0 + 8u * (3 + 2 * kPStages + b); };
   if (tid == 0) {
-    s_fail = 0;
     mbar_init(a_full, 1);
     for (uint32_t s = 0; s < kPStages; ++s) {
       mbar_init(b_full(s), 1);
@@ -217,32 +264,31 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
   const uint32_t tmem = tmem_base_sh;
   const uint32_t a_addr = uint32_t(__cvta_generic_to_shared(A0));
   const uint32_t b_addr = uint32_t(__cvta_generic_to_shared(B0));
-  const int ngt = 2 * a.ntiles;  // tiles of both passes
-  auto fail = [&]() {
-    set_device_error(a.err, kErrTimeout);
-    atomicExch(&s_fail, 1);
-  };
+  const int T = a.ntiles;
+  const int nload = 3 * T;  // centroid tiles loaded: T hi (pass 1), then hi and lo of each tile (pass 2)
   auto acc_col = [&](int m, uint32_t b) { return uint32_t((m * 2 + int(b)) * 128); };
 
   if (warp == 8) {
-    // ---------------- TMA: the CTA's two query tiles, then every centroid tile twice
+    // ---------------- TMA: the CTA's query tiles, then the centroid tiles
     if (lane == 0) {
-      mbar_arrive_expect(a_full, uint32_t(2 * TB));
-      bulk_copy_1d(a_addr, a.qtiles + size_t(blockIdx.x) * 2 * TB, uint32_t(2 * TB), a_full);
-      int gt = 0;
-      for (; gt < ngt; ++gt) {
-        const uint32_t s = uint32_t(gt % kPStages), u = uint32_t(gt / kPStages);
+      mbar_arrive_expect(a_full, uint32_t(4 * TB));
+      bulk_copy_1d(a_addr, a.qtiles + size_t(blockIdx.x) * 4 * TB, uint32_t(4 * TB), a_full);
+      int j = 0;
+      for (; j < nload; ++j) {
+        const uint32_t s = uint32_t(j % kPStages), u = uint32_t(j / kPStages);
         if (u > 0 && !mbar_wait(b_empty(s), (u - 1) & 1)) {
-          fail();
+          set_device_error(a.err, kErrTimeout);
           break;
         }
-        const int t = gt % a.ntiles;
+        const int r = j - T;
+        const int tile = j < T ? j : (r >> 1) + ((r & 1) ? T : 0);
         mbar_arrive_expect(b_full(s), uint32_t(TB));
-        bulk_copy_1d(b_addr + s * uint32_t(TB), a.ctiles + size_t(t) * TB, uint32_t(TB), b_full(s));
+        bulk_copy_1d(b_addr + s * uint32_t(TB), a.ctiles + size_t(tile) * TB, uint32_t(TB), b_full(s));
       }
       // no copy may still be landing when the CTA exits
       mbar_wait(a_full, 0);
-      for (int s = 0; s < kPStages && s < gt; ++s) mbar_wait(b_full(uint32_t(s)), uint32_t((gt - 1 - s) / kPStages) & 1);
+      for (int s = 0; s < kPStages && s < j; ++s)
+        mbar_wait(b_full(uint32_t(s)), uint32_t((j - 1 - s) / kPStages) & 1);
     }
     __syncwarp();
   } else if (warp == 9) {
@@ -250,27 +296,50 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
     if (lane == 0) {
       const uint32_t idesc = f16_idesc(kPRows, kPRows);
       const uint32_t sbo = uint32_t(a.Kp / 8) * 128;
+      const int nks = a.Kp / 16;
       bool ok = mbar_wait(a_full, 0);
-      if (!ok) fail();
-      int gt = 0;
-      for (; ok && gt < ngt; ++gt) {
-        const uint32_t s = uint32_t(gt % kPStages), u = uint32_t(gt / kPStages);
+      int j = 0;
+      // acc(m, b) (+)= A tile `at + m` times the centroid tile in stage s
+      auto mma_tile = [&](int at, uint32_t s, uint32_t b, bool acc) {
+        for (int m = 0; m < 2; ++m)
+          for (int ks = 0; ks < nks; ++ks)
+            umma_f16(tmem + acc_col(m, b), smem_desc(a_addr + uint32_t((at + m) * TB + ks * 256), 128, sbo),
+                     smem_desc(b_addr + s * uint32_t(TB) + uint32_t(ks * 256), 128, sbo), idesc,
+                     (acc || ks > 0) ? 1u : 0u);
+      };
+      // wait for centroid load j; its stage in s
+      auto next_b = [&](uint32_t& s) {
+        s = uint32_t(j % kPStages);
+        const bool r = mbar_wait(b_full(s), uint32_t(j / kPStages) & 1);
+        fence_after_sync();
+        return r;
+      };
+      for (int gt = 0; ok && gt < 2 * T; ++gt) {
         const uint32_t b = uint32_t(gt & 1), ub = uint32_t(gt >> 1);
-        if (!mbar_wait(b_full(s), u & 1) || (ub > 0 && !mbar_wait(acc_empty(b), (ub - 1) & 1))) {
-          fail();
+        uint32_t s = 0;
+        if ((ub > 0 && !mbar_wait(acc_empty(b), (ub - 1) & 1)) || !next_b(s)) {
+          ok = false;
           break;
         }
-        fence_after_sync();
-        for (int m = 0; m < 2; ++m)
-          for (int ks = 0; ks < a.Kp / 16; ++ks)
-            umma_f16(tmem + acc_col(m, b), smem_desc(a_addr + uint32_t(m * TB + ks * 256), 128, sbo),
-                     smem_desc(b_addr + s * uint32_t(TB) + uint32_t(ks * 256), 128, sbo), idesc,
-                     ks > 0 ? 1u : 0u);
+        mma_tile(0, s, b, false);  // <q_hi, c_hi>
+        if (gt >= T) mma_tile(2, s, b, true);  // + <q_lo, c_hi>
         umma_commit(b_empty(s));
+        ++j;
+        if (gt >= T) {
+          if (!next_b(s)) {
+            ok = false;
+            break;
+          }
+          mma_tile(0, s, b, true);  // + <q_hi, c_lo>
+          umma_commit(b_empty(s));
+          ++j;
+        }
         umma_commit(mma_done(b));
       }
-      // no MMA may still be running when TMEM is freed
-      if (gt > 0) mbar_wait(mma_done(uint32_t((gt - 1) & 1)), uint32_t(((gt - 1) >> 1) & 1));
+      if (!ok) set_device_error(a.err, kErrTimeout);
+      // no MMA may still be running when TMEM is freed: the last commit
+      // tracks every MMA issued before it
+      if (j > 0) mbar_wait(b_empty(uint32_t((j - 1) % kPStages)), uint32_t((j - 1) / kPStages) & 1);
     }
     __syncwarp();
   } else {
@@ -280,25 +349,22 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
     const bool valid = q < a.nq;
     const uint32_t lane_base = uint32_t(qd * 32) << 16;
     const int ngroups_chunks = a.ngr * a.mch;  // chunks that form the bound groups
-    float top[8];  // the group's largest chunk maxima, descending
+    float top[JTH];  // the group's largest chunk maxima, descending
 #pragma unroll
-    for (int j = 0; j < 8; ++j) top[j] = -CUDART_INF_F;
+    for (int j = 0; j < JTH; ++j) top[j] = -CUDART_INF_F;
     float bound = CUDART_INF_F, thr = CUDART_INF_F;
     int n = 0, in_group = 0;  // chunks of the current bound group seen
-    // this thread's row of the value stage: value i of a chunk at word i * kPThreads + tid
-    float* stage = reinterpret_cast<float*>(sm + (2 + kPStages) * size_t(TB)) + tid;
-    int32_t* out = a.cand + (valid ? q : 0) * int64_t(a.cap);
-    float* outv = a.cval + (valid ? q : 0) * int64_t(a.cap);
-    for (int gt = 0; gt < ngt; ++gt) {
+    uint64_t* out = a.keys + (valid ? q : 0) * int64_t(a.cap);
+    for (int gt = 0; gt < 2 * T; ++gt) {
       const uint32_t b = uint32_t(gt & 1), ub = uint32_t(gt >> 1);
       if (!mbar_wait(mma_done(b), ub & 1)) {
-        fail();
+        set_device_error(a.err, kErrTimeout);
         break;
       }
       fence_after_sync();
-      const bool pass1 = gt < a.ntiles;
-      const int t = pass1 ? gt : gt - a.ntiles;
-      if (gt == a.ntiles) thr = bound - (valid ? a.delta2[q] : 0.0f);
+      const bool pass1 = gt < T;
+      const int t = pass1 ? gt : gt - T;
+      if (gt == T) thr = bound - (valid ? a.dthr[q] : 0.0f);
       // the tile's 128 columns in one load (a TMEM load issued while the
       // tensor core is busy has a long latency), then release the accumulator
       float vt[kPRows];
@@ -308,52 +374,38 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
       if (lane == 0) mbar_arrive(acc_empty(b));
 #pragma unroll
       for (int c = 0; c < kPRows / 32; ++c) {
-        float v[32];
-#pragma unroll
-        for (int i = 0; i < 32; ++i) v[i] = vt[c * 32 + i];
-        float mx = -CUDART_INF_F;
-#pragma unroll
-        for (int i = 0; i < 32; i += 2) mx = fmax3(mx, v[i], v[i + 1]);
+        const float* v = vt + c * 32;
+        const float mx = max32(v);
         const int gc = t * (kPRows / 32) + c;  // 32-column chunk index
         if (pass1) {
           if (gc < ngroups_chunks) {
             float x = mx;
 #pragma unroll
-            for (int j = 0; j < 8; ++j) {
+            for (int j = 0; j < JTH; ++j) {
               const float hi = fmaxf(top[j], x);
               x = fminf(top[j], x);
               top[j] = hi;
             }
             if (++in_group == a.mch) {
-              // at least jth centroids of this group reach top[jth - 1]
-              float tj = top[0];
+              // at least JTH centroids of this group reach top[JTH - 1]
+              bound = fminf(bound, top[JTH - 1]);
 #pragma unroll
-              for (int j = 1; j < 8; ++j) tj = j == a.jth - 1 ? top[j] : tj;
-              bound = fminf(bound, tj);
-#pragma unroll
-              for (int j = 0; j < 8; ++j) top[j] = -CUDART_INF_F;
+              for (int j = 0; j < JTH; ++j) top[j] = -CUDART_INF_F;
               in_group = 0;
             }
           }
         } else if (mx >= thr && valid) {
-          // append the columns at or above thr, in increasing index order
+          // append the columns at or above thr
           const int col0 = gc * 32;
           uint32_t hit = 0;
 #pragma unroll
           for (int i = 0; i < 32; ++i) hit |= (v[i] >= thr ? 1u : 0u) << i;
           const int nreal = max(0, min(32, a.nlist - col0));  // columns beyond nlist are padding
           hit &= nreal == 32 ? ~0u : ((1u << nreal) - 1u);
-          if (hit) {
-#pragma unroll
-            for (int i = 0; i < 32; ++i) stage[i * kPThreads] = v[i];
-          }
           while (hit) {
             const int i = __ffs(hit) - 1;
             hit &= hit - 1;
-            if (n < a.cap) {
-              out[n] = col0 + i;
-              outv[n] = stage[i * kPThreads];
-            }
+            if (n < a.cap) out[n] = list_key(pick32(v, i), col0 + i);
             ++n;
           }
         }
@@ -368,8 +420,86 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
   }
 }
 
+// Sort the warp's n (a power of two, <= 256) keys in shared memory into
+// descending order.
+__device__ __forceinline__ void warp_sort_desc(uint64_t* key, int n) {
+  const int lane = threadIdx.x & 31;
+  for (int size = 2; size <= n; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = lane; i < (n >> 1); i += 32) {
+        const int lo = 2 * i - (i & (stride - 1));
+        const int hi = lo + stride;
+        const bool desc = (lo & size) == 0;
+        const uint64_t klo = key[lo], khi = key[hi];
+        if (desc ? khi > klo : klo > khi) {
+          key[lo] = khi;
+          key[hi] = klo;
+        }
+      }
+      __syncwarp();
+    }
+  }
+}
+
+// Top nprobe of each query's list by its unique keys: the nprobe-th largest
+// key T by a bit search (stopping once exactly nprobe keys are >= T), the
+// keys >= T sorted.  A list that overflowed (or, defensively, holds fewer
+// than nprobe entries) is queued for probe_exact_kernel.  One warp per query.
+constexpr int kSelWarpsPerBlock = 4;
+__global__ void __launch_bounds__(kSelWarpsPerBlock * 32) probe_select_kernel(
+    int64_t nq, const uint64_t* __restrict__ keys, const int* __restrict__ cnt, int cap, int k,
+    const float* __restrict__ qinv, int* __restrict__ nexact, int32_t* __restrict__ exact_q,
+    int32_t* __restrict__ out_probes, float* __restrict__ out_cs) {
+  __shared__ uint64_t ss[kSelWarpsPerBlock][256];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const unsigned lt = (1u << lane) - 1u;
+  const int64_t nw = int64_t(gridDim.x) * kSelWarpsPerBlock;
+  int p2 = 1;
+  while (p2 < k) p2 <<= 1;
+  for (int64_t q = int64_t(blockIdx.x) * kSelWarpsPerBlock + w; q < nq; q += nw) {
+    const int n = cnt[q];
+    if (n > cap || n < k) {
+      if (lane == 0) exact_q[atomicAdd(nexact, 1)] = int32_t(q);
+      continue;
+    }
+    const uint64_t* lk = keys + q * int64_t(cap);
+    uint64_t T = 0;
+    int cT = n;  // keys >= T
+    for (int bit = 63; bit >= 0 && cT > k; --bit) {
+      const uint64_t t = T | (uint64_t(1) << bit);
+      int c0 = 0;
+      for (int i = lane; i < n; i += 32) c0 += __ldg(lk + i) >= t ? 1 : 0;
+      const int c = int(__reduce_add_sync(kFull, uint32_t(c0)));
+      if (c >= k) {
+        T = t;
+        cT = c;
+      }
+    }
+    // exactly k keys are >= T
+    int m = 0;
+    for (int base = 0; base < n; base += 32) {
+      const int i = base + lane;
+      const uint64_t key = i < n ? __ldg(lk + i) : 0;
+      const bool keep = i < n && key >= T;
+      const unsigned bal = __ballot_sync(kFull, keep);
+      if (keep) ss[w][m + __popc(bal & lt)] = key;
+      m += __popc(bal);
+    }
+    for (int i = k + lane; i < p2; i += 32) ss[w][i] = 0;
+    __syncwarp();
+    warp_sort_desc(ss[w], p2);
+    const float inv = qinv[q];
+    for (int i = lane; i < k; i += 32) {
+      const uint64_t key = ss[w][i];
+      out_probes[q * k + i] = int32_t(~uint32_t(key));
+      out_cs[q * k + i] = float_from_order_key(uint32_t(key >> 32)) * inv;
+    }
+    __syncwarp();
+  }
+}
+
 // Centroids again as fp32 rows of Kp floats (zero padded), so every row is
-// 16-byte aligned for the exact rescoring below.
+// 16-byte aligned for the exact scoring below.
 __global__ void centroid_rows_kernel(const float* __restrict__ C, int nlist, int D, int Kp,
                                      float* __restrict__ out) {
   const int64_t total = int64_t(nlist) * Kp;
@@ -380,83 +510,48 @@ __global__ void centroid_rows_kernel(const float* __restrict__ C, int nlist, int
   }
 }
 
-// Exact top-nprobe of every query from its list: fp32 <q, c> of the listed
-// centroids (every centroid when the list overflowed), the nprobe-th largest
-// order key T bit by bit, the centroids above T plus the lowest-index ones at
-// T, sorted by (score desc, p asc).  One warp per query; the warp scores
-// eight candidates per step (four groups of eight lanes, two candidates each,
-// a lane holding Kp / 8 dims).  Keys of a list live in shared memory; an
-// overflowed list uses the warp's global scratch row of nlist keys.
-constexpr int kFinWarpsPerBlock = 4;
-constexpr int kFinCap = 1024;
-__global__ void __launch_bounds__(kFinWarpsPerBlock * 32) probe_finish_kernel(
-    const float* __restrict__ Q, int64_t nq, int D, const float* __restrict__ Cp, int Kp, int nlist,
-    const int32_t* __restrict__ cand, const float* __restrict__ cval, const float* __restrict__ delta2,
-    const int* __restrict__ cnt, int cap, int k, uint32_t* __restrict__ scratch,
+// Exact top-nprobe of the queued queries: fp32 <q, c> of every centroid, the
+// nprobe-th largest order key T bit by bit, the centroids above T plus the
+// lowest-index ones at T, sorted by (score desc, p asc).  One warp per
+// query; the warp scores eight centroids per step (four groups of eight
+// lanes, two centroids each, a lane holding Kp / 8 dims).  Keys live in the
+// warp's global scratch row of nlist keys.
+constexpr int kExactWarpsPerBlock = 4;
+__global__ void __launch_bounds__(kExactWarpsPerBlock * 32) probe_exact_kernel(
+    const float* __restrict__ Q, int D, const float* __restrict__ Cp, int Kp, int nlist,
+    const int* __restrict__ nexact, const int32_t* __restrict__ exact_q, int k, uint32_t* __restrict__ scratch,
     int32_t* __restrict__ out_probes, float* __restrict__ out_cs) {
-  __shared__ uint32_t skeys[kFinWarpsPerBlock][kFinCap];
-  __shared__ int32_t sids[kFinWarpsPerBlock][kFinCap];
-  __shared__ uint32_t sk[kFinWarpsPerBlock][256];
-  __shared__ int32_t si[kFinWarpsPerBlock][256];
+  __shared__ uint64_t ss[kExactWarpsPerBlock][256];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int grp = lane >> 3, sub = lane & 7;
-  const int64_t gw = int64_t(blockIdx.x) * kFinWarpsPerBlock + w;
-  const int64_t nw = int64_t(gridDim.x) * kFinWarpsPerBlock;
+  const unsigned lt = (1u << lane) - 1u;
+  const int64_t gw = int64_t(blockIdx.x) * kExactWarpsPerBlock + w;
+  const int64_t nw = int64_t(gridDim.x) * kExactWarpsPerBlock;
   const int nf = Kp / 4;  // float4 of a row; lane sub takes f = sub + 8 j (Kp <= 128)
-  for (int64_t q = gw; q < nq; q += nw) {
+  uint32_t* keys = scratch + gw * int64_t(nlist);
+  const int nx = *nexact;
+  int p2 = 1;
+  while (p2 < k) p2 <<= 1;
+  for (int64_t e = gw; e < nx; e += nw) {
+    const int64_t q = exact_q[e];
     float4 qv[4];
 #pragma unroll
     for (int j = 0; j < 4; ++j) {
-      float e[4];
+      float v[4];
 #pragma unroll
       for (int c = 0; c < 4; ++c) {
         const int d = (sub + 8 * j) * 4 + c;
-        e[c] = (sub + 8 * j < nf && d < D) ? Q[q * D + d] : 0.0f;
+        v[c] = (sub + 8 * j < nf && d < D) ? Q[q * D + d] : 0.0f;
       }
-      qv[j] = make_float4(e[0], e[1], e[2], e[3]);
+      qv[j] = make_float4(v[0], v[1], v[2], v[3]);
     }
-    const int nc = cnt[q];
-    const bool all = nc > cap;
-    const int32_t* cl = cand + q * int64_t(cap);
-    uint32_t* keys = all ? scratch + gw * int64_t(nlist) : skeys[w];
-    int n = all ? nlist : nc;
-    if (!all) {
-      // Keep only the listed centroids whose a is within 2 delta of the k-th
-      // largest a (A_k): the k centroids at or above A_k score at least
-      // A_k - delta, so no centroid below A_k - 2 delta is in the top k.
-      const float* cv = cval + q * int64_t(cap);
-      for (int i = lane; i < n; i += 32) keys[i] = float_order_key(cv[i]);
-      __syncwarp();
-      uint32_t Ak = 0u;
-      for (int bit = 31; bit >= 0; --bit) {
-        const uint32_t t = Ak | (1u << bit);
-        int c0 = 0;
-        for (int i = lane; i < n; i += 32) c0 += keys[i] >= t ? 1 : 0;
-        if (int(__reduce_add_sync(kFull, uint32_t(c0))) >= k) Ak = t;
-      }
-      const uint32_t lim = float_order_key(float_from_order_key(Ak) - delta2[q]);
-      const unsigned lt = (1u << lane) - 1u;
-      int m = 0;
-      for (int base = 0; base < n; base += 32) {
-        const int i = base + lane;
-        const bool keep = i < n && keys[i] >= lim;
-        const unsigned bal = __ballot_sync(kFull, keep);
-        const int id = keep ? cl[i] : 0;
-        __syncwarp();
-        if (keep) sids[w][m + __popc(bal & lt)] = id;
-        m += __popc(bal);
-      }
-      __syncwarp();
-      cl = sids[w];
-      n = m;
-    }
-    for (int i0 = 0; i0 < n; i0 += 8) {
+    for (int i0 = 0; i0 < nlist; i0 += 8) {
       float acc[2];
       int idx[2];
 #pragma unroll
       for (int u = 0; u < 2; ++u) {
         idx[u] = i0 + 4 * u + grp;
-        const int p = idx[u] < n ? (all ? idx[u] : cl[idx[u]]) : 0;
+        const int p = idx[u] < nlist ? idx[u] : 0;
         const float4* c4 = reinterpret_cast<const float4*>(Cp + int64_t(p) * Kp);
         float s = 0.0f;
 #pragma unroll
@@ -475,7 +570,7 @@ __global__ void __launch_bounds__(kFinWarpsPerBlock * 32) probe_finish_kernel(
       for (int u = 0; u < 2; ++u) {
 #pragma unroll
         for (int o = 4; o; o >>= 1) acc[u] += __shfl_xor_sync(kFull, acc[u], o);
-        if (sub == 0 && idx[u] < n) keys[idx[u]] = float_order_key(acc[u]);
+        if (sub == 0 && idx[u] < nlist) keys[idx[u]] = float_order_key(acc[u]);
       }
     }
     __syncwarp();
@@ -484,66 +579,35 @@ __global__ void __launch_bounds__(kFinWarpsPerBlock * 32) probe_finish_kernel(
     for (int bit = 31; bit >= 0; --bit) {
       const uint32_t t = T | (1u << bit);
       int c0 = 0;
-      for (int i = lane; i < n; i += 32) c0 += keys[i] >= t ? 1 : 0;
+      for (int i = lane; i < nlist; i += 32) c0 += keys[i] >= t ? 1 : 0;
       if (int(__reduce_add_sync(kFull, uint32_t(c0))) >= k) T = t;
     }
     // keys above T (fewer than k), then the lowest-index keys equal to T
-    const unsigned lt = (1u << lane) - 1u;
     int ngt = 0, neq = 0, ngt_tot = 0;
-    for (int base = 0; base < n; base += 32) {
+    for (int base = 0; base < nlist; base += 32) {
       const int i = base + lane;
-      ngt_tot += __popc(__ballot_sync(kFull, i < n && keys[i] > T));
+      ngt_tot += __popc(__ballot_sync(kFull, i < nlist && keys[i] > T));
     }
-    for (int base = 0; base < n; base += 32) {
+    for (int base = 0; base < nlist; base += 32) {
       const int i = base + lane;
-      const uint32_t key = i < n ? keys[i] : 0u;
-      const bool gtr = i < n && key > T, eq = i < n && key == T;
+      const uint32_t key = i < nlist ? keys[i] : 0u;
+      const bool gtr = i < nlist && key > T, eq = i < nlist && key == T;
       const unsigned bg = __ballot_sync(kFull, gtr), be = __ballot_sync(kFull, eq);
-      const int p = i < n ? (all ? i : cl[i]) : 0;
-      if (gtr) {
-        const int at = ngt + __popc(bg & lt);
-        sk[w][at] = key;
-        si[w][at] = p;
-      }
+      if (gtr) ss[w][ngt + __popc(bg & lt)] = (uint64_t(key) << 32) | uint64_t(~uint32_t(i));
       if (eq) {
         const int at = ngt_tot + neq + __popc(be & lt);
-        if (at < k) {
-          sk[w][at] = key;
-          si[w][at] = p;
-        }
+        if (at < k) ss[w][at] = (uint64_t(key) << 32) | uint64_t(~uint32_t(i));
       }
       ngt += __popc(bg);
       neq += __popc(be);
     }
-    int p2 = 1;
-    while (p2 < k) p2 <<= 1;
-    for (int i = k + lane; i < p2; i += 32) {
-      sk[w][i] = 0u;
-      si[w][i] = INT_MAX;
-    }
+    for (int i = k + lane; i < p2; i += 32) ss[w][i] = 0;
     __syncwarp();
-    for (int size = 2; size <= p2; size <<= 1) {
-      for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        for (int i = lane; i < (p2 >> 1); i += 32) {
-          const int lo = 2 * i - (i & (stride - 1));
-          const int hi = lo + stride;
-          const bool asc = (lo & size) == 0;
-          const uint32_t klo = sk[w][lo], khi = sk[w][hi];
-          const int32_t ilo = si[w][lo], ihi = si[w][hi];
-          const bool swap = asc ? better(khi, ihi, klo, ilo) : better(klo, ilo, khi, ihi);
-          if (swap) {
-            sk[w][lo] = khi;
-            sk[w][hi] = klo;
-            si[w][lo] = ihi;
-            si[w][hi] = ilo;
-          }
-        }
-        __syncwarp();
-      }
-    }
+    warp_sort_desc(ss[w], p2);
     for (int i = lane; i < k; i += 32) {
-      out_probes[q * k + i] = si[w][i];
-      out_cs[q * k + i] = float_from_order_key(sk[w][i]);
+      const uint64_t key = ss[w][i];
+      out_probes[q * k + i] = int32_t(~uint32_t(key));
+      out_cs[q * k + i] = float_from_order_key(uint32_t(key >> 32));
     }
     __syncwarp();
   }
@@ -559,13 +623,13 @@ cudaError_t probe_prepare(rslm_index* ix, cudaStream_t s) {
   const int Kp = (ix->D + 15) / 16 * 16;
   if (Kp > 128) return cudaSuccess;  // the fused probe keeps whole rows in one K chunk
   const int ntiles = (ix->nlist + kPRows - 1) / kPRows;
-  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&ix->ctiles), size_t(ntiles) * tile_bytes(Kp));
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&ix->ctiles), size_t(2) * ntiles * tile_bytes(Kp));
   if (e != cudaSuccess) return e;
   e = cudaMalloc(reinterpret_cast<void**>(&ix->cmeta), 4 * sizeof(float));
   if (e != cudaSuccess) return e;
   e = cudaMalloc(reinterpret_cast<void**>(&ix->crows), size_t(ix->nlist) * Kp * sizeof(float));
   if (e != cudaSuccess) return e;
-  ix->device_bytes += int64_t(ntiles) * tile_bytes(Kp) + 16 + int64_t(ix->nlist) * Kp * 4;
+  ix->device_bytes += int64_t(2) * ntiles * tile_bytes(Kp) + 16 + int64_t(ix->nlist) * Kp * 4;
   centroid_rows_kernel<<<152 * 4, 256, 0, s>>>(ix->centroids, ix->nlist, ix->D, Kp, ix->crows);
   centroid_stats_kernel<<<1, 1024, 0, s>>>(ix->centroids, ix->nlist, ix->D, ix->cmeta);
   centroid_tiles_kernel<<<152 * 4, 256, 0, s>>>(ix->centroids, ix->nlist, ix->D, Kp, ix->cmeta, ix->ctiles);
@@ -579,32 +643,36 @@ cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64
   const int ntiles = (ix->nlist + kPRows - 1) / kPRows;
   const int64_t nblk = (nq + kPQ - 1) / kPQ;
   const int64_t nqp = nblk * kPQ;  // queries padded to whole CTAs
-  const int cap = kFinCap;
+  const int cap = kListCap;
   int sms = 152, dev = 0;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
-  const int fin_blocks = sms * 8;
-  const int64_t scratch_row = ix->nlist;
+  const int sel_blocks = sms * 8, exact_blocks = sms * 2;
   size_t bytes = 0;
   auto take = [&](size_t n) {
     size_t at = bytes;
     bytes += (n + 255) / 256 * 256;
     return at;
   };
-  const size_t o_qt = take(size_t(nblk) * 2 * tile_bytes(Kp)), o_d = take(size_t(nq) * 4),
-               o_cand = take(size_t(nq) * cap * 4), o_cval = take(size_t(nq) * cap * 4),
-               o_cnt = take(size_t(nq) * 4),
-               o_scr = take(size_t(fin_blocks) * kFinWarpsPerBlock * scratch_row * 4);
+  const size_t o_qt = take(size_t(nblk) * 4 * tile_bytes(Kp)), o_d = take(size_t(nq) * 4),
+               o_inv = take(size_t(nq) * 4), o_keys = take(size_t(nq) * cap * 8), o_cnt = take(size_t(nq) * 4),
+               o_nx = take(4), o_xq = take(size_t(nq) * 4),
+               o_scr = take(size_t(exact_blocks) * kExactWarpsPerBlock * ix->nlist * 4);
   uint8_t* ws = nullptr;
   cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, s);
   if (e != cudaSuccess) return e;
-  query_tiles_kernel<<<unsigned((nqp + 7) / 8 < 152 * 64 ? (nqp + 7) / 8 : 152 * 64), 256, 0, s>>>(
-      queries, nq, nqp, ix->D, Kp, ix->cmeta, ws + o_qt, reinterpret_cast<float*>(ws + o_d));
-  e = cudaGetLastError();
+  int* nexact = reinterpret_cast<int*>(ws + o_nx);
+  e = cudaMemsetAsync(nexact, 0, sizeof(int), s);
+  if (e == cudaSuccess) {
+    query_tiles_kernel<<<unsigned((nqp + 7) / 8 < 152 * 64 ? (nqp + 7) / 8 : 152 * 64), 256, 0, s>>>(
+        queries, nq, nqp, ix->D, Kp, ix->cmeta, ws + o_qt, reinterpret_cast<float*>(ws + o_d),
+        reinterpret_cast<float*>(ws + o_inv));
+    e = cudaGetLastError();
+  }
   if (e == cudaSuccess) {
     ProbeArgs a;
     a.qtiles = ws + o_qt;
     a.ctiles = ix->ctiles;
-    a.delta2 = reinterpret_cast<const float*>(ws + o_d);
+    a.dthr = reinterpret_cast<const float*>(ws + o_d);
     a.nq = nq;
     a.nlist = ix->nlist;
     a.Kp = Kp;
@@ -613,35 +681,40 @@ cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64
     // the largest jth in {8, 4, 2, 1} whose ceil(nprobe / jth) groups of at
     // least jth chunks fit in the nlist / 32 whole chunks
     const int nch = ix->nlist / 32;
+    int jth = 1;
     for (int j = 8; j >= 1; j >>= 1) {
       const int ng = (nprobe + j - 1) / j;
       if (nch / ng >= j || j == 1) {
-        a.jth = j;
+        jth = j;
         a.ngr = ng;
         a.mch = nch / ng;
         break;
       }
     }
     a.cap = cap;
-    a.cand = reinterpret_cast<int32_t*>(ws + o_cand);
-    a.cval = reinterpret_cast<float*>(ws + o_cval);
+    a.keys = reinterpret_cast<uint64_t*>(ws + o_keys);
     a.cnt = reinterpret_cast<int*>(ws + o_cnt);
     a.err = ix->d_err;
     // at least 116 KB, so one CTA per SM: each CTA holds all 512 TMEM columns
-    const size_t smem = std::max(size_t(2 + kPStages) * tile_bytes(Kp) + size_t(32) * kPThreads * 4,
-                                 size_t(116) * 1024);
-    e = cudaFuncSetAttribute(probe_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+    const size_t smem = std::max(size_t(4 + kPStages) * tile_bytes(Kp), size_t(116) * 1024);
+    auto kern = jth == 8 ? probe_kernel<8> : jth == 4 ? probe_kernel<4> : jth == 2 ? probe_kernel<2> : probe_kernel<1>;
+    e = cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     if (e == cudaSuccess) {
-      probe_kernel<<<unsigned(nblk), kPThreads, smem, s>>>(a);
+      kern<<<unsigned(nblk), kPThreads, smem, s>>>(a);
       e = cudaGetLastError();
     }
   }
   if (e == cudaSuccess) {
-    probe_finish_kernel<<<unsigned(fin_blocks), kFinWarpsPerBlock * 32, 0, s>>>(
-        queries, nq, ix->D, ix->crows, Kp, ix->nlist, reinterpret_cast<const int32_t*>(ws + o_cand),
-        reinterpret_cast<const float*>(ws + o_cval), reinterpret_cast<const float*>(ws + o_d),
-        reinterpret_cast<const int*>(ws + o_cnt), cap, nprobe, reinterpret_cast<uint32_t*>(ws + o_scr),
+    probe_select_kernel<<<unsigned(sel_blocks), kSelWarpsPerBlock * 32, 0, s>>>(
+        nq, reinterpret_cast<const uint64_t*>(ws + o_keys), reinterpret_cast<const int*>(ws + o_cnt), cap,
+        nprobe, reinterpret_cast<const float*>(ws + o_inv), nexact, reinterpret_cast<int32_t*>(ws + o_xq),
         out_probes, out_cs);
+    e = cudaGetLastError();
+  }
+  if (e == cudaSuccess) {
+    probe_exact_kernel<<<unsigned(exact_blocks), kExactWarpsPerBlock * 32, 0, s>>>(
+        queries, ix->D, ix->crows, Kp, ix->nlist, nexact, reinterpret_cast<const int32_t*>(ws + o_xq), nprobe,
+        reinterpret_cast<uint32_t*>(ws + o_scr), out_probes, out_cs);
     e = cudaGetLastError();
   }
   cudaError_t f = cudaFreeAsync(ws, s);
