@@ -45,10 +45,11 @@ namespace {
 constexpr int kPRows = 128;       // rows (queries or centroids) per operand tile
 constexpr int kPQ = 2 * kPRows;   // queries per CTA (two M blocks)
 constexpr int kPStages = 3;       // centroid tiles in flight
-constexpr int kPThreads = 10 * 32;  // warps 0-7 epilogue, 8 TMA, 9 MMA
-constexpr int kPEpiWarps = 8;
+constexpr int kPEpiWarps = 16;    // (M block, column half, TMEM lane quarter)
+constexpr int kPThreads = (kPEpiWarps + 2) * 32;  // then one TMA and one MMA warp
+constexpr int kPTmaWarp = kPEpiWarps, kPMmaWarp = kPEpiWarps + 1;
 constexpr uint32_t kPCols = 512;  // TMEM: (M block, buffer) accumulators of 128 columns
-constexpr int kListCap = 1024;    // listed centroids per query before the exact fallback
+constexpr int kListCapMin = 1024;  // listed centroids per query (at least 8 nprobe) before the exact fallback
 
 __host__ __device__ constexpr int tile_bytes(int Kp) { return kPRows * Kp * 2; }
 
@@ -206,6 +207,34 @@ __device__ __forceinline__ float pick32(const float* v, int i) {
   return (i & 16) ? d1 : d0;
 }
 
+// Bit b of a chunk's hit mask stands for column 4 (b mod 8) + b / 8.
+__host__ __device__ constexpr int mask_bit_col(int b) { return 4 * (b & 7) + (b >> 3); }
+
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+  uint32_t d;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(d) : "r"(a), "r"(b), "r"(sel));
+  return d;
+}
+
+// Mask of the columns of a 32-column chunk below thr, in mask-bit order: the
+// signs of v - thr (paired fp32 arithmetic; exact zero for v == thr), their
+// sign bytes gathered four at a time by byte permutes (selector nibbles with
+// bit 3 set replicate a byte's sign), one bit of each kept.
+__device__ __forceinline__ uint32_t miss_mask(const float* v, float thr) {
+  const uint64_t one2 = f2pack(1.0f, 1.0f), nthr2 = f2pack(-thr, -thr);
+  uint32_t miss = 0;
+#pragma unroll
+  for (int g = 0; g < 8; ++g) {
+    float d[4];
+    f2unpack(fma2(f2pack(v[4 * g], v[4 * g + 1]), one2, nthr2), d[0], d[1]);
+    f2unpack(fma2(f2pack(v[4 * g + 2], v[4 * g + 3]), one2, nthr2), d[2], d[3]);
+    const uint32_t s01 = prmt(__float_as_uint(d[0]), __float_as_uint(d[1]), 0x00fbu);
+    const uint32_t s23 = prmt(__float_as_uint(d[2]), __float_as_uint(d[3]), 0x00fbu);
+    miss |= prmt(s01, s23, 0x5410u) & (0x01010101u << g);  // column 4g + k at bit 8k + g
+  }
+  return miss;
+}
+
 // List entry: larger key = better (a3 desc, then p asc); keys are unique.
 __device__ __forceinline__ uint64_t list_key(float a, int p) {
   return (uint64_t(float_order_key(a)) << 32) | uint64_t(~uint32_t(p));
@@ -216,12 +245,15 @@ struct ProbeArgs {
   const uint8_t* ctiles;
   const float* dthr;
   int64_t nq;
-  // bound groups: ngr groups of mch consecutive 32-column chunks; a group
-  // contributes its JTH-largest chunk maximum (JTH * ngr >= nprobe)
-  int nlist, Kp, ntiles, nprobe, mch, ngr;
+  // bound groups: the whole 32-column chunks (index < nlist / 32) of column
+  // half h (chunks 2h and 2h + 1 of every tile), in order, form ngr[h]
+  // groups of mch[h] chunks; a group contributes its JTH-largest chunk
+  // maximum, and JTH (ngr[0] + ngr[1]) >= nprobe
+  int nlist, Kp, ntiles, nprobe;
+  int mch[2], ngr[2];
   int cap;
-  uint64_t* keys;  // [nq * cap] list_key of the listed centroids
-  int* cnt;        // [nq]
+  uint64_t* keys;  // [nq][cap]: list_key of the centroids listed by half 0, then (at cap / 2) half 1
+  int* cnt;        // [nq][2]: entries listed by each half (more than cap / 2: overflow)
   int* err;
 };
 
@@ -230,6 +262,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
   extern __shared__ __align__(128) uint8_t sm[];
   __shared__ __align__(8) uint64_t bars[1 + 2 * kPStages + 4];
   __shared__ uint32_t tmem_base_sh;
+  __shared__ float half_bound[2][kPQ];  // pass-1 bound of each query from each column half
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int TB = tile_bytes(a.Kp);
   uint8_t* A0 = sm;            // query tiles: hi M0, hi M1, lo M0, lo M1
@@ -268,7 +301,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
   const int nload = 3 * T;  // centroid tiles loaded: T hi (pass 1), then hi and lo of each tile (pass 2)
   auto acc_col = [&](int m, uint32_t b) { return uint32_t((m * 2 + int(b)) * 128); };
 
-  if (warp == 8) {
+  if (warp == kPTmaWarp) {
     // ---------------- TMA: the CTA's query tiles, then the centroid tiles
     if (lane == 0) {
       mbar_arrive_expect(a_full, uint32_t(4 * TB));
@@ -291,7 +324,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
         mbar_wait(b_full(uint32_t(s)), uint32_t((j - 1 - s) / kPStages) & 1);
     }
     __syncwarp();
-  } else if (warp == 9) {
+  } else if (warp == kPMmaWarp) {
     // ---------------- MMA issue: both M blocks against each centroid tile
     if (lane == 0) {
       const uint32_t idesc = f16_idesc(kPRows, kPRows);
@@ -343,50 +376,61 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
     }
     __syncwarp();
   } else {
-    // ---------------- epilogue: thread = one query row of M block m
-    const int m = warp >> 2, qd = warp & 3;
-    const int64_t q = int64_t(blockIdx.x) * kPQ + m * kPRows + qd * 32 + lane;
+    // ---------------- epilogue: thread = one query row of M block m, 64
+    // columns (column half h) of every tile
+    const int m = warp >> 3, h = (warp >> 2) & 1, qd = warp & 3;
+    const int row = m * kPRows + qd * 32 + lane;  // query within the CTA
+    const int64_t q = int64_t(blockIdx.x) * kPQ + row;
     const bool valid = q < a.nq;
     const uint32_t lane_base = uint32_t(qd * 32) << 16;
-    const int ngroups_chunks = a.ngr * a.mch;  // chunks that form the bound groups
+    const int nwhole = a.nlist / 32;                 // whole chunks
+    const int ngroups_chunks = a.ngr[h] * a.mch[h];  // this half's chunks that form its groups
+    const int mch = a.mch[h];
     float top[JTH];  // the group's largest chunk maxima, descending
 #pragma unroll
     for (int j = 0; j < JTH; ++j) top[j] = -CUDART_INF_F;
     float bound = CUDART_INF_F, thr = CUDART_INF_F;
     int n = 0, in_group = 0;  // chunks of the current bound group seen
-    uint64_t* out = a.keys + (valid ? q : 0) * int64_t(a.cap);
+    bool dead = false;        // a wait timed out: skip the work, keep the barrier
+    uint64_t* out = a.keys + (valid ? q : 0) * int64_t(a.cap) + h * (a.cap / 2);  // this half's segment
     for (int gt = 0; gt < 2 * T; ++gt) {
+      if (gt == T) {
+        // B1 of the query: the smaller of the two halves' bounds
+        half_bound[h][row] = bound;
+        asm volatile("bar.sync 1, %0;" ::"n"(kPEpiWarps * 32) : "memory");
+        bound = fminf(half_bound[0][row], half_bound[1][row]);
+        thr = bound - (valid ? a.dthr[q] : 0.0f);
+      }
+      if (dead) continue;
       const uint32_t b = uint32_t(gt & 1), ub = uint32_t(gt >> 1);
       if (!mbar_wait(mma_done(b), ub & 1)) {
         set_device_error(a.err, kErrTimeout);
-        break;
+        dead = true;
+        continue;
       }
       fence_after_sync();
       const bool pass1 = gt < T;
       const int t = pass1 ? gt : gt - T;
-      if (gt == T) thr = bound - (valid ? a.dthr[q] : 0.0f);
-      // the tile's 128 columns in one load (a TMEM load issued while the
-      // tensor core is busy has a long latency), then release the accumulator
-      float vt[kPRows];
-      tmem_ld128(tmem + lane_base + acc_col(m, b), vt);
+      // this half's 64 columns in one load, then release the accumulator
+      float vt[64];
+      tmem_ld64(tmem + lane_base + acc_col(m, b) + uint32_t(h * 64), vt);
       fence_before_sync();
       __syncwarp();
       if (lane == 0) mbar_arrive(acc_empty(b));
 #pragma unroll
-      for (int c = 0; c < kPRows / 32; ++c) {
+      for (int c = 0; c < 2; ++c) {
         const float* v = vt + c * 32;
-        const float mx = max32(v);
-        const int gc = t * (kPRows / 32) + c;  // 32-column chunk index
+        const int gc = t * (kPRows / 32) + 2 * h + c;  // 32-column chunk index
         if (pass1) {
-          if (gc < ngroups_chunks) {
-            float x = mx;
+          if (gc < nwhole && 2 * t + c < ngroups_chunks) {
+            float x = max32(v);
 #pragma unroll
             for (int j = 0; j < JTH; ++j) {
               const float hi = fmaxf(top[j], x);
               x = fminf(top[j], x);
               top[j] = hi;
             }
-            if (++in_group == a.mch) {
+            if (++in_group == mch) {
               // at least JTH centroids of this group reach top[JTH - 1]
               bound = fminf(bound, top[JTH - 1]);
 #pragma unroll
@@ -394,24 +438,26 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
               in_group = 0;
             }
           }
-        } else if (mx >= thr && valid) {
+        } else if (valid) {
           // append the columns at or above thr
           const int col0 = gc * 32;
-          uint32_t hit = 0;
+          uint32_t hit = ~miss_mask(v, thr);
+          float vp[32];  // the chunk in mask-bit order
 #pragma unroll
-          for (int i = 0; i < 32; ++i) hit |= (v[i] >= thr ? 1u : 0u) << i;
-          const int nreal = max(0, min(32, a.nlist - col0));  // columns beyond nlist are padding
-          hit &= nreal == 32 ? ~0u : ((1u << nreal) - 1u);
+          for (int b = 0; b < 32; ++b) vp[b] = v[mask_bit_col(b)];
           while (hit) {
-            const int i = __ffs(hit) - 1;
+            const int b = __ffs(hit) - 1;
             hit &= hit - 1;
-            if (n < a.cap) out[n] = list_key(pick32(v, i), col0 + i);
-            ++n;
+            const int col = col0 + mask_bit_col(b);
+            if (col < a.nlist) {  // columns beyond nlist are padding
+              if (n < a.cap / 2) out[n] = list_key(pick32(vp, b), col);
+              ++n;
+            }
           }
         }
       }
     }
-    if (valid) a.cnt[q] = n;
+    if (valid) a.cnt[2 * q + h] = n;
   }
   __syncthreads();
   if (warp == 0) {
@@ -441,10 +487,68 @@ __device__ __forceinline__ void warp_sort_desc(uint64_t* key, int n) {
   }
 }
 
-// Top nprobe of each query's list by its unique keys: the nprobe-th largest
-// key T by a bit search (stopping once exactly nprobe keys are >= T), the
-// keys >= T sorted.  A list that overflowed (or, defensively, holds fewer
-// than nprobe entries) is queued for probe_exact_kernel.  One warp per query.
+// The keys >= the k-th largest of a warp's list, the list held as J keys
+// per lane (element lane + 32 j; 0 beyond the list, smaller than any real
+// key), compacted into out[0, k).  T is found bit by bit, first over the
+// high words below their common prefix, then, only if the k-th largest
+// high word is tied, over the low words; the search stops as soon as
+// exactly k keys are >= T.
+template <int J>
+__device__ __forceinline__ void select_top_regs(const uint64_t (&r)[J], int n, int k, uint64_t* out) {
+  const int lane = threadIdx.x & 31;
+  const unsigned lt = (1u << lane) - 1u;
+  uint32_t hmax = 0u, hmin = ~0u;
+#pragma unroll
+  for (int j = 0; j < J; ++j) {
+    if (lane + 32 * j < n) {
+      const uint32_t h = uint32_t(r[j] >> 32);
+      hmax = max(hmax, h);
+      hmin = min(hmin, h);
+    }
+  }
+  hmax = __reduce_max_sync(kFull, hmax);
+  hmin = __reduce_min_sync(kFull, hmin);
+  const int L = __clz(hmax ^ hmin);  // bits shared by every high word
+  uint32_t Th = L == 0 ? 0u : (hmax & (~0u << (32 - L)));
+  int cT = n;  // keys with high word >= Th
+  for (int bit = 31 - L; bit >= 0 && cT > k; --bit) {
+    const uint32_t t = Th | (1u << bit);
+    int c = 0;
+#pragma unroll
+    for (int j = 0; j < J; ++j) c += uint32_t(r[j] >> 32) >= t ? 1 : 0;
+    c = int(__reduce_add_sync(kFull, uint32_t(c)));
+    if (c >= k) {
+      Th = t;
+      cT = c;
+    }
+  }
+  uint64_t T = uint64_t(Th) << 32;
+  for (int bit = 31; bit >= 0 && cT > k; --bit) {
+    const uint64_t t = T | (uint64_t(1) << bit);
+    int c = 0;
+#pragma unroll
+    for (int j = 0; j < J; ++j) c += r[j] >= t ? 1 : 0;
+    c = int(__reduce_add_sync(kFull, uint32_t(c)));
+    if (c >= k) {
+      T = t;
+      cT = c;
+    }
+  }
+  int m = 0;
+#pragma unroll
+  for (int j = 0; j < J; ++j) {
+    const bool keep = lane + 32 * j < n && r[j] >= T;
+    const unsigned bal = __ballot_sync(kFull, keep);
+    if (keep) out[m + __popc(bal & lt)] = r[j];
+    m += __popc(bal);
+  }
+}
+
+// Top nprobe of each query's list (the two column halves' segments) by its
+// unique keys, sorted.  Lists of up to 256 entries are selected in
+// registers; longer ones by the same bit search over the list in global
+// memory.  A list with an overflowed segment (or, defensively, fewer than
+// nprobe entries) is queued for probe_exact_kernel.  One warp per query.
 constexpr int kSelWarpsPerBlock = 4;
 __global__ void __launch_bounds__(kSelWarpsPerBlock * 32) probe_select_kernel(
     int64_t nq, const uint64_t* __restrict__ keys, const int* __restrict__ cnt, int cap, int k,
@@ -457,33 +561,47 @@ __global__ void __launch_bounds__(kSelWarpsPerBlock * 32) probe_select_kernel(
   int p2 = 1;
   while (p2 < k) p2 <<= 1;
   for (int64_t q = int64_t(blockIdx.x) * kSelWarpsPerBlock + w; q < nq; q += nw) {
-    const int n = cnt[q];
-    if (n > cap || n < k) {
+    const int half = cap / 2, n0 = cnt[2 * q], n1 = cnt[2 * q + 1], n = n0 + n1;
+    if (n0 > half || n1 > half || n < k) {
       if (lane == 0) exact_q[atomicAdd(nexact, 1)] = int32_t(q);
       continue;
     }
+    // entry e of the list: the first n0 from half 0's segment, then half 1's
     const uint64_t* lk = keys + q * int64_t(cap);
-    uint64_t T = 0;
-    int cT = n;  // keys >= T
-    for (int bit = 63; bit >= 0 && cT > k; --bit) {
-      const uint64_t t = T | (uint64_t(1) << bit);
-      int c0 = 0;
-      for (int i = lane; i < n; i += 32) c0 += __ldg(lk + i) >= t ? 1 : 0;
-      const int c = int(__reduce_add_sync(kFull, uint32_t(c0)));
-      if (c >= k) {
-        T = t;
-        cT = c;
+    auto entry = [&](int e) { return __ldg(lk + (e < n0 ? e : half + e - n0)); };
+    if (n <= 128) {
+      uint64_t r[4];
+#pragma unroll
+      for (int j = 0; j < 4; ++j) r[j] = lane + 32 * j < n ? entry(lane + 32 * j) : 0;
+      select_top_regs<4>(r, n, k, ss[w]);
+    } else if (n <= 256) {
+      uint64_t r[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) r[j] = lane + 32 * j < n ? entry(lane + 32 * j) : 0;
+      select_top_regs<8>(r, n, k, ss[w]);
+    } else {
+      uint64_t T = 0;
+      int cT = n;  // keys >= T
+      for (int bit = 63; bit >= 0 && cT > k; --bit) {
+        const uint64_t t = T | (uint64_t(1) << bit);
+        int c0 = 0;
+        for (int i = lane; i < n; i += 32) c0 += entry(i) >= t ? 1 : 0;
+        const int c = int(__reduce_add_sync(kFull, uint32_t(c0)));
+        if (c >= k) {
+          T = t;
+          cT = c;
+        }
       }
-    }
-    // exactly k keys are >= T
-    int m = 0;
-    for (int base = 0; base < n; base += 32) {
-      const int i = base + lane;
-      const uint64_t key = i < n ? __ldg(lk + i) : 0;
-      const bool keep = i < n && key >= T;
-      const unsigned bal = __ballot_sync(kFull, keep);
-      if (keep) ss[w][m + __popc(bal & lt)] = key;
-      m += __popc(bal);
+      // exactly k keys are >= T
+      int m = 0;
+      for (int base = 0; base < n; base += 32) {
+        const int i = base + lane;
+        const uint64_t key = i < n ? entry(i) : 0;
+        const bool keep = i < n && key >= T;
+        const unsigned bal = __ballot_sync(kFull, keep);
+        if (keep) ss[w][m + __popc(bal & lt)] = key;
+        m += __popc(bal);
+      }
     }
     for (int i = k + lane; i < p2; i += 32) ss[w][i] = 0;
     __syncwarp();
@@ -643,7 +761,7 @@ cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64
   const int ntiles = (ix->nlist + kPRows - 1) / kPRows;
   const int64_t nblk = (nq + kPQ - 1) / kPQ;
   const int64_t nqp = nblk * kPQ;  // queries padded to whole CTAs
-  const int cap = kListCap;
+  const int cap = std::max(kListCapMin, 8 * nprobe);
   int sms = 152, dev = 0;
   if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
   const int sel_blocks = sms * 8, exact_blocks = sms * 2;
@@ -654,7 +772,7 @@ cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64
     return at;
   };
   const size_t o_qt = take(size_t(nblk) * 4 * tile_bytes(Kp)), o_d = take(size_t(nq) * 4),
-               o_inv = take(size_t(nq) * 4), o_keys = take(size_t(nq) * cap * 8), o_cnt = take(size_t(nq) * 4),
+               o_inv = take(size_t(nq) * 4), o_keys = take(size_t(nq) * cap * 8), o_cnt = take(size_t(nq) * 8),
                o_nx = take(4), o_xq = take(size_t(nq) * 4),
                o_scr = take(size_t(exact_blocks) * kExactWarpsPerBlock * ix->nlist * 4);
   uint8_t* ws = nullptr;
@@ -678,16 +796,19 @@ cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64
     a.Kp = Kp;
     a.ntiles = ntiles;
     a.nprobe = nprobe;
-    // the largest jth in {8, 4, 2, 1} whose ceil(nprobe / jth) groups of at
-    // least jth chunks fit in the nlist / 32 whole chunks
+    // whole chunks of each column half (chunk g is in half (g mod 4) / 2),
+    // then the largest jth in {8, 4, 2, 1} for which ceil(nprobe / jth)
+    // groups of at least jth chunks fit in the two halves, split evenly
     const int nch = ix->nlist / 32;
+    const int hc[2] = {2 * (nch / 4) + std::min(nch % 4, 2), 2 * (nch / 4) + std::max(nch % 4 - 2, 0)};
     int jth = 1;
     for (int j = 8; j >= 1; j >>= 1) {
-      const int ng = (nprobe + j - 1) / j;
-      if (nch / ng >= j || j == 1) {
+      const int G = (nprobe + j - 1) / j, f0 = hc[0] / j, f1 = hc[1] / j;
+      if (f0 + f1 >= G || j == 1) {
         jth = j;
-        a.ngr = ng;
-        a.mch = nch / ng;
+        a.ngr[0] = std::min(f0, std::max(G - f1, (G + 1) / 2));
+        a.ngr[1] = G - a.ngr[0];
+        for (int h = 0; h < 2; ++h) a.mch[h] = a.ngr[h] > 0 ? hc[h] / a.ngr[h] : 1;
         break;
       }
     }
