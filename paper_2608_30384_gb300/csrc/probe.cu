@@ -46,8 +46,11 @@ constexpr int kPRows = 128;       // rows (queries or centroids) per operand til
 constexpr int kPQ = 2 * kPRows;   // queries per CTA (two M blocks)
 constexpr int kPStages = 3;       // centroid tiles in flight
 constexpr int kPEpiWarps = 16;    // (M block, column half, TMEM lane quarter)
-constexpr int kPThreads = (kPEpiWarps + 2) * 32;  // then one TMA and one MMA warp
-constexpr int kPTmaWarp = kPEpiWarps, kPMmaWarp = kPEpiWarps + 1;
+// then one TMA warp and one MMA-issuing warp per M block: the tensor core
+// queues only about two MMAs, so a lone issuer's barrier waits would leave
+// it idle; two issuers cover each other's waits
+constexpr int kPThreads = (kPEpiWarps + 3) * 32;
+constexpr int kPTmaWarp = kPEpiWarps, kPMmaWarp0 = kPEpiWarps + 1;
 constexpr uint32_t kPCols = 512;  // TMEM: (M block, buffer) accumulators of 128 columns
 constexpr int kListCapMin = 1024;  // listed centroids per query (at least 8 nprobe) before the exact fallback
 
@@ -260,7 +263,7 @@ struct ProbeArgs {
 template <int JTH>
 __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_constant__ ProbeArgs a) {
   extern __shared__ __align__(128) uint8_t sm[];
-  __shared__ __align__(8) uint64_t bars[1 + 2 * kPStages + 4];
+  __shared__ __align__(8) uint64_t bars[1 + 2 * kPStages + 8];
   __shared__ uint32_t tmem_base_sh;
   __shared__ float half_bound[2][kPQ];  // pass-1 bound of each query from each column half
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
@@ -271,18 +274,20 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
   const uint32_t a_full = bar0;
   auto b_full = [&](uint32_t s) { return bar0 + 8u * (1 + s); };
   auto b_empty = [&](uint32_t s) { return bar0 + 8u * (1 + kPStages + s); };
-  auto mma_done = [&](uint32_t b) { return bar0 + 8u * (1 + 2 * kPStages + b); };
-  auto acc_empty = [&](uint32_t b) { return bar0 + 8u * (3 + 2 * kPStages + b); };
+  // accumulator (M block m, buffer b): MMAs done / read by the epilogue
+  auto mma_done = [&](int m, uint32_t b) { return bar0 + 8u * (1 + 2 * kPStages + 2 * m + b); };
+  auto acc_empty = [&](int m, uint32_t b) { return bar0 + 8u * (5 + 2 * kPStages + 2 * m + b); };
   if (tid == 0) {
     mbar_init(a_full, 1);
     for (uint32_t s = 0; s < kPStages; ++s) {
       mbar_init(b_full(s), 1);
-      mbar_init(b_empty(s), 1);
+      mbar_init(b_empty(s), 2);  // one commit per MMA-issuing warp
     }
-    for (uint32_t b = 0; b < 2; ++b) {
-      mbar_init(mma_done(b), 1);
-      mbar_init(acc_empty(b), kPEpiWarps);
-    }
+    for (int m = 0; m < 2; ++m)
+      for (uint32_t b = 0; b < 2; ++b) {
+        mbar_init(mma_done(m, b), 1);
+        mbar_init(acc_empty(m, b), kPEpiWarps / 2);
+      }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
   if (warp == 0) {
@@ -324,21 +329,21 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
         mbar_wait(b_full(uint32_t(s)), uint32_t((j - 1 - s) / kPStages) & 1);
     }
     __syncwarp();
-  } else if (warp == kPMmaWarp) {
-    // ---------------- MMA issue: both M blocks against each centroid tile
+  } else if (warp >= kPMmaWarp0) {
+    // ---------------- MMA issue: M block m against each centroid tile
+    const int m = warp - kPMmaWarp0;
     if (lane == 0) {
       const uint32_t idesc = f16_idesc(kPRows, kPRows);
       const uint32_t sbo = uint32_t(a.Kp / 8) * 128;
       const int nks = a.Kp / 16;
       bool ok = mbar_wait(a_full, 0);
-      int j = 0;
+      int j = 0, last = -1;
       // acc(m, b) (+)= A tile `at + m` times the centroid tile in stage s
       auto mma_tile = [&](int at, uint32_t s, uint32_t b, bool acc) {
-        for (int m = 0; m < 2; ++m)
-          for (int ks = 0; ks < nks; ++ks)
-            umma_f16(tmem + acc_col(m, b), smem_desc(a_addr + uint32_t((at + m) * TB + ks * 256), 128, sbo),
-                     smem_desc(b_addr + s * uint32_t(TB) + uint32_t(ks * 256), 128, sbo), idesc,
-                     (acc || ks > 0) ? 1u : 0u);
+        for (int ks = 0; ks < nks; ++ks)
+          umma_f16(tmem + acc_col(m, b), smem_desc(a_addr + uint32_t((at + m) * TB + ks * 256), 128, sbo),
+                   smem_desc(b_addr + s * uint32_t(TB) + uint32_t(ks * 256), 128, sbo), idesc,
+                   (acc || ks > 0) ? 1u : 0u);
       };
       // wait for centroid load j; its stage in s
       auto next_b = [&](uint32_t& s) {
@@ -350,7 +355,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
       for (int gt = 0; ok && gt < 2 * T; ++gt) {
         const uint32_t b = uint32_t(gt & 1), ub = uint32_t(gt >> 1);
         uint32_t s = 0;
-        if ((ub > 0 && !mbar_wait(acc_empty(b), (ub - 1) & 1)) || !next_b(s)) {
+        if ((ub > 0 && !mbar_wait(acc_empty(m, b), (ub - 1) & 1)) || !next_b(s)) {
           ok = false;
           break;
         }
@@ -367,12 +372,13 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
           umma_commit(b_empty(s));
           ++j;
         }
-        umma_commit(mma_done(b));
+        umma_commit(mma_done(m, b));
+        last = gt;
       }
       if (!ok) set_device_error(a.err, kErrTimeout);
-      // no MMA may still be running when TMEM is freed: the last commit
-      // tracks every MMA issued before it
-      if (j > 0) mbar_wait(b_empty(uint32_t((j - 1) % kPStages)), uint32_t((j - 1) / kPStages) & 1);
+      // no MMA may still be running when TMEM is freed: this warp's last
+      // commit tracks every MMA it issued
+      if (last >= 0) mbar_wait(mma_done(m, uint32_t(last & 1)), uint32_t(last >> 1) & 1);
     }
     __syncwarp();
   } else {
@@ -403,7 +409,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
       }
       if (dead) continue;
       const uint32_t b = uint32_t(gt & 1), ub = uint32_t(gt >> 1);
-      if (!mbar_wait(mma_done(b), ub & 1)) {
+      if (!mbar_wait(mma_done(m, b), ub & 1)) {
         set_device_error(a.err, kErrTimeout);
         dead = true;
         continue;
@@ -416,7 +422,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
       tmem_ld64(tmem + lane_base + acc_col(m, b) + uint32_t(h * 64), vt);
       fence_before_sync();
       __syncwarp();
-      if (lane == 0) mbar_arrive(acc_empty(b));
+      if (lane == 0) mbar_arrive(acc_empty(m, b));
 #pragma unroll
       for (int c = 0; c < 2; ++c) {
         const float* v = vt + c * 32;
