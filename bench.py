@@ -262,10 +262,9 @@ def launches_per_step(w: W.Workload, nq: int, batched: bool) -> int:
         n = math.ceil(nq / qc) * (2 if w.nprobe <= 256 else 1)
     n += 1                   # query rotation
     # batched: two probe-list inversions (count, list scan, item table,
-    # scatter), query split, first-probe pass, threshold (warp kernel + block
-    # fallback), tensor-core scan, finalize (warp kernel + block fallback),
-    # overflow re-scan; else one scan
-    n += 8 + 1 + 1 + 2 + 1 + 2 + 1 if batched else 1
+    # scatter), query split, first-probe pass, threshold, tensor-core scan,
+    # finalize (warp kernel + block fallback), overflow re-scan; else one scan
+    n += 8 + 1 + 1 + 1 + 1 + 2 + 1 if batched else 1
     if w.rescore_bits:
         n += 2               # second rotation + rescore
     return n

@@ -155,62 +155,23 @@ __device__ uint32_t block_kth_key(const float* s, int n, int k, uint32_t* hist, 
   return prefix;
 }
 
-// theta_q = k-th best score of the query's first probed partition (all of its
-// candidates are in the buffer), lowered by a relative margin of 1e-6; -inf
-// when that partition has fewer than k rows.
+// theta_q bounds the query's k-th best score from below: k distinct
+// candidates of its first probed partition (all of whose scores are in the
+// buffer) reach the k-th largest of the maxima of 256 interleaved groups
+// (element i in group i mod 256); lowered by a relative margin of 1e-6;
+// -inf when that partition has fewer than k rows.  One warp per query; the
+// k-th largest group maximum is found bit by bit.
 __device__ __forceinline__ float theta_from(float t) { return t - 1e-6f * fabsf(t) - 1e-30f; }
 
-__global__ void theta_kernel(const float* __restrict__ buf_s, const int* __restrict__ cnt, int cap,
-                             int k, float* __restrict__ theta, const int* __restrict__ only_if) {
-  __shared__ uint32_t hist[256];
-  __shared__ uint32_t sh[2];
-  const int64_t q = blockIdx.x;
-  if (only_if && only_if[q] == 0) return;
-  const int n = min(cnt[q], cap);
-  float t = -CUDART_INF_F;
-  if (n >= k) {
-    const float* s = buf_s + q * cap;
-    if (n == k) {
-      // smallest of the n scores
-      float m = CUDART_INF_F;
-      for (int i = threadIdx.x; i < n; i += blockDim.x) m = fminf(m, s[i]);
-      for (int o = 16; o; o >>= 1) m = fminf(m, __shfl_xor_sync(kFull, m, o));
-      if ((threadIdx.x & 31) == 0) hist[threadIdx.x >> 5] = __float_as_uint(m);
-      __syncthreads();
-      if (threadIdx.x == 0) {
-        for (int w = 0; w < int(blockDim.x >> 5); ++w) m = fminf(m, __uint_as_float(hist[w]));
-        hist[255] = __float_as_uint(m);
-      }
-      __syncthreads();
-      t = __uint_as_float(hist[255]);
-    } else {
-      t = float_from_order_key(block_kth_key(s, n, k, hist, sh));
-    }
-    t = theta_from(t);
-  }
-  if (threadIdx.x == 0) theta[q] = t;
-}
-
-// The same theta_q by one warp per query.  Bound: the k-th largest of the
-// maxima of 256 interleaved groups (element i in group i mod 256) is at most
-// the k-th largest score; the scores at or above it (usually about k) are
-// compacted into shared memory and their k-th largest found bit by bit.  A
-// query with more than kThetaCap of them sets need_block[q] for theta_kernel.
-constexpr int kThetaCap = 512;
 __global__ void __launch_bounds__(256) theta_warp_kernel(const float* __restrict__ buf_s,
                                                          const int* __restrict__ cnt, int64_t nq, int cap,
-                                                         int k, float* __restrict__ theta,
-                                                         int* __restrict__ need_block) {
-  __shared__ uint32_t ck[8][kThetaCap];
+                                                         int k, float* __restrict__ theta) {
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t q = int64_t(blockIdx.x) * 8 + w;
   if (q >= nq) return;
   const int n = min(cnt[q], cap);
   if (n < k) {
-    if (lane == 0) {
-      theta[q] = -CUDART_INF_F;
-      need_block[q] = 0;
-    }
+    if (lane == 0) theta[q] = -CUDART_INF_F;
     return;
   }
   const float* s = buf_s + q * cap;
@@ -224,7 +185,7 @@ __global__ void __launch_bounds__(256) theta_warp_kernel(const float* __restrict
       if (i < n) gm[c] = max(gm[c], float_order_key(s[i]));
     }
   }
-  // the largest t with #{gm >= t} >= k
+  // the largest t with #{gm >= t} >= k (groups without an element hold 0)
   uint32_t bound = 0u;
   for (int bit = 31; bit >= 0; --bit) {
     const uint32_t t = bound | (1u << bit);
@@ -233,33 +194,7 @@ __global__ void __launch_bounds__(256) theta_warp_kernel(const float* __restrict
     for (int c = 0; c < 8; ++c) c0 += gm[c] >= t ? 1 : 0;
     if (int(__reduce_add_sync(kFull, uint32_t(c0))) >= k) bound = t;
   }
-  const unsigned lt = (1u << lane) - 1u;
-  int m = 0;
-  for (int base = 0; base < n; base += 32) {
-    const int i = base + lane;
-    const uint32_t key = i < n ? float_order_key(s[i]) : 0u;
-    const bool hit = i < n && key >= bound;
-    const unsigned bal = __ballot_sync(kFull, hit);
-    const int at = m + __popc(bal & lt);
-    if (hit && at < kThetaCap) ck[w][at] = key;
-    m += __popc(bal);
-  }
-  if (m > kThetaCap) {
-    if (lane == 0) need_block[q] = 1;
-    return;
-  }
-  __syncwarp();
-  uint32_t res = 0u;
-  for (int bit = 31; bit >= 0; --bit) {
-    const uint32_t t = res | (1u << bit);
-    int c0 = 0;
-    for (int e = lane; e < m; e += 32) c0 += ck[w][e] >= t ? 1 : 0;
-    if (int(__reduce_add_sync(kFull, uint32_t(c0))) >= k) res = t;
-  }
-  if (lane == 0) {
-    theta[q] = theta_from(float_from_order_key(res));
-    need_block[q] = 0;
-  }
+  if (lane == 0) theta[q] = theta_from(float_from_order_key(bound));
 }
 
 struct BatchArgs {
@@ -1596,13 +1531,12 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   }
   if (e == cudaSuccess) e = cudaMemsetAsync(ac, 0, size_t(nq) * 4, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(bc, 0, size_t(nq) * 4, s);
-  // Pass 1: every candidate of each query's first probed partition; its
-  // exact k-th best score bounds the query's k-th best score from below.
+  // Pass 1: every candidate of each query's first probed partition; k of
+  // them reach theta, which bounds the query's k-th best score from below.
   if (e == cudaSuccess)
     e = run_batched(ix, L[0], qhi, qlo, qinv, Dp16, nullptr, as, ap, ac, capA, work, false, s);
   if (e == cudaSuccess) {
-    theta_warp_kernel<<<unsigned((nq + 7) / 8), 256, 0, s>>>(as, ac, nq, capA, k, theta, ovf);
-    theta_kernel<<<unsigned(nq), 256, 0, s>>>(as, ac, capA, k, theta, ovf);
+    theta_warp_kernel<<<unsigned((nq + 7) / 8), 256, 0, s>>>(as, ac, nq, capA, k, theta);
     e = cudaGetLastError();
   }
   // Pass 2: all probed partitions, keeping candidates >= theta.
