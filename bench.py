@@ -47,9 +47,12 @@ CLOCK_FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_eve
                 "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
 SCAN_SOURCES = {
     "scan_kernel": ["paper_2608_30384_gb300/csrc/search.cu", "paper_2608_30384_gb300/csrc/device_common.cuh"],
-    "batched_scan_kernel": ["paper_2608_30384_gb300/csrc/batched.cu",
+    "batched_pipe_kernel": ["paper_2608_30384_gb300/csrc/batched.cu",
                             "paper_2608_30384_gb300/csrc/device_common.cuh",
                             "paper_2608_30384_gb300/csrc/tcgen05.cuh"],
+    "batched_kpipe_kernel": ["paper_2608_30384_gb300/csrc/batched.cu",
+                             "paper_2608_30384_gb300/csrc/device_common.cuh",
+                             "paper_2608_30384_gb300/csrc/tcgen05.cuh"],
 }
 
 
@@ -422,7 +425,7 @@ def run_gpu(args):
     kern_avg_s = kern_ms / max(1, kern_n) / 1e3
     trec = traffic_record(w.name, kern_name)
     traffic = (trec["dram_bytes_per_candidate"] * cand_per_step) if trec else None
-    if kern_name == "batched_scan_kernel":
+    if kern_name.startswith("batched_"):
         # dense contraction: 2 D flops per candidate (the fp16 hi/lo split is
         # counted once); one launch scores the whole step's candidates
         flops = 2.0 * w.D * cand_per_step

@@ -1458,7 +1458,8 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
                          : (g == 2 ? batched_kpipe_kernel<2, true> : batched_kpipe_kernel<4, true>));
   e = cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
-  cudaEvent_t stop = profile ? prof_start(ix, s, "batched_scan_kernel") : nullptr;
+  cudaEvent_t stop =
+      profile ? prof_start(ix, s, b.nkc == 1 ? "batched_pipe_kernel" : "batched_kpipe_kernel") : nullptr;
   pk<<<sms, kPipeThreads, smem, s>>>(b);
   prof_stop(stop, s);
   return cudaGetLastError();
