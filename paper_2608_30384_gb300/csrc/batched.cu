@@ -21,6 +21,7 @@
 #include <cuda_runtime.h>
 #include <math_constants.h>
 
+#include <algorithm>
 #include <climits>
 
 #include "device_common.cuh"
@@ -89,6 +90,66 @@ __global__ void scatter_pairs_kernel(const int32_t* __restrict__ probes, const f
     const int p = probes[src];
     if (p < 0 || p >= nlist) continue;
     const int at = off[p] + atomicAdd(&fill[p], 1);
+    lq[at] = int32_t(i / eff);
+    lcs[at] = cs[src];
+  }
+}
+
+// The same inversion without a global atomic per pair, for nlist small
+// enough for a shared-memory histogram: block b takes the pairs
+// [b chunk, (b + 1) chunk) and writes their per-partition counts to row b of
+// ghist; hist_prefix_kernel turns every column into its exclusive prefix over
+// blocks (cnt[p] = the total); scatter_hist_kernel places block b's pairs of
+// partition p at off[p] + ghist[b][p] + their rank inside the block.
+constexpr int kHistBlocks = 2 * 152;
+constexpr int kHistMaxList = 24576;  // shared-memory histogram: nlist ints
+__global__ void __launch_bounds__(1024) hist_pairs_kernel(const int32_t* __restrict__ probes, int64_t nq,
+                                                          int stride, int eff, int nlist, int64_t chunk,
+                                                          int* __restrict__ ghist, int* err) {
+  extern __shared__ int h[];
+  for (int p = threadIdx.x; p < nlist; p += blockDim.x) h[p] = 0;
+  __syncthreads();
+  const int64_t npairs = nq * eff;
+  const int64_t lo = blockIdx.x * chunk, hi = min(npairs, lo + chunk);
+  for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+    const int p = probes[(i / eff) * stride + i % eff];
+    if (p >= 0 && p < nlist) atomicAdd(&h[p], 1);
+    else set_device_error(err, kErrBadProbe);
+  }
+  __syncthreads();
+  for (int p = threadIdx.x; p < nlist; p += blockDim.x) ghist[int64_t(blockIdx.x) * nlist + p] = h[p];
+}
+
+__global__ void hist_prefix_kernel(int* __restrict__ ghist, int nb, int nlist, int* __restrict__ cnt) {
+  const int p = blockIdx.x * blockDim.x + threadIdx.x;
+  if (p >= nlist) return;
+  int run = 0;
+#pragma unroll 8
+  for (int b = 0; b < nb; ++b) {
+    const int v = ghist[int64_t(b) * nlist + p];
+    ghist[int64_t(b) * nlist + p] = run;
+    run += v;
+  }
+  cnt[p] = run;
+}
+
+__global__ void __launch_bounds__(1024) scatter_hist_kernel(const int32_t* __restrict__ probes,
+                                                            const float* __restrict__ cs, int64_t nq,
+                                                            int stride, int eff, int nlist, int64_t chunk,
+                                                            const int* __restrict__ off,
+                                                            const int* __restrict__ ghist,
+                                                            int32_t* __restrict__ lq, float* __restrict__ lcs) {
+  extern __shared__ int base[];
+  for (int p = threadIdx.x; p < nlist; p += blockDim.x)
+    base[p] = off[p] + ghist[int64_t(blockIdx.x) * nlist + p];
+  __syncthreads();
+  const int64_t npairs = nq * eff;
+  const int64_t lo = blockIdx.x * chunk, hi = min(npairs, lo + chunk);
+  for (int64_t i = lo + threadIdx.x; i < hi; i += blockDim.x) {
+    const int64_t src = (i / eff) * stride + i % eff;
+    const int p = probes[src];
+    if (p < 0 || p >= nlist) continue;
+    const int at = atomicAdd(&base[p], 1);
     lq[at] = int32_t(i / eff);
     lcs[at] = cs[src];
   }
@@ -1379,7 +1440,8 @@ namespace {
 // Per-partition query lists of the probe pairs (q, j < eff).
 struct Lists {
   int* cnt;
-  int* fill;
+  int* fill;   // global-atomic path only
+  int* ghist;  // shared-memory histogram path: kHistBlocks x nlist (shared by both lists)
   int* off;
   int* items;
   int32_t* lq;
@@ -1391,6 +1453,22 @@ cudaError_t build_lists(const rslm_index* ix, const int32_t* probes, const float
                         int stride, int eff, const Lists& L, cudaStream_t s) {
   const int nlist = ix->nlist;
   const int64_t npairs = nq * eff;
+  if (nlist <= kHistMaxList) {
+    const int64_t chunk = std::max<int64_t>(2048, (npairs + kHistBlocks - 1) / kHistBlocks);
+    const int nb = int(std::max<int64_t>(1, (npairs + chunk - 1) / chunk));
+    const size_t hs = size_t(nlist) * 4;
+    cudaError_t e = cudaFuncSetAttribute(hist_pairs_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(hs));
+    if (e == cudaSuccess)
+      e = cudaFuncSetAttribute(scatter_hist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(hs));
+    if (e != cudaSuccess) return e;
+    hist_pairs_kernel<<<nb, 1024, hs, s>>>(probes, nq, stride, eff, nlist, chunk, L.ghist, ix->d_err);
+    hist_prefix_kernel<<<(nlist + 255) / 256, 256, 0, s>>>(L.ghist, nb, nlist, L.cnt);
+    scan_lists_kernel<<<1, 1024, 0, s>>>(L.cnt, nlist, L.off, L.items);
+    item_part_kernel<<<blocks_for(nlist, 256, 152 * 4), 256, 0, s>>>(L.items, nlist, L.item_p);
+    scatter_hist_kernel<<<nb, 1024, hs, s>>>(probes, cs, nq, stride, eff, nlist, chunk, L.off, L.ghist, L.lq,
+                                              L.lcs);
+    return cudaGetLastError();
+  }
   cudaError_t e = cudaMemsetAsync(L.cnt, 0, size_t(nlist) * 4, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(L.fill, 0, size_t(nlist) * 4, s);
   if (e != cudaSuccess) return e;
@@ -1484,6 +1562,7 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
     return at;
   };
   size_t oL[2][7];
+  const size_t o_ghist = take(nlist <= kHistMaxList ? size_t(kHistBlocks) * nlist * 4 : 4);
   for (int l = 0; l < 2; ++l) {
     const int64_t np = l ? npairs : nq;
     oL[l][0] = take(size_t(nlist) * 4);
@@ -1506,7 +1585,7 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   Lists L[2];
   for (int l = 0; l < 2; ++l)
     L[l] = Lists{reinterpret_cast<int*>(ws + oL[l][0]), reinterpret_cast<int*>(ws + oL[l][1]),
-                 reinterpret_cast<int*>(ws + oL[l][2]), reinterpret_cast<int*>(ws + oL[l][3]),
+                 reinterpret_cast<int*>(ws + o_ghist), reinterpret_cast<int*>(ws + oL[l][2]), reinterpret_cast<int*>(ws + oL[l][3]),
                  reinterpret_cast<int32_t*>(ws + oL[l][4]), reinterpret_cast<float*>(ws + oL[l][5]),
                  reinterpret_cast<int*>(ws + oL[l][6])};
   __half* qhi = reinterpret_cast<__half*>(ws + o_qhi);
