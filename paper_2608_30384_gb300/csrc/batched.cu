@@ -1315,21 +1315,17 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
 // overflowed marks the query for the single-query re-scan.
 __global__ void finalize_kernel(const float* __restrict__ buf_s, const int32_t* __restrict__ buf_p,
                                 const int* __restrict__ cnt, int cap, const int64_t* __restrict__ ids,
-                                int k, int* __restrict__ overflow, int64_t* __restrict__ out_ids,
-                                float* __restrict__ out_scores, const int* __restrict__ only_if) {
+                                int k, const int* __restrict__ qlist, const int* __restrict__ qcount,
+                                int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
   extern __shared__ __align__(16) uint8_t fsm[];
   __shared__ uint32_t hist[256];
   __shared__ uint32_t sh_prefix[2];
   __shared__ uint32_t sh_n;
-  const int64_t q = blockIdx.x;
-  if (only_if && only_if[q] == 0) return;
+  const int nlisted = *qcount;
+  for (int e = blockIdx.x; e < nlisted; e += gridDim.x) {
+  const int64_t q = qlist[e];
   const int tid = threadIdx.x;
   const int n = cnt[q];
-  if (n > cap) {
-    if (tid == 0) overflow[q] = 1;
-    return;
-  }
-  if (tid == 0) overflow[q] = 0;
   int p2 = 1;
   while (p2 < k + 64) p2 <<= 1;
   float* key = reinterpret_cast<float*>(fsm);
@@ -1364,17 +1360,21 @@ __global__ void finalize_kernel(const float* __restrict__ buf_s, const int32_t* 
     out_ids[q * k + i] = ok ? idv[i] : -1;
     out_scores[q * k + i] = ok ? key[i] : -CUDART_INF_F;
   }
+  __syncthreads();  // the next listed query reuses the shared buffers
+  }
 }
 
 // The same result by one warp per query for buffers of at most kFinCap
-// candidates: sort them in shared memory by (score desc, id asc).  A buffer
-// with more sets need_block[q] for finalize_kernel.
+// candidates: sort them in shared memory by (score desc, id asc).  A longer
+// buffer is listed for finalize_kernel, an overflowed one (more than cap
+// candidates) for the single-query re-scan.
 constexpr int kFinCap = 512;
 constexpr int kFinWarps = 4;
 __global__ void __launch_bounds__(kFinWarps * 32) finalize_warp_kernel(
     const float* __restrict__ buf_s, const int32_t* __restrict__ buf_p, const int* __restrict__ cnt,
-    int64_t nq, int cap, const int64_t* __restrict__ ids, int k, int* __restrict__ overflow,
-    int* __restrict__ need_block, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
+    int64_t nq, int cap, const int64_t* __restrict__ ids, int k, int* __restrict__ ovf_list,
+    int* __restrict__ blk_list, int* __restrict__ counts, int64_t* __restrict__ out_ids,
+    float* __restrict__ out_scores) {
   __shared__ uint32_t fk[kFinWarps][kFinCap];
   __shared__ int64_t fi[kFinWarps][kFinCap];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
@@ -1382,9 +1382,10 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_warp_kernel(
   if (q >= nq) return;
   const int n = cnt[q];
   if (n > cap || n > kFinCap) {
+    // counts[0]: overflowed queries, counts[1]: queries for the block kernel
     if (lane == 0) {
-      overflow[q] = n > cap ? 1 : 0;
-      need_block[q] = n > cap ? 0 : 1;
+      if (n > cap) ovf_list[atomicAdd(&counts[0], 1)] = int(q);
+      else blk_list[atomicAdd(&counts[1], 1)] = int(q);
     }
     return;
   }
@@ -1420,10 +1421,6 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_warp_kernel(
     const bool ok = i < n && fi[w][i] != LLONG_MAX;
     out_ids[q * k + i] = ok ? fi[w][i] : -1;
     out_scores[q * k + i] = ok ? float_from_order_key(fk[w][i]) : -CUDART_INF_F;
-  }
-  if (lane == 0) {
-    overflow[q] = 0;
-    need_block[q] = 0;
   }
 }
 
@@ -1578,7 +1575,7 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
                o_as = take(size_t(nq) * capA * 4), o_ap = take(size_t(nq) * capA * 4),
                o_ac = take(size_t(nq) * 4), o_bs = take(size_t(nq) * cap * 4),
                o_bp = take(size_t(nq) * cap * 4), o_bc = take(size_t(nq) * 4),
-               o_ovf = take(size_t(nq) * 4), o_work = take(4);
+               o_ovf = take(size_t(nq) * 4), o_work = take(4), o_fcounts = take(8);
   uint8_t* ws = nullptr;
   cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, s);
   if (e != cudaSuccess) return e;
@@ -1600,6 +1597,7 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   int* bc = reinterpret_cast<int*>(ws + o_bc);
   int* ovf = reinterpret_cast<int*>(ws + o_ovf);
   int* work = reinterpret_cast<int*>(ws + o_work);
+  int* fcounts = reinterpret_cast<int*>(ws + o_fcounts);
 
   // lists: L[0] the first probe of every query, L[1] all probe pairs
   e = build_lists(ix, probes, cs, nq, nprobe, 1, L[0], s);
@@ -1628,17 +1626,22 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
     const size_t smem = size_t(p2) * 12;
     e = cudaFuncSetAttribute(finalize_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
     if (e == cudaSuccess) {
-      // ac (the first pass's counts) is free again: it holds the hand-over flags
-      finalize_warp_kernel<<<unsigned((nq + kFinWarps - 1) / kFinWarps), kFinWarps * 32, 0, s>>>(
-          bs, bp, bc, nq, cap, ix->ids, k, ovf, ac, out_ids, out_scores);
-      finalize_kernel<<<unsigned(nq), 256, smem, s>>>(bs, bp, bc, cap, ix->ids, k, ovf, out_ids, out_scores,
-                                                      ac);
-      e = cudaGetLastError();
+      // ac (the first pass's counts) is free again: it lists the queries
+      // handed to the block kernel; ovf lists the overflowed ones
+      e = cudaMemsetAsync(fcounts, 0, 2 * sizeof(int), s);
+      if (e == cudaSuccess) {
+        finalize_warp_kernel<<<unsigned((nq + kFinWarps - 1) / kFinWarps), kFinWarps * 32, 0, s>>>(
+            bs, bp, bc, nq, cap, ix->ids, k, ovf, ac, fcounts, out_ids, out_scores);
+        finalize_kernel<<<unsigned(std::min<int64_t>(nq, 2 * 152)), 256, smem, s>>>(
+            bs, bp, bc, cap, ix->ids, k, ac, fcounts + 1, out_ids, out_scores);
+        e = cudaGetLastError();
+      }
     }
   }
   // Queries whose buffer overflowed: exact single-query scan of all probes.
   if (e == cudaSuccess)
-    e = launch_scan_strided(ix, qrot, nq, probes, nprobe, cs, nprobe, k, k, out_ids, out_scores, ovf, s);
+    e = launch_scan_listed(ix, qrot, nq, probes, nprobe, cs, nprobe, k, out_ids, out_scores, ovf, fcounts,
+                           s);
   cudaError_t f = cudaFreeAsync(ws, s);
   return e != cudaSuccess ? e : f;
 }

@@ -30,6 +30,11 @@ cudaError_t launch_scan_strided(const rslm_index* ix, const float* qrot, int64_t
                                 const int32_t* probes, int probe_stride, const float* cs, int nprobe,
                                 int k, int out_k, int64_t* out_ids, float* out_scores,
                                 const int* only_if, cudaStream_t s);
+// The same scan of the queries qlist[0 .. *qcount) (a device-side count of
+// at most nq), by a fixed grid whose blocks stride over the list.
+cudaError_t launch_scan_listed(const rslm_index* ix, const float* qrot, int64_t nq, const int32_t* probes,
+                               int probe_stride, const float* cs, int nprobe, int k, int64_t* out_ids,
+                               float* out_scores, const int* qlist, const int* qcount, cudaStream_t s);
 // Partition-major scan on the tensor cores (batched.cu); output as launch_scan.
 cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t nq,
                                 const int32_t* probes, const float* cs, int nprobe, int k,

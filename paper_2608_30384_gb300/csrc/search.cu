@@ -294,6 +294,9 @@ struct ScanArgs {
   int nprobe;        // probes scanned per query (the first nprobe of each list)
   int probe_stride;  // row stride of probes / cs
   const int* only_if;  // optional: scan query q only if only_if[q] != 0
+  // optional: scan the queries qlist[0 .. *qcount) instead, blocks striding
+  const int* qlist;
+  const int* qcount;
   int k;
   int out_k;
   const uint8_t* codes;
@@ -381,7 +384,9 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   extern __shared__ __align__(16) uint8_t ssm[];
   __shared__ int scratch[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, W = blockDim.x >> 5;
-  const int64_t q = blockIdx.x;
+  const int nrun = a.qlist ? *a.qcount : 1;
+  for (int run0 = a.qlist ? int(blockIdx.x) : 0; run0 < nrun; run0 += a.qlist ? int(gridDim.x) : 1) {
+  const int64_t q = a.qlist ? int64_t(a.qlist[run0]) : int64_t(blockIdx.x);
   if (a.only_if && a.only_if[q] == 0) return;
   // The table starts on a 256-byte boundary of the shared window (up to 255
   // bytes of padding are reserved by the launcher).
@@ -530,6 +535,8 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
     a.out_ids[q * a.out_k + e] = ok ? id : -1;
     a.out_scores[q * a.out_k + e] = ok ? mkey[e] : -CUDART_INF_F;
   }
+  __syncthreads();  // the next listed query rebuilds the shared tables
+  }
 }
 
 // ---------------------------------------------------------------- rescore
@@ -604,11 +611,14 @@ __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ Re
 template <int CH>
 cudaError_t launch_scan_ch(const rslm_index* ix, const ScanArgs& a, int64_t nq, size_t smem,
                            cudaStream_t s) {
+  // listed queries: a fixed grid strides over the list, whose length is on the device
+  const int64_t grid = a.qlist ? (nq < 2 * 152 ? nq : 2 * 152) : nq;
   cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        int(smem));
   if (e != cudaSuccess) return e;
-  cudaEvent_t stop = a.only_if == nullptr && a.nprobe > 1 ? prof_start(ix, s, "scan_kernel") : nullptr;
-  scan_kernel<CH><<<unsigned(nq), 256, smem, s>>>(a);
+  cudaEvent_t stop =
+      a.only_if == nullptr && a.qlist == nullptr && a.nprobe > 1 ? prof_start(ix, s, "scan_kernel") : nullptr;
+  scan_kernel<CH><<<unsigned(grid), 256, smem, s>>>(a);
   prof_stop(stop, s);
   return cudaGetLastError();
 }
@@ -652,12 +662,15 @@ cudaError_t launch_scan(const rslm_index* ix, const float* qrot, int64_t nq, con
                              nullptr, s);
 }
 
-cudaError_t launch_scan_strided(const rslm_index* ix, const float* qrot, int64_t nq,
-                                const int32_t* probes, int probe_stride, const float* cs, int nprobe,
-                                int k, int out_k, int64_t* out_ids, float* out_scores,
-                                const int* only_if, cudaStream_t s) {
+namespace {
+cudaError_t launch_scan_impl(const rslm_index* ix, const float* qrot, int64_t nq, const int32_t* probes,
+                             int probe_stride, const float* cs, int nprobe, int k, int out_k,
+                             int64_t* out_ids, float* out_scores, const int* only_if, const int* qlist,
+                             const int* qcount, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
   ScanArgs a;
+  a.qlist = qlist;
+  a.qcount = qcount;
   a.qrot = qrot;
   a.Dp = ix->cs1.Dp;
   a.probes = probes;
@@ -695,6 +708,22 @@ cudaError_t launch_scan_strided(const rslm_index* ix, const float* qrot, int64_t
     case 8: return launch_scan_ch<8>(ix, a, nq, smem, s);
     default: return launch_scan_ch<4>(ix, a, nq, smem, s);
   }
+}
+}  // namespace
+
+cudaError_t launch_scan_strided(const rslm_index* ix, const float* qrot, int64_t nq,
+                                const int32_t* probes, int probe_stride, const float* cs, int nprobe,
+                                int k, int out_k, int64_t* out_ids, float* out_scores,
+                                const int* only_if, cudaStream_t s) {
+  return launch_scan_impl(ix, qrot, nq, probes, probe_stride, cs, nprobe, k, out_k, out_ids, out_scores,
+                          only_if, nullptr, nullptr, s);
+}
+
+cudaError_t launch_scan_listed(const rslm_index* ix, const float* qrot, int64_t nq, const int32_t* probes,
+                               int probe_stride, const float* cs, int nprobe, int k, int64_t* out_ids,
+                               float* out_scores, const int* qlist, const int* qcount, cudaStream_t s) {
+  return launch_scan_impl(ix, qrot, nq, probes, probe_stride, cs, nprobe, k, k, out_ids, out_scores, nullptr,
+                          qlist, qcount, s);
 }
 
 cudaError_t launch_rescore(const rslm_index* ix, const float* qrot2, int64_t nq,
