@@ -120,17 +120,38 @@ __global__ void __launch_bounds__(1024) hist_pairs_kernel(const int32_t* __restr
   for (int p = threadIdx.x; p < nlist; p += blockDim.x) ghist[int64_t(blockIdx.x) * nlist + p] = h[p];
 }
 
-__global__ void hist_prefix_kernel(int* __restrict__ ghist, int nb, int nlist, int* __restrict__ cnt) {
-  const int p = blockIdx.x * blockDim.x + threadIdx.x;
+// The column prefix in two steps over segments of kHistSeg rows, one thread
+// per (column, segment): segment sums, then each segment's rows rewritten
+// from the sum of the segments above it.
+constexpr int kHistSeg = 16;
+__global__ void hist_segsum_kernel(const int* __restrict__ ghist, int nb, int nlist, int* __restrict__ segsum) {
+  const int p = blockIdx.x * blockDim.x + threadIdx.x, seg = blockIdx.y;
+  if (p >= nlist) return;
+  int sum = 0;
+#pragma unroll
+  for (int r = 0; r < kHistSeg; ++r) {
+    const int b = seg * kHistSeg + r;
+    if (b < nb) sum += ghist[int64_t(b) * nlist + p];
+  }
+  segsum[int64_t(seg) * nlist + p] = sum;
+}
+
+__global__ void hist_prefix_kernel(int* __restrict__ ghist, const int* __restrict__ segsum, int nb, int nlist,
+                                   int* __restrict__ cnt) {
+  const int p = blockIdx.x * blockDim.x + threadIdx.x, seg = blockIdx.y;
   if (p >= nlist) return;
   int run = 0;
-#pragma unroll 8
-  for (int b = 0; b < nb; ++b) {
-    const int v = ghist[int64_t(b) * nlist + p];
-    ghist[int64_t(b) * nlist + p] = run;
-    run += v;
+  for (int s2 = 0; s2 < seg; ++s2) run += segsum[int64_t(s2) * nlist + p];
+#pragma unroll
+  for (int r = 0; r < kHistSeg; ++r) {
+    const int b = seg * kHistSeg + r;
+    if (b < nb) {
+      const int v = ghist[int64_t(b) * nlist + p];
+      ghist[int64_t(b) * nlist + p] = run;
+      run += v;
+    }
   }
-  cnt[p] = run;
+  if (seg == int(gridDim.y) - 1) cnt[p] = run;
 }
 
 __global__ void __launch_bounds__(1024) scatter_hist_kernel(const int32_t* __restrict__ probes,
@@ -1438,7 +1459,8 @@ namespace {
 struct Lists {
   int* cnt;
   int* fill;   // global-atomic path only
-  int* ghist;  // shared-memory histogram path: kHistBlocks x nlist (shared by both lists)
+  int* ghist;   // shared-memory histogram path: kHistBlocks x nlist (shared by both lists)
+  int* segsum;  // and its segment sums: kHistBlocks / kHistSeg (rounded up) x nlist
   int* off;
   int* items;
   int32_t* lq;
@@ -1459,7 +1481,9 @@ cudaError_t build_lists(const rslm_index* ix, const int32_t* probes, const float
       e = cudaFuncSetAttribute(scatter_hist_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(hs));
     if (e != cudaSuccess) return e;
     hist_pairs_kernel<<<nb, 1024, hs, s>>>(probes, nq, stride, eff, nlist, chunk, L.ghist, ix->d_err);
-    hist_prefix_kernel<<<(nlist + 255) / 256, 256, 0, s>>>(L.ghist, nb, nlist, L.cnt);
+    const dim3 pg((nlist + 255) / 256, (nb + kHistSeg - 1) / kHistSeg);
+    hist_segsum_kernel<<<pg, 256, 0, s>>>(L.ghist, nb, nlist, L.segsum);
+    hist_prefix_kernel<<<pg, 256, 0, s>>>(L.ghist, L.segsum, nb, nlist, L.cnt);
     scan_lists_kernel<<<1, 1024, 0, s>>>(L.cnt, nlist, L.off, L.items);
     item_part_kernel<<<blocks_for(nlist, 256, 152 * 4), 256, 0, s>>>(L.items, nlist, L.item_p);
     scatter_hist_kernel<<<nb, 1024, hs, s>>>(probes, cs, nq, stride, eff, nlist, chunk, L.off, L.ghist, L.lq,
@@ -1560,6 +1584,8 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   };
   size_t oL[2][7];
   const size_t o_ghist = take(nlist <= kHistMaxList ? size_t(kHistBlocks) * nlist * 4 : 4);
+  const size_t o_segsum =
+      take(nlist <= kHistMaxList ? size_t((kHistBlocks + kHistSeg - 1) / kHistSeg) * nlist * 4 : 4);
   for (int l = 0; l < 2; ++l) {
     const int64_t np = l ? npairs : nq;
     oL[l][0] = take(size_t(nlist) * 4);
@@ -1582,7 +1608,8 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   Lists L[2];
   for (int l = 0; l < 2; ++l)
     L[l] = Lists{reinterpret_cast<int*>(ws + oL[l][0]), reinterpret_cast<int*>(ws + oL[l][1]),
-                 reinterpret_cast<int*>(ws + o_ghist), reinterpret_cast<int*>(ws + oL[l][2]), reinterpret_cast<int*>(ws + oL[l][3]),
+                 reinterpret_cast<int*>(ws + o_ghist), reinterpret_cast<int*>(ws + o_segsum),
+                 reinterpret_cast<int*>(ws + oL[l][2]), reinterpret_cast<int*>(ws + oL[l][3]),
                  reinterpret_cast<int32_t*>(ws + oL[l][4]), reinterpret_cast<float*>(ws + oL[l][5]),
                  reinterpret_cast<int*>(ws + oL[l][6])};
   __half* qhi = reinterpret_cast<__half*>(ws + o_qhi);
