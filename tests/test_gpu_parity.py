@@ -234,6 +234,13 @@ def test_batched_scan_overflow_fallback():
                          seed=12)), batched=True)
 
 
+def test_batched_scan_many_partitions():
+    """More partitions (25000) than the shared-memory histograms of the
+    probe-list inversion hold (24576): the global-atomic inversion path."""
+    _scan_parity(Case(Wl("np", 60_000, 16, 25_000, 0.5, False, 0.5, "true", 200, 4, 0, 16, 10, 10,
+                         seed=21)), batched=True)
+
+
 @pytest.mark.parametrize("bits,D", [(4, 128), (2, 96), (1, 128), (4, 256), (1, 768), (2, 300),
                                     (1, 256), (2, 768), (4, 768), (1, 384)])
 def test_batched_scan_many_queries_per_partition(bits, D):
