@@ -157,6 +157,110 @@ def decode(A, enc_codes, L_u16, G_u16, bits: int, D: int) -> np.ndarray:
     return Gh[:, None] * (A + Lh[:, None] * (uhat @ R))
 
 
+# ------------------------------------------------------------ Rslm4Lite
+# Sec. 3.4 (Rslm4Lite paragraph) and Sec. 3.5 (relative quantization): for
+# D >= 64 the first 16 rotated coordinates take the K=8 (3-bit) codebook,
+# which leaves the top bit of each of their 4-bit codes free; the UE7M9
+# local scale is stored in those 16 bits, so the packed row is exactly
+# ceil(D/2) bytes.  RelApproxGlobal-Rslm4Lite does the same over the first
+# 32 coordinates and stores the UE4M12 global scale in the second 16 bits.
+
+LITE_MIN_D = 64
+
+
+def lite_head(global_scale: bool) -> int:
+    """Leading coordinates on the K=8 codebook: 32 with the global scale, else 16."""
+    return 32 if global_scale else 16
+
+
+def encode_lite(X, A, global_scale: bool = True) -> Encoded:
+    """Rslm4Lite encoding of residuals X - A (steps 1-6 of ``encode``).
+
+    The rotation and the EVT scale are those of the 4-bit codec.  Step 3
+    quantizes coordinates j < H (H = ``lite_head``) with the K=8 levels and
+    the others with the K=16 levels.  After steps 4-6 the scale codes are
+    embedded: bit i of the UE7M9 code is the top bit of code i, and with
+    the global scale bit i of the UE4M12 code is the top bit of code 16 + i
+    (i = 0 .. 15, least significant bit first).  ``codes`` holds the stored
+    4-bit values (level index | scale bit << 3).
+    """
+    X = np.asarray(X, dtype=np.float64)
+    A = np.asarray(A, dtype=np.float64)
+    n, D = X.shape
+    if D < LITE_MIN_D:
+        raise ValueError(f"Rslm4Lite needs D >= {LITE_MIN_D}")
+    H = lite_head(global_scale)
+    cb8, cb16 = codebook(3), codebook(4)
+    R = rotation_matrix(D, rotation_mode(4, D))
+
+    r = X - A                                   # step 1
+    z = r @ R.T
+    m = np.max(np.abs(z), axis=1)
+    factor = np.where(m > 0, e_max(D) / np.where(m > 0, m, 1.0), 0.0)
+    u = z * factor[:, None]                     # step 2 (g = 1: no padding)
+
+    levels = np.zeros((n, D), dtype=np.int64)   # step 3
+    levels[:, :H] = cb8.assign(u[:, :H, None])
+    levels[:, H:] = cb16.assign(u[:, H:, None])
+    uhat = np.empty((n, D))
+    uhat[:, :H] = cb8.C[levels[:, :H], 0]
+    uhat[:, H:] = cb16.C[levels[:, H:], 0]
+
+    nr = np.linalg.norm(r, axis=1)              # step 4
+    nu = np.linalg.norm(uhat, axis=1)
+    L = np.where(nu > 0, nr / np.where(nu > 0, nu, 1.0), 0.0)
+    L_u16 = UE7M9.encode(L)
+    Lhat = UE7M9.decode(L_u16)
+    rt = Lhat[:, None] * (uhat @ R)             # step 5
+    if global_scale:                            # step 6
+        na = np.linalg.norm(A + rt, axis=1)
+        G = np.where(na > 0, np.linalg.norm(X, axis=1) / np.where(na > 0, na, 1.0), 0.0)
+    else:
+        G = np.ones(n)
+    G_u16 = UE4M12.encode(G)
+    Ghat = UE4M12.decode(G_u16)
+    recon = Ghat[:, None] * (A + rt)
+
+    codes = levels.copy()                       # scale bits into the free top bits
+    for i in range(16):
+        codes[:, i] |= ((L_u16 >> i) & 1) << 3
+        if global_scale:
+            codes[:, 16 + i] |= ((G_u16 >> i) & 1) << 3
+    return Encoded(4, rotation_mode(4, D), D, 1, codes, L_u16, G_u16, Lhat, Ghat, uhat, u, recon, L, G)
+
+
+def unpack_lite(codes, global_scale: bool = True):
+    """Stored Rslm4Lite codes (n, D) -> (level indices, UE7M9 codes, UE4M12 codes).
+
+    Without the global scale the UE4M12 code is that of 1.0.
+    """
+    codes = np.asarray(codes, dtype=np.int64)
+    H = lite_head(global_scale)
+    levels = codes.copy()
+    levels[:, :H] &= 7
+    L_u16 = np.zeros(codes.shape[0], dtype=np.int64)
+    G_u16 = np.zeros(codes.shape[0], dtype=np.int64)
+    for i in range(16):
+        L_u16 |= ((codes[:, i] >> 3) & 1) << i
+        if global_scale:
+            G_u16 |= ((codes[:, 16 + i] >> 3) & 1) << i
+    if not global_scale:
+        G_u16[:] = UE4M12.encode(np.ones(1))[0]
+    return levels, L_u16, G_u16
+
+
+def decode_lite(A, codes, D: int, global_scale: bool = True) -> np.ndarray:
+    """Reconstruction Ghat (a + Lhat R^T uhat) from stored Rslm4Lite codes."""
+    A = np.asarray(A, dtype=np.float64)
+    levels, L_u16, G_u16 = unpack_lite(codes, global_scale)
+    H = lite_head(global_scale)
+    uhat = np.empty((levels.shape[0], D))
+    uhat[:, :H] = codebook(3).C[levels[:, :H], 0]
+    uhat[:, H:] = codebook(4).C[levels[:, H:], 0]
+    R = rotation_matrix(D, rotation_mode(4, D))
+    return UE4M12.decode(G_u16)[:, None] * (A + UE7M9.decode(L_u16)[:, None] * (uhat @ R))
+
+
 def pack_nibbles(codes: np.ndarray) -> np.ndarray:
     """(n, ngroups) codes < 16 -> (n, ceil(ngroups/2)) uint8, low nibble first."""
     codes = np.asarray(codes, dtype=np.int64)

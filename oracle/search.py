@@ -26,7 +26,7 @@ from dataclasses import dataclass, field
 
 import numpy as np
 
-from oracle.codec import Encoded, encode
+from oracle.codec import Encoded, encode, encode_lite
 from oracle.rotation import rotation_matrix, rotation_mode
 
 
@@ -50,18 +50,21 @@ class OracleIndex:
 
 
 def build_index(X, ids, assign, centroids, bits: int, rescore_bits: int = 0,
-                global_scale: bool = True) -> OracleIndex:
+                global_scale: bool = True, lite: bool = False) -> OracleIndex:
     """Encode rows X (ids, partition ``assign``) against their centroids.
 
-    Stage 1 quantizes r = x - c_p with ``bits`` per dimension.  With
-    ``rescore_bits`` > 0, stage 2 quantizes x - a2 with a2 the stage-1
-    reconstruction, using ``rescore_bits`` per dimension.
+    Stage 1 quantizes r = x - c_p with ``bits`` per dimension (``lite``:
+    Rslm4Lite, bits must be 4).  With ``rescore_bits`` > 0, stage 2
+    quantizes x - a2 with a2 the stage-1 reconstruction, using
+    ``rescore_bits`` per dimension.
     """
     X = np.asarray(X, dtype=np.float64)
     C = np.asarray(centroids, dtype=np.float64)
     assign = np.asarray(assign, dtype=np.int64)
     A1 = C[assign]
-    st1 = encode(X, A1, bits, global_scale=global_scale)
+    if lite and bits != 4:
+        raise ValueError("Rslm4Lite is a 4-bit codec")
+    st1 = encode_lite(X, A1, global_scale) if lite else encode(X, A1, bits, global_scale=global_scale)
     st2 = None
     if rescore_bits:
         st2 = encode(X, st1.recon, rescore_bits, global_scale=global_scale)
