@@ -63,6 +63,19 @@ typedef enum {
  * the global scale is then 1. */
 #define RSLM_GLOBAL_SCALE 1u
 
+/* Flag for rslm_index_create.  Set: the scoring codes are Rslm4Lite (Sec.
+ * 3.4, Rslm4Lite paragraph; with RSLM_GLOBAL_SCALE, RelApproxGlobal-
+ * Rslm4Lite, Sec. 3.5.2).  score_bits must be 4 and dim >= 64.  The first
+ * 16 rotated coordinates (32 with RSLM_GLOBAL_SCALE) are quantized with the
+ * K = 8 levels of the 3-bit codec; bit i of the UE7M9 local-scale code is
+ * stored as the top bit of code i and, with RSLM_GLOBAL_SCALE, bit i of the
+ * UE4M12 global-scale code as the top bit of code 16 + i (i = 0 .. 15), so a
+ * row is exactly ceil(dim / 2) code bytes.  The single-query scan reads the
+ * scales from those bits; the index also keeps the decoded scale pair per
+ * row (the `local_scale` / `global_scale` of rslm_export_codes and
+ * rslm_import_codes, which then move codes that include the scale bits). */
+#define RSLM_LITE 2u
+
 typedef struct rslm_index rslm_index;
 
 /* Shape of an index, filled by rslm_index_describe. */
@@ -94,7 +107,7 @@ typedef struct {
  *   Specifications").
  * rescore_bits: 0 (no rescoring) or 4: bits of the rescoring codes, which
  *   quantize x - a2 with a2 the full first-stage reconstruction (Sec. 5.2).
- * flags: RSLM_GLOBAL_SCALE or 0.
+ * flags: RSLM_GLOBAL_SCALE and / or RSLM_LITE, or 0.
  * On success *out receives the index; release it with rslm_index_destroy. */
 rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids,
                               int32_t score_bits, int32_t rescore_bits, uint32_t flags,

@@ -168,7 +168,9 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
   RSLM_ARG(nlist >= 1, "nlist must be >= 1");
   RSLM_ARG(score_bits == 1 || score_bits == 2 || score_bits == 4, "score_bits must be 1, 2 or 4");
   RSLM_ARG(rescore_bits == 0 || rescore_bits == 4, "rescore_bits must be 0 or 4");
-  RSLM_ARG((flags & ~RSLM_GLOBAL_SCALE) == 0, "unknown flag bits");
+  RSLM_ARG((flags & ~(RSLM_GLOBAL_SCALE | RSLM_LITE)) == 0, "unknown flag bits");
+  RSLM_ARG(!(flags & RSLM_LITE) || (score_bits == 4 && dim >= 64),
+           "RSLM_LITE needs score_bits == 4 and dim >= 64");
   RSLM_ARG(centroids, "centroids is NULL");
   {
     CodecSpec probe_spec;
@@ -197,6 +199,16 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
   ix->flags = flags;
   ix->rot1 = make_rot_spec(dim, score_bits);
   make_codec_spec(score_bits, dim, true, &ix->cs1);
+  if (flags & RSLM_LITE) {
+    CodecSpec k8;
+    make_codec_spec(3, 0, true, &k8);
+    ix->cs1.lite_h = (flags & RSLM_GLOBAL_SCALE) ? 32 : 16;
+    for (int i = 0; i < 8; ++i) {
+      ix->cs1.cb8d[i] = k8.cbd[i];
+      ix->cs1.cb8f[i] = k8.cbf[i];
+      if (i < 7) ix->cs1.thr8[i] = k8.thr[i];
+    }
+  }
   if (rescore_bits) {
     ix->rot2 = make_rot_spec(dim, rescore_bits);
     make_codec_spec(rescore_bits, dim, false, &ix->cs2);

@@ -287,6 +287,8 @@ struct BatchArgs {
   int nlist;
   int stride, chunk, g, Dp16, nkc;
   uint32_t cbbits[64];  // codebook components as binary16 bits, K x g
+  int lite_h;            // Rslm4Lite: leading coordinates on the K = 8 levels (0: none)
+  uint32_t cb8bits[8];   // their levels as binary16 bits
   const int* off;       // [nlist + 1] per-partition query list offsets
   const int* items;     // [nlist + 1] per-partition work-item offsets
   const int* item_p;    // [items[nlist]] partition of each work item
@@ -378,17 +380,21 @@ constexpr int kScaleBytes = kMR * 4;  // a tile's (L | G << 16) words
 // 256-entry table held once per lane (entry (byte, lane) at word byte * 32 +
 // lane), so the 32 lookups of a warp always fall into 32 distinct banks.
 constexpr int kByteTableBytes = 256 * 32 * 4;
+// Rslm4Lite head bytes: (3-bit code | 3-bit code << 3) -> two halves, 64
+// entries (the top bits, which hold the scale codes, are dropped)
+constexpr int kLiteTableBytes = 64 * 4;
 __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
   return size_t(2) * kSlotBytes + size_t(kSlabs) * slab_bytes(g) + size_t(kScaleStages) * kScaleBytes + 32 * 4 +
-         (g == 1 ? kByteTableBytes : 0);
+         (g == 1 ? kByteTableBytes + kLiteTableBytes : 0);
 }
 
 // Half dh (32 columns = 64 halves = 64 / G codes) of a row's A operand from
 // the row's code words wd (G = 1: 16 words; byte -> column through the
 // per-lane table t256; G = 2, 4: nibble -> halves through t32).
-template <int G>
+template <int G, bool LITE>
 __device__ __forceinline__ void decode_half(const uint32_t* wd, int dh, const uint32_t* t256,
-                                            const uint32_t* t32, int lane, uint32_t (&av)[32]) {
+                                            const uint32_t* t32, int lane, uint32_t (&av)[32],
+                                            int lite_words, const uint32_t* t64) {
   if constexpr (G == 1) {
     // one byte (two codes) -> one 32-bit column (low half = even position)
     const uint32_t* tl = t256 + lane;
@@ -396,6 +402,18 @@ __device__ __forceinline__ void decode_half(const uint32_t* wd, int dh, const ui
     for (int w = 0; w < 8; ++w)
 #pragma unroll
       for (int bb = 0; bb < 4; ++bb) av[4 * w + bb] = tl[((wd[8 * dh + w] >> (8 * bb)) & 255u) << 5];
+    // Rslm4Lite: the first lite_words (<= 4) words hold K = 8 codes under
+    // the scale bits (static indices keep av in registers)
+    if constexpr (LITE) {
+#pragma unroll
+      for (int w = 0; w < 4; ++w)
+        if (w < lite_words)
+#pragma unroll
+          for (int bb = 0; bb < 4; ++bb) {
+            const uint32_t byte = (wd[8 * dh + w] >> (8 * bb)) & 255u;
+            av[4 * w + bb] = t64[(byte & 7u) | ((byte >> 1) & 0x38u)];
+          }
+    }
   } else if constexpr (G == 2) {
 #pragma unroll
     for (int w = 0; w < 4; ++w)
@@ -483,7 +501,7 @@ __device__ __forceinline__ void epilogue_row(const BatchArgs& a, const float (&v
   }
 }
 
-template <int G, bool DENSE>
+template <int G, bool DENSE, bool LITE>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
   extern __shared__ __align__(128) uint8_t psm[];
   uint8_t* slab0 = psm + 2 * kSlotBytes;
@@ -498,11 +516,13 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   const int CH = a.chunk;
 
   uint32_t* t256 = t32 + 32;  // G = 1 only
+  uint32_t* t64 = t256 + 256 * 32;  // G = 1 only: Rslm4Lite head
   if (G == 1) {
     for (int e = tid; e < 256 * 32; e += blockDim.x) {
       const uint32_t byte = uint32_t(e) >> 5;  // low nibble -> low half (even position)
       t256[e] = a.cbbits[byte & 15u] | (a.cbbits[byte >> 4] << 16);
     }
+    for (int e = tid; e < 64; e += blockDim.x) t64[e] = a.cb8bits[e & 7] | (a.cb8bits[e >> 3] << 16);
   } else if (G == 2) {
     for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[2 * c] | (a.cbbits[2 * c + 1] << 16);
   } else {
@@ -802,7 +822,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
 #pragma unroll
         for (int dh = 0; dh < 2; ++dh) {
           uint32_t av[32];
-          decode_half<G>(wd, dh, t256, t32, lane, av);
+          decode_half<G, LITE>(wd, dh, t256, t32, lane, av, dh == 0 ? a.lite_h / 8 : 0, t64);
           tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
         }
         fence_before_sync();
@@ -895,10 +915,10 @@ constexpr int kKSlot = (kNQ * 16 + int(sizeof(ItemDesc)) + 127) / 128 * 128;  //
 constexpr int kKOffQinv = kNQ * 8, kKOffQid = kNQ * 12, kKOffDesc = kNQ * 16;
 __host__ __device__ constexpr size_t kpipe_smem_bytes(int g) {
   return size_t(2) * kBStageBytes + size_t(2) * kKSlot + size_t(kSlabs) * slab_bytes(g) +
-         size_t(kScaleStages) * kScaleBytes + 32 * 4 + (g == 1 ? kByteTableBytes : 0);
+         size_t(kScaleStages) * kScaleBytes + 32 * 4 + (g == 1 ? kByteTableBytes + kLiteTableBytes : 0);
 }
 
-template <int G, bool DENSE>
+template <int G, bool DENSE, bool LITE>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __grid_constant__ BatchArgs a) {
   extern __shared__ __align__(128) uint8_t psm[];
   uint8_t* bst0 = psm;                               // B ring
@@ -907,6 +927,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
   uint32_t* scl0 = reinterpret_cast<uint32_t*>(slab0 + kSlabs * slab_bytes(G));
   uint32_t* t32 = scl0 + kScaleStages * kMR;
   uint32_t* t256 = t32 + 32;  // G = 1 only
+  uint32_t* t64 = t256 + 256 * 32;  // G = 1 only: Rslm4Lite head
   __shared__ __align__(8) uint64_t bars[12 + 2 * kSlabs + 2 * kKR + 2 * kScaleStages];
   __shared__ uint32_t tmem_base_sh;
   __shared__ int s_fail;
@@ -917,6 +938,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
       const uint32_t byte = uint32_t(e) >> 5;
       t256[e] = a.cbbits[byte & 15u] | (a.cbbits[byte >> 4] << 16);
     }
+    for (int e = tid; e < 64; e += blockDim.x) t64[e] = a.cb8bits[e & 7] | (a.cb8bits[e >> 3] << 16);
   } else if (G == 2) {
     for (int c = tid; c < 16; c += blockDim.x) t32[c] = a.cbbits[2 * c] | (a.cbbits[2 * c + 1] << 16);
   } else {
@@ -1254,7 +1276,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
 #pragma unroll
             for (int dh = 0; dh < 2; ++dh) {
               uint32_t av[32];
-              decode_half<G>(wd, dh, t256, t32, lane, av);
+              decode_half<G, LITE>(wd, dh, t256, t32, lane, av, (kc == 0 && dh == 0) ? a.lite_h / 8 : 0,
+                                   t64);
               tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(ab) + uint32_t(dh * 32), av);
             }
             fence_before_sync();
@@ -1518,6 +1541,8 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   b.Dp16 = Dp16;
   b.nkc = (Dp16 + kKC - 1) / kKC;
   for (int i = 0; i < 64; ++i) b.cbbits[i] = __half_as_ushort(__float2half_rn(c1.cbf[i]));
+  b.lite_h = c1.lite_h;
+  for (int i = 0; i < 8; ++i) b.cb8bits[i] = __half_as_ushort(__float2half_rn(c1.cb8f[i]));
   b.off = L.off;
   b.items = L.items;
   b.item_p = L.item_p;
@@ -1546,15 +1571,17 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   using K = void (*)(BatchArgs);
   K pk;
   if (one)
-    pk = theta ? (g == 1 ? batched_pipe_kernel<1, false>
-                         : (g == 2 ? batched_pipe_kernel<2, false> : batched_pipe_kernel<4, false>))
-               : (g == 1 ? batched_pipe_kernel<1, true>
-                         : (g == 2 ? batched_pipe_kernel<2, true> : batched_pipe_kernel<4, true>));
+    pk = b.lite_h ? (theta ? batched_pipe_kernel<1, false, true> : batched_pipe_kernel<1, true, true>)
+         : theta  ? (g == 1 ? batched_pipe_kernel<1, false, false>
+                            : (g == 2 ? batched_pipe_kernel<2, false, false> : batched_pipe_kernel<4, false, false>))
+                  : (g == 1 ? batched_pipe_kernel<1, true, false>
+                            : (g == 2 ? batched_pipe_kernel<2, true, false> : batched_pipe_kernel<4, true, false>));
   else
-    pk = theta ? (g == 1 ? batched_kpipe_kernel<1, false>
-                         : (g == 2 ? batched_kpipe_kernel<2, false> : batched_kpipe_kernel<4, false>))
-               : (g == 1 ? batched_kpipe_kernel<1, true>
-                         : (g == 2 ? batched_kpipe_kernel<2, true> : batched_kpipe_kernel<4, true>));
+    pk = b.lite_h ? (theta ? batched_kpipe_kernel<1, false, true> : batched_kpipe_kernel<1, true, true>)
+         : theta  ? (g == 1 ? batched_kpipe_kernel<1, false, false>
+                            : (g == 2 ? batched_kpipe_kernel<2, false, false> : batched_kpipe_kernel<4, false, false>))
+                  : (g == 1 ? batched_kpipe_kernel<1, true, false>
+                            : (g == 2 ? batched_kpipe_kernel<2, true, false> : batched_kpipe_kernel<4, true, false>));
   e = cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
   cudaEvent_t stop =

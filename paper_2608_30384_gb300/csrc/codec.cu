@@ -64,6 +64,8 @@ struct EncodeArgs {
 struct CodecTables {
   double cb[64];
   double thr[15];
+  double cb8[8];  // Rslm4Lite head (K = 8)
+  double thr8[7];
 };
 
 // Nearest codeword of the group starting at u (Sec. 3.2): 1-D by the count
@@ -108,6 +110,19 @@ __device__ uint32_t quantize_stage(double* A, double* tmp, const RotSpec& rs, co
   __syncwarp();
   for (int b = lane; b < cs.code_bytes; b += 32) {
     const int g0 = 2 * b, g1 = 2 * b + 1;
+    if (g0 < cs.lite_h) {
+      // Rslm4Lite head (g = 1, lite_h even): the K = 8 levels; the top bits
+      // stay clear for the scale codes
+      int c0 = 0, c1 = 0;
+      for (int i = 0; i < 7; ++i) {
+        c0 += (A[g0] >= ct.thr8[i]);
+        c1 += (A[g1] >= ct.thr8[i]);
+      }
+      put(b, uint32_t(c0 | (c1 << 4)));
+      A[g0] = ct.cb8[c0];
+      A[g1] = ct.cb8[c1];
+      continue;
+    }
     const int c0 = nearest_code(A + g0 * cs.g, cs, ct);
     const int c1 = g1 < cs.ngroups ? nearest_code(A + g1 * cs.g, cs, ct) : 0;
     put(b, uint32_t(c0 | (c1 << 4)));
@@ -143,6 +158,10 @@ __global__ void encode_kernel(const __grid_constant__ EncodeArgs a) {
   for (int i = threadIdx.x; i < 15; i += blockDim.x) {
     ct1.thr[i] = a.cs1.thr[i];
     ct2.thr[i] = a.cs2.thr[i];
+  }
+  for (int i = threadIdx.x; i < 8; i += blockDim.x) {
+    ct1.cb8[i] = a.cs1.cb8d[i];
+    if (i < 7) ct1.thr8[i] = a.cs1.thr8[i];
   }
   __syncthreads();
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, W = blockDim.x >> 5;
@@ -194,6 +213,18 @@ __global__ void encode_kernel(const __grid_constant__ EncodeArgs a) {
       const double G = na2 > 0.0 ? sqrt(nx2) / sqrt(na2) : 0.0;
       Gu1 = ue_encode(G, 4, 12);
       Gh1 = ue_decode(Gu1, 4, 12);
+    }
+    if (a.cs1.lite_h) {
+      // Rslm4Lite: bit i of the UE7M9 code into the top bit of code i, and
+      // of the UE4M12 code into that of code 16 + i (lite_h = 32); code j
+      // is the low (even j) or high (odd j) nibble of byte j / 2
+      __syncwarp();
+      if (lane < a.cs1.lite_h / 2) {
+        const int b = lane;
+        uint8_t* pb = tile + ((b / ch) * kTile + rin) * ch + (b % ch);
+        auto bit = [&](int j) { return j < 16 ? (Lu1 >> j) & 1u : (Gu1 >> (j - 16)) & 1u; };
+        *pb = uint8_t(*pb | (bit(2 * b) << 3) | (bit(2 * b + 1) << 7));
+      }
     }
     if (lane == 0) {
       a.scales1[slot] = Lu1 | (Gu1 << 16);

@@ -56,6 +56,13 @@ struct CodecSpec {
   float cbf[64];  // K x g codewords (binary16-exact)
   double cbd[64];
   double thr[15]; // 1-D decision thresholds (midpoints of adjacent levels)
+  // Rslm4Lite (Sec. 3.4): the first lite_h coordinates (0, 16 or 32) take
+  // the K=8 levels; the UE7M9 code sits in the top bits of codes 0-15 and,
+  // with lite_h = 32, the UE4M12 code in those of codes 16-31
+  int lite_h;
+  double cb8d[8];
+  float cb8f[8];
+  double thr8[7];
 };
 
 // Host-side tables (tables.cpp).

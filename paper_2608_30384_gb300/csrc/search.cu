@@ -310,6 +310,8 @@ struct ScanArgs {
   int ngroups;
   int g;
   float cb[64];
+  int lite_h;    // Rslm4Lite: leading coordinates on the K = 8 levels (0: none);
+  float cb8[8];  // their levels; the scale codes are read from the codes' top bits
   int64_t* out_ids;
   float* out_scores;
   int* err;
@@ -379,6 +381,14 @@ __device__ __forceinline__ void warp_insert(float* sc, int* ps, int& cnt, int k,
   cnt = newcnt;
 }
 
+// The top bits of a word's eight 4-bit codes, code k's at bit k.
+__device__ __forceinline__ uint32_t nibble_tops(uint32_t w) {
+  uint32_t t = (w >> 3) & 0x11111111u;
+  t = (t | (t >> 3)) & 0x03030303u;
+  t = (t | (t >> 6)) & 0x000F000Fu;
+  return (t | (t >> 12)) & 0xFFu;
+}
+
 template <int CH>
 __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanArgs a) {
   extern __shared__ __align__(16) uint8_t ssm[];
@@ -410,7 +420,9 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   for (int e = tid; e < a.lut_groups * 16; e += blockDim.x) {
     const int grp = e >> 4, code = e & 15;
     float v = 0.0f;
-    if (grp < a.ngroups)
+    if (grp < a.lite_h)
+      v = qr[grp] * a.cb8[code & 7];  // the top bit is a scale bit (g = 1)
+    else if (grp < a.ngroups)
       for (int j = 0; j < a.g; ++j) v = fmaf(qr[grp * a.g + j], a.cb[code * a.g + j], v);
     lut[(2 * (grp >> 3) + (grp & 1)) * 64 + ((grp & 7) >> 1) * 16 + code] = v;
   }
@@ -455,11 +467,23 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
     const float csj = a.cs[q * a.probe_stride + j];
     const uint8_t* tp = a.codes + slot0 * a.stride;
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+    uint32_t hb[4] = {0u, 0u, 0u, 0u};  // Rslm4Lite: UE7M9 | UE4M12 << 16 from the top bits
     for (int c = 0; c < nch; ++c) {
       uint32_t w[4][CH / 4];
 #pragma unroll
       for (int r = 0; r < 4; ++r)
         load_chunk<CH>(tp + (size_t(c) * kTile + r * 32 + lane) * CH, w[r]);
+      if (c * CH < a.lite_h / 2) {
+        // word wi of the row holds codes 8 wi .. 8 wi + 7: their top bits are
+        // bits 8 wi .. 8 wi + 7 of the scale pair
+#pragma unroll
+        for (int v = 0; v < CH / 4; ++v) {
+          const int wi = c * (CH / 4) + v;
+          if (wi < a.lite_h / 8)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) hb[r] |= nibble_tops(w[r][v]) << (8 * wi);
+        }
+      }
 #pragma unroll
       for (int v = 0; v < CH / 4; ++v) {
         // bits 8.. of the addresses of this word's even / odd positions
@@ -485,7 +509,7 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
       const int pos = int(slot0) + row;
       float s = -CUDART_INF_F;
       if (valid) {
-        const uint32_t sc = __ldg(a.scales + slot0 + row);
+        const uint32_t sc = a.lite_h ? (a.lite_h == 32 ? hb[r] : (hb[r] | (7u << 28))) : __ldg(a.scales + slot0 + row);
         s = ue4m12_to_f32(sc >> 16) * fmaf(ue7m9_to_f32(sc & 0xffffu), acc[r], csj);
       }
       const bool cand = valid && (cnt < a.k || s > thr || (s == thr && pos < thr_pos));
@@ -691,6 +715,8 @@ cudaError_t launch_scan_impl(const rslm_index* ix, const float* qrot, int64_t nq
   a.ngroups = ix->cs1.ngroups;
   a.g = ix->cs1.g;
   for (int i = 0; i < 64; ++i) a.cb[i] = ix->cs1.cbf[i];
+  a.lite_h = ix->cs1.lite_h;
+  for (int i = 0; i < 8; ++i) a.cb8[i] = ix->cs1.cb8f[i];
   a.out_ids = out_ids;
   a.out_scores = out_scores;
   a.err = ix->d_err;

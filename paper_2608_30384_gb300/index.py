@@ -13,11 +13,12 @@ class Index:
     """
 
     def __init__(self, centroids, score_bits: int, rescore_bits: int = 0, global_scale: bool = True,
-                 stream=None):
+                 stream=None, lite: bool = False):
         nlist, dim = centroids.shape
         self.device = centroids.device
+        flags = (B.RSLM_GLOBAL_SCALE if global_scale else 0) | (B.RSLM_LITE if lite else 0)
         self.handle = B.rslm_index_create(dim, nlist, centroids.contiguous(), score_bits, rescore_bits,
-                                          B.RSLM_GLOBAL_SCALE if global_scale else 0, stream)
+                                          flags, stream)
 
     @property
     def desc(self) -> dict:

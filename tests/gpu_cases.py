@@ -5,6 +5,7 @@ from __future__ import annotations
 import numpy as np
 
 from oracle import codec, constants as K, search
+from oracle.rotation import rotation_matrix, rotation_mode
 from paper_2608_30384_gb300 import workloads as W
 
 
@@ -25,20 +26,22 @@ def ue_near_tie(v, fmt: K.UEFormat, rel: float = 1e-9) -> np.ndarray:
 class Case:
     """A workload, its oracle index and (lazily) its GPU index."""
 
-    def __init__(self, w: W.Workload, nq: int | None = None, global_scale: bool = True):
+    def __init__(self, w: W.Workload, nq: int | None = None, global_scale: bool = True, lite: bool = False):
         self.w = w
         self.X, self.A = W.database(w)
         self.C = W.ivf_centroids(w, self.X, self.A)
         self.Q = W.queries(w, nq)
         self.global_scale = global_scale
+        self.lite = lite
         self.oracle = search.build_index(self.X, np.arange(w.N), self.A, self.C, w.bits,
-                                         w.rescore_bits, global_scale=global_scale)
+                                         w.rescore_bits, global_scale=global_scale, lite=lite)
         self._gpu = None
 
     def gpu_index(self, encode: bool = True):
         import torch
         from paper_2608_30384_gb300 import Index
-        ix = Index(torch.from_numpy(self.C).cuda(), self.w.bits, self.w.rescore_bits, self.global_scale)
+        ix = Index(torch.from_numpy(self.C).cuda(), self.w.bits, self.w.rescore_bits, self.global_scale,
+                   lite=self.lite)
         ix.reserve(torch.from_numpy(self.A).cuda())
         if encode:
             ix.encode(torch.from_numpy(self.X).cuda(), 0)
@@ -90,4 +93,51 @@ def check_stage(gpu_codes, gpu_L, gpu_G, enc, X, A, bits, global_scale, name):
         Lu, Gu, Le, Ge = codec.scales_from_codes(X[r:r + 1], A[r:r + 1], bits, got[r:r + 1], global_scale)
         assert abs(int(gpu_L[r]) - int(Lu[0])) <= (1 if ue_near_tie(Le, K.UE7M9)[0] else 0)
         assert abs(int(gpu_G[r]) - int(Gu[0])) <= (1 if ue_near_tie(Ge, K.UE4M12)[0] else 0)
+    return ok
+
+
+def check_lite_stage(gpu_codes, gpu_L, gpu_G, enc, X, A, global_scale, name):
+    """Encode parity of Rslm4Lite scoring codes, with the rules of
+    ``check_stage``: the level codes (K = 8 head, K = 16 tail) bit-exact
+    except near their decision boundaries, the scale codes embedded in the
+    head's top bits equal to the decoded pair the index keeps, and both equal
+    to the oracle's except at rounding ties (or, on a row with a boundary
+    flip, to the scales the GPU's own levels imply)."""
+    D = enc.D
+    H = codec.lite_head(global_scale)
+    got = codec.unpack_nibbles(gpu_codes, D)
+    lv, eL, eG = codec.unpack_lite(got, global_scale)
+    assert np.array_equal(eL, gpu_L.astype(np.int64)), f"{name}: embedded UE7M9 code != kept scale"
+    if global_scale:
+        assert np.array_equal(eG, gpu_G.astype(np.int64)), f"{name}: embedded UE4M12 code != kept scale"
+    olv, _, _ = codec.unpack_lite(enc.codes, global_scale)
+    mism = lv != olv
+    near = np.zeros_like(mism)
+    for lo, hi, cb in ((0, H, K.codebook(3)), (H, D, K.codebook(4))):
+        d = np.abs(enc.u[:, lo:hi, None] - cb.thresholds[None, None, :])
+        near[:, lo:hi] = d.min(axis=-1) < 1e-5
+    assert np.all(near[mism]), f"{name}: level mismatch away from a decision boundary"
+    assert mism.sum() <= max(1, 1e-4 * mism.size), f"{name}: {mism.sum()} mismatched codes"
+    ok = ~mism.any(1)
+    for gv, ov, ex, fmt in ((gpu_L, enc.L_u16, enc.L_exact, K.UE7M9), (gpu_G, enc.G_u16, enc.G_exact, K.UE4M12)):
+        bad = ok & (gv.astype(np.int64) != ov)
+        if bad.any():
+            tie = ue_near_tie(ex[bad], fmt)
+            assert np.all(tie) and np.all(np.abs(gv[bad].astype(np.int64) - ov[bad]) <= 1), \
+                f"{name}: {bad.sum()} scale codes differ away from rounding ties"
+    for r in np.nonzero(~ok)[0]:
+        # the scales the GPU's levels imply: steps 4-6 with those codewords
+        uhat = np.empty(D)
+        uhat[:H] = K.codebook(3).C[lv[r, :H], 0]
+        uhat[H:] = K.codebook(4).C[lv[r, H:], 0]
+        Rm = rotation_matrix(D, rotation_mode(4, D))
+        rr = np.asarray(X[r], dtype=np.float64) - A[r]
+        L = np.linalg.norm(rr) / np.linalg.norm(uhat)
+        Lu = int(K.UE7M9.encode(np.array([L]))[0])
+        assert abs(int(gpu_L[r]) - Lu) <= (1 if ue_near_tie(np.array([L]), K.UE7M9)[0] else 0)
+        if global_scale:
+            rt = K.UE7M9.decode(np.array([Lu]))[0] * (uhat @ Rm)
+            G = np.linalg.norm(X[r]) / np.linalg.norm(A[r] + rt)
+            Gu = int(K.UE4M12.encode(np.array([G]))[0])
+            assert abs(int(gpu_G[r]) - Gu) <= (1 if ue_near_tie(np.array([G]), K.UE4M12)[0] else 0)
     return ok

@@ -13,7 +13,7 @@ import pytest
 from oracle import codec, constants as K, search
 from oracle.rotation import rotation_matrix, rotation_mode
 from paper_2608_30384_gb300 import workloads as W
-from tests.gpu_cases import Case, check_stage
+from tests.gpu_cases import Case, check_lite_stage, check_stage
 from tests.lib_util import check_topk, ensure_library, score_tol
 
 torch = pytest.importorskip("torch")
@@ -250,6 +250,37 @@ def test_batched_scan_many_queries_per_partition(bits, D):
     K chunks (D = 300: a partial last chunk)."""
     _scan_parity(Case(Wl(f"mq{bits}", 20_000, D, 8, 0.5, False, 0.5, "mean", 600, bits, 0, 3, 10, 10,
                          seed=13 + bits)), batched=True)
+
+
+# ------------------------------------------------------------- Rslm4Lite
+# Sec. 3.4: the scale codes ride in the top bits of the first 16 (32 with the
+# global scale) codes, which take the K = 8 levels.  D = 100 exercises 4-byte
+# code chunks and a partial last group; D = 768 the several-K-chunk kernel.
+LITE = {
+    "l128": Wl("l128", 30_000, 128, 24, 0.5, False, 0.5, "mean", 48, 4, 0, 6, 10, 10, seed=31),
+    "l100": Wl("l100", 20_000, 100, 16, 0.5, True, None, "mean", 48, 4, 0, 4, 10, 10, seed=32),
+    "l768": Wl("l768", 8_000, 768, 8, 0.5, True, None, "mean", 48, 4, 0, 3, 10, 10, seed=33),
+}
+
+
+@pytest.mark.parametrize("name", sorted(LITE))
+@pytest.mark.parametrize("gs", [True, False])
+def test_lite_encode_parity(name, gs):
+    case = Case(LITE[name], global_scale=gs, lite=True)
+    ix = case.gpu_index()
+    c1, L1, G1 = (t.cpu().numpy() for t in ix.export_codes(1))
+    assert c1.shape[1] == (case.w.D + 1) // 2
+    check_lite_stage(c1, L1, G1, case.oracle.stage1, case.X, case.C[case.A].astype(np.float64), gs, name)
+
+
+@pytest.mark.parametrize("name", sorted(LITE))
+@pytest.mark.parametrize("gs", [True, False])
+@pytest.mark.parametrize("batched", [False, True])
+def test_lite_scan_parity(name, gs, batched):
+    """Scan of imported oracle Rslm4Lite codes: the single-query kernel reads
+    the scales from the codes' top bits, the tensor-core kernels decode the
+    head through the K = 8 table."""
+    _scan_parity(Case(LITE[name], global_scale=gs, lite=True), batched=batched)
 
 
 def test_rescore_parity_on_oracle_codes(case):
