@@ -69,10 +69,19 @@ def parse_args():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--scan", default="auto", choices=["auto", "gemv", "batched"],
                     help="scan form; auto = rslm_search's rule (batched when nq*nprobe >= 16*nlist)")
-    return ap.parse_args()
+    ap.add_argument("--lite", action="store_true",
+                    help="Rslm4Lite scoring codes (4-bit workloads, D >= 64): scales in the codes' top bits")
+    args = ap.parse_args()
+    if args.lite:
+        w = W.WORKLOADS[args.config]
+        if w.bits != 4 or w.D < 64:
+            ap.error("--lite needs a 4-bit workload with D >= 64")
+    return args
 
 
-def workload_label(w: W.Workload) -> str:
+def workload_label(w: W.Workload, lite: bool = False) -> str:
+    if lite:
+        return f"{w.name} with Rslm4Lite scoring codes: {w.description}"
     return f"{w.name}: {w.description}"
 
 
@@ -184,7 +193,7 @@ def dist_setup(args):
 
 
 # --------------------------------------------------------- oracle (CPU) leg
-def oracle_sample(w: W.Workload, A, C, Q, n_queries: int):
+def oracle_sample(w: W.Workload, A, C, Q, n_queries: int, lite: bool = False):
     """Oracle index over the rows of the partitions the sample queries probe
     (those rows are regenerated from their seeds)."""
     from oracle import search as osearch
@@ -192,7 +201,7 @@ def oracle_sample(w: W.Workload, A, C, Q, n_queries: int):
     parts = np.unique(probes)
     rows = np.nonzero(np.isin(A, parts))[0]
     X, _ = W.rows(w, rows)
-    index = osearch.build_index(X, rows, A[rows], C, w.bits, w.rescore_bits)
+    index = osearch.build_index(X, rows, A[rows], C, w.bits, w.rescore_bits, lite=lite)
     sizes = np.bincount(A, minlength=w.P)
     cand = int(sizes[probes].sum())
     return index, cand, len(rows)
@@ -230,7 +239,7 @@ def run_reference(args):
     C = W.ivf_centroids(w)
     nqs = min(SAMPLE_QUERIES[w.name], w.nq)
     Q = W.queries(w, nqs)
-    index, cand, nrows = oracle_sample(w, A, C, Q, nqs)
+    index, cand, nrows = oracle_sample(w, A, C, Q, nqs, args.lite)
     for _ in range(args.warmup):
         oracle_time(w, index, Q, nqs, cand, 0.0)
     t0 = time.perf_counter()
@@ -243,7 +252,7 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": workload_label(w), "nq_per_step": nqs},
+            "data": "synthetic", "config": {"workload": workload_label(w, args.lite), "nq_per_step": nqs},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -298,7 +307,7 @@ def run_gpu(args):
     nq = w.nq
 
     # index build (not timed as part of the step)
-    ix = Index(torch.from_numpy(C).to(dev), w.bits, w.rescore_bits)
+    ix = Index(torch.from_numpy(C).to(dev), w.bits, w.rescore_bits, lite=args.lite)
     ix.reserve(torch.from_numpy(A).to(dev))
     torch.cuda.synchronize()
     encode_s = 0.0
@@ -348,7 +357,8 @@ def run_gpu(args):
     ix.sync()
     sizes = torch.bincount(torch.from_numpy(A).to(dev).long(), minlength=w.P)
     cand_per_step = int(sizes[probes.long()].sum().item())
-    bytes_per_cand = desc["code_bytes"] + 4  # codes + UE7M9 + UE4M12 scales
+    # codes + UE7M9 + UE4M12 scales (Rslm4Lite: the scales are inside the codes)
+    bytes_per_cand = desc["code_bytes"] + (0 if args.lite else 4)
 
     E = lambda: torch.cuda.Event(enable_timing=True)  # noqa: E731
     starts = [E() for _ in range(args.steps)]
@@ -423,7 +433,7 @@ def run_gpu(args):
     hbm_peak, tensor_peak, peak_kind = load_peaks()
     scan_bytes = cand_per_step * bytes_per_cand
     kern_avg_s = kern_ms / max(1, kern_n) / 1e3
-    trec = traffic_record(w.name, kern_name)
+    trec = traffic_record(w.name + ("-lite" if args.lite else ""), kern_name)
     traffic = (trec["dram_bytes_per_candidate"] * cand_per_step) if trec else None
     if kern_name.startswith("batched_"):
         # dense contraction: 2 D flops per candidate (the fp16 hi/lo split is
@@ -445,7 +455,7 @@ def run_gpu(args):
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         nqs = min(SAMPLE_QUERIES[w.name], nq)
-        index, cand, nrows = oracle_sample(w, A, C, Q, nqs)
+        index, cand, nrows = oracle_sample(w, A, C, Q, nqs, args.lite)
         cval, passes, dt = oracle_time(w, index, Q, nqs, cand, args.cpu_seconds)
         cpu = {"value": cval, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": f"{nqs} of the {nq} queries of {w.name} ({cand} candidates per pass) x {passes} "
@@ -457,7 +467,7 @@ def run_gpu(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": workload_label(w), "nq": nq, "nprobe": w.nprobe, "k": w.k,
+            "config": {"workload": workload_label(w, args.lite), "nq": nq, "nprobe": w.nprobe, "k": w.k,
                        "k_final": w.k_final, "score_bits": w.bits, "rescore_bits": w.rescore_bits,
                        "l2": (f"L2 flushed between timed steps (a {4 * L2_BYTES / 1e6:.0f} MB buffer "
                               f"overwritten, not timed): the {(scan_bytes_index(desc) + rescore_bytes_index(desc)) / 1e6:.0f}"
