@@ -14,7 +14,13 @@ for the top-k) with the score identities of Sec. 3.5:
 * Rescoring (Sec. 2.1 and Sec. 5.2): the survivors of the first stage are
   rescored from higher-bit codes of the second residual x - a2, where the
   approximation a2 is the full first-stage reconstruction, so <q, a2> is the
-  first-stage score itself.
+  first-stage score itself ("reading B", the default).  Reading A: a2 is the
+  first stage's own approximation (the centroid), so the second stage is an
+  independent, finer code of the same residual and its score is
+  Ghat2 (<q, c> + Lhat2 <R2 q, uhat2>).
+* Full-vector quantization (Sec. 3.5, first paragraph: the codec applied to
+  x itself): the approximation is 0, the partitions only route the probe,
+  and a score is Ghat Lhat <R q, uhat>.
 
 Orders: probes by (<q, c_p> descending, p ascending); candidates by (score
 descending, id ascending).  Missing results are id -1 with score -inf.
@@ -44,13 +50,16 @@ class OracleIndex:
     stage1: Encoded
     stage2: Encoded | None
     members: dict = field(default_factory=dict)  # partition -> row positions
+    reading: str = "B"             # rescoring approximation: "B" stage-1 reconstruction, "A" centroid
+    full_vector: bool = False      # the approximation is 0 (no residual)
 
     def rows_of(self, p: int) -> np.ndarray:
         return self.members.get(int(p), np.zeros(0, dtype=np.int64))
 
 
 def build_index(X, ids, assign, centroids, bits: int, rescore_bits: int = 0,
-                global_scale: bool = True, lite: bool = False) -> OracleIndex:
+                global_scale: bool = True, lite: bool = False, reading: str = "B",
+                full_vector: bool = False) -> OracleIndex:
     """Encode rows X (ids, partition ``assign``) against their centroids.
 
     Stage 1 quantizes r = x - c_p with ``bits`` per dimension (``lite``:
@@ -64,15 +73,19 @@ def build_index(X, ids, assign, centroids, bits: int, rescore_bits: int = 0,
     A1 = C[assign]
     if lite and bits != 4:
         raise ValueError("Rslm4Lite is a 4-bit codec")
+    if reading not in ("A", "B"):
+        raise ValueError("reading is 'A' or 'B'")
+    if full_vector:
+        A1 = np.zeros_like(A1)
     st1 = encode_lite(X, A1, global_scale) if lite else encode(X, A1, bits, global_scale=global_scale)
     st2 = None
     if rescore_bits:
-        st2 = encode(X, st1.recon, rescore_bits, global_scale=global_scale)
+        st2 = encode(X, st1.recon if reading == "B" else A1, rescore_bits, global_scale=global_scale)
     members = {}
     for p in np.unique(assign):
         members[int(p)] = np.nonzero(assign == p)[0]
     return OracleIndex(X.shape[1], bits, rescore_bits, global_scale, C,
-                       np.asarray(ids, dtype=np.int64), assign, st1, st2, members)
+                       np.asarray(ids, dtype=np.int64), assign, st1, st2, members, reading, full_vector)
 
 
 def order_desc(scores: np.ndarray, ids: np.ndarray) -> np.ndarray:
@@ -122,7 +135,8 @@ def stage1_scores(index: OracleIndex, q, probes, cs):
         if r.size == 0:
             continue
         dot = st.uhat[r] @ qb
-        sc.append(st.Ghat[r] * (c + st.Lhat[r] * dot))
+        a_term = 0.0 if index.full_vector else c
+        sc.append(st.Ghat[r] * (a_term + st.Lhat[r] * dot))
         rows.append(r)
     if not rows:
         return np.zeros(0, dtype=np.int64), np.zeros(0)
@@ -137,7 +151,11 @@ def scan(index: OracleIndex, q, probes, cs, k: int):
 
 
 def rescore(index: OracleIndex, q, cand_ids, cand_scores, k_final: int):
-    """Stage-2 scores Ghat2 (s1 + Lhat2 <R2 q, uhat2>) and their top k_final."""
+    """Stage-2 scores Ghat2 (<q, a2> + Lhat2 <R2 q, uhat2>) and their top k_final.
+
+    <q, a2> is the stage-1 score s1 (reading B), or <q, c> of the row's
+    partition (reading A; 0 for full-vector codes).
+    """
     st = index.stage2
     qb = rotate_query(q, index.rescore_bits)
     pos_of = {int(i): j for j, i in enumerate(index.ids)}
@@ -147,7 +165,13 @@ def rescore(index: OracleIndex, q, cand_ids, cand_scores, k_final: int):
     r = np.array([pos_of[int(i)] for i in cid], dtype=np.int64)
     if r.size == 0:
         return take_top(np.zeros(0), np.zeros(0, dtype=np.int64), k_final) + (np.zeros(0),)
-    s2 = st.Ghat[r] * (s1 + st.Lhat[r] * (st.uhat[r] @ qb))
+    if index.reading == "B":
+        a_term = s1
+    elif index.full_vector:
+        a_term = np.zeros(r.size)
+    else:
+        a_term = index.centroids[index.assign[r]] @ np.asarray(q, dtype=np.float64)
+    s2 = st.Ghat[r] * (a_term + st.Lhat[r] * (st.uhat[r] @ qb))
     ids, scores = take_top(s2, cid, k_final)
     return ids, scores, s2
 
