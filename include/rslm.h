@@ -76,6 +76,20 @@ typedef enum {
  * rslm_import_codes, which then move codes that include the scale bits). */
 #define RSLM_LITE 2u
 
+/* Flag for rslm_index_create.  Set: the rescoring codes quantize x - c with
+ * c the partition centroid, the first stage's own approximation ("reading
+ * A": an independent finer code of the same residual), and rescoring scores
+ * are G2 (<q, c> + L2 <R2 q, u2^>).  Clear ("reading B", Sec. 5.2): they
+ * quantize x - a2 with a2 the full first-stage reconstruction, scored
+ * G2 (s1 + L2 <R2 q, u2^>).  Needs rescore_bits > 0. */
+#define RSLM_RESCORE_READING_A 4u
+
+/* Flag for rslm_index_create.  Set: full-vector quantization (Sec. 3.5,
+ * first paragraph): the codes quantize x itself (approximation 0).  The
+ * partitions only route the probe; scores are G L <R q, u^> (no <q, c>
+ * term, so rslm_scan ignores its cs argument). */
+#define RSLM_FULL_VECTOR 8u
+
 typedef struct rslm_index rslm_index;
 
 /* Shape of an index, filled by rslm_index_describe. */
@@ -107,7 +121,8 @@ typedef struct {
  *   Specifications").
  * rescore_bits: 0 (no rescoring) or 4: bits of the rescoring codes, which
  *   quantize x - a2 with a2 the full first-stage reconstruction (Sec. 5.2).
- * flags: RSLM_GLOBAL_SCALE and / or RSLM_LITE, or 0.
+ * flags: any of RSLM_GLOBAL_SCALE, RSLM_LITE, RSLM_RESCORE_READING_A,
+ *   RSLM_FULL_VECTOR, or 0.
  * On success *out receives the index; release it with rslm_index_destroy. */
 rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids,
                               int32_t score_bits, int32_t rescore_bits, uint32_t flags,

@@ -19,6 +19,8 @@ LIB_PATH = os.path.join(_HERE, "librslm.so")
 
 RSLM_GLOBAL_SCALE = 1
 RSLM_LITE = 2
+RSLM_RESCORE_READING_A = 4
+RSLM_FULL_VECTOR = 8
 STATUS = {0: "RSLM_OK", 1: "RSLM_ERR_INVALID_ARG", 2: "RSLM_ERR_OUT_OF_MEMORY", 3: "RSLM_ERR_CUDA",
           4: "RSLM_ERR_TIMEOUT", 5: "RSLM_ERR_STATE", 6: "RSLM_ERR_DEVICE", 7: "RSLM_ERR_INTERNAL"}
 

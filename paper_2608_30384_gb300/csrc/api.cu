@@ -65,7 +65,7 @@ cudaError_t dev_alloc(rslm_index* ix, T** p, size_t count) {
 void free_all(rslm_index* ix) {
   void* ptrs[] = {ix->centroids, ix->part_off, ix->part_n, ix->assign, ix->slot_of_row, ix->ids,
                   ix->codes1,    ix->scales1,  ix->codes2, ix->scales2, ix->d_err,   ix->ctiles,
-                  ix->cmeta,     ix->crows};
+                  ix->cmeta,     ix->crows,    ix->crot2};
   for (void* p : ptrs)
     if (p) cudaFree(p);
   if (ix->cublas) cublasDestroy(reinterpret_cast<cublasHandle_t>(ix->cublas));
@@ -168,7 +168,9 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
   RSLM_ARG(nlist >= 1, "nlist must be >= 1");
   RSLM_ARG(score_bits == 1 || score_bits == 2 || score_bits == 4, "score_bits must be 1, 2 or 4");
   RSLM_ARG(rescore_bits == 0 || rescore_bits == 4, "rescore_bits must be 0 or 4");
-  RSLM_ARG((flags & ~(RSLM_GLOBAL_SCALE | RSLM_LITE)) == 0, "unknown flag bits");
+  RSLM_ARG((flags & ~(RSLM_GLOBAL_SCALE | RSLM_LITE | RSLM_RESCORE_READING_A | RSLM_FULL_VECTOR)) == 0,
+           "unknown flag bits");
+  RSLM_ARG(!(flags & RSLM_RESCORE_READING_A) || rescore_bits > 0, "RSLM_RESCORE_READING_A needs rescoring codes");
   RSLM_ARG(!(flags & RSLM_LITE) || (score_bits == 4 && dim >= 64),
            "RSLM_LITE needs score_bits == 4 and dim >= 64");
   RSLM_ARG(centroids, "centroids is NULL");
@@ -221,6 +223,11 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
                         cudaMemcpyDeviceToDevice, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(ix->d_err, 0, sizeof(int), s);
   if (e == cudaSuccess) e = probe_prepare(ix, s);
+  if (e == cudaSuccess && (flags & RSLM_RESCORE_READING_A) && !(flags & RSLM_FULL_VECTOR)) {
+    // reading A scores <q, c> in the rescoring rotation: R2 c of every centroid
+    e = dev_alloc(ix, &ix->crot2, size_t(nlist) * ix->cs2.Dp);
+    if (e == cudaSuccess) e = launch_rotate_rows(ix->rot2, ix->centroids, nlist, ix->crot2, ix->cs2.Dp, s);
+  }
   if (e == cudaSuccess) e = cudaStreamSynchronize(s);
   if (e != cudaSuccess) {
     free_all(ix);

@@ -91,7 +91,7 @@ __global__ void scatter_pairs_kernel(const int32_t* __restrict__ probes, const f
     if (p < 0 || p >= nlist) continue;
     const int at = off[p] + atomicAdd(&fill[p], 1);
     lq[at] = int32_t(i / eff);
-    lcs[at] = cs[src];
+    lcs[at] = cs ? cs[src] : 0.0f;  // no cs: full-vector codes
   }
 }
 
@@ -172,7 +172,7 @@ __global__ void __launch_bounds__(1024) scatter_hist_kernel(const int32_t* __res
     if (p < 0 || p >= nlist) continue;
     const int at = atomicAdd(&base[p], 1);
     lq[at] = int32_t(i / eff);
-    lcs[at] = cs[src];
+    lcs[at] = cs ? cs[src] : 0.0f;  // no cs: full-vector codes
   }
 }
 
@@ -1654,8 +1654,9 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   int* fcounts = reinterpret_cast<int*>(ws + o_fcounts);
 
   // lists: L[0] the first probe of every query, L[1] all probe pairs
-  e = build_lists(ix, probes, cs, nq, nprobe, 1, L[0], s);
-  if (e == cudaSuccess) e = build_lists(ix, probes, cs, nq, nprobe, nprobe, L[1], s);
+  const float* lcs = (ix->flags & RSLM_FULL_VECTOR) ? nullptr : cs;  // full-vector codes: no <q, c> term
+  e = build_lists(ix, probes, lcs, nq, nprobe, 1, L[0], s);
+  if (e == cudaSuccess) e = build_lists(ix, probes, lcs, nq, nprobe, nprobe, L[1], s);
   if (e == cudaSuccess) {
     split_queries_kernel<<<blocks_for(nq, 8, 152 * 32), 256, 0, s>>>(qrot, nq, c1.Dp, Dp16, qhi, qlo,
                                                                       qinv);

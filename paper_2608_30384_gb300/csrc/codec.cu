@@ -58,6 +58,8 @@ struct EncodeArgs {
   int D;
   int global_scale;
   int stage2;
+  int full_vector;  // approximation 0 instead of the centroid (Sec. 3.5)
+  int reading_a;    // stage 2 against the stage-1 approximation, not its reconstruction
   int buflen;
 };
 
@@ -176,12 +178,14 @@ __global__ void encode_kernel(const __grid_constant__ EncodeArgs a) {
     const int p = a.assign[gid];
     const int64_t slot = a.slot_of_row[gid];
     const float* x = a.x + i * D;
+    // the stage-1 approximation: the centroid, or 0 for full-vector codes
     const float* c = a.centroids + int64_t(p) * D;
+    const double cw = a.full_vector ? 0.0 : 1.0;
 
     // ---- stage 1: residual against the centroid (Sec. 3.5, Sec. 5.5.1)
     double nr2 = 0.0, nx2 = 0.0;
     for (int d = lane; d < D; d += 32) {
-      const double xv = x[d], cv = c[d];
+      const double xv = x[d], cv = cw * c[d];
       const double r = xv - cv;
       A[d] = r;
       nr2 += r * r;
@@ -199,14 +203,14 @@ __global__ void encode_kernel(const __grid_constant__ EncodeArgs a) {
         [&](int b, uint32_t v) { tile[((b / ch) * kTile + rin) * ch + (b % ch)] = uint8_t(v); }, &Lh1);
     uint32_t Gu1 = one_ue4m12;
     double Gh1 = 1.0;
-    if (a.global_scale || a.stage2) {
+    if (a.global_scale || (a.stage2 && !a.reading_a)) {
       warp_rotate(A, T, a.rot1, tb1, true, lane);  // A = R^T uhat
     }
     if (a.global_scale) {
       // Sec. 3.5.2: G = ||x|| / ||c + Lhat R^T uhat||
       double na2 = 0.0;
       for (int d = lane; d < D; d += 32) {
-        const double v = double(c[d]) + Lh1 * A[d];
+        const double v = cw * double(c[d]) + Lh1 * A[d];
         na2 += v * v;
       }
       na2 = warp_sum(na2);
@@ -232,10 +236,11 @@ __global__ void encode_kernel(const __grid_constant__ EncodeArgs a) {
     }
     if (!a.stage2) continue;
 
-    // ---- stage 2: residual against the full stage-1 reconstruction (Sec. 5.2)
+    // ---- stage 2: residual against the full stage-1 reconstruction (Sec.
+    // 5.2), or against the stage-1 approximation itself (reading A)
     double nr2b = 0.0;
     for (int d = lane; d < D; d += 32) {
-      const double ap = Gh1 * (double(c[d]) + Lh1 * A[d]);
+      const double ap = a.reading_a ? cw * double(c[d]) : Gh1 * (cw * double(c[d]) + Lh1 * A[d]);
       Ap[d] = ap;
       const double r = double(x[d]) - ap;
       A[d] = r;
@@ -356,6 +361,8 @@ cudaError_t launch_encode(const rslm_index* ix, const float* x, int64_t row_begi
   a.D = ix->D;
   a.global_scale = (ix->flags & RSLM_GLOBAL_SCALE) ? 1 : 0;
   a.stage2 = ix->rescore_bits ? 1 : 0;
+  a.full_vector = (ix->flags & RSLM_FULL_VECTOR) ? 1 : 0;
+  a.reading_a = (ix->flags & RSLM_RESCORE_READING_A) ? 1 : 0;
   int len = ix->D;
   if (ix->cs1.Dp > len) len = ix->cs1.Dp;
   if (ix->rescore_bits && ix->cs2.Dp > len) len = ix->cs2.Dp;

@@ -106,6 +106,7 @@ struct rslm_index {
   uint8_t* ctiles = nullptr;    // fused probe: centroids * 2^sC as fp16 operand tiles (D <= 128)
   float* cmeta = nullptr;       // fused probe: max|c|, max||c||^2, 2^sC, max||c|| 2^sC
   float* crows = nullptr;       // fused probe: centroids as fp32 rows of Kp floats
+  float* crot2 = nullptr;       // rescoring reading A: R2 c of every centroid [nlist * Dp2]
   void* cublas = nullptr;       // cublasHandle_t
   int64_t device_bytes = 0;
   // profiling of the dominant scan kernel

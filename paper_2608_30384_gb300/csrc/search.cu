@@ -464,7 +464,7 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
     const int t = it - tpref[j];
     const int64_t slot0 = a.part_off[p] + int64_t(t) * kTile;
     const int nvalid = min(kTile, a.part_n[p] - t * kTile);
-    const float csj = a.cs[q * a.probe_stride + j];
+    const float csj = a.cs ? a.cs[q * a.probe_stride + j] : 0.0f;  // no cs: full-vector codes
     const uint8_t* tp = a.codes + slot0 * a.stride;
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     uint32_t hb[4] = {0u, 0u, 0u, 0u};  // Rslm4Lite: UE7M9 | UE4M12 << 16 from the top bits
@@ -578,6 +578,11 @@ struct RescoreArgs {
   int stride2;
   int code_bytes2;
   float lv[16];
+  // <q, a2>: reading B the stage-1 score; reading A <R2 q, R2 c> of the row's
+  // partition (crot2, assign); 0 for full-vector codes (zero_a)
+  const float* crot2;
+  const int32_t* assign;
+  int zero_a;
   int64_t* out_ids;
   float* out_scores;
   int* err;
@@ -614,8 +619,16 @@ __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ Re
         }
         acc = warp_sum(acc);
         const uint32_t sc = __ldg(a.scales2 + slot);
-        const float s1 = a.cand_scores[q * a.k + j];
-        s2 = ue4m12_to_f32(sc >> 16) * fmaf(ue7m9_to_f32(sc & 0xffffu), acc, s1);
+        float a2 = a.cand_scores[q * a.k + j];  // reading B: <q, a2> = s1
+        if (a.zero_a) {
+          a2 = 0.0f;
+        } else if (a.crot2) {
+          const float* cr = a.crot2 + int64_t(a.assign[cid]) * a.Dp2;
+          float c = 0.0f;
+          for (int d = lane; d < a.Dp2; d += 32) c = fmaf(q2[d], __ldg(cr + d), c);
+          a2 = warp_sum(c);
+        }
+        s2 = ue4m12_to_f32(sc >> 16) * fmaf(ue7m9_to_f32(sc & 0xffffu), acc, a2);
         id = cid;
       }
     }
@@ -698,7 +711,7 @@ cudaError_t launch_scan_impl(const rslm_index* ix, const float* qrot, int64_t nq
   a.qrot = qrot;
   a.Dp = ix->cs1.Dp;
   a.probes = probes;
-  a.cs = cs;
+  a.cs = (ix->flags & RSLM_FULL_VECTOR) ? nullptr : cs;
   a.nprobe = nprobe;
   a.probe_stride = probe_stride;
   a.only_if = only_if;
@@ -770,6 +783,10 @@ cudaError_t launch_rescore(const rslm_index* ix, const float* qrot2, int64_t nq,
   a.stride2 = ix->cs2.stride;
   a.code_bytes2 = ix->cs2.code_bytes;
   for (int i = 0; i < 16; ++i) a.lv[i] = ix->cs2.cbf[i];
+  const bool reading_a = (ix->flags & RSLM_RESCORE_READING_A) != 0;
+  a.zero_a = reading_a && (ix->flags & RSLM_FULL_VECTOR) ? 1 : 0;
+  a.crot2 = reading_a ? ix->crot2 : nullptr;
+  a.assign = ix->assign;
   a.out_ids = out_ids;
   a.out_scores = out_scores;
   a.err = ix->d_err;

@@ -13,10 +13,14 @@ class Index:
     """
 
     def __init__(self, centroids, score_bits: int, rescore_bits: int = 0, global_scale: bool = True,
-                 stream=None, lite: bool = False):
+                 stream=None, lite: bool = False, reading: str = "B", full_vector: bool = False):
         nlist, dim = centroids.shape
         self.device = centroids.device
-        flags = (B.RSLM_GLOBAL_SCALE if global_scale else 0) | (B.RSLM_LITE if lite else 0)
+        if reading not in ("A", "B"):
+            raise ValueError("reading is 'A' or 'B'")
+        flags = ((B.RSLM_GLOBAL_SCALE if global_scale else 0) | (B.RSLM_LITE if lite else 0)
+                 | (B.RSLM_RESCORE_READING_A if reading == "A" else 0)
+                 | (B.RSLM_FULL_VECTOR if full_vector else 0))
         self.handle = B.rslm_index_create(dim, nlist, centroids.contiguous(), score_bits, rescore_bits,
                                           flags, stream)
 

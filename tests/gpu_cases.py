@@ -26,22 +26,26 @@ def ue_near_tie(v, fmt: K.UEFormat, rel: float = 1e-9) -> np.ndarray:
 class Case:
     """A workload, its oracle index and (lazily) its GPU index."""
 
-    def __init__(self, w: W.Workload, nq: int | None = None, global_scale: bool = True, lite: bool = False):
+    def __init__(self, w: W.Workload, nq: int | None = None, global_scale: bool = True, lite: bool = False,
+                 reading: str = "B", full_vector: bool = False):
         self.w = w
         self.X, self.A = W.database(w)
         self.C = W.ivf_centroids(w, self.X, self.A)
         self.Q = W.queries(w, nq)
         self.global_scale = global_scale
         self.lite = lite
+        self.reading = reading
+        self.full_vector = full_vector
         self.oracle = search.build_index(self.X, np.arange(w.N), self.A, self.C, w.bits,
-                                         w.rescore_bits, global_scale=global_scale, lite=lite)
+                                         w.rescore_bits, global_scale=global_scale, lite=lite,
+                                         reading=reading, full_vector=full_vector)
         self._gpu = None
 
     def gpu_index(self, encode: bool = True):
         import torch
         from paper_2608_30384_gb300 import Index
         ix = Index(torch.from_numpy(self.C).cuda(), self.w.bits, self.w.rescore_bits, self.global_scale,
-                   lite=self.lite)
+                   lite=self.lite, reading=self.reading, full_vector=self.full_vector)
         ix.reserve(torch.from_numpy(self.A).cuda())
         if encode:
             ix.encode(torch.from_numpy(self.X).cuda(), 0)
@@ -60,6 +64,14 @@ class Case:
                             torch.from_numpy(s2.L_u16.astype(np.uint16)).cuda(),
                             torch.from_numpy(s2.G_u16.astype(np.uint16)).cuda())
         torch.cuda.synchronize()
+
+    def approximations(self):
+        """The stage-1 and stage-2 approximations of every row (float64)."""
+        A1 = self.C[self.A].astype(np.float64)
+        if self.full_vector:
+            A1 = np.zeros_like(A1)
+        A2 = A1 if self.reading == "A" else self.oracle.stage1.recon
+        return A1, A2
 
     # ---------------------------------------------------------- references
     def qnorm(self, i):

@@ -80,7 +80,7 @@ def _encode_check(case):
     ix = case.gpu_index()
     w = case.w
     c1, L1, G1 = (t.cpu().numpy() for t in ix.export_codes(1))
-    A1 = case.C[case.A].astype(np.float64)
+    A1, A2 = case.approximations()
     ok = check_stage(c1, L1, G1, case.oracle.stage1, case.X, A1, w.bits, case.global_scale, "stage 1")
     if w.rescore_bits:
         c2, L2, G2 = (t.cpu().numpy() for t in ix.export_codes(2))
@@ -89,7 +89,7 @@ def _encode_check(case):
         sub = codec.Encoded(st2.bits, st2.mode, st2.D, st2.g, st2.codes[sel], st2.L_u16[sel],
                             st2.G_u16[sel], st2.Lhat[sel], st2.Ghat[sel], st2.uhat[sel], st2.u[sel],
                             st2.recon[sel], st2.L_exact[sel], st2.G_exact[sel])
-        check_stage(c2[sel], L2[sel], G2[sel], sub, case.X[sel], case.oracle.stage1.recon[sel],
+        check_stage(c2[sel], L2[sel], G2[sel], sub, case.X[sel], A2[sel],
                      w.rescore_bits, case.global_scale, "stage 2")
     return ix
 
@@ -250,6 +250,28 @@ def test_batched_scan_many_queries_per_partition(bits, D):
     K chunks (D = 300: a partial last chunk)."""
     _scan_parity(Case(Wl(f"mq{bits}", 20_000, D, 8, 0.5, False, 0.5, "mean", 600, bits, 0, 3, 10, 10,
                          seed=13 + bits)), batched=True)
+
+
+# ---------------------------------------------- relative-mode variants
+# Rescoring reading A (codes of x - c, scored with <q, c>) and full-vector
+# codes (approximation 0), Sec. 3.5 / Sec. 5.2.  C2-like: 2-bit scoring,
+# 4-bit rescoring, D = 96 (two FWHT blocks).
+REL = Wl("rel", 20_000, 96, 16, 0.5, False, 0.5, "mean", 40, 2, 4, 4, 60, 10, seed=41)
+
+
+@pytest.mark.parametrize("reading,full_vector", [("A", False), ("B", True), ("A", True)])
+def test_relative_variants_encode_parity(reading, full_vector):
+    _encode_check(Case(REL, reading=reading, full_vector=full_vector))
+
+
+@pytest.mark.parametrize("reading,full_vector", [("A", False), ("B", True), ("A", True)])
+@pytest.mark.parametrize("batched", [False, True])
+def test_relative_variants_scan_and_rescore_parity(reading, full_vector, batched):
+    """Stage 1 ignores <q, c> for full-vector codes; rescoring reading A
+    adds <q, c> of the row's partition (from the rotated centroids)."""
+    case = Case(REL, reading=reading, full_vector=full_vector)
+    _scan_parity(case, batched=batched)
+    test_rescore_parity_on_oracle_codes(case)
 
 
 # ------------------------------------------------------------- Rslm4Lite
