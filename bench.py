@@ -71,6 +71,9 @@ def parse_args():
                     help="scan form; auto = rslm_search's rule (batched when nq*nprobe >= 16*nlist)")
     ap.add_argument("--lite", action="store_true",
                     help="Rslm4Lite scoring codes (4-bit workloads, D >= 64): scales in the codes' top bits")
+    ap.add_argument("--reading", default="B", choices=["A", "B"],
+                    help="rescoring approximation: B the stage-1 reconstruction (default), A the centroid")
+    ap.add_argument("--full-vector", action="store_true", help="codes of x itself (approximation 0)")
     args = ap.parse_args()
     if args.lite:
         w = W.WORKLOADS[args.config]
@@ -79,9 +82,11 @@ def parse_args():
     return args
 
 
-def workload_label(w: W.Workload, lite: bool = False) -> str:
-    if lite:
-        return f"{w.name} with Rslm4Lite scoring codes: {w.description}"
+def workload_label(w: W.Workload, lite: bool = False, reading: str = "B", full_vector: bool = False) -> str:
+    mods = (["Rslm4Lite scoring codes"] if lite else []) + (["full-vector codes"] if full_vector else []) \
+        + (["rescoring reading A"] if reading == "A" and w.rescore_bits else [])
+    if mods:
+        return f"{w.name} with {', '.join(mods)}: {w.description}"
     return f"{w.name}: {w.description}"
 
 
@@ -193,7 +198,8 @@ def dist_setup(args):
 
 
 # --------------------------------------------------------- oracle (CPU) leg
-def oracle_sample(w: W.Workload, A, C, Q, n_queries: int, lite: bool = False):
+def oracle_sample(w: W.Workload, A, C, Q, n_queries: int, lite: bool = False, reading: str = "B",
+                  full_vector: bool = False):
     """Oracle index over the rows of the partitions the sample queries probe
     (those rows are regenerated from their seeds)."""
     from oracle import search as osearch
@@ -201,7 +207,8 @@ def oracle_sample(w: W.Workload, A, C, Q, n_queries: int, lite: bool = False):
     parts = np.unique(probes)
     rows = np.nonzero(np.isin(A, parts))[0]
     X, _ = W.rows(w, rows)
-    index = osearch.build_index(X, rows, A[rows], C, w.bits, w.rescore_bits, lite=lite)
+    index = osearch.build_index(X, rows, A[rows], C, w.bits, w.rescore_bits, lite=lite,
+                                reading=reading if w.rescore_bits else "B", full_vector=full_vector)
     sizes = np.bincount(A, minlength=w.P)
     cand = int(sizes[probes].sum())
     return index, cand, len(rows)
@@ -239,7 +246,7 @@ def run_reference(args):
     C = W.ivf_centroids(w)
     nqs = min(SAMPLE_QUERIES[w.name], w.nq)
     Q = W.queries(w, nqs)
-    index, cand, nrows = oracle_sample(w, A, C, Q, nqs, args.lite)
+    index, cand, nrows = oracle_sample(w, A, C, Q, nqs, args.lite, args.reading, args.full_vector)
     for _ in range(args.warmup):
         oracle_time(w, index, Q, nqs, cand, 0.0)
     t0 = time.perf_counter()
@@ -252,7 +259,7 @@ def run_reference(args):
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": dt * 1e3 / args.steps,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic", "config": {"workload": workload_label(w, args.lite), "nq_per_step": nqs},
+            "data": "synthetic", "config": {"workload": workload_label(w, args.lite, args.reading, args.full_vector), "nq_per_step": nqs},
             "cpu_baseline": {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                              "sample": sample},
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
@@ -307,7 +314,8 @@ def run_gpu(args):
     nq = w.nq
 
     # index build (not timed as part of the step)
-    ix = Index(torch.from_numpy(C).to(dev), w.bits, w.rescore_bits, lite=args.lite)
+    ix = Index(torch.from_numpy(C).to(dev), w.bits, w.rescore_bits, lite=args.lite,
+               reading=args.reading if w.rescore_bits else "B", full_vector=args.full_vector)
     ix.reserve(torch.from_numpy(A).to(dev))
     torch.cuda.synchronize()
     encode_s = 0.0
@@ -455,7 +463,7 @@ def run_gpu(args):
     cpu = None
     if rank == 0 and ws == 1 and not args.no_cpu_baseline:
         nqs = min(SAMPLE_QUERIES[w.name], nq)
-        index, cand, nrows = oracle_sample(w, A, C, Q, nqs, args.lite)
+        index, cand, nrows = oracle_sample(w, A, C, Q, nqs, args.lite, args.reading, args.full_vector)
         cval, passes, dt = oracle_time(w, index, Q, nqs, cand, args.cpu_seconds)
         cpu = {"value": cval, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle",
                "sample": f"{nqs} of the {nq} queries of {w.name} ({cand} candidates per pass) x {passes} "
@@ -467,7 +475,7 @@ def run_gpu(args):
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": ws, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_per_step, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": workload_label(w, args.lite), "nq": nq, "nprobe": w.nprobe, "k": w.k,
+            "config": {"workload": workload_label(w, args.lite, args.reading, args.full_vector), "nq": nq, "nprobe": w.nprobe, "k": w.k,
                        "k_final": w.k_final, "score_bits": w.bits, "rescore_bits": w.rescore_bits,
                        "l2": (f"L2 flushed between timed steps (a {4 * L2_BYTES / 1e6:.0f} MB buffer "
                               f"overwritten, not timed): the {(scan_bytes_index(desc) + rescore_bytes_index(desc)) / 1e6:.0f}"
