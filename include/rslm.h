@@ -244,6 +244,20 @@ rslm_status rslm_import_codes(rslm_index* index, int32_t which, int64_t row_begi
                               const uint8_t* codes, const uint16_t* local_scale,
                               const uint16_t* global_scale, void* stream);
 
+/* Decompression (Sec. 4; the inverse of the codec): the reconstructions of
+ * rows [row_begin, row_begin + rows) from the stored codes and scales of
+ * stage `which` (1: scoring, 2: rescoring), computed in float64 and written
+ * to out: device [rows * dim] float32, row-major.
+ *   which = 1: Ghat (a + Lhat R^T uhat) with a = the row's centroid (0 for
+ *     RSLM_FULL_VECTOR);
+ *   which = 2: Ghat2 (a2 + Lhat2 R2^T uhat2) with a2 = the stage-1
+ *     reconstruction, or the stage-1 approximation with
+ *     RSLM_RESCORE_READING_A.
+ * Errors: RSLM_ERR_INVALID_ARG (bad which, range, NULL out),
+ * RSLM_ERR_STATE before rslm_index_reserve.  Asynchronous on `stream`. */
+rslm_status rslm_decompress(const rslm_index* index, int32_t which, int64_t row_begin, int64_t rows,
+                            float* out, void* stream);
+
 /* Codebook of a bit rate (Sec. 3.2) as the library uses it: host out
  * [K * g] float32 values (binary16-exact), K = 16.  *K_out, *g_out: host.
  * Needs no GPU. */

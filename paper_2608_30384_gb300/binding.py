@@ -46,6 +46,7 @@ SIGNATURES = {
     "rslm_e_max": (ctypes.c_int, [_I32, ctypes.POINTER(_D)]),
     "rslm_profile_enable": (ctypes.c_int, [_P, _I32]),
     "rslm_profile_read": (ctypes.c_int, [_P, ctypes.POINTER(_D), ctypes.POINTER(_I64), _P, _I32]),
+    "rslm_decompress": (ctypes.c_int, [_P, _I32, _I64, _I64, _P, _P]),
     "rslm_sync": (ctypes.c_int, [_P, _P]),
     "rslm_last_error": (ctypes.c_char_p, []),
     "rslm_index_destroy": (None, [_P]),
@@ -264,6 +265,14 @@ def rslm_e_max(dim) -> float:
 
 def rslm_profile_enable(index, on=True):
     _check(lib().rslm_profile_enable(_ptr(index), int(bool(on))))
+
+
+def rslm_decompress(index, which, row_begin, rows, out, stream=None):
+    """Reconstructions of rows [row_begin, row_begin + rows) of stage ``which`` into out [rows, dim]."""
+    import torch
+    dim = rslm_index_describe(index)["dim"]
+    _check(lib().rslm_decompress(_ptr(index), which, row_begin, rows,
+                                 _dev(out, torch.float32, "out", rows * dim), _stream(stream)))
 
 
 def rslm_profile_read(index):

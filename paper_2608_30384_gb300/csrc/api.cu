@@ -488,6 +488,18 @@ rslm_status rslm_export_codes(const rslm_index* ix, int32_t which, int64_t row_b
   return RSLM_OK;
 }
 
+rslm_status rslm_decompress(const rslm_index* ix, int32_t which, int64_t row_begin, int64_t rows, float* out,
+                            void* stream) {
+  RSLM_ARG(ix, "index is NULL");
+  RSLM_ARG(which == 1 || (which == 2 && ix->rescore_bits), "which must be 1, or 2 with rescoring codes");
+  if (!ix->slot_of_row) return fail(RSLM_ERR_STATE, "rslm_index_reserve has not been called");
+  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin + rows <= ix->n_rows, "row range out of bounds");
+  RSLM_ARG(rows == 0 || out, "NULL array");
+  DeviceGuard g(ix->device);
+  RSLM_CK(launch_decompress(ix, which, row_begin, rows, out, as_stream(stream)), "decompress launch");
+  return RSLM_OK;
+}
+
 rslm_status rslm_import_codes(rslm_index* ix, int32_t which, int64_t row_begin, int64_t rows,
                               const uint8_t* codes, const uint16_t* local_scale,
                               const uint16_t* global_scale, void* stream) {

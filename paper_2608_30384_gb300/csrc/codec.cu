@@ -270,6 +270,88 @@ __global__ void encode_kernel(const __grid_constant__ EncodeArgs a) {
   }
 }
 
+// Decompression (Sec. 4, the inverse of the codec): the reconstruction
+// Ghat (a + Lhat R^T uhat) of each row from its stored codes and scales, in
+// float64 like the encoder, written as float32.  Stage 1: a = the centroid
+// (0 for full-vector codes).  Stage 2: a = the stage-1 reconstruction
+// (reading B) or the stage-1 approximation (reading A).  One warp per row.
+struct DecompArgs {
+  RotSpec rot1, rot2;
+  CodecSpec cs1, cs2;
+  int64_t row_begin, rows;
+  const float* centroids;
+  const int32_t* assign;
+  const int32_t* slot_of_row;
+  const uint8_t* codes1;  // tile-interleaved
+  const uint32_t* scales1;
+  const uint8_t* codes2;  // row-major
+  const uint32_t* scales2;
+  int D, which, full_vector, reading_a, buflen;
+  float* out;             // [rows * D]
+};
+
+// Codewords of a stored row into u[0, Dp) (zero beyond D); `byte(b)` reads
+// code byte b.
+template <typename Byte>
+__device__ __forceinline__ void decode_codewords(double* u, const CodecSpec& cs, int D, int lane, Byte byte) {
+  for (int g = lane; g < cs.ngroups; g += 32) {
+    const uint32_t code = (uint32_t(byte(g >> 1)) >> (4 * (g & 1))) & 15u;
+    if (g < cs.lite_h) {
+      u[g] = cs.cb8d[code & 7u];  // Rslm4Lite head: the top bit is a scale bit
+    } else {
+      for (int j = 0; j < cs.g; ++j) {
+        const int d = g * cs.g + j;
+        u[d] = d < D ? cs.cbd[code * cs.g + j] : 0.0;
+      }
+    }
+  }
+}
+
+__global__ void decompress_kernel(const __grid_constant__ DecompArgs a) {
+  extern __shared__ double dsm[];
+  __shared__ RotTables tb1, tb2;
+  load_rot_tables(&tb1, a.rot1);
+  load_rot_tables(&tb2, a.rot2);
+  __syncthreads();
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, W = blockDim.x >> 5;
+  double* U = dsm + size_t(warp) * 3 * a.buflen;
+  double* T = U + a.buflen;
+  double* R1 = T + a.buflen;  // stage-1 reconstruction
+  const int D = a.D;
+  const double cw = a.full_vector ? 0.0 : 1.0;
+  for (int64_t i = int64_t(blockIdx.x) * W + warp; i < a.rows; i += int64_t(gridDim.x) * W) {
+    const int64_t gid = a.row_begin + i;
+    const int64_t slot = a.slot_of_row[gid];
+    const float* c = a.centroids + int64_t(a.assign[gid]) * D;
+    const uint8_t* tile = a.codes1 + (slot >> 7) * kTile * a.cs1.stride;
+    const int rin = int(slot & 127), ch = a.cs1.chunk;
+    decode_codewords(U, a.cs1, D, lane,
+                     [&](int b) { return tile[((b / ch) * kTile + rin) * ch + (b % ch)]; });
+    __syncwarp();
+    warp_rotate(U, T, a.rot1, tb1, true, lane);  // R^T uhat
+    const uint32_t sc1 = a.scales1[slot];
+    const double Lh1 = ue_decode(sc1 & 0xffffu, 7, 9), Gh1 = ue_decode(sc1 >> 16, 4, 12);
+    for (int d = lane; d < D; d += 32) R1[d] = Gh1 * (cw * double(c[d]) + Lh1 * U[d]);
+    __syncwarp();
+    if (a.which == 1) {
+      for (int d = lane; d < D; d += 32) a.out[i * D + d] = float(R1[d]);
+      __syncwarp();
+      continue;
+    }
+    const uint8_t* row2 = a.codes2 + slot * a.cs2.stride;
+    decode_codewords(U, a.cs2, D, lane, [&](int b) { return row2[b]; });
+    __syncwarp();
+    warp_rotate(U, T, a.rot2, tb2, true, lane);
+    const uint32_t sc2 = a.scales2[slot];
+    const double Lh2 = ue_decode(sc2 & 0xffffu, 7, 9), Gh2 = ue_decode(sc2 >> 16, 4, 12);
+    for (int d = lane; d < D; d += 32) {
+      const double a2 = a.reading_a ? cw * double(c[d]) : R1[d];
+      a.out[i * D + d] = float(Gh2 * (a2 + Lh2 * U[d]));
+    }
+    __syncwarp();
+  }
+}
+
 struct ExportArgs {
   const int32_t* slot_of_row;
   int64_t row_begin, rows;
@@ -376,6 +458,44 @@ cudaError_t launch_encode(const rslm_index* ix, const float* x, int64_t row_begi
       cudaFuncSetAttribute(encode_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
   encode_kernel<<<grid_for(rows, warps, 152 * 16), warps * 32, smem, s>>>(a);
+  return cudaGetLastError();
+}
+
+cudaError_t launch_decompress(const rslm_index* ix, int which, int64_t row_begin, int64_t rows, float* out,
+                              cudaStream_t s) {
+  if (rows == 0) return cudaSuccess;
+  DecompArgs a;
+  a.rot1 = ix->rot1;
+  a.rot2 = ix->rescore_bits ? ix->rot2 : ix->rot1;
+  a.cs1 = ix->cs1;
+  a.cs2 = ix->rescore_bits ? ix->cs2 : ix->cs1;
+  a.row_begin = row_begin;
+  a.rows = rows;
+  a.centroids = ix->centroids;
+  a.assign = ix->assign;
+  a.slot_of_row = ix->slot_of_row;
+  a.codes1 = ix->codes1;
+  a.scales1 = ix->scales1;
+  a.codes2 = ix->codes2;
+  a.scales2 = ix->scales2;
+  a.D = ix->D;
+  a.which = which;
+  a.full_vector = (ix->flags & RSLM_FULL_VECTOR) ? 1 : 0;
+  a.reading_a = (ix->flags & RSLM_RESCORE_READING_A) ? 1 : 0;
+  a.out = out;
+  int len = ix->D;
+  if (ix->cs1.Dp > len) len = ix->cs1.Dp;
+  if (ix->rescore_bits && ix->cs2.Dp > len) len = ix->cs2.Dp;
+  a.buflen = (len + 3) / 4 * 4;
+  const size_t per_warp = size_t(3) * a.buflen * sizeof(double);
+  int warps = int((96 * 1024) / per_warp);
+  if (warps > 8) warps = 8;
+  if (warps < 1) warps = 1;
+  const size_t smem = per_warp * warps;
+  cudaError_t e =
+      cudaFuncSetAttribute(decompress_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  decompress_kernel<<<grid_for(rows, warps, 152 * 16), warps * 32, smem, s>>>(a);
   return cudaGetLastError();
 }
 

@@ -12,6 +12,10 @@ cudaError_t launch_rotate_rows(const RotSpec& rot, const float* in, int64_t n, f
                                cudaStream_t s);
 cudaError_t launch_encode(const rslm_index* ix, const float* x, int64_t row_begin, int64_t rows,
                           cudaStream_t s);
+// Reconstructions of rows [row_begin, row_begin + rows) from stage `which`'s
+// codes (codec.cu): [rows * D] float32.
+cudaError_t launch_decompress(const rslm_index* ix, int which, int64_t row_begin, int64_t rows, float* out,
+                              cudaStream_t s);
 cudaError_t launch_export_import(const rslm_index* ix, int which, int64_t row_begin, int64_t rows,
                                  uint8_t* codes, uint16_t* lscale, uint16_t* gscale, bool import,
                                  cudaStream_t s);

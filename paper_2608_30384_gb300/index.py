@@ -98,6 +98,15 @@ class Index:
         B.rslm_export_codes(self.handle, which, row_begin, rows, codes, L, G, stream)
         return codes, L, G
 
+    def decompress(self, which: int = 1, row_begin: int = 0, rows: int | None = None, stream=None):
+        """Reconstructed vectors [rows, dim] of stage ``which`` (float32)."""
+        import torch
+        d = self.desc
+        rows = d["n_rows"] - row_begin if rows is None else rows
+        out = torch.empty((rows, d["dim"]), dtype=torch.float32, device=self.device)
+        B.rslm_decompress(self.handle, which, row_begin, rows, out, stream)
+        return out
+
     def import_codes(self, which, row_begin, codes, L, G, stream=None):
         B.rslm_import_codes(self.handle, which, row_begin, codes.shape[0], codes.contiguous(),
                             L.contiguous(), G.contiguous(), stream)

@@ -252,6 +252,50 @@ def test_batched_scan_many_queries_per_partition(bits, D):
                          seed=13 + bits)), batched=True)
 
 
+# ------------------------------------------------------------ decompress
+def _decompress_check(case):
+    """rslm_decompress of both stages against the oracle's decode of the
+    GPU's own exported codes and scales (Sec. 4): equal up to the float32
+    rounding of the output."""
+    w = case.w
+    ix = case.gpu_index()
+    A1, _ = case.approximations()
+    c1, L1, G1 = (t.cpu().numpy().astype(np.int64) for t in ix.export_codes(1))
+    ng1 = case.oracle.stage1.codes.shape[1]
+    if case.lite:
+        ref1 = codec.decode_lite(A1, codec.unpack_nibbles(c1, w.D), w.D, case.global_scale)
+    else:
+        ref1 = codec.decode(A1, codec.unpack_nibbles(c1, ng1), L1, G1, w.bits, w.D)
+    tol = 1e-6 * float(np.abs(case.X).max()) + 1e-6
+    got1 = ix.decompress(1).cpu().numpy()
+    assert np.allclose(got1, ref1, rtol=1e-6, atol=tol), np.abs(got1 - ref1).max()
+    if w.rescore_bits:
+        c2, L2, G2 = (t.cpu().numpy().astype(np.int64) for t in ix.export_codes(2))
+        A2 = A1 if case.reading == "A" else ref1
+        ref2 = codec.decode(A2, codec.unpack_nibbles(c2, case.oracle.stage2.codes.shape[1]), L2, G2,
+                            w.rescore_bits, w.D)
+        got2 = ix.decompress(2).cpu().numpy()
+        assert np.allclose(got2, ref2, rtol=1e-6, atol=tol), np.abs(got2 - ref2).max()
+        # the rescoring reconstruction is closer to x than the scoring one
+        e1 = np.linalg.norm(got1 - case.X, axis=1).mean()
+        e2 = np.linalg.norm(got2 - case.X, axis=1).mean()
+        assert e2 < e1
+
+
+def test_decompress_parity(case):
+    _decompress_check(case)
+
+
+@pytest.mark.parametrize("kind", ["lite", "reading_a", "full_vector"])
+def test_decompress_parity_variants(kind):
+    if kind == "lite":
+        case = Case(Wl("dl", 6_000, 128, 8, 0.5, False, 0.5, "mean", 8, 4, 0, 3, 10, 10, seed=51), lite=True)
+    else:
+        case = Case(Wl("dv", 6_000, 96, 8, 0.5, False, 0.5, "mean", 8, 2, 4, 3, 40, 10, seed=52),
+                    reading="A" if kind == "reading_a" else "B", full_vector=kind == "full_vector")
+    _decompress_check(case)
+
+
 # ---------------------------------------------- relative-mode variants
 # Rescoring reading A (codes of x - c, scored with <q, c>) and full-vector
 # codes (approximation 0), Sec. 3.5 / Sec. 5.2.  C2-like: 2-bit scoring,
