@@ -74,6 +74,9 @@ def parse_args():
     ap.add_argument("--reading", default="B", choices=["A", "B"],
                     help="rescoring approximation: B the stage-1 reconstruction (default), A the centroid")
     ap.add_argument("--full-vector", action="store_true", help="codes of x itself (approximation 0)")
+    ap.add_argument("--recall", type=int, default=0, metavar="N",
+                    help="diagnostic: recall of the final top-k of the first N queries against exact "
+                         "float64 MIPS over the whole database (computed while the index is built)")
     args = ap.parse_args()
     if args.lite:
         w = W.WORKLOADS[args.config]
@@ -195,6 +198,39 @@ def dist_setup(args):
     if ws != args.gpus:
         raise SystemExit(f"--gpus {args.gpus} but WORLD_SIZE={ws}")
     return ws, rank, local
+
+
+# ------------------------------------------------------ recall diagnostic
+class ExactTopK:
+    """Exact maximum-inner-product top-k (float64, ties to the lower row id)
+    of a few queries over database rows streamed in blocks."""
+
+    def __init__(self, Q, k):
+        self.Q = np.asarray(Q, dtype=np.float64)
+        self.k = k
+        self.sc = np.full((len(Q), 0), -np.inf)
+        self.ids = np.zeros((len(Q), 0), dtype=np.int64)
+
+    def add(self, X, lo):
+        S = self.Q @ np.asarray(X, dtype=np.float64).T
+        ids = np.broadcast_to(np.arange(lo, lo + X.shape[0]), S.shape)
+        sc = np.concatenate([self.sc, S], axis=1)
+        ii = np.concatenate([self.ids, ids], axis=1)
+        keep = np.argpartition(-sc, min(self.k, sc.shape[1] - 1), axis=1)[:, :self.k + 1] \
+            if sc.shape[1] > self.k + 1 else np.tile(np.arange(sc.shape[1]), (len(sc), 1))
+        sc = np.take_along_axis(sc, keep, 1)
+        ii = np.take_along_axis(ii, keep, 1)
+        o = np.lexsort((ii, -sc), axis=1)[:, :self.k]
+        self.sc = np.take_along_axis(sc, o, 1)
+        self.ids = np.take_along_axis(ii, o, 1)
+
+    def recall(self, found):
+        """Recall@k@k (share of the exact top k returned) and Recall@1@k."""
+        n = len(self.Q)
+        rk = np.mean([len(set(found[i].tolist()) & set(self.ids[i].tolist())) / self.k for i in range(n)])
+        r1 = np.mean([self.ids[i, 0] in set(found[i].tolist()) for i in range(n)])
+        return {"queries": n, "k": self.k, "recall_k_at_k": float(rk), "recall_1_at_k": float(r1),
+                "exact": "float64 maximum inner product over every database row"}
 
 
 # --------------------------------------------------------- oracle (CPU) leg
@@ -319,6 +355,7 @@ def run_gpu(args):
     ix.reserve(torch.from_numpy(A).to(dev))
     torch.cuda.synchronize()
     encode_s = 0.0
+    exact = ExactTopK(Q[:args.recall], w.k_final) if args.recall else None
     for lo, X in W.row_blocks(w, 1 << 20):
         Xd = torch.from_numpy(X).to(dev)
         torch.cuda.synchronize()
@@ -327,6 +364,8 @@ def run_gpu(args):
         ix.sync()
         encode_s += time.perf_counter() - t0
         del Xd
+        if exact is not None:
+            exact.add(X, lo)
     desc = ix.desc
 
     Qd = torch.from_numpy(Q).to(dev)
@@ -497,6 +536,8 @@ def run_gpu(args):
             "e2e": e2e,
             "gpu_launches": launches_per_step(w, nq, batched) * args.steps,
             "clocks": clocks,
+            "recall": (exact.recall((f_ids if w.rescore_bits else s1_ids)[:args.recall].cpu().numpy())
+                       if exact is not None else None),
         }
         print(json.dumps(line), flush=True)
     if ws > 1:
