@@ -281,6 +281,32 @@ def unpack_nibbles(packed: np.ndarray, ngroups: int) -> np.ndarray:
     return out
 
 
+def pack_bits3(codes: np.ndarray) -> np.ndarray:
+    """(n, ngroups) codes < 8 -> (n, ceil(3 ngroups / 8)) uint8: Rslm3's 3-bit
+    stream, code i at bits 3i .. 3i + 2 (least significant bit first), byte j
+    holding stream bits 8j .. 8j + 7."""
+    codes = np.asarray(codes, dtype=np.int64)
+    n, ng = codes.shape
+    nb = (3 * ng + 7) // 8
+    out = np.zeros((n, nb), dtype=np.int64)
+    for i in range(ng):
+        for t in range(3):
+            bit = 3 * i + t
+            out[:, bit // 8] |= ((codes[:, i] >> t) & 1) << (bit % 8)
+    return out.astype(np.uint8)
+
+
+def unpack_bits3(packed: np.ndarray, ngroups: int) -> np.ndarray:
+    """Inverse of ``pack_bits3``."""
+    packed = np.asarray(packed, dtype=np.int64)
+    out = np.zeros((packed.shape[0], ngroups), dtype=np.int64)
+    for i in range(ngroups):
+        for t in range(3):
+            bit = 3 * i + t
+            out[:, i] |= ((packed[:, bit // 8] >> (bit % 8)) & 1) << t
+    return out
+
+
 def bytes_per_vector(D: int, bits: int, n_scales: int = 1) -> int:
     """Packed size: ceil(D b / 8) code bytes plus 2 bytes per stored scale."""
     return math.ceil(D * bits / 8) + 2 * n_scales

@@ -188,3 +188,30 @@ def test_empty_partition_and_fewer_candidates_than_k():
     assert res["ids"][0].tolist() == [-1] * 10
     res = search.search(idx, q, nprobe=4, k=20)
     assert (res["ids"][0] >= 0).sum() == 12
+
+
+# --------------------------------------------------------------- Rslm3
+def test_rslm3_packing_by_hand_and_round_trip():
+    """Rslm3 (Sec. 3.4: 3 bits per dimension, K = 8) packs 8 codes into 3
+    bytes, least significant bit first: codes 1, 2, 3, 4, 5, 6, 7, 0 give
+    the stream 001 010 011 100 101 110 111 000 read from bit 0 upwards."""
+    codes = np.array([[1, 2, 3, 4, 5, 6, 7, 0]])
+    packed = codec.pack_bits3(codes)
+    bits = "".join(format(int(b), "08b")[::-1] for b in packed[0])  # bit 0 first
+    assert bits == "".join(format(c, "03b")[::-1] for c in codes[0])
+    assert packed.shape == (1, 3)
+    rng = np.random.default_rng(3)
+    for ng in (1, 7, 8, 100, 128, 1536):
+        c = rng.integers(0, 8, (5, ng))
+        p = codec.pack_bits3(c)
+        assert p.shape[1] == (3 * ng + 7) // 8 == codec.bytes_per_vector(ng, 3, 0)
+        assert np.array_equal(codec.unpack_bits3(p, ng), c)
+
+
+def test_rslm3_codes_are_the_nearest_of_eight_levels():
+    X, C, a = _data(200, 128, seed=17)
+    enc = codec.encode(X, C[a], 3)
+    lv = K.codebook(3).C[:, 0]
+    d = np.abs(enc.u[:, :, None] - lv[None, None, :])
+    assert enc.codes.max() < 8
+    assert np.array_equal(enc.codes, np.argmin(d, axis=-1))
