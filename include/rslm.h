@@ -100,7 +100,8 @@ typedef struct {
   int32_t rescore_bits;   /* 0 or 4 */
   int32_t group;          /* g: coordinates per 4-bit code (4, 2, 1 for b = 1, 2, 4) */
   int32_t padded_dim;     /* D' = g * ceil(D / g): width of a rotated scoring query */
-  int32_t code_bytes;     /* ceil(D' / g / 2): canonical scoring-code bytes per row */
+  int32_t code_bytes;     /* canonical scoring-code bytes per row: ceil(D' / g / 2)
+                             (ceil(3 D / 8) for score_bits = 3) */
   int32_t rescore_group;
   int32_t rescore_padded_dim;
   int32_t rescore_code_bytes;
@@ -117,7 +118,10 @@ typedef struct {
  *   afterwards).  They are the approximations a of the first stage (IVF
  *   centroids, Sec. 5.5.1).
  * score_bits: bits per dimension of the scoring codes: 1 (4-D codebook,
- *   K = 16), 2 (2-D, K = 16) or 4 (1-D, K = 16) (Sec. 3.2, Table "Rslm Codec
+ *   K = 16), 2 (2-D, K = 16), 3 (1-D, K = 8: Rslm3, eight codes packed in
+ *   3 bytes, code i at bits 3i .. 3i + 2 of the row's byte stream, least
+ *   significant bit first; scanned by the single-query kernel in both
+ *   regimes) or 4 (1-D, K = 16) (Sec. 3.2, Table "Rslm Codec
  *   Specifications").
  * rescore_bits: 0 (no rescoring) or 4: bits of the rescoring codes, which
  *   quantize x - a2 with a2 the full first-stage reconstruction (Sec. 5.2).
@@ -231,7 +235,7 @@ rslm_status rslm_search(const rslm_index* index, const float* queries, int64_t n
 /* Canonical codes of rows [row_begin, row_begin + rows): which = 1 scoring,
  * 2 rescoring.  codes: device [rows * code_bytes] uint8, row-major by row id,
  * the code of group i in the low nibble of byte i/2 when i is even, the high
- * nibble when odd.  Code values index the codebook in ascending order (1-D)
+ * nibble when odd (3-bit codes: bits 3i .. 3i + 2 of the row's byte stream).  Code values index the codebook in ascending order (1-D)
  * or in lexicographic codeword order (2-D, 4-D).  local_scale / global_scale:
  * device [rows] uint16 (UE7M9 / UE4M12 codes). */
 rslm_status rslm_export_codes(const rslm_index* index, int32_t which, int64_t row_begin,

@@ -166,7 +166,7 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
   *out = nullptr;
   RSLM_ARG(dim >= 1 && dim <= kMaxDim, "dim must be in [1, 4096]");
   RSLM_ARG(nlist >= 1, "nlist must be >= 1");
-  RSLM_ARG(score_bits == 1 || score_bits == 2 || score_bits == 4, "score_bits must be 1, 2 or 4");
+  RSLM_ARG(score_bits >= 1 && score_bits <= 4, "score_bits must be 1, 2, 3 or 4");
   RSLM_ARG(rescore_bits == 0 || rescore_bits == 4, "rescore_bits must be 0 or 4");
   RSLM_ARG((flags & ~(RSLM_GLOBAL_SCALE | RSLM_LITE | RSLM_RESCORE_READING_A | RSLM_FULL_VECTOR)) == 0,
            "unknown flag bits");

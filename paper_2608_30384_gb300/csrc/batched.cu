@@ -1597,6 +1597,8 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
                                 const int32_t* probes, const float* cs, int nprobe, int k,
                                 int64_t* out_ids, float* out_scores, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
+  // Rslm3's 3-bit rows have no tensor-core decode: the single-query scan serves them
+  if (ix->cs1.bits == 3) return launch_scan(ix, qrot, nq, probes, cs, nprobe, k, k, out_ids, out_scores, s);
   const CodecSpec& c1 = ix->cs1;
   const int Dp16 = (c1.Dp + 15) / 16 * 16;
   const int nlist = ix->nlist;

@@ -110,7 +110,23 @@ __device__ uint32_t quantize_stage(double* A, double* tmp, const RotSpec& rs, co
   const double f = m > 0.0 ? cs.emax / m : 0.0;
   for (int d = lane; d < cs.Dp; d += 32) A[d] = d < D ? A[d] * f : 0.0;
   __syncwarp();
-  for (int b = lane; b < cs.code_bytes; b += 32) {
+  if (cs.bits == 3) {
+    // Rslm3 (g = 1, K = 8): eight codes per 3 bytes, code i at stream bits 3i ..
+    for (int o = lane; o * 8 < cs.ngroups; o += 32) {
+      uint32_t v = 0;
+      for (int i = 0; i < 8; ++i) {
+        const int gi = 8 * o + i;
+        if (gi < cs.ngroups) {
+          const int c = nearest_code(A + gi, cs, ct);
+          v |= uint32_t(c) << (3 * i);
+          A[gi] = ct.cb[c];
+        }
+      }
+      for (int t = 0; t < 3; ++t)
+        if (3 * o + t < cs.code_bytes) put(3 * o + t, (v >> (8 * t)) & 255u);
+    }
+  }
+  for (int b = lane; cs.bits != 3 && b < cs.code_bytes; b += 32) {
     const int g0 = 2 * b, g1 = 2 * b + 1;
     if (g0 < cs.lite_h) {
       // Rslm4Lite head (g = 1, lite_h even): the K = 8 levels; the top bits
@@ -295,7 +311,14 @@ struct DecompArgs {
 template <typename Byte>
 __device__ __forceinline__ void decode_codewords(double* u, const CodecSpec& cs, int D, int lane, Byte byte) {
   for (int g = lane; g < cs.ngroups; g += 32) {
-    const uint32_t code = (uint32_t(byte(g >> 1)) >> (4 * (g & 1))) & 15u;
+    uint32_t code;
+    if (cs.bits == 3) {  // Rslm3: bits 3g .. 3g + 2 of the byte stream
+      const int bit = 3 * g, b0 = bit >> 3;
+      const uint32_t two = uint32_t(byte(b0)) | (b0 + 1 < cs.code_bytes ? uint32_t(byte(b0 + 1)) << 8 : 0u);
+      code = (two >> (bit & 7)) & 7u;
+    } else {
+      code = (uint32_t(byte(g >> 1)) >> (4 * (g & 1))) & 15u;
+    }
     if (g < cs.lite_h) {
       u[g] = cs.cb8d[code & 7u];  // Rslm4Lite head: the top bit is a scale bit
     } else {

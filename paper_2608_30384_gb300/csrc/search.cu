@@ -389,7 +389,7 @@ __device__ __forceinline__ uint32_t nibble_tops(uint32_t w) {
   return (t | (t >> 12)) & 0xFFu;
 }
 
-template <int CH>
+template <int CH, bool B3>
 __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanArgs a) {
   extern __shared__ __align__(16) uint8_t ssm[];
   __shared__ int scratch[32];
@@ -417,7 +417,14 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   // code's shared-memory address is then (block << 8) | (64 k + 4 code):
   // one byte permute per code builds it (see the scan loop).
   const float* qr = a.qrot + q * a.Dp;
-  for (int e = tid; e < a.lut_groups * 16; e += blockDim.x) {
+  if constexpr (B3) {
+    // Rslm3: T[position][code] at lut[8 position + code]
+    for (int e = tid; e < a.lut_groups * 8; e += blockDim.x) {
+      const int pos = e >> 3;
+      lut[e] = pos < a.ngroups ? qr[pos] * a.cb[e & 7] : 0.0f;
+    }
+  }
+  for (int e = tid; !B3 && e < a.lut_groups * 16; e += blockDim.x) {
     const int grp = e >> 4, code = e & 15;
     float v = 0.0f;
     if (grp < a.lite_h)
@@ -468,7 +475,29 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
     const uint8_t* tp = a.codes + slot0 * a.stride;
     float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     uint32_t hb[4] = {0u, 0u, 0u, 0u};  // Rslm4Lite: UE7M9 | UE4M12 << 16 from the top bits
-    for (int c = 0; c < nch; ++c) {
+    if constexpr (B3) {
+      // Rslm3: 32 codes per three words (chunks of 4 bytes), code k at bits
+      // 3k .. 3k + 2 of the 96-bit group
+      for (int g3 = 0; g3 < nch / 3; ++g3) {
+        uint32_t w[4][3];
+#pragma unroll
+        for (int r = 0; r < 4; ++r)
+#pragma unroll
+          for (int t = 0; t < 3; ++t)
+            w[r][t] = __ldg(reinterpret_cast<const uint32_t*>(tp + (size_t(3 * g3 + t) * kTile + r * 32 + lane) * 4));
+        const float* lg = lut + g3 * 32 * 8;
+#pragma unroll
+        for (int kk = 0; kk < 32; ++kk) {
+          const int bit = 3 * kk, wi = bit >> 5, sh = bit & 31;
+#pragma unroll
+          for (int r = 0; r < 4; ++r) {
+            const uint32_t code = sh <= 29 ? (w[r][wi] >> sh) & 7u : __funnelshift_r(w[r][wi], w[r][wi + 1], sh) & 7u;
+            acc[r] += lg[kk * 8 + int(code)];
+          }
+        }
+      }
+    }
+    for (int c = 0; !B3 && c < nch; ++c) {
       uint32_t w[4][CH / 4];
 #pragma unroll
       for (int r = 0; r < 4; ++r)
@@ -645,17 +674,17 @@ __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ Re
   }
 }
 
-template <int CH>
+template <int CH, bool B3>
 cudaError_t launch_scan_ch(const rslm_index* ix, const ScanArgs& a, int64_t nq, size_t smem,
                            cudaStream_t s) {
   // listed queries: a fixed grid strides over the list, whose length is on the device
   const int64_t grid = a.qlist ? (nq < 2 * 152 ? nq : 2 * 152) : nq;
-  cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH, B3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        int(smem));
   if (e != cudaSuccess) return e;
   cudaEvent_t stop =
       a.only_if == nullptr && a.qlist == nullptr && a.nprobe > 1 ? prof_start(ix, s, "scan_kernel") : nullptr;
-  scan_kernel<CH><<<unsigned(grid), 256, smem, s>>>(a);
+  scan_kernel<CH, B3><<<unsigned(grid), 256, smem, s>>>(a);
   prof_stop(stop, s);
   return cudaGetLastError();
 }
@@ -724,7 +753,8 @@ cudaError_t launch_scan_impl(const rslm_index* ix, const float* qrot, int64_t nq
   a.part_n = ix->part_n;
   a.nlist = ix->nlist;
   a.stride = ix->cs1.stride;
-  a.lut_groups = 2 * ix->cs1.stride;
+  const bool b3 = ix->cs1.bits == 3;
+  a.lut_groups = b3 ? (ix->cs1.ngroups + 31) / 32 * 32 : 2 * ix->cs1.stride;
   a.ngroups = ix->cs1.ngroups;
   a.g = ix->cs1.g;
   for (int i = 0; i < 64; ++i) a.cb[i] = ix->cs1.cbf[i];
@@ -736,16 +766,17 @@ cudaError_t launch_scan_impl(const rslm_index* ix, const float* qrot, int64_t nq
   const int W = 8;
   int np2 = 1;
   while (np2 < W * k) np2 <<= 1;
-  const size_t lut_bytes = size_t(a.lut_groups) * 16 * 4;
+  const size_t lut_bytes = size_t(a.lut_groups) * (b3 ? 8 : 16) * 4;
   const size_t merge_bytes = ((size_t(np2) * 4 + 15) & ~size_t(15)) + size_t(np2) * 8;
   size_t region = lut_bytes > merge_bytes ? lut_bytes : merge_bytes;
   region = (region + 15) & ~size_t(15);
   a.lut_region = int(region);
   const size_t smem = 256 + region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
+  if (b3) return launch_scan_ch<4, true>(ix, a, nq, smem, s);
   switch (ix->cs1.chunk) {
-    case 16: return launch_scan_ch<16>(ix, a, nq, smem, s);
-    case 8: return launch_scan_ch<8>(ix, a, nq, smem, s);
-    default: return launch_scan_ch<4>(ix, a, nq, smem, s);
+    case 16: return launch_scan_ch<16, false>(ix, a, nq, smem, s);
+    case 8: return launch_scan_ch<8, false>(ix, a, nq, smem, s);
+    default: return launch_scan_ch<4, false>(ix, a, nq, smem, s);
   }
 }
 }  // namespace

@@ -178,7 +178,14 @@ bool make_codec_spec(int bits, int D, bool interleaved, CodecSpec* out) {
     c.ngroups = (D + c.g - 1) / c.g;
     c.Dp = c.ngroups * c.g;
     c.code_bytes = (c.ngroups + 1) / 2;
-    if (interleaved) {
+    if (bits == 3) {
+      // Rslm3: a 3-bit stream, 8 codes in 3 bytes; the device rows hold whole
+      // groups of 32 codes (three 32-bit words), interleaved word by word
+      c.code_bytes = (3 * c.ngroups + 7) / 8;
+      c.stride = (c.ngroups + 31) / 32 * 12;
+      c.chunk = interleaved ? 4 : 0;
+      if (!interleaved) c.stride = (c.stride + 15) / 16 * 16;
+    } else if (interleaved) {
       c.stride = (c.code_bytes + 3) / 4 * 4;
       c.chunk = c.stride % 16 == 0 ? 16 : (c.stride % 8 == 0 ? 8 : 4);
     } else {

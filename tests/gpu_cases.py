@@ -55,7 +55,8 @@ class Case:
     def import_oracle_codes(self, ix):
         import torch
         st = self.oracle.stage1
-        ix.import_codes(1, 0, torch.from_numpy(codec.pack_nibbles(st.codes)).cuda(),
+        pack = codec.pack_bits3 if self.w.bits == 3 else codec.pack_nibbles
+        ix.import_codes(1, 0, torch.from_numpy(pack(st.codes)).cuda(),
                         torch.from_numpy(st.L_u16.astype(np.uint16)).cuda(),
                         torch.from_numpy(st.G_u16.astype(np.uint16)).cuda())
         if self.oracle.stage2 is not None:
@@ -88,7 +89,7 @@ def check_stage(gpu_codes, gpu_L, gpu_G, enc, X, A, bits, global_scale, name):
     flip the scales the GPU's own codes imply.  Returns the rows without a
     code flip."""
     ng = enc.codes.shape[1]
-    got = codec.unpack_nibbles(gpu_codes, ng)
+    got = codec.unpack_bits3(gpu_codes, ng) if bits == 3 else codec.unpack_nibbles(gpu_codes, ng)
     mism = got != enc.codes
     near = codec.near_threshold(enc.u, bits, 1e-5)
     assert np.all(near[mism]), f"{name}: code mismatch away from a decision boundary"

@@ -265,7 +265,8 @@ def _decompress_check(case):
     if case.lite:
         ref1 = codec.decode_lite(A1, codec.unpack_nibbles(c1, w.D), w.D, case.global_scale)
     else:
-        ref1 = codec.decode(A1, codec.unpack_nibbles(c1, ng1), L1, G1, w.bits, w.D)
+        unpack = codec.unpack_bits3 if w.bits == 3 else codec.unpack_nibbles
+        ref1 = codec.decode(A1, unpack(c1, ng1), L1, G1, w.bits, w.D)
     tol = 1e-6 * float(np.abs(case.X).max()) + 1e-6
     got1 = ix.decompress(1).cpu().numpy()
     assert np.allclose(got1, ref1, rtol=1e-6, atol=tol), np.abs(got1 - ref1).max()
@@ -294,6 +295,33 @@ def test_decompress_parity_variants(kind):
         case = Case(Wl("dv", 6_000, 96, 8, 0.5, False, 0.5, "mean", 8, 2, 4, 3, 40, 10, seed=52),
                     reading="A" if kind == "reading_a" else "B", full_vector=kind == "full_vector")
     _decompress_check(case)
+
+
+# ----------------------------------------------------------------- Rslm3
+# Sec. 3.4: 3 bits per dimension on the K = 8 levels, eight codes in 3 bytes.
+# D = 100: a partial last 32-code group (and 4-bit rescoring on top);
+# D = 768: many groups.
+R3 = {
+    "r3a": Wl("r3a", 20_000, 128, 16, 0.5, False, 0.5, "mean", 40, 3, 0, 4, 10, 10, seed=61),
+    "r3b": Wl("r3b", 15_000, 100, 12, 0.5, True, None, "mean", 40, 3, 4, 4, 60, 10, seed=62),
+    "r3c": Wl("r3c", 6_000, 768, 8, 0.5, True, None, "mean", 24, 3, 0, 3, 10, 10, seed=63),
+}
+
+
+@pytest.mark.parametrize("name", sorted(R3))
+def test_rslm3_encode_and_decompress_parity(name):
+    case = Case(R3[name])
+    ix = _encode_check(case)
+    assert ix.desc["code_bytes"] == (3 * case.w.D + 7) // 8
+    _decompress_check(case)
+
+
+@pytest.mark.parametrize("name", sorted(R3))
+@pytest.mark.parametrize("batched", [False, True])
+def test_rslm3_scan_parity(name, batched):
+    """The single-query kernel's 3-bit path (the tensor-core regime hands
+    3-bit rows to it)."""
+    _scan_parity(Case(R3[name]), batched=batched)
 
 
 # ---------------------------------------------- relative-mode variants

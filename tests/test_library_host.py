@@ -64,7 +64,7 @@ def test_argument_checks_need_no_gpu(L):
     dummy = ctypes.c_void_p(16)
     # bad dim, nlist, bits, rescore bits; an unknown flag; RSLM_LITE below
     # D = 64 or with 2-bit codes; RSLM_RESCORE_READING_A without rescoring codes
-    cases = [(0, 4, 4, 0, 1), (4097, 4, 4, 0, 1), (64, 0, 4, 0, 1), (64, 4, 3, 0, 1),
+    cases = [(0, 4, 4, 0, 1), (4097, 4, 4, 0, 1), (64, 0, 4, 0, 1), (64, 4, 5, 0, 1), (64, 4, 3, 0, 2),
              (64, 4, 4, 2, 1), (64, 4, 4, 0, 16), (48, 4, 4, 0, 2), (64, 4, 2, 0, 2), (64, 4, 4, 0, 4)]
     for dim, nlist, bits, rb, flags in cases:
         st = lib.rslm_index_create(dim, nlist, dummy, bits, rb, flags, None, ctypes.byref(out))
