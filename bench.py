@@ -74,19 +74,24 @@ def parse_args():
     ap.add_argument("--reading", default="B", choices=["A", "B"],
                     help="rescoring approximation: B the stage-1 reconstruction (default), A the centroid")
     ap.add_argument("--full-vector", action="store_true", help="codes of x itself (approximation 0)")
+    ap.add_argument("--score-bits", type=int, default=None, choices=[1, 2, 3, 4],
+                    help="override the workload's scoring bit rate (3: Rslm3)")
     ap.add_argument("--recall", type=int, default=0, metavar="N",
                     help="diagnostic: recall of the final top-k of the first N queries against exact "
                          "float64 MIPS over the whole database (computed while the index is built)")
     args = ap.parse_args()
     if args.lite:
         w = W.WORKLOADS[args.config]
-        if w.bits != 4 or w.D < 64:
+        if (args.score_bits or w.bits) != 4 or w.D < 64:
             ap.error("--lite needs a 4-bit workload with D >= 64")
     return args
 
 
 def workload_label(w: W.Workload, lite: bool = False, reading: str = "B", full_vector: bool = False) -> str:
-    mods = (["Rslm4Lite scoring codes"] if lite else []) + (["full-vector codes"] if full_vector else []) \
+    base = W.WORKLOADS.get(w.name)
+    mods = ([f"{w.bits}-bit scoring codes" + (" (Rslm3)" if w.bits == 3 else "")]
+            if base is not None and w.bits != base.bits else []) \
+        + (["Rslm4Lite scoring codes"] if lite else []) + (["full-vector codes"] if full_vector else []) \
         + (["rescoring reading A"] if reading == "A" and w.rescore_bits else [])
     if mods:
         return f"{w.name} with {', '.join(mods)}: {w.description}"
@@ -278,6 +283,8 @@ def run_reference(args):
     w = W.WORKLOADS[args.config]
     if args.nq:
         w = w.scaled(nq=args.nq)
+    if args.score_bits:
+        w = w.scaled(bits=args.score_bits)
     A = W.assignment(w)
     C = W.ivf_centroids(w)
     nqs = min(SAMPLE_QUERIES[w.name], w.nq)
@@ -342,6 +349,8 @@ def run_gpu(args):
     w = W.WORKLOADS[args.config]
     if args.nq:
         w = w.scaled(nq=args.nq)
+    if args.score_bits:
+        w = w.scaled(bits=args.score_bits)
     # the database is generated in 2^20-row blocks straight into the encoder,
     # so no configuration holds it in host memory
     A = W.assignment(w)
@@ -480,7 +489,8 @@ def run_gpu(args):
     hbm_peak, tensor_peak, peak_kind = load_peaks()
     scan_bytes = cand_per_step * bytes_per_cand
     kern_avg_s = kern_ms / max(1, kern_n) / 1e3
-    trec = traffic_record(w.name + ("-lite" if args.lite else ""), kern_name)
+    bits_tag = f"-{w.bits}bit" if args.score_bits and args.score_bits != W.WORKLOADS[w.name].bits else ""
+    trec = traffic_record(w.name + bits_tag + ("-lite" if args.lite else ""), kern_name)
     traffic = (trec["dram_bytes_per_candidate"] * cand_per_step) if trec else None
     if kern_name.startswith("batched_"):
         # dense contraction: 2 D flops per candidate (the fp16 hi/lo split is
