@@ -77,8 +77,9 @@ def parse_args():
     ap.add_argument("--score-bits", type=int, default=None, choices=[1, 2, 3, 4],
                     help="override the workload's scoring bit rate (3: Rslm3)")
     ap.add_argument("--recall", type=int, default=0, metavar="N",
-                    help="diagnostic: recall of the final top-k of the first N queries against exact "
-                         "float64 MIPS over the whole database (computed while the index is built)")
+                    help="diagnostic: recall of the first N queries against exact float64 MIPS over "
+                         "the whole database (computed while the index is built): Recall@k@k of the "
+                         "final top-k, and Recall@20@20/30/40 from one untimed deeper search")
     args = ap.parse_args()
     if args.lite:
         w = W.WORKLOADS[args.config]
@@ -229,13 +230,26 @@ class ExactTopK:
         self.sc = np.take_along_axis(sc, o, 1)
         self.ids = np.take_along_axis(ii, o, 1)
 
-    def recall(self, found):
-        """Recall@k@k (share of the exact top k returned) and Recall@1@k."""
+    def recall_at(self, found, x):
+        """Recall@x@y (Sec. 4, quality metrics): the share of the exact top x
+        among the y results returned per query (y = found's width)."""
+        assert x <= self.k
         n = len(self.Q)
-        rk = np.mean([len(set(found[i].tolist()) & set(self.ids[i].tolist())) / self.k for i in range(n)])
-        r1 = np.mean([self.ids[i, 0] in set(found[i].tolist()) for i in range(n)])
-        return {"queries": n, "k": self.k, "recall_k_at_k": float(rk), "recall_1_at_k": float(r1),
-                "exact": "float64 maximum inner product over every database row"}
+        return float(np.mean([len(set(found[i].tolist()) & set(self.ids[i, :x].tolist())) / x
+                              for i in range(n)]))
+
+    def recall(self, found, deep=None):
+        """Recall@k@k and Recall@1@k of the final top k (found: [n, k]); with
+        deep ([n, 40] results of a deeper search), Recall@20@20, @20@30 and
+        @20@40 from its prefixes."""
+        k = found.shape[1]
+        out = {"queries": len(self.Q), "k": k, "recall_k_at_k": self.recall_at(found, k),
+               "recall_1_at_k": self.recall_at(found, 1),
+               "exact": "float64 maximum inner product over every database row"}
+        if deep is not None:
+            for y in (20, 30, 40):
+                out[f"recall_20_at_{y}"] = self.recall_at(deep[:, :y], 20)
+        return out
 
 
 # --------------------------------------------------------- oracle (CPU) leg
@@ -364,7 +378,7 @@ def run_gpu(args):
     ix.reserve(torch.from_numpy(A).to(dev))
     torch.cuda.synchronize()
     encode_s = 0.0
-    exact = ExactTopK(Q[:args.recall], w.k_final) if args.recall else None
+    exact = ExactTopK(Q[:args.recall], max(w.k_final, 20)) if args.recall else None
     for lo, X in W.row_blocks(w, 1 << 20):
         Xd = torch.from_numpy(X).to(dev)
         torch.cuda.synchronize()
@@ -486,6 +500,16 @@ def run_gpu(args):
                "d2h_bytes_per_step": int(h_ids.numel() * 8 + h_sc.numel() * 4),
                "ms_per_step": ems / args.steps}
 
+    # recall diagnostic (untimed): the final top-k of the timed steps, and
+    # one deeper search (40 results) of the same queries for Recall@20@y
+    recall = None
+    if exact is not None:
+        n = args.recall
+        final = (f_ids if w.rescore_bits else s1_ids)[:n].cpu().numpy()
+        deep_ids, _ = ix.search(Qd[:n].contiguous(), w.nprobe, max(w.k, 40), k_final=40)
+        ix.sync()
+        recall = exact.recall(final, deep_ids.cpu().numpy())
+
     hbm_peak, tensor_peak, peak_kind = load_peaks()
     scan_bytes = cand_per_step * bytes_per_cand
     kern_avg_s = kern_ms / max(1, kern_n) / 1e3
@@ -546,8 +570,7 @@ def run_gpu(args):
             "e2e": e2e,
             "gpu_launches": launches_per_step(w, nq, batched) * args.steps,
             "clocks": clocks,
-            "recall": (exact.recall((f_ids if w.rescore_bits else s1_ids)[:args.recall].cpu().numpy())
-                       if exact is not None else None),
+            "recall": recall,
         }
         print(json.dumps(line), flush=True)
     if ws > 1:

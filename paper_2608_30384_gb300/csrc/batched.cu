@@ -383,6 +383,18 @@ constexpr int kByteTableBytes = 256 * 32 * 4;
 // Rslm4Lite head bytes: (3-bit code | 3-bit code << 3) -> two halves, 64
 // entries (the top bits, which hold the scale codes, are dropped)
 constexpr int kLiteTableBytes = 64 * 4;
+// Code formats of the scoring rows: codes of 4 bits (g = 1, 2, 4), the
+// same with the Rslm4Lite head, and Rslm3's 3-bit stream (g = 1).  Rslm3
+// decodes two codes (6 stream bits) per lookup through a 64-entry table
+// held once per lane (entry (pair, lane) at word pair * 32 + lane), which
+// takes the place of the 256-entry byte table.
+constexpr int kFmtNibble = 0, kFmtLite = 1, kFmt3 = 2;
+// Code words of one row in a K chunk of 128 coordinates.
+__host__ __device__ constexpr int row_words(int g, int fmt) { return fmt == kFmt3 ? 12 : 16 / g; }
+// Code bytes of klen (<= 128) coordinates of a row.
+__host__ __device__ constexpr int row_bytes(int klen, int g, int fmt) {
+  return fmt == kFmt3 ? (3 * klen + 7) / 8 : (klen + 2 * g - 1) / (2 * g);
+}
 __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
   return size_t(2) * kSlotBytes + size_t(kSlabs) * slab_bytes(g) + size_t(kScaleStages) * kScaleBytes + 32 * 4 +
          (g == 1 ? kByteTableBytes + kLiteTableBytes : 0);
@@ -390,12 +402,29 @@ __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
 
 // Half dh (32 columns = 64 halves = 64 / G codes) of a row's A operand from
 // the row's code words wd (G = 1: 16 words; byte -> column through the
-// per-lane table t256; G = 2, 4: nibble -> halves through t32).
-template <int G, bool LITE>
+// per-lane table t256; G = 2, 4: nibble -> halves through t32; Rslm3: 12
+// words, three per 32 codes, code i of a group at its bits 3i .. 3i + 2, so
+// column m of the group is its 6-bit field 6m .. 6m + 5, looked up in the
+// per-lane pair table held in t256's place).
+template <int G, int FMT>
 __device__ __forceinline__ void decode_half(const uint32_t* wd, int dh, const uint32_t* t256,
                                             const uint32_t* t32, int lane, uint32_t (&av)[32],
                                             int lite_words, const uint32_t* t64) {
-  if constexpr (G == 1) {
+  if constexpr (FMT == kFmt3) {
+    const uint32_t* tl = t256 + lane;
+#pragma unroll
+    for (int j = 0; j < 2; ++j) {
+      const uint32_t w0 = wd[6 * dh + 3 * j], w1 = wd[6 * dh + 3 * j + 1], w2 = wd[6 * dh + 3 * j + 2];
+#pragma unroll
+      for (int m = 0; m < 16; ++m) {
+        const int bit = 6 * m, wi = bit >> 5, sh = bit & 31;
+        const uint32_t lo = wi == 0 ? w0 : (wi == 1 ? w1 : w2);
+        const uint32_t hi = wi == 0 ? w1 : w2;
+        const uint32_t v = (sh <= 26 ? lo >> sh : __funnelshift_r(lo, hi, sh)) & 63u;
+        av[16 * j + m] = tl[v << 5];
+      }
+    }
+  } else if constexpr (G == 1) {
     // one byte (two codes) -> one 32-bit column (low half = even position)
     const uint32_t* tl = t256 + lane;
 #pragma unroll
@@ -404,7 +433,7 @@ __device__ __forceinline__ void decode_half(const uint32_t* wd, int dh, const ui
       for (int bb = 0; bb < 4; ++bb) av[4 * w + bb] = tl[((wd[8 * dh + w] >> (8 * bb)) & 255u) << 5];
     // Rslm4Lite: the first lite_words (<= 4) words hold K = 8 codes under
     // the scale bits (static indices keep av in registers)
-    if constexpr (LITE) {
+    if constexpr (FMT == kFmtLite) {
 #pragma unroll
       for (int w = 0; w < 4; ++w)
         if (w < lite_words)
@@ -501,7 +530,7 @@ __device__ __forceinline__ void epilogue_row(const BatchArgs& a, const float (&v
   }
 }
 
-template <int G, bool DENSE, bool LITE>
+template <int G, bool DENSE, int FMT>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
   extern __shared__ __align__(128) uint8_t psm[];
   uint8_t* slab0 = psm + 2 * kSlotBytes;
@@ -517,7 +546,12 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
 
   uint32_t* t256 = t32 + 32;  // G = 1 only
   uint32_t* t64 = t256 + 256 * 32;  // G = 1 only: Rslm4Lite head
-  if (G == 1) {
+  if (FMT == kFmt3) {
+    for (int e = tid; e < 64 * 32; e += blockDim.x) {
+      const uint32_t pair = uint32_t(e) >> 5;  // even code in the low 3 bits -> low half
+      t256[e] = a.cbbits[pair & 7u] | (a.cbbits[pair >> 3] << 16);
+    }
+  } else if (G == 1) {
     for (int e = tid; e < 256 * 32; e += blockDim.x) {
       const uint32_t byte = uint32_t(e) >> 5;  // low nibble -> low half (even position)
       t256[e] = a.cbbits[byte & 15u] | (a.cbbits[byte >> 4] << 16);
@@ -585,7 +619,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   const uint32_t scl_addr0 = uint32_t(__cvta_generic_to_shared(scl0));
   const int n_items = a.items[a.nlist];
   const int klen = a.Dp16;  // single K chunk
-  const int nbytes = (klen + 2 * G - 1) / (2 * G);
+  const int nbytes = row_bytes(klen, G, FMT);
   const int c1 = min((nbytes + CH - 1) / CH, a.stride / CH);  // code chunks of a row used
   const uint32_t slab_len = uint32_t(c1 * kMR * CH);
   auto slot = [&](uint32_t s) { return psm + s * kSlotBytes; };
@@ -783,15 +817,15 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           ok = false;
           break;
         }
-        // the 64 / G bytes = 16 / G words of row r (half dh: words dh * NW ..)
-        constexpr int NW = 8 / G;
-        uint32_t wd[2 * NW];
+        // the code words of row r (half dh: words dh * NW / 2 ..)
+        constexpr int NW = row_words(G, FMT);
+        uint32_t wd[NW];
         {
           const uint8_t* sl = slab0 + sb * slab_bytes(G);
-          if (CH == 16) {
+          if (FMT != kFmt3 && CH == 16) {
             // whole 16-byte chunks (G = 1: four, G = 2: two, G = 4: one)
 #pragma unroll
-            for (int v = 0; v < (2 * NW) / 4; ++v) {
+            for (int v = 0; v < NW / 4; ++v) {
               uint4 x = make_uint4(0, 0, 0, 0);
               if (v < c1) x = *reinterpret_cast<const uint4*>(sl + (v * kMR + r) * 16);
               wd[4 * v] = x.x;
@@ -801,7 +835,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
             }
           } else {
 #pragma unroll
-            for (int w = 0; w < 2 * NW; ++w) {
+            for (int w = 0; w < NW; ++w) {
               const int byte = 4 * w;
               const int c = byte / CH;
               wd[w] = c < c1 ? *reinterpret_cast<const uint32_t*>(sl + (c * kMR + r) * CH + (byte % CH))
@@ -822,7 +856,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
 #pragma unroll
         for (int dh = 0; dh < 2; ++dh) {
           uint32_t av[32];
-          decode_half<G, LITE>(wd, dh, t256, t32, lane, av, dh == 0 ? a.lite_h / 8 : 0, t64);
+          decode_half<G, FMT>(wd, dh, t256, t32, lane, av, dh == 0 ? a.lite_h / 8 : 0, t64);
           tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
         }
         fence_before_sync();
@@ -918,7 +952,7 @@ __host__ __device__ constexpr size_t kpipe_smem_bytes(int g) {
          size_t(kScaleStages) * kScaleBytes + 32 * 4 + (g == 1 ? kByteTableBytes + kLiteTableBytes : 0);
 }
 
-template <int G, bool DENSE, bool LITE>
+template <int G, bool DENSE, int FMT>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __grid_constant__ BatchArgs a) {
   extern __shared__ __align__(128) uint8_t psm[];
   uint8_t* bst0 = psm;                               // B ring
@@ -933,7 +967,12 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
   __shared__ int s_fail;
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
   const int CH = a.chunk;
-  if (G == 1) {
+  if (FMT == kFmt3) {
+    for (int e = tid; e < 64 * 32; e += blockDim.x) {
+      const uint32_t pair = uint32_t(e) >> 5;
+      t256[e] = a.cbbits[pair & 7u] | (a.cbbits[pair >> 3] << 16);
+    }
+  } else if (G == 1) {
     for (int e = tid; e < 256 * 32; e += blockDim.x) {
       const uint32_t byte = uint32_t(e) >> 5;
       t256[e] = a.cbbits[byte & 15u] | (a.cbbits[byte >> 4] << 16);
@@ -1004,7 +1043,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
   const int n_items = a.items[a.nlist];
   const int nkc = a.nkc;
   // bytes of a full K chunk of a row; its code chunks [kc * cpk, kc * cpk + cpk)
-  const int kc_bytes = kKC / (2 * G);
+  const int kc_bytes = row_bytes(kKC, G, FMT);
   const int cpk = kc_bytes / CH;
   const int nchunks_row = a.stride / CH;
   auto klen_of = [&](int kc) { return min(kKC, a.Dp16 - kc * kKC); };
@@ -1253,12 +1292,12 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
               ok = false;
               break;
             }
-            constexpr int NW = 8 / G;
-            uint32_t wd[2 * NW];
+            constexpr int NW = row_words(G, FMT);
+            uint32_t wd[NW];
             {
               const uint8_t* sl = slab0 + sb * slab_bytes(G);
 #pragma unroll
-              for (int w = 0; w < 2 * NW; ++w) {
+              for (int w = 0; w < NW; ++w) {
                 const int byte = 4 * w;
                 const int c = byte / CH;
                 wd[w] = c < c_n ? *reinterpret_cast<const uint32_t*>(sl + (c * kMR + row) * CH + (byte % CH)) : 0u;
@@ -1276,7 +1315,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
 #pragma unroll
             for (int dh = 0; dh < 2; ++dh) {
               uint32_t av[32];
-              decode_half<G, LITE>(wd, dh, t256, t32, lane, av, (kc == 0 && dh == 0) ? a.lite_h / 8 : 0,
+              decode_half<G, FMT>(wd, dh, t256, t32, lane, av, (kc == 0 && dh == 0) ? a.lite_h / 8 : 0,
                                    t64);
               tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(ab) + uint32_t(dh * 32), av);
             }
@@ -1571,17 +1610,23 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   using K = void (*)(BatchArgs);
   K pk;
   if (one)
-    pk = b.lite_h ? (theta ? batched_pipe_kernel<1, false, true> : batched_pipe_kernel<1, true, true>)
-         : theta  ? (g == 1 ? batched_pipe_kernel<1, false, false>
-                            : (g == 2 ? batched_pipe_kernel<2, false, false> : batched_pipe_kernel<4, false, false>))
-                  : (g == 1 ? batched_pipe_kernel<1, true, false>
-                            : (g == 2 ? batched_pipe_kernel<2, true, false> : batched_pipe_kernel<4, true, false>));
+    pk = c1.bits == 3 ? (theta ? batched_pipe_kernel<1, false, kFmt3> : batched_pipe_kernel<1, true, kFmt3>)
+         : b.lite_h   ? (theta ? batched_pipe_kernel<1, false, kFmtLite> : batched_pipe_kernel<1, true, kFmtLite>)
+         : theta      ? (g == 1   ? batched_pipe_kernel<1, false, kFmtNibble>
+                         : g == 2 ? batched_pipe_kernel<2, false, kFmtNibble>
+                                  : batched_pipe_kernel<4, false, kFmtNibble>)
+                      : (g == 1   ? batched_pipe_kernel<1, true, kFmtNibble>
+                         : g == 2 ? batched_pipe_kernel<2, true, kFmtNibble>
+                                  : batched_pipe_kernel<4, true, kFmtNibble>);
   else
-    pk = b.lite_h ? (theta ? batched_kpipe_kernel<1, false, true> : batched_kpipe_kernel<1, true, true>)
-         : theta  ? (g == 1 ? batched_kpipe_kernel<1, false, false>
-                            : (g == 2 ? batched_kpipe_kernel<2, false, false> : batched_kpipe_kernel<4, false, false>))
-                  : (g == 1 ? batched_kpipe_kernel<1, true, false>
-                            : (g == 2 ? batched_kpipe_kernel<2, true, false> : batched_kpipe_kernel<4, true, false>));
+    pk = c1.bits == 3 ? (theta ? batched_kpipe_kernel<1, false, kFmt3> : batched_kpipe_kernel<1, true, kFmt3>)
+         : b.lite_h   ? (theta ? batched_kpipe_kernel<1, false, kFmtLite> : batched_kpipe_kernel<1, true, kFmtLite>)
+         : theta      ? (g == 1   ? batched_kpipe_kernel<1, false, kFmtNibble>
+                         : g == 2 ? batched_kpipe_kernel<2, false, kFmtNibble>
+                                  : batched_kpipe_kernel<4, false, kFmtNibble>)
+                      : (g == 1   ? batched_kpipe_kernel<1, true, kFmtNibble>
+                         : g == 2 ? batched_kpipe_kernel<2, true, kFmtNibble>
+                                  : batched_kpipe_kernel<4, true, kFmtNibble>);
   e = cudaFuncSetAttribute(pk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
   if (e != cudaSuccess) return e;
   cudaEvent_t stop =
@@ -1597,8 +1642,6 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
                                 const int32_t* probes, const float* cs, int nprobe, int k,
                                 int64_t* out_ids, float* out_scores, cudaStream_t s) {
   if (nq == 0) return cudaSuccess;
-  // Rslm3's 3-bit rows have no tensor-core decode: the single-query scan serves them
-  if (ix->cs1.bits == 3) return launch_scan(ix, qrot, nq, probes, cs, nprobe, k, k, out_ids, out_scores, s);
   const CodecSpec& c1 = ix->cs1;
   const int Dp16 = (c1.Dp + 15) / 16 * 16;
   const int nlist = ix->nlist;

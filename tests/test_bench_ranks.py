@@ -11,6 +11,7 @@ import socket
 import subprocess
 import sys
 
+import numpy as np
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
@@ -81,3 +82,28 @@ def test_reference_arm_runs_on_rank_zero_only():
 def test_world_size_must_match_gpus():
     r = _run_bench(0, 2, ["--impl", "reference", "--gpus", "1", "--config", "C1", "--steps", "1"])
     assert r.returncode != 0 and "WORLD_SIZE" in (r.stderr + r.stdout)
+
+
+def test_exact_topk_and_recall_at():
+    """The recall diagnostic's exact top-k, streamed over row blocks, equals
+    a full sort (score desc, row asc); Recall@x@y counts the exact top x
+    among y results."""
+    b = _bench()
+    rng = np.random.default_rng(5)
+    X = rng.standard_normal((1000, 16))
+    X[500] = X[20]  # a tie: the lower row comes first
+    Q = rng.standard_normal((4, 16))
+    ex = b.ExactTopK(Q, 25)
+    for lo in range(0, 1000, 300):
+        ex.add(X[lo:lo + 300], lo)
+    S = Q @ X.T
+    for i in range(4):
+        o = np.lexsort((np.arange(1000), -S[i]))[:25]
+        assert np.array_equal(ex.ids[i], o)
+    truth = ex.ids
+    found = np.concatenate([truth[:, :15], np.full((4, 25), -1)], axis=1)  # 40 results
+    assert ex.recall_at(found, 20) == 0.75
+    assert ex.recall_at(found[:, :10], 20) == 0.5
+    r = ex.recall(truth[:, :10], found)
+    assert r["recall_k_at_k"] == 1.0 and r["recall_1_at_k"] == 1.0
+    assert (r["recall_20_at_20"], r["recall_20_at_30"], r["recall_20_at_40"]) == (0.75, 0.75, 0.75)

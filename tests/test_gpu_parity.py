@@ -242,7 +242,7 @@ def test_batched_scan_many_partitions():
 
 
 @pytest.mark.parametrize("bits,D", [(4, 128), (2, 96), (1, 128), (4, 256), (1, 768), (2, 300),
-                                    (1, 256), (2, 768), (4, 768), (1, 384)])
+                                    (1, 256), (2, 768), (4, 768), (1, 384), (3, 128), (3, 300)])
 def test_batched_scan_many_queries_per_partition(bits, D):
     """About 225 queries per partition: two work items per partition (N = 128
     and a partial N), about 20 row tiles each, so the pipelined kernels'
@@ -319,9 +319,20 @@ def test_rslm3_encode_and_decompress_parity(name):
 @pytest.mark.parametrize("name", sorted(R3))
 @pytest.mark.parametrize("batched", [False, True])
 def test_rslm3_scan_parity(name, batched):
-    """The single-query kernel's 3-bit path (the tensor-core regime hands
-    3-bit rows to it)."""
+    """Both scan forms on 3-bit rows: the single-query kernel's shift /
+    funnel-shift extraction and the tensor-core decode of 6-bit code pairs
+    (D = 768: six K chunks)."""
     _scan_parity(Case(R3[name]), batched=batched)
+
+
+def test_rslm3_search_end_to_end_batched():
+    """rslm_search on 3-bit scoring codes with enough queries per probed
+    list for the tensor-core regime, then 4-bit rescoring."""
+    case = Case(Wl("r3e", 20_000, 128, 8, 0.5, True, None, "mean", 200, 3, 4, 3, 40, 10, seed=64))
+    assert case.w.nq * case.w.nprobe >= 16 * case.w.P
+    ix = case.gpu_index(encode=False)
+    case.import_oracle_codes(ix)
+    _end_to_end(case, ix)
 
 
 # ---------------------------------------------- relative-mode variants
