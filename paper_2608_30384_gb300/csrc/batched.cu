@@ -400,6 +400,36 @@ __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
          (g == 1 ? kByteTableBytes + kLiteTableBytes : 0);
 }
 
+// The NW code words of row r of a slab whose rows are interleaved in
+// chunks of CH bytes (chunk c of row r at (c * kMR + r) * CH; CH is 16, 8
+// or 4); words of the nch chunks present, zeros after them.  The branch
+// picks a path with constant chunk arithmetic.
+template <int NW>
+__device__ __forceinline__ void load_row_words(const uint8_t* sl, int r, int CH, int nch, uint32_t (&wd)[NW]) {
+  if (CH == 16) {
+#pragma unroll
+    for (int v = 0; v < NW / 4; ++v) {
+      uint4 x = make_uint4(0, 0, 0, 0);
+      if (v < nch) x = *reinterpret_cast<const uint4*>(sl + (v * kMR + r) * 16);
+      wd[4 * v] = x.x;
+      wd[4 * v + 1] = x.y;
+      wd[4 * v + 2] = x.z;
+      wd[4 * v + 3] = x.w;
+    }
+  } else if (CH == 8) {
+#pragma unroll
+    for (int v = 0; v < NW / 2; ++v) {
+      uint2 x = make_uint2(0, 0);
+      if (v < nch) x = *reinterpret_cast<const uint2*>(sl + (v * kMR + r) * 8);
+      wd[2 * v] = x.x;
+      wd[2 * v + 1] = x.y;
+    }
+  } else {
+#pragma unroll
+    for (int w = 0; w < NW; ++w) wd[w] = w < nch ? *reinterpret_cast<const uint32_t*>(sl + (w * kMR + r) * 4) : 0u;
+  }
+}
+
 // Half dh (32 columns = 64 halves = 64 / G codes) of a row's A operand from
 // the row's code words wd (G = 1: 16 words; byte -> column through the
 // per-lane table t256; G = 2, 4: nibble -> halves through t32; Rslm3: 12
@@ -820,29 +850,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         // the code words of row r (half dh: words dh * NW / 2 ..)
         constexpr int NW = row_words(G, FMT);
         uint32_t wd[NW];
-        {
-          const uint8_t* sl = slab0 + sb * slab_bytes(G);
-          if (FMT != kFmt3 && CH == 16) {
-            // whole 16-byte chunks (G = 1: four, G = 2: two, G = 4: one)
-#pragma unroll
-            for (int v = 0; v < NW / 4; ++v) {
-              uint4 x = make_uint4(0, 0, 0, 0);
-              if (v < c1) x = *reinterpret_cast<const uint4*>(sl + (v * kMR + r) * 16);
-              wd[4 * v] = x.x;
-              wd[4 * v + 1] = x.y;
-              wd[4 * v + 2] = x.z;
-              wd[4 * v + 3] = x.w;
-            }
-          } else {
-#pragma unroll
-            for (int w = 0; w < NW; ++w) {
-              const int byte = 4 * w;
-              const int c = byte / CH;
-              wd[w] = c < c1 ? *reinterpret_cast<const uint32_t*>(sl + (c * kMR + r) * CH + (byte % CH))
-                             : 0u;
-            }
-          }
-        }
+        load_row_words<NW>(slab0 + sb * slab_bytes(G), r, FMT == kFmt3 ? 4 : CH, c1, wd);
         __syncwarp();
         if (lane == 0) mbar_arrive(slab_empty(sb));
         // A buffer b is free once the MMAs of tile gt - 2 have completed
@@ -1294,15 +1302,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
             }
             constexpr int NW = row_words(G, FMT);
             uint32_t wd[NW];
-            {
-              const uint8_t* sl = slab0 + sb * slab_bytes(G);
-#pragma unroll
-              for (int w = 0; w < NW; ++w) {
-                const int byte = 4 * w;
-                const int c = byte / CH;
-                wd[w] = c < c_n ? *reinterpret_cast<const uint32_t*>(sl + (c * kMR + row) * CH + (byte % CH)) : 0u;
-              }
-            }
+            load_row_words<NW>(slab0 + sb * slab_bytes(G), row, FMT == kFmt3 ? 4 : CH, c_n, wd);
             __syncwarp();
             if (lane == 0) mbar_arrive(slab_empty(sb));
             const uint32_t ab = aseq & 1, au = aseq >> 1;
