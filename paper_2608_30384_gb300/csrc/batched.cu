@@ -1132,27 +1132,32 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
           // loads in batches of four 16-byte pieces, then shared stores (lane =
           // query row: a warp's stores fill whole 128-byte rows); see the
           // single-chunk kernel on why not cp.async
+          // both of a thread's queries in one batch: 16 loads in flight
+          constexpr int U = kNQ / kLoadThreads;
+          for (int k0 = 0; k0 < k8n; k0 += 4) {
+            uint4 hv[U][4], lv[U][4];
 #pragma unroll
-          for (int u = 0; u < kNQ / kLoadThreads; ++u) {
-            const int j = lt + u * kLoadThreads;
-            const bool v = qs[u] >= 0;
-            const int64_t base = int64_t(v ? qs[u] : 0) * a.Dp16 + kc * kKC;
-            for (int k0 = 0; k0 < k8n; k0 += 4) {
-              uint4 hv[4], lv[4];
+            for (int u = 0; u < U; ++u) {
+              const bool v = qs[u] >= 0;
+              const int64_t base = int64_t(v ? qs[u] : 0) * a.Dp16 + kc * kKC;
 #pragma unroll
               for (int e = 0; e < 4; ++e) {
-                hv[e] = make_uint4(0, 0, 0, 0);
-                lv[e] = make_uint4(0, 0, 0, 0);
+                hv[u][e] = make_uint4(0, 0, 0, 0);
+                lv[u][e] = make_uint4(0, 0, 0, 0);
                 if (v && k0 + e < k8n) {
-                  hv[e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + (k0 + e) * 8));
-                  lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
+                  hv[u][e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + (k0 + e) * 8));
+                  lv[u][e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
                 }
               }
+            }
+#pragma unroll
+            for (int u = 0; u < U; ++u) {
+              const int j = lt + u * kLoadThreads;
 #pragma unroll
               for (int e = 0; e < 4; ++e)
                 if (k0 + e < k8n) {
-                  *reinterpret_cast<uint4*>(dst + tile_off(j, k0 + e)) = hv[e];
-                  *reinterpret_cast<uint4*>(dst + kTileBytes + tile_off(j, k0 + e)) = lv[e];
+                  *reinterpret_cast<uint4*>(dst + tile_off(j, k0 + e)) = hv[u][e];
+                  *reinterpret_cast<uint4*>(dst + kTileBytes + tile_off(j, k0 + e)) = lv[u][e];
                 }
             }
           }
