@@ -26,7 +26,7 @@
  * - An index may be searched concurrently from several host threads on
  *   different streams once it is fully encoded; building (reserve, encode,
  *   import) must not overlap any other call on the same index.
- * - Limits: 1 <= dim <= 4096; nlist >= 1; score_bits in {1, 2, 4};
+ * - Limits: 1 <= dim <= 4096; nlist >= 1; score_bits in {1, 2, 3, 4};
  *   rescore_bits in {0, 4}; n <= 2^31 - 1 rows; 1 <= nprobe <= min(nlist,
  *   4096); 1 <= k <= 256; 1 <= k_final <= k; with score_bits = 4, dim <=
  *   3200 (the scan keeps a per-query table in shared memory).  Violations return
@@ -120,8 +120,8 @@ typedef struct {
  * score_bits: bits per dimension of the scoring codes: 1 (4-D codebook,
  *   K = 16), 2 (2-D, K = 16), 3 (1-D, K = 8: Rslm3, eight codes packed in
  *   3 bytes, code i at bits 3i .. 3i + 2 of the row's byte stream, least
- *   significant bit first; scanned by the single-query kernel in both
- *   regimes) or 4 (1-D, K = 16) (Sec. 3.2, Table "Rslm Codec
+ *   significant bit first; the tensor-core scan decodes two codes (6 bits)
+ *   per table lookup) or 4 (1-D, K = 16) (Sec. 3.2, Table "Rslm Codec
  *   Specifications").
  * rescore_bits: 0 (no rescoring) or 4: bits of the rescoring codes, which
  *   quantize x - a2 with a2 the full first-stage reconstruction (Sec. 5.2).
@@ -235,8 +235,9 @@ rslm_status rslm_search(const rslm_index* index, const float* queries, int64_t n
 /* Canonical codes of rows [row_begin, row_begin + rows): which = 1 scoring,
  * 2 rescoring.  codes: device [rows * code_bytes] uint8, row-major by row id,
  * the code of group i in the low nibble of byte i/2 when i is even, the high
- * nibble when odd (3-bit codes: bits 3i .. 3i + 2 of the row's byte stream).  Code values index the codebook in ascending order (1-D)
- * or in lexicographic codeword order (2-D, 4-D).  local_scale / global_scale:
+ * nibble when odd (3-bit codes: bits 3i .. 3i + 2 of the row's byte
+ * stream).  Code values index the codebook in ascending order (1-D) or in
+ * lexicographic codeword order (2-D, 4-D).  local_scale / global_scale:
  * device [rows] uint16 (UE7M9 / UE4M12 codes). */
 rslm_status rslm_export_codes(const rslm_index* index, int32_t which, int64_t row_begin,
                               int64_t rows, uint8_t* codes, uint16_t* local_scale,
