@@ -347,7 +347,7 @@ rslm_status rslm_encode(rslm_index* ix, const float* vectors, int64_t row_begin,
                         void* stream) {
   RSLM_ARG(ix, "index is NULL");
   if (!ix->slot_of_row) return fail(RSLM_ERR_STATE, "rslm_index_reserve has not been called");
-  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin + rows <= ix->n_rows,
+  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin <= ix->n_rows && rows <= ix->n_rows - row_begin,
            "rows [row_begin, row_begin + rows) outside the reserved rows");
   RSLM_ARG(rows == 0 || vectors, "vectors is NULL");
   DeviceGuard g(ix->device);
@@ -479,7 +479,8 @@ rslm_status rslm_export_codes(const rslm_index* ix, int32_t which, int64_t row_b
   RSLM_ARG(ix, "index is NULL");
   RSLM_ARG(which == 1 || (which == 2 && ix->rescore_bits), "which must be 1, or 2 with rescoring codes");
   if (!ix->slot_of_row) return fail(RSLM_ERR_STATE, "rslm_index_reserve has not been called");
-  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin + rows <= ix->n_rows, "row range out of bounds");
+  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin <= ix->n_rows && rows <= ix->n_rows - row_begin,
+           "row range out of bounds");
   RSLM_ARG(rows == 0 || (codes && local_scale && global_scale), "NULL array");
   DeviceGuard g(ix->device);
   RSLM_CK(launch_export_import(ix, which, row_begin, rows, codes, local_scale, global_scale, false,
@@ -493,7 +494,8 @@ rslm_status rslm_decompress(const rslm_index* ix, int32_t which, int64_t row_beg
   RSLM_ARG(ix, "index is NULL");
   RSLM_ARG(which == 1 || (which == 2 && ix->rescore_bits), "which must be 1, or 2 with rescoring codes");
   if (!ix->slot_of_row) return fail(RSLM_ERR_STATE, "rslm_index_reserve has not been called");
-  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin + rows <= ix->n_rows, "row range out of bounds");
+  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin <= ix->n_rows && rows <= ix->n_rows - row_begin,
+           "row range out of bounds");
   RSLM_ARG(rows == 0 || out, "NULL array");
   DeviceGuard g(ix->device);
   RSLM_CK(launch_decompress(ix, which, row_begin, rows, out, as_stream(stream)), "decompress launch");
@@ -506,7 +508,8 @@ rslm_status rslm_import_codes(rslm_index* ix, int32_t which, int64_t row_begin, 
   RSLM_ARG(ix, "index is NULL");
   RSLM_ARG(which == 1 || (which == 2 && ix->rescore_bits), "which must be 1, or 2 with rescoring codes");
   if (!ix->slot_of_row) return fail(RSLM_ERR_STATE, "rslm_index_reserve has not been called");
-  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin + rows <= ix->n_rows, "row range out of bounds");
+  RSLM_ARG(row_begin >= 0 && rows >= 0 && row_begin <= ix->n_rows && rows <= ix->n_rows - row_begin,
+           "row range out of bounds");
   RSLM_ARG(rows == 0 || (codes && local_scale && global_scale), "NULL array");
   DeviceGuard g(ix->device);
   RSLM_CK(launch_export_import(ix, which, row_begin, rows, const_cast<uint8_t*>(codes),

@@ -511,6 +511,14 @@ def test_edge_cases():
     assert ei.value.status == 1
     with pytest.raises(RslmError):
         ix.search(Q, 2, 300)
+    # a row range whose end overflows int64 is rejected before any launch
+    from paper_2608_30384_gb300 import binding as Bnd
+    small = torch.empty((1, 32), device="cuda")
+    lib, h, buf = Bnd.lib(), Bnd._ptr(ix.handle), small.data_ptr()
+    assert lib.rslm_decompress(h, 1, 2 ** 62, 2 ** 62, buf, None) == 1
+    assert lib.rslm_export_codes(h, 1, 2 ** 62, 2 ** 62, buf, buf, buf, None) == 1
+    assert lib.rslm_import_codes(h, 1, 2 ** 62, 2 ** 62, buf, buf, buf, None) == 1
+    assert lib.rslm_encode(h, buf, 2 ** 62, 2 ** 62, None) == 1
 
 
 def test_state_errors():
