@@ -94,9 +94,14 @@ def workload_label(w: W.Workload, lite: bool = False, reading: str = "B", full_v
             if base is not None and w.bits != base.bits else []) \
         + (["Rslm4Lite scoring codes"] if lite else []) + (["full-vector codes"] if full_vector else []) \
         + (["rescoring reading A"] if reading == "A" and w.rescore_bits else [])
+    desc = w.description
+    if base is not None and w.bits != base.bits:
+        # the workload's own text names its stock bit rate
+        for tail in ("-bit codes", "-bit scoring"):
+            desc = desc.replace(f"{base.bits}{tail}", f"{w.bits}{tail}")
     if mods:
-        return f"{w.name} with {', '.join(mods)}: {w.description}"
-    return f"{w.name}: {w.description}"
+        return f"{w.name} with {', '.join(mods)}: {desc}"
+    return f"{w.name}: {desc}"
 
 
 # ------------------------------------------------------------------ helpers
