@@ -15,6 +15,8 @@ import pytest
 
 import tests.test_oracle_codec as TC
 import tests.test_oracle_constants as TK
+import tests.test_oracle_lite as TL
+import tests.test_oracle_relative as TRel
 import tests.test_oracle_rotation as TR
 from oracle import codec, constants as K, rotation, search
 
@@ -52,7 +54,14 @@ def test_pins_pass_on_the_unmutated_oracle(mutate):
                        (TC.test_probe_order_and_padding, ()),
                        (TK.test_ue7m9_and_ue4m12_formats, ()),
                        (TK.test_1d_assignment_tie_goes_up, ()),
-                       (TR.test_matches_factor_product, (300, "two")))
+                       (TR.test_matches_factor_product, (300, "two")),
+                       (TL.test_scale_bits_in_the_top_bits, (True,)),
+                       (TRel.test_reading_a_codes_are_the_finer_codec_of_x_minus_c, ()),
+                       (TRel.test_rescore_score_identity, ("B",)),
+                       (TRel.test_full_vector_codes_encode_x_itself, ()),
+                       (TR.test_mode_rule, ()),
+                       (TR.test_orthogonal_and_inverse, (96, "single")),
+                       (TR.test_overlap_block_is_applied_last, ()))
 
 
 def test_transposed_rotation_in_the_codec(mutate):
@@ -143,3 +152,81 @@ def test_ties_ordered_by_descending_id(mutate):
     mutate.setattr(search, "order_desc", lambda scores, ids: np.lexsort((-ids, -scores)))
     assert _caught((TC.test_probe_order_and_padding, ()),
                    (TC.test_empty_partition_and_fewer_candidates_than_k, ()))
+
+
+def test_lite_scale_bits_one_code_late(mutate):
+    orig = codec.encode_lite
+
+    def shifted(X, A, global_scale=True):
+        enc = orig(X, A, global_scale)
+        codes = enc.codes.copy()
+        top = (codes[:, :16] >> 3) & 1
+        codes[:, :16] = (codes[:, :16] & 7) | (np.roll(top, 1, axis=1) << 3)
+        enc.codes = codes
+        return enc
+
+    mutate.setattr(codec, "encode_lite", shifted)
+    assert _caught((TL.test_scale_bits_in_the_top_bits, (True,)))
+
+
+def test_reading_a_built_as_reading_b(mutate):
+    orig = search.build_index
+
+    def always_b(*args, **kw):
+        kw["reading"] = "B"
+        return orig(*args, **kw)
+
+    mutate.setattr(search, "build_index", always_b)
+    assert _caught((TRel.test_reading_a_codes_are_the_finer_codec_of_x_minus_c, ()))
+
+
+def test_rescoring_without_its_global_scale(mutate):
+    orig = search.rescore
+
+    def no_g2(index, *args):
+        st = index.stage2
+        saved = st.Ghat
+        st.Ghat = np.ones_like(saved)
+        try:
+            return orig(index, *args)
+        finally:
+            st.Ghat = saved
+
+    mutate.setattr(search, "rescore", no_g2)
+    assert _caught((TRel.test_rescore_score_identity, ("B",)), (TRel.test_rescore_score_identity, ("A",)))
+
+
+def test_full_vector_scores_keep_the_centroid_term(mutate):
+    orig = search.stage1_scores
+
+    def with_cq(index, *args):
+        saved = index.full_vector
+        index.full_vector = False
+        try:
+            return orig(index, *args)
+        finally:
+            index.full_vector = saved
+
+    mutate.setattr(search, "stage1_scores", with_cq)
+    assert _caught((TRel.test_full_vector_codes_encode_x_itself, ()))
+
+
+def test_rotation_mode_rule_flipped(mutate):
+    mutate.setattr(rotation, "rotation_mode", lambda bits, D: "two" if bits == 4 else "single")
+    assert _caught((TR.test_mode_rule, ()))
+
+
+def test_hadamard_left_unnormalised(mutate):
+    mutate.setattr(rotation, "hadamard", rotation.hadamard_unnormalized)
+    assert _caught((TR.test_orthogonal_and_inverse, (96, "single")))
+
+
+def test_overlapping_block_applied_first(mutate):
+    orig = rotation.block_starts
+
+    def overlap_first(D):
+        s = orig(D)
+        return s[-1:] + s[:-1] if D % rotation.block_size(D) else s
+
+    mutate.setattr(rotation, "block_starts", overlap_first)
+    assert _caught((TR.test_overlap_block_is_applied_last, ()))
