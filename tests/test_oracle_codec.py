@@ -215,3 +215,25 @@ def test_rslm3_codes_are_the_nearest_of_eight_levels():
     d = np.abs(enc.u[:, :, None] - lv[None, None, :])
     assert enc.codes.max() < 8
     assert np.array_equal(enc.codes, np.argmin(d, axis=-1))
+
+
+@pytest.mark.parametrize("bits", [1, 2, 3, 4])
+def test_near_threshold_marks_only_boundary_groups(bits):
+    """The tolerance set of the code comparisons: groups placed exactly on a
+    decision boundary (a 1-D threshold, or the midpoint of two codewords)
+    are marked, groups at a codeword are not."""
+    cb = K.codebook(bits)
+    g = cb.g
+    n = cb.K - 1
+    at_code = cb.C[:n].reshape(1, n * g)                    # group j = codeword j
+    mid = 0.5 * (cb.C[:n] + cb.C[1:n + 1])                  # between codewords j and j + 1
+    if g == 1:
+        assert np.allclose(mid[:, 0], cb.thresholds)
+    # a midpoint is a boundary only if no other codeword is nearer than its two
+    d = ((mid[:, None, :] - cb.C[None, :, :]) ** 2).sum(-1)
+    own = ((mid - cb.C[:n]) ** 2).sum(-1)
+    boundary = np.sort(d, axis=1)[:, 0] >= own - 1e-12
+    assert not codec.near_threshold(at_code, bits).any()
+    marked = codec.near_threshold(mid.reshape(1, n * g), bits)[0]
+    assert np.array_equal(marked, boundary)
+    assert boundary.any()
