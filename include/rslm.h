@@ -152,6 +152,20 @@ rslm_status rslm_index_reserve(rslm_index* index, const int32_t* assignment, int
 rslm_status rslm_encode(rslm_index* index, const float* vectors, int64_t row_begin, int64_t rows,
                         void* stream);
 
+/* One call from vectors to an encoded index (the encode half of the
+ * problem statement of Sec. 5.5.1: residuals of the vectors against their
+ * partitions' centroids, coded as in Sec. 3.4 / 3.5): rslm_index_create
+ * with (dim, nlist, centroids, score_bits, rescore_bits, flags), then
+ * rslm_index_reserve(assignment, n), then rslm_encode of all n rows.
+ * vectors: device [n * dim] float32; assignment: device [n] int32 in
+ * [0, nlist); centroids: device [nlist * dim] float32 (copied).  The same
+ * limits and errors as those calls; on any failure nothing is returned in
+ * *out and the partial index is released.  Synchronizes `stream` (as
+ * rslm_index_reserve does); the encode itself is queued on it. */
+rslm_status rslm_encode_all(const float* vectors, const int32_t* assignment, int64_t n, int32_t dim,
+                            int32_t nlist, const float* centroids, int32_t score_bits,
+                            int32_t rescore_bits, uint32_t flags, void* stream, rslm_index** out);
+
 /* Rotate query rows with the rotation of the scoring codes (which = 1) or of
  * the rescoring codes (which = 2) (Sec. 3.1.3; done once per query, Sec. 5.4).
  * queries: device [nq * dim] float32.  out: device [nq * padded_dim] (or
@@ -290,6 +304,22 @@ rslm_status rslm_profile_read(rslm_index* index, double* total_ms, int64_t* laun
 /* Wait for `stream`, then report and clear the index's sticky device error
  * flag (RSLM_ERR_DEVICE) or a pending CUDA error (RSLM_ERR_CUDA). */
 rslm_status rslm_sync(const rslm_index* index, void* stream);
+
+/* Event counters of the index since its creation (a diagnostic for tests
+ * and benchmarks; not a paper quantity).  Waits for the device, then writes
+ * the first n (1..4) counters into out (host int64):
+ *   out[0] queries whose tensor-core (batched) scan kept fewer than k
+ *          candidates although the first probed partition gave a finite
+ *          threshold; they are answered by the exact single-query scan.
+ *          The two passes compute a row's score by the same arithmetic, so
+ *          a nonzero value means a fault of the batched path;
+ *   out[1] queries whose batched candidate buffer overflowed (many scores at
+ *          the threshold); also answered by the exact scan (expected, rare);
+ *   out[2] queries whose fused-probe candidate list overflowed (many
+ *          centroid scores tied at the bound); answered by the exact probe;
+ *   out[3] reserved, 0.
+ * RSLM_ERR_INVALID_ARG for a NULL argument or n outside [1, 4]. */
+rslm_status rslm_counters(const rslm_index* index, int64_t* out, int32_t n);
 
 /* Message of the last failing call on this thread ("" if none). */
 const char* rslm_last_error(void);

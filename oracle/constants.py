@@ -2,7 +2,7 @@
 
 Test infrastructure only: see ``oracle/__init__.py``.
 
-Readings of the paper taken here (each also listed in the design doc):
+Readings of the paper taken here, where it leaves a value or a rule open:
 
 * Sec. 3.1.2 fixes a 256-entry pseudo-random sign table S1 and a 128-entry
   permutation P but does not print them.  They are drawn here from the

@@ -32,6 +32,7 @@ SIGNATURES = {
     "rslm_index_describe": (ctypes.c_int, [_P, _P]),
     "rslm_index_reserve": (ctypes.c_int, [_P, _P, _I64, _P]),
     "rslm_encode": (ctypes.c_int, [_P, _P, _I64, _I64, _P]),
+    "rslm_encode_all": (ctypes.c_int, [_P, _P, _I64, _I32, _I32, _P, _I32, _I32, _U32, _P, ctypes.POINTER(_P)]),
     "rslm_rotate_queries": (ctypes.c_int, [_P, _I32, _P, _I64, _P, _P]),
     "rslm_probe": (ctypes.c_int, [_P, _P, _I64, _I32, _P, _P, _P]),
     "rslm_probe_noalloc": (ctypes.c_int, [_P, _P, _I64, _I32, _P, _P, _P]),
@@ -48,6 +49,7 @@ SIGNATURES = {
     "rslm_profile_read": (ctypes.c_int, [_P, ctypes.POINTER(_D), ctypes.POINTER(_I64), _P, _I32]),
     "rslm_decompress": (ctypes.c_int, [_P, _I32, _I64, _I64, _P, _P]),
     "rslm_sync": (ctypes.c_int, [_P, _P]),
+    "rslm_counters": (ctypes.c_int, [_P, ctypes.POINTER(_I64), _I32]),
     "rslm_last_error": (ctypes.c_char_p, []),
     "rslm_index_destroy": (None, [_P]),
 }
@@ -159,6 +161,20 @@ def rslm_encode(index, vectors, row_begin, rows=None, stream=None):
     rows = vectors.shape[0] if rows is None else rows
     _check(lib().rslm_encode(_ptr(index), _dev(vectors, torch.float32, "vectors"), row_begin, rows,
                              _stream(stream)))
+
+
+def rslm_encode_all(vectors, assignment, centroids, score_bits, rescore_bits=0, flags=RSLM_GLOBAL_SCALE,
+                    stream=None) -> IndexHandle:
+    """Create, reserve and encode an index from vectors [n, dim] in one call."""
+    import torch
+    n, dim = vectors.shape
+    nlist = centroids.shape[0]
+    out = _P()
+    _check(lib().rslm_encode_all(_dev(vectors, torch.float32, "vectors", n * dim),
+                                 _dev(assignment, torch.int32, "assignment", n), n, dim, nlist,
+                                 _dev(centroids, torch.float32, "centroids", nlist * dim), score_bits,
+                                 rescore_bits, flags, _stream(stream), ctypes.byref(out)))
+    return IndexHandle(out.value)
 
 
 def rslm_rotate_queries(index, which, queries, out, stream=None):
@@ -285,6 +301,16 @@ def rslm_profile_read(index):
 
 def rslm_sync(index, stream=None):
     _check(lib().rslm_sync(_ptr(index), _stream(stream)))
+
+
+COUNTERS = ("batched_short_rescans", "batched_overflow_rescans", "probe_exact_fallbacks")
+
+
+def rslm_counters(index) -> dict:
+    """Event counters of the index since creation (waits for the device)."""
+    out = (_I64 * 4)()
+    _check(lib().rslm_counters(_ptr(index), out, 4))
+    return dict(zip(COUNTERS, (int(v) for v in out)))
 
 
 def rslm_last_error() -> str:

@@ -1,7 +1,8 @@
 """Build librslm.so in-tree with nvcc for sm_103a (GB300).
 
 Translation units compile in parallel into ``_build/`` and link into
-``paper_2608_30384_gb300/librslm.so`` together with cuBLAS (the probe GEMM).
+``paper_2608_30384_gb300/librslm.so`` (CUDA runtime only: no CUDA library
+kernels).
 Run ``python -m paper_2608_30384_gb300.build`` or call ``build_library()``.
 """
 
@@ -56,7 +57,7 @@ def build_library(verbose: bool = False, extra_flags=()) -> str:
     with ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
         objs = list(ex.map(compile_one, SOURCES))
     tmp = LIB + ".tmp"
-    cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *objs, "-lcublas"]
+    cmd = [nvcc, *ARCH, "-shared", "-o", tmp, *objs]
     res = subprocess.run(cmd, capture_output=True, text=True)
     if res.returncode != 0:
         raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")

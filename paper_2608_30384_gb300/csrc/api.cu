@@ -1,5 +1,4 @@
 // api.cu -- the extern "C" entry points of librslm (declared in include/rslm.h).
-#include <cublas_v2.h>
 #include <cuda_runtime.h>
 
 #include <algorithm>
@@ -16,7 +15,6 @@ using namespace rslm;
 namespace {
 
 thread_local std::string g_last_error;
-std::mutex g_cublas_mutex;  // one cuBLAS handle per index; calls that use it are serialised
 
 rslm_status fail(rslm_status st, const std::string& msg) {
   g_last_error = msg;
@@ -64,15 +62,15 @@ cudaError_t dev_alloc(rslm_index* ix, T** p, size_t count) {
 
 void free_all(rslm_index* ix) {
   void* ptrs[] = {ix->centroids, ix->part_off, ix->part_n, ix->assign, ix->slot_of_row, ix->ids,
-                  ix->codes1,    ix->scales1,  ix->codes2, ix->scales2, ix->d_err,   ix->ctiles,
-                  ix->cmeta,     ix->crows,    ix->crot2};
+                  ix->codes1,    ix->scales1,  ix->codes2, ix->scales2, ix->d_err,   ix->ctiles, ix->d_counters,
+                  ix->cmeta,     ix->crows,    ix->crot2,   ix->cgemm};
   for (void* p : ptrs)
     if (p) cudaFree(p);
-  if (ix->cublas) cublasDestroy(reinterpret_cast<cublasHandle_t>(ix->cublas));
 }
 
-// Probe stage shared by rslm_probe and rslm_search: <q, c_p> for all p by one
-// SGEMM per query chunk, then top-nprobe selection.
+// Probe stage shared by rslm_probe and rslm_search (Sec. 5.5.1 step 3): the
+// fused tensor-core probe where it applies (padded D <= 128, nlist >= 32
+// nprobe), otherwise the tensor-core score GEMM with a row selection.
 rslm_status run_probe(const rslm_index* ix, const float* queries, int64_t nq, int nprobe,
                       int32_t* out_probes, float* out_cs, cudaStream_t s) {
   if (nq == 0) return RSLM_OK;
@@ -80,39 +78,8 @@ rslm_status run_probe(const rslm_index* ix, const float* queries, int64_t nq, in
     RSLM_CK(launch_probe_fused(ix, queries, nq, nprobe, out_probes, out_cs, s), "fused probe launch");
     return RSLM_OK;
   }
-  const int64_t budget = int64_t(64) << 20;  // floats in the score chunk (256 MB)
-  const int64_t ld = (int64_t(ix->nlist) + 3) & ~int64_t(3);  // row stride, 16-byte multiple
-  int64_t qc = budget / ld;
-  if (qc < 1) qc = 1;
-  if (qc > nq) qc = nq;
-  float* S = nullptr;
-  RSLM_CK(cudaMallocAsync(reinterpret_cast<void**>(&S), size_t(qc) * (ld + 1) * sizeof(float), s),
-          "cudaMallocAsync(probe scores)");
-  int* flags = reinterpret_cast<int*>(S + size_t(qc) * ld);  // one int per query row
-  rslm_status st = RSLM_OK;
-  {
-    std::lock_guard<std::mutex> lock(g_cublas_mutex);
-    cublasHandle_t h = reinterpret_cast<cublasHandle_t>(ix->cublas);
-    cublasSetStream(h, s);
-    const float one = 1.0f, zero = 0.0f;
-    for (int64_t q0 = 0; q0 < nq && st == RSLM_OK; q0 += qc) {
-      const int64_t n = std::min(qc, nq - q0);
-      // Row-major S[n x nlist] = Q[n x D] C^T, i.e. column-major S^T = C^T^T Q^T.
-      cublasStatus_t cb = cublasSgemm(h, CUBLAS_OP_T, CUBLAS_OP_N, ix->nlist, int(n), ix->D, &one,
-                                      ix->centroids, ix->D, queries + q0 * ix->D, ix->D, &zero, S,
-                                      int(ld));
-      if (cb != CUBLAS_STATUS_SUCCESS) {
-        st = fail(RSLM_ERR_CUDA, "cublasSgemm failed with status " + std::to_string(int(cb)));
-        break;
-      }
-      cudaError_t e = launch_select_topn(S, n, ld, ix->nlist, nprobe, out_probes + q0 * nprobe,
-                                         out_cs + q0 * nprobe, flags, s);
-      if (e != cudaSuccess) st = cuda_fail(e, "select_topn launch");
-    }
-  }
-  cudaError_t e = cudaFreeAsync(S, s);
-  if (st == RSLM_OK && e != cudaSuccess) st = cuda_fail(e, "cudaFreeAsync");
-  return st;
+  RSLM_CK(launch_probe_gemm(ix, queries, nq, nprobe, out_probes, out_cs, s), "probe GEMM launch");
+  return RSLM_OK;
 }
 
 rslm_status check_query_args(const rslm_index* ix, int64_t nq, int nprobe) {
@@ -218,10 +185,12 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
   cudaStream_t s = as_stream(stream);
   cudaError_t e = dev_alloc(ix, &ix->centroids, size_t(nlist) * dim);
   if (e == cudaSuccess) e = dev_alloc(ix, &ix->d_err, 1);
+  if (e == cudaSuccess) e = dev_alloc(ix, &ix->d_counters, kNumCounters);
   if (e == cudaSuccess)
     e = cudaMemcpyAsync(ix->centroids, centroids, size_t(nlist) * dim * sizeof(float),
                         cudaMemcpyDeviceToDevice, s);
   if (e == cudaSuccess) e = cudaMemsetAsync(ix->d_err, 0, sizeof(int), s);
+  if (e == cudaSuccess) e = cudaMemsetAsync(ix->d_counters, 0, kNumCounters * sizeof(unsigned long long), s);
   if (e == cudaSuccess) e = probe_prepare(ix, s);
   if (e == cudaSuccess && (flags & RSLM_RESCORE_READING_A) && !(flags & RSLM_FULL_VECTOR)) {
     // reading A scores <q, c> in the rescoring rotation: R2 c of every centroid
@@ -234,16 +203,6 @@ rslm_status rslm_index_create(int32_t dim, int32_t nlist, const float* centroids
     delete ix;
     return cuda_fail(e, "rslm_index_create");
   }
-  cublasHandle_t h;
-  if (cublasCreate(&h) != CUBLAS_STATUS_SUCCESS) {
-    free_all(ix);
-    delete ix;
-    return fail(RSLM_ERR_CUDA, "cublasCreate failed");
-  }
-  // FP32 GEMM with float32 accuracy, allowed to run as BF16x9 on the tensor
-  // cores when cuBLAS finds that faster.
-  cublasSetMathMode(h, CUBLAS_FP32_EMULATED_BF16X9_MATH);
-  ix->cublas = h;
   *out = ix;
   return RSLM_OK;
 }
@@ -340,6 +299,26 @@ rslm_status rslm_index_reserve(rslm_index* ix, const int32_t* assignment, int64_
   ix->n_rows = n;
   ix->n_slots = n_slots;
   ix->max_part_n = *std::max_element(pn.begin(), pn.end());
+  return RSLM_OK;
+}
+
+rslm_status rslm_encode_all(const float* vectors, const int32_t* assignment, int64_t n, int32_t dim,
+                            int32_t nlist, const float* centroids, int32_t score_bits,
+                            int32_t rescore_bits, uint32_t flags, void* stream, rslm_index** out) {
+  RSLM_ARG(out, "out is NULL");
+  *out = nullptr;
+  RSLM_ARG(n == 0 || vectors, "vectors is NULL");
+  rslm_index* ix = nullptr;
+  rslm_status st = rslm_index_create(dim, nlist, centroids, score_bits, rescore_bits, flags, stream, &ix);
+  if (st != RSLM_OK) return st;
+  st = rslm_index_reserve(ix, assignment, n, stream);
+  if (st == RSLM_OK) st = rslm_encode(ix, vectors, 0, n, stream);
+  if (st != RSLM_OK) {
+    const std::string msg = g_last_error;
+    rslm_index_destroy(ix);
+    return fail(st, msg);
+  }
+  *out = ix;
   return RSLM_OK;
 }
 
@@ -562,6 +541,17 @@ rslm_status rslm_sync(const rslm_index* ix, void* stream) {
 }
 
 const char* rslm_last_error(void) { return g_last_error.c_str(); }
+
+rslm_status rslm_counters(const rslm_index* ix, int64_t* out, int32_t n) {
+  RSLM_ARG(ix && out, "NULL argument");
+  RSLM_ARG(n >= 1 && n <= kNumCounters, "n must be in [1, 4]");
+  DeviceGuard g(ix->device);
+  RSLM_CK(cudaDeviceSynchronize(), "device synchronize");
+  unsigned long long h[kNumCounters] = {};
+  RSLM_CK(cudaMemcpy(h, ix->d_counters, sizeof(h), cudaMemcpyDeviceToHost), "read counters");
+  for (int i = 0; i < n; ++i) out[i] = int64_t(h[i]);
+  return RSLM_OK;
+}
 
 rslm_status rslm_profile_enable(rslm_index* ix, int32_t on) {
   RSLM_ARG(ix, "index is NULL");

@@ -633,6 +633,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  __syncwarp();  // warp 0 again converged: tcgen05.alloc is .sync.aligned
   if (warp == 0) {
     const uint32_t dst = uint32_t(__cvta_generic_to_shared(&tmem_base_sh));
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst),
@@ -666,8 +667,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
     const int k8n = klen / 8;
     for (uint32_t seq = 0;; ++seq) {
       const uint32_t s = seq & 1, use = seq >> 1;
-      bool ok = !(use > 0 && !mbar_wait(item_empty(s), (use - 1) & 1));
+      bool ok = !(use > 0 && !mbar_wait_warp(item_empty(s), (use - 1) & 1));
       if (!ok) fail();
+      fence_proxy_async();  // the MMAs' reads of this slot (async proxy) before its new generic stores
       uint8_t* sb = slot(s);
       ItemDesc* d = reinterpret_cast<ItemDesc*>(sb + kOffDesc);
       if (lt == 0) {
@@ -833,7 +835,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
     bool ok = true;
     for (uint32_t seq = 0; ok; ++seq) {
       const uint32_t s = seq & 1;
-      if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+      if (!mbar_wait_warp(item_full(s), (seq >> 1) & 1)) {
         fail();
         break;
       }
@@ -842,7 +844,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
       for (int t = 0; t < ntiles; ++t, ++gt) {
         const uint32_t sb = gt % kSlabs, us = gt / kSlabs;
-        if (!mbar_wait(slab_full(sb), us & 1)) {
+        if (!mbar_wait_warp(slab_full(sb), us & 1)) {
           fail();
           ok = false;
           break;
@@ -851,15 +853,17 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         constexpr int NW = row_words(G, FMT);
         uint32_t wd[NW];
         load_row_words<NW>(slab0 + sb * slab_bytes(G), r, FMT == kFmt3 ? 4 : CH, c1, wd);
+        fence_proxy_async();  // generic reads of the slab before the next bulk copy into it
         __syncwarp();
         if (lane == 0) mbar_arrive(slab_empty(sb));
         // A buffer b is free once the MMAs of tile gt - 2 have completed
         const uint32_t b = gt & 1, u = gt >> 1;
-        if (u > 0 && !mbar_wait(a_free(b), (u - 1) & 1)) {
+        if (u > 0 && !mbar_wait_warp(a_free(b), (u - 1) & 1)) {
           fail();
           ok = false;
           break;
         }
+        __syncwarp();  // converged for the .sync.aligned tcgen05.st (also on a buffer's first use)
         fence_after_sync();
 #pragma unroll
         for (int dh = 0; dh < 2; ++dh) {
@@ -881,7 +885,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
     bool ok = true;
     for (uint32_t seq = 0; ok; ++seq) {
       const uint32_t s = seq & 1;
-      if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+      if (!mbar_wait_warp(item_full(s), (seq >> 1) & 1)) {
         fail();
         break;
       }
@@ -901,12 +905,15 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row);
         // the tile's scales (scale stage ss)
         const uint32_t ss = gt % kScaleStages;
-        if (!mbar_wait(scale_full(ss), (gt / kScaleStages) & 1)) {
+        if (!mbar_wait_warp(scale_full(ss), (gt / kScaleStages) & 1)) {
           fail();
           ok = false;
           break;
         }
         const uint32_t sc = scl0[ss * kMR + row];
+        // the generic read must be ordered before the next bulk copy into
+        // this stage (async proxy) that the release below allows
+        fence_proxy_async();
         __syncwarp();
         if (lane == 0) mbar_arrive(scale_empty(ss));
         float L = 0.0f, Gs = 0.0f;
@@ -914,7 +921,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           L = ue7m9_to_f32(sc & 0xffffu);
           Gs = ue4m12_to_f32(sc >> 16);
         }
-        if (!mbar_wait(acc_full(b), u & 1)) {
+        if (!mbar_wait_warp(acc_full(b), u & 1)) {
           fail();
           ok = false;
           break;
@@ -1034,6 +1041,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  __syncwarp();  // warp 0 again converged: tcgen05.alloc is .sync.aligned
   if (warp == 0) {
     const uint32_t dst = uint32_t(__cvta_generic_to_shared(&tmem_base_sh));
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst),
@@ -1070,7 +1078,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
     bool ok = true;
     for (uint32_t seq = 0; ok; ++seq) {
       const uint32_t s = seq & 1, use = seq >> 1;
-      if (use > 0 && !mbar_wait(item_empty(s), (use - 1) & 1)) {
+      if (use > 0 && !mbar_wait_warp(item_empty(s), (use - 1) & 1)) {
         fail();
         ok = false;
       }
@@ -1122,11 +1130,12 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
       for (int g = 0; g < ngroups && ok; ++g) {
         for (int kc = 0; kc < nkc; ++kc, ++bseq) {
           const uint32_t bs = bseq & 1, bu = bseq >> 1;
-          if (bu > 0 && !mbar_wait(b_empty(bs), (bu - 1) & 1)) {
+          if (bu > 0 && !mbar_wait_warp(b_empty(bs), (bu - 1) & 1)) {
             fail();
             ok = false;
             break;
           }
+          fence_proxy_async();  // the MMAs' reads of this stage (async proxy) before its new generic stores
           uint8_t* dst = bst0 + bs * kBStageBytes;
           const int k8n = klen_of(kc) / 8;
           // loads in batches of four 16-byte pieces, then shared stores (lane =
@@ -1287,7 +1296,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
     bool ok = true;
     for (uint32_t seq = 0; ok; ++seq) {
       const uint32_t s = seq & 1;
-      if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+      if (!mbar_wait_warp(item_full(s), (seq >> 1) & 1)) {
         fail();
         break;
       }
@@ -1300,7 +1309,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
           const int c_n = min(cpk, nchunks_row - kc * cpk);  // code chunks of this K chunk
           for (int r = 0; r < R; ++r, ++sseq, ++aseq) {
             const uint32_t sb = sseq % kSlabs;
-            if (!mbar_wait(slab_full(sb), (sseq / kSlabs) & 1)) {
+            if (!mbar_wait_warp(slab_full(sb), (sseq / kSlabs) & 1)) {
               fail();
               ok = false;
               break;
@@ -1308,14 +1317,16 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
             constexpr int NW = row_words(G, FMT);
             uint32_t wd[NW];
             load_row_words<NW>(slab0 + sb * slab_bytes(G), row, FMT == kFmt3 ? 4 : CH, c_n, wd);
+            fence_proxy_async();  // generic reads of the slab before the next bulk copy into it
             __syncwarp();
             if (lane == 0) mbar_arrive(slab_empty(sb));
             const uint32_t ab = aseq & 1, au = aseq >> 1;
-            if (au > 0 && !mbar_wait(a_free(ab), (au - 1) & 1)) {
+            if (au > 0 && !mbar_wait_warp(a_free(ab), (au - 1) & 1)) {
               fail();
               ok = false;
               break;
             }
+            __syncwarp();  // converged for the .sync.aligned tcgen05.st (also on a buffer's first use)
             fence_after_sync();
 #pragma unroll
             for (int dh = 0; dh < 2; ++dh) {
@@ -1340,7 +1351,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
     bool ok = true;
     for (uint32_t seq = 0; ok; ++seq) {
       const uint32_t s = seq & 1;
-      if (!mbar_wait(item_full(s), (seq >> 1) & 1)) {
+      if (!mbar_wait_warp(item_full(s), (seq >> 1) & 1)) {
         fail();
         break;
       }
@@ -1358,12 +1369,15 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
         const int nvalid = min(kMR, nrows - t * kMR);
         const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row);
         const uint32_t ss = cseq % kScaleStages;
-        if (!mbar_wait(scale_full(ss), (cseq / kScaleStages) & 1)) {
+        if (!mbar_wait_warp(scale_full(ss), (cseq / kScaleStages) & 1)) {
           fail();
           ok = false;
           break;
         }
         const uint32_t sc = scl0[ss * kMR + row];
+        // the generic read must be ordered before the next bulk copy into
+        // this stage (async proxy) that the release below allows
+        fence_proxy_async();
         __syncwarp();
         if (lane == 0) mbar_arrive(scale_empty(ss));
         float L = 0.0f, Gs = 0.0f;
@@ -1371,7 +1385,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
           L = ue7m9_to_f32(sc & 0xffffu);
           Gs = ue4m12_to_f32(sc >> 16);
         }
-        if (!mbar_wait(acc_full(r), accu[r] & 1)) {
+        if (!mbar_wait_warp(acc_full(r), accu[r] & 1)) {
           fail();
           ok = false;
           break;
@@ -1455,25 +1469,33 @@ __global__ void finalize_kernel(const float* __restrict__ buf_s, const int32_t* 
 // The same result by one warp per query for buffers of at most kFinCap
 // candidates: sort them in shared memory by (score desc, id asc).  A longer
 // buffer is listed for finalize_kernel, an overflowed one (more than cap
-// candidates) for the single-query re-scan.
+// candidates) for the single-query re-scan.  So is a buffer with fewer than
+// k candidates under a finite theta: k candidates of the first probed list
+// reach theta, so pass 2 must keep at least k, and a shorter list means the
+// two passes disagreed; the exact re-scan answers it and ctr counts it.
 constexpr int kFinCap = 512;
 constexpr int kFinWarps = 4;
 __global__ void __launch_bounds__(kFinWarps * 32) finalize_warp_kernel(
     const float* __restrict__ buf_s, const int32_t* __restrict__ buf_p, const int* __restrict__ cnt,
-    int64_t nq, int cap, const int64_t* __restrict__ ids, int k, int* __restrict__ ovf_list,
-    int* __restrict__ blk_list, int* __restrict__ counts, int64_t* __restrict__ out_ids,
-    float* __restrict__ out_scores) {
+    int64_t nq, int cap, const int64_t* __restrict__ ids, int k, const float* __restrict__ theta,
+    int* __restrict__ ovf_list, int* __restrict__ blk_list, int* __restrict__ counts,
+    unsigned long long* __restrict__ ctr, int64_t* __restrict__ out_ids, float* __restrict__ out_scores) {
   __shared__ uint32_t fk[kFinWarps][kFinCap];
   __shared__ int64_t fi[kFinWarps][kFinCap];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const int64_t q = int64_t(blockIdx.x) * kFinWarps + w;
   if (q >= nq) return;
   const int n = cnt[q];
-  if (n > cap || n > kFinCap) {
-    // counts[0]: overflowed queries, counts[1]: queries for the block kernel
+  const bool short_list = n < k && theta[q] > -CUDART_INF_F;
+  if (n > cap || n > kFinCap || short_list) {
+    // counts[0]: queries for the exact re-scan, counts[1]: queries for the block kernel
     if (lane == 0) {
-      if (n > cap) ovf_list[atomicAdd(&counts[0], 1)] = int(q);
-      else blk_list[atomicAdd(&counts[1], 1)] = int(q);
+      if (n > cap || short_list) {
+        ovf_list[atomicAdd(&counts[0], 1)] = int(q);
+        atomicAdd(&ctr[short_list ? kCtrBatchedShort : kCtrBatchedOverflow], 1ull);
+      } else {
+        blk_list[atomicAdd(&counts[1], 1)] = int(q);
+      }
     }
     return;
   }
@@ -1736,14 +1758,14 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
       e = cudaMemsetAsync(fcounts, 0, 2 * sizeof(int), s);
       if (e == cudaSuccess) {
         finalize_warp_kernel<<<unsigned((nq + kFinWarps - 1) / kFinWarps), kFinWarps * 32, 0, s>>>(
-            bs, bp, bc, nq, cap, ix->ids, k, ovf, ac, fcounts, out_ids, out_scores);
+            bs, bp, bc, nq, cap, ix->ids, k, theta, ovf, ac, fcounts, ix->d_counters, out_ids, out_scores);
         finalize_kernel<<<unsigned(std::min<int64_t>(nq, 2 * 152)), 256, smem, s>>>(
             bs, bp, bc, cap, ix->ids, k, ac, fcounts + 1, out_ids, out_scores);
         e = cudaGetLastError();
       }
     }
   }
-  // Queries whose buffer overflowed: exact single-query scan of all probes.
+  // Queries whose buffer overflowed (or came out short): exact single-query scan of all probes.
   if (e == cudaSuccess)
     e = launch_scan_listed(ix, qrot, nq, probes, nprobe, cs, nprobe, k, out_ids, out_scores, ovf, fcounts,
                            s);

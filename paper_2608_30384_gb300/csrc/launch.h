@@ -47,12 +47,15 @@ cudaError_t launch_rescore(const rslm_index* ix, const float* qrot2, int64_t nq,
                            const int64_t* cand_ids, const float* cand_scores, int k, int k_final,
                            int64_t* out_ids, float* out_scores, cudaStream_t s);
 
-// Fused tensor-core probe (probe.cu).  probe_prepare builds the centroid
-// operand of an index with D <= 128 (a no-op otherwise);
-// probe_fused_supported says whether launch_probe_fused can serve nprobe.
+// Tensor-core probes (probe.cu).  probe_prepare builds the centroid
+// operands (the GEMM's for every shape, the fused probe's for padded
+// D <= 128); probe_fused_supported says whether launch_probe_fused can serve
+// nprobe; launch_probe_gemm serves every shape (score matrix + selection).
 cudaError_t probe_prepare(rslm_index* ix, cudaStream_t s);
 bool probe_fused_supported(const rslm_index* ix, int nprobe);
 cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64_t nq, int nprobe,
                                int32_t* out_probes, float* out_cs, cudaStream_t s);
+cudaError_t launch_probe_gemm(const rslm_index* ix, const float* queries, int64_t nq, int nprobe,
+                              int32_t* out_probes, float* out_cs, cudaStream_t s);
 
 }  // namespace rslm

@@ -290,6 +290,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
       }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
+  __syncwarp();  // warp 0 again converged: tcgen05.alloc is .sync.aligned
   if (warp == 0) {
     const uint32_t dst = uint32_t(__cvta_generic_to_shared(&tmem_base_sh));
     asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst), "r"(kPCols)
@@ -409,7 +410,7 @@ __global__ void __launch_bounds__(kPThreads, 1) probe_kernel(const __grid_consta
       }
       if (dead) continue;
       const uint32_t b = uint32_t(gt & 1), ub = uint32_t(gt >> 1);
-      if (!mbar_wait(mma_done(m, b), ub & 1)) {
+      if (!mbar_wait_warp(mma_done(m, b), ub & 1)) {
         set_device_error(a.err, kErrTimeout);
         dead = true;
         continue;
@@ -559,7 +560,7 @@ constexpr int kSelWarpsPerBlock = 4;
 __global__ void __launch_bounds__(kSelWarpsPerBlock * 32) probe_select_kernel(
     int64_t nq, const uint64_t* __restrict__ keys, const int* __restrict__ cnt, int cap, int k,
     const float* __restrict__ qinv, int* __restrict__ nexact, int32_t* __restrict__ exact_q,
-    int32_t* __restrict__ out_probes, float* __restrict__ out_cs) {
+    unsigned long long* __restrict__ ctr, int32_t* __restrict__ out_probes, float* __restrict__ out_cs) {
   __shared__ uint64_t ss[kSelWarpsPerBlock][256];
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
   const unsigned lt = (1u << lane) - 1u;
@@ -569,7 +570,10 @@ __global__ void __launch_bounds__(kSelWarpsPerBlock * 32) probe_select_kernel(
   for (int64_t q = int64_t(blockIdx.x) * kSelWarpsPerBlock + w; q < nq; q += nw) {
     const int half = cap / 2, n0 = cnt[2 * q], n1 = cnt[2 * q + 1], n = n0 + n1;
     if (n0 > half || n1 > half || n < k) {
-      if (lane == 0) exact_q[atomicAdd(nexact, 1)] = int32_t(q);
+      if (lane == 0) {
+        exact_q[atomicAdd(nexact, 1)] = int32_t(q);
+        atomicAdd(&ctr[kCtrProbeExact], 1ull);
+      }
       continue;
     }
     // entry e of the list: the first n0 from half 0's segment, then half 1's
@@ -737,6 +741,278 @@ __global__ void __launch_bounds__(kExactWarpsPerBlock * 32) probe_exact_kernel(
   }
 }
 
+// ------------------------------------------------------------ probe GEMM
+// For every other shape (padded D > 128, or fewer than 32 nprobe
+// centroids) the probe scores form the matrix S = Q C^T, nq x nlist, which
+// probe_gemm_kernel computes on the tensor cores and the row selection
+// kernels then reduce to the top nprobe of each row.  Operands are split
+// like the fused probe's (x = x_hi + x_lo, scaled by powers of two) and
+// S = (<q_hi, c_hi> + <q_lo, c_hi> + <q_hi, c_lo>) / (2^sq 2^sC), within
+// delta3 = 2^-14 ||q|| max ||c|| of <q, c> (the bound of the fused probe's
+// second pass; the accumulation runs over K chunks of 32 dims instead of
+// one chunk of up to 128).
+//
+// Pre-tiled operand blocks, one 1-D bulk copy each: for every tile of
+// kGM = 128 queries (kGN = 256 centroids) and every K chunk of kGK = 32
+// dims, the hi block then the lo block, each K-major without swizzle (core
+// matrices of 8 rows x 16 bytes; K-adjacent ones 128 bytes apart, 8-row
+// groups 512 bytes apart).
+constexpr int kGM = 128, kGN = 256, kGK = 32;
+constexpr int kGStages = 4;
+constexpr int kGSbo = (kGK / 8) * 128;                  // bytes between 8-row groups
+constexpr int kGBlockA = 2 * kGM * kGK * 2;             // hi + lo of a query block (16 KB)
+constexpr int kGBlockB = 2 * kGN * kGK * 2;             // hi + lo of a centroid block (32 KB)
+constexpr int kGStageBytes = kGBlockA + kGBlockB;
+constexpr int kGEpiWarps = 8;                           // (lane quadrant, column half of 128)
+constexpr int kGTmaWarp = kGEpiWarps, kGMmaWarp = kGEpiWarps + 1;
+constexpr int kGThreads = (kGEpiWarps + 2) * 32;
+constexpr uint32_t kGCols = 512;                        // two accumulators of 256 columns
+
+__host__ __device__ constexpr int gemm_kchunks(int D) { return (D + kGK - 1) / kGK; }
+
+__device__ __forceinline__ uint32_t gblock_off(int r, int k) {
+  return uint32_t((r >> 3) * kGSbo + (k >> 3) * 128 + (r & 7) * 16 + (k & 7) * 2);
+}
+
+// Centroid blocks [N tile][K chunk] of c * 2^sC (meta[2] = 2^sC, set by
+// centroid_tiles_meta_kernel); rows beyond nlist and dims beyond D are zero.
+__global__ void centroid_gemm_blocks_kernel(const float* __restrict__ C, int nlist, int D,
+                                            const float* __restrict__ meta, uint8_t* __restrict__ out) {
+  const float sc = meta[2];
+  const int nkc = gemm_kchunks(D), ntn = (nlist + kGN - 1) / kGN;
+  const int64_t total = int64_t(ntn) * kGN * nkc * (kGK / 8);
+  for (int64_t i = blockIdx.x * int64_t(blockDim.x) + threadIdx.x; i < total;
+       i += int64_t(gridDim.x) * blockDim.x) {
+    const int k8 = int(i % (nkc * (kGK / 8)));  // 8-dim group of the row
+    const int64_t p = i / (nkc * (kGK / 8));
+    __align__(16) __half h[8], l[8];
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      const int d = k8 * 8 + j;
+      split_half((p < nlist && d < D) ? C[p * D + d] * sc : 0.0f, h[j], l[j]);
+    }
+    const int kc = k8 / (kGK / 8), kk = (k8 % (kGK / 8)) * 8;
+    uint8_t* blk = out + (size_t(p / kGN) * nkc + kc) * kGBlockB;
+    const uint32_t off = gblock_off(int(p % kGN), kk);
+    *reinterpret_cast<uint4*>(blk + off) = *reinterpret_cast<const uint4*>(h);
+    *reinterpret_cast<uint4*>(blk + kGBlockB / 2 + off) = *reinterpret_cast<const uint4*>(l);
+  }
+}
+
+// 2^sC from the centroids' largest |c| (meta[0]), as centroid_tiles_kernel
+// does for the fused probe.
+__global__ void centroid_tiles_meta_kernel(float* __restrict__ meta) {
+  const float sc = ldexpf(1.0f, pow2_exp_for(meta[0]));
+  meta[2] = sc;
+  meta[3] = sqrtf(meta[1]) * sc;
+}
+
+// Query blocks [M tile][K chunk] of q * 2^sq for the nq queries (rows up to
+// the next multiple of kGM are zero); qinv[q] = 1 / (2^sq 2^sC).
+__global__ void query_gemm_blocks_kernel(const float* __restrict__ Q, int64_t nq, int D,
+                                         const float* __restrict__ meta, uint8_t* __restrict__ out,
+                                         float* __restrict__ qinv) {
+  const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, W = blockDim.x >> 5;
+  const int nkc = gemm_kchunks(D);
+  const int64_t nqp = (nq + kGM - 1) / kGM * kGM;
+  for (int64_t q = int64_t(blockIdx.x) * W + warp; q < nqp; q += int64_t(gridDim.x) * W) {
+    float m = 0.0f;
+    if (q < nq)
+      for (int d = lane; d < D; d += 32) m = fmaxf(m, fabsf(Q[q * D + d]));
+#pragma unroll
+    for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
+    const int sq = pow2_exp_for(m);
+    const float sc = ldexpf(1.0f, sq);
+    const int r = int(q % kGM);
+    for (int k8 = lane; k8 < nkc * (kGK / 8); k8 += 32) {
+      __align__(16) __half h[8], l[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int d = k8 * 8 + j;
+        split_half((q < nq && d < D) ? Q[q * D + d] * sc : 0.0f, h[j], l[j]);
+      }
+      const int kc = k8 / (kGK / 8), kk = (k8 % (kGK / 8)) * 8;
+      uint8_t* blk = out + (size_t(q / kGM) * nkc + kc) * kGBlockA;
+      const uint32_t off = gblock_off(r, kk);
+      *reinterpret_cast<uint4*>(blk + off) = *reinterpret_cast<const uint4*>(h);
+      *reinterpret_cast<uint4*>(blk + kGBlockA / 2 + off) = *reinterpret_cast<const uint4*>(l);
+    }
+    if (lane == 0 && q < nq) qinv[q] = ldexpf(1.0f, -sq) / meta[2];
+  }
+}
+
+struct GemmArgs {
+  const uint8_t* qblk;  // query blocks of this call's nq queries
+  const uint8_t* cblk;  // centroid blocks of the index
+  const float* qinv;
+  int64_t nq;
+  int nlist, nkc, ntm, ntn;
+  float* S;    // [nq][ld] fp32 scores
+  int64_t ld;  // row stride of S, a multiple of 4
+  int* err;
+};
+
+// Persistent CTAs, one per SM, take the (M tile, N tile) units in M-major
+// order (CTAs running at the same time share query blocks in L2).  Roles:
+//   warp 8  lane 0 streams each unit's (query, centroid) block pairs of all K
+//           chunks through kGStages shared-memory stages;
+//   warp 9  lane 0 issues three 128 x 256 x 16 MMAs per 16 dims into one of
+//           two 256-column TMEM accumulators (the epilogue of one unit
+//           overlaps the next unit's MMAs);
+//   warps 0-7 read their lane quadrant's 128 columns, scale each row by its
+//           qinv and store the scores.
+// Every wait is bounded; a timeout sets the error flag and ends every role.
+__global__ void __launch_bounds__(kGThreads, 1) probe_gemm_kernel(const __grid_constant__ GemmArgs a) {
+  extern __shared__ __align__(128) uint8_t gsm[];
+  __shared__ __align__(8) uint64_t bars[2 * kGStages + 5];
+  __shared__ uint32_t tmem_base_sh;
+  __shared__ int s_fail;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
+  auto full = [&](uint32_t s) { return bar0 + 8u * s; };
+  auto empty = [&](uint32_t s) { return bar0 + 8u * (kGStages + s); };
+  auto acc_full = [&](uint32_t b) { return bar0 + 8u * (2 * kGStages + b); };
+  auto acc_empty = [&](uint32_t b) { return bar0 + 8u * (2 * kGStages + 2 + b); };
+  const uint32_t drain = bar0 + 8u * (2 * kGStages + 4);  // every MMA of the CTA completed
+  if (tid == 0) {
+    s_fail = 0;
+    mbar_init(drain, 1);
+    for (uint32_t s = 0; s < kGStages; ++s) {
+      mbar_init(full(s), 1);
+      mbar_init(empty(s), 1);
+    }
+    for (uint32_t b = 0; b < 2; ++b) {
+      mbar_init(acc_full(b), 1);
+      mbar_init(acc_empty(b), kGEpiWarps);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncwarp();  // warp 0 again converged: tcgen05.alloc is .sync.aligned
+  if (warp == 0) {
+    const uint32_t dst = uint32_t(__cvta_generic_to_shared(&tmem_base_sh));
+    asm volatile("tcgen05.alloc.cta_group::1.sync.aligned.shared::cta.b32 [%0], %1;" ::"r"(dst), "r"(kGCols)
+                 : "memory");
+    asm volatile("tcgen05.relinquish_alloc_permit.cta_group::1.sync.aligned;" ::: "memory");
+  }
+  fence_before_sync();
+  __syncthreads();
+  fence_after_sync();
+  const uint32_t tmem = tmem_base_sh;
+  const uint32_t sm_addr = uint32_t(__cvta_generic_to_shared(gsm));
+  const int64_t nunits = int64_t(a.ntm) * a.ntn;
+  auto failed = [&]() { return *reinterpret_cast<volatile int*>(&s_fail) != 0; };
+  auto fail = [&]() {
+    set_device_error(a.err, kErrTimeout);
+    atomicExch(&s_fail, 1);
+  };
+
+  if (warp == kGTmaWarp) {
+    if (lane == 0) {
+      uint32_t it = 0;
+      bool ok = true;
+      for (int64_t u = blockIdx.x; ok && u < nunits && !failed(); u += gridDim.x) {
+        const int64_t mt = u / a.ntn, nt = u % a.ntn;
+        for (int kc = 0; kc < a.nkc; ++kc, ++it) {
+          const uint32_t s = it % kGStages, use = it / kGStages;
+          if (use > 0 && !mbar_wait(empty(s), (use - 1) & 1)) {
+            fail();
+            ok = false;
+            break;
+          }
+          const uint32_t dst = sm_addr + s * uint32_t(kGStageBytes);
+          mbar_arrive_expect(full(s), uint32_t(kGStageBytes));
+          bulk_copy_1d(dst, a.qblk + (size_t(mt) * a.nkc + kc) * kGBlockA, uint32_t(kGBlockA), full(s));
+          bulk_copy_1d(dst + kGBlockA, a.cblk + (size_t(nt) * a.nkc + kc) * kGBlockB, uint32_t(kGBlockB), full(s));
+        }
+      }
+      // no copy may still be landing when the CTA exits
+      for (uint32_t s = 0; s < kGStages && s < it; ++s) mbar_wait(full(s), ((it - 1 - s) / kGStages) & 1);
+    }
+    __syncwarp();
+  } else if (warp == kGMmaWarp) {
+    if (lane == 0) {
+      const uint32_t idesc = f16_idesc(kGM, kGN);
+      uint32_t it = 0, nb = 0;
+      bool ok = true;
+      for (int64_t u = blockIdx.x; ok && u < nunits && !failed(); u += gridDim.x, ++nb) {
+        const uint32_t b = nb & 1, ub = nb >> 1;
+        if (ub > 0 && !mbar_wait(acc_empty(b), (ub - 1) & 1)) {
+          fail();
+          break;
+        }
+        fence_after_sync();
+        const uint32_t acc = tmem + b * uint32_t(kGN);
+        for (int kc = 0; kc < a.nkc; ++kc, ++it) {
+          const uint32_t s = it % kGStages;
+          if (!mbar_wait(full(s), (it / kGStages) & 1)) {
+            fail();
+            ok = false;
+            break;
+          }
+          fence_after_sync();
+          const uint32_t ahi = sm_addr + s * uint32_t(kGStageBytes), alo = ahi + kGBlockA / 2;
+          const uint32_t bhi = ahi + kGBlockA, blo = bhi + kGBlockB / 2;
+#pragma unroll
+          for (int ks = 0; ks < kGK / 16; ++ks) {
+            const uint32_t o = uint32_t(ks * 256);
+            umma_f16(acc, smem_desc(ahi + o, 128, kGSbo), smem_desc(bhi + o, 128, kGSbo), idesc,
+                     (kc > 0 || ks > 0) ? 1u : 0u);
+            umma_f16(acc, smem_desc(alo + o, 128, kGSbo), smem_desc(bhi + o, 128, kGSbo), idesc, 1u);
+            umma_f16(acc, smem_desc(ahi + o, 128, kGSbo), smem_desc(blo + o, 128, kGSbo), idesc, 1u);
+          }
+          umma_commit(empty(s));
+        }
+        if (!ok) break;
+        umma_commit(acc_full(b));
+      }
+      // no MMA may still be running when TMEM is freed (also after a timeout):
+      // a commit tracks every MMA this thread issued
+      umma_commit(drain);
+      mbar_wait(drain, 0);
+    }
+    __syncwarp();
+  } else {
+    // epilogue: rows of quadrant warp % 4, columns (warp / 4) * 128 ..
+    const int quad = warp & 3, ch = warp >> 2;
+    const int row = quad * 32 + lane;
+    uint32_t nb = 0;
+    for (int64_t u = blockIdx.x; u < nunits && !failed(); u += gridDim.x, ++nb) {
+      const int64_t mt = u / a.ntn, nt = u % a.ntn;
+      const uint32_t b = nb & 1, ub = nb >> 1;
+      if (!mbar_wait_warp(acc_full(b), ub & 1)) {
+        fail();
+        break;
+      }
+      fence_after_sync();
+      const int64_t q = mt * kGM + row;
+      const bool valid = q < a.nq;
+      const float inv = valid ? a.qinv[q] : 0.0f;
+      float* dst = a.S + (valid ? q : 0) * a.ld;
+#pragma unroll 1
+      for (int c = 0; c < 4; ++c) {
+        float v[32];
+        tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + b * uint32_t(kGN) + uint32_t(ch * 128 + c * 32), v);
+        const int64_t col0 = nt * kGN + ch * 128 + c * 32;
+        if (valid) {
+#pragma unroll
+          for (int j = 0; j < 32; j += 4)
+            if (col0 + j < a.ld)
+              *reinterpret_cast<float4*>(dst + col0 + j) =
+                  make_float4(v[j] * inv, v[j + 1] * inv, v[j + 2] * inv, v[j + 3] * inv);
+        }
+      }
+      fence_before_sync();
+      __syncwarp();
+      if (lane == 0) mbar_arrive(acc_empty(b));
+    }
+  }
+  __syncthreads();
+  if (warp == 0) {
+    fence_after_sync();
+    asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kGCols) : "memory");
+  }
+}
+
 }  // namespace
 
 bool probe_fused_supported(const rslm_index* ix, int nprobe) {
@@ -744,20 +1020,80 @@ bool probe_fused_supported(const rslm_index* ix, int nprobe) {
 }
 
 cudaError_t probe_prepare(rslm_index* ix, cudaStream_t s) {
-  const int Kp = (ix->D + 15) / 16 * 16;
-  if (Kp > 128) return cudaSuccess;  // the fused probe keeps whole rows in one K chunk
-  const int ntiles = (ix->nlist + kPRows - 1) / kPRows;
-  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&ix->ctiles), size_t(2) * ntiles * tile_bytes(Kp));
+  // centroid statistics and scale (both probes)
+  cudaError_t e = cudaMalloc(reinterpret_cast<void**>(&ix->cmeta), 4 * sizeof(float));
   if (e != cudaSuccess) return e;
-  e = cudaMalloc(reinterpret_cast<void**>(&ix->cmeta), 4 * sizeof(float));
+  ix->device_bytes += 16;
+  centroid_stats_kernel<<<1, 1024, 0, s>>>(ix->centroids, ix->nlist, ix->D, ix->cmeta);
+  centroid_tiles_meta_kernel<<<1, 1, 0, s>>>(ix->cmeta);
+  // probe GEMM operand (every shape)
+  const size_t gbytes = size_t((ix->nlist + kGN - 1) / kGN) * gemm_kchunks(ix->D) * kGBlockB;
+  e = cudaMalloc(reinterpret_cast<void**>(&ix->cgemm), gbytes);
+  if (e != cudaSuccess) return e;
+  ix->device_bytes += int64_t(gbytes);
+  centroid_gemm_blocks_kernel<<<152 * 4, 256, 0, s>>>(ix->centroids, ix->nlist, ix->D, ix->cmeta, ix->cgemm);
+  const int Kp = (ix->D + 15) / 16 * 16;
+  if (Kp > 128) return cudaGetLastError();  // the fused probe keeps whole rows in one K chunk
+  const int ntiles = (ix->nlist + kPRows - 1) / kPRows;
+  e = cudaMalloc(reinterpret_cast<void**>(&ix->ctiles), size_t(2) * ntiles * tile_bytes(Kp));
   if (e != cudaSuccess) return e;
   e = cudaMalloc(reinterpret_cast<void**>(&ix->crows), size_t(ix->nlist) * Kp * sizeof(float));
   if (e != cudaSuccess) return e;
-  ix->device_bytes += int64_t(2) * ntiles * tile_bytes(Kp) + 16 + int64_t(ix->nlist) * Kp * 4;
+  ix->device_bytes += int64_t(2) * ntiles * tile_bytes(Kp) + int64_t(ix->nlist) * Kp * 4;
   centroid_rows_kernel<<<152 * 4, 256, 0, s>>>(ix->centroids, ix->nlist, ix->D, Kp, ix->crows);
-  centroid_stats_kernel<<<1, 1024, 0, s>>>(ix->centroids, ix->nlist, ix->D, ix->cmeta);
   centroid_tiles_kernel<<<152 * 4, 256, 0, s>>>(ix->centroids, ix->nlist, ix->D, Kp, ix->cmeta, ix->ctiles);
   return cudaGetLastError();
+}
+
+cudaError_t launch_probe_gemm(const rslm_index* ix, const float* queries, int64_t nq, int nprobe,
+                              int32_t* out_probes, float* out_cs, cudaStream_t s) {
+  if (nq == 0) return cudaSuccess;
+  const int nkc = gemm_kchunks(ix->D);
+  const int64_t ld = (int64_t(ix->nlist) + 3) & ~int64_t(3);  // row stride of S, a 16-byte multiple
+  const int64_t budget = int64_t(64) << 20;                   // floats of S per query chunk (256 MB)
+  int64_t qc = std::max<int64_t>(kGM, budget / ld / kGM * kGM);
+  qc = std::min(qc, (nq + kGM - 1) / kGM * kGM);
+  size_t bytes = 0;
+  auto take = [&](size_t n) {
+    size_t at = bytes;
+    bytes += (n + 255) / 256 * 256;
+    return at;
+  };
+  const size_t o_S = take(size_t(qc) * ld * 4), o_flags = take(size_t(qc) * 4),
+               o_qb = take(size_t(qc / kGM) * nkc * kGBlockA), o_inv = take(size_t(qc) * 4);
+  uint8_t* ws = nullptr;
+  cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, s);
+  if (e != cudaSuccess) return e;
+  int sms = 152, dev = 0;
+  if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+  const size_t smem = size_t(kGStages) * kGStageBytes;
+  e = cudaFuncSetAttribute(probe_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  for (int64_t q0 = 0; q0 < nq && e == cudaSuccess; q0 += qc) {
+    const int64_t n = std::min(qc, nq - q0);
+    const int64_t nqp = (n + kGM - 1) / kGM * kGM;
+    query_gemm_blocks_kernel<<<unsigned(std::min<int64_t>((nqp + 7) / 8, int64_t(sms) * 64)), 256, 0, s>>>(
+        queries + q0 * ix->D, n, ix->D, ix->cmeta, ws + o_qb, reinterpret_cast<float*>(ws + o_inv));
+    GemmArgs a;
+    a.qblk = ws + o_qb;
+    a.cblk = ix->cgemm;
+    a.qinv = reinterpret_cast<const float*>(ws + o_inv);
+    a.nq = n;
+    a.nlist = ix->nlist;
+    a.nkc = nkc;
+    a.ntm = int(nqp / kGM);
+    a.ntn = (ix->nlist + kGN - 1) / kGN;
+    a.S = reinterpret_cast<float*>(ws + o_S);
+    a.ld = ld;
+    a.err = ix->d_err;
+    const int64_t units = int64_t(a.ntm) * a.ntn;
+    probe_gemm_kernel<<<unsigned(std::min<int64_t>(units, sms)), kGThreads, smem, s>>>(a);
+    e = cudaGetLastError();
+    if (e == cudaSuccess)
+      e = launch_select_topn(a.S, n, ld, ix->nlist, nprobe, out_probes + q0 * nprobe, out_cs + q0 * nprobe,
+                             reinterpret_cast<int*>(ws + o_flags), s);
+  }
+  cudaError_t f = cudaFreeAsync(ws, s);
+  return e != cudaSuccess ? e : f;
 }
 
 cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64_t nq, int nprobe,
@@ -835,7 +1171,7 @@ cudaError_t launch_probe_fused(const rslm_index* ix, const float* queries, int64
     probe_select_kernel<<<unsigned(sel_blocks), kSelWarpsPerBlock * 32, 0, s>>>(
         nq, reinterpret_cast<const uint64_t*>(ws + o_keys), reinterpret_cast<const int*>(ws + o_cnt), cap,
         nprobe, reinterpret_cast<const float*>(ws + o_inv), nexact, reinterpret_cast<int32_t*>(ws + o_xq),
-        out_probes, out_cs);
+        ix->d_counters, out_probes, out_cs);
     e = cudaGetLastError();
   }
   if (e == cudaSuccess) {

@@ -1,7 +1,8 @@
 // probe_noalloc.cu -- rslm_probe_noalloc: the probe step without device allocation.
 //
-// rslm_probe computes the <query, centroid> matrix of a query chunk in a
-// temporary buffer from the stream-ordered allocator and runs cuBLAS on it.
+// rslm_probe keeps its working buffers (query operands, candidate lists or a
+// <query, centroid> score chunk) in temporary memory from the stream-ordered
+// allocator.
 // Some callers cannot allocate on the query path: applications whose device
 // memory is entirely owned by another allocator (a framework's caching
 // allocator, or a fixed budget handed out up front), and latency-critical
@@ -38,10 +39,16 @@ static __device__ __align__(256) float g_probe_scratch[kScratchFloats];
 std::mutex g_scratch_mu;
 float* g_scratch_ptr[kMaxDevices] = {};
 
-// Device address of g_probe_scratch on `dev` (which must be current).
+// Device address of g_probe_scratch on `dev`, which must be the current
+// device: the address is cached per device, so a lookup made with another
+// device current would poison every later call on `dev`.
 cudaError_t scratch_address(int dev, float** out) {
   std::lock_guard<std::mutex> lock(g_scratch_mu);
   if (!g_scratch_ptr[dev]) {
+    int cur = -1;
+    cudaError_t e0 = cudaGetDevice(&cur);
+    if (e0 != cudaSuccess) return e0;
+    if (cur != dev) return cudaErrorInvalidDevice;
     void* p = nullptr;
     cudaError_t e = cudaGetSymbolAddress(&p, g_probe_scratch);
     if (e != cudaSuccess) return e;
@@ -120,12 +127,18 @@ extern "C" rslm_status rslm_probe_noalloc(const rslm_index* ix, const float* que
     return set_last_error(RSLM_ERR_INVALID_ARG, "device ordinal beyond the scratch table");
   if (nq == 0) return RSLM_OK;
   int prev = -1;
-  cudaGetDevice(&prev);
-  if (prev != ix->device) cudaSetDevice(ix->device);
+  cudaError_t e = cudaGetDevice(&prev);
+  if (e != cudaSuccess)
+    return set_last_error(RSLM_ERR_CUDA, std::string("cudaGetDevice: ") + cudaGetErrorString(e));
+  if (prev != ix->device) {
+    e = cudaSetDevice(ix->device);
+    if (e != cudaSuccess)
+      return set_last_error(RSLM_ERR_CUDA, std::string("cudaSetDevice: ") + cudaGetErrorString(e));
+  }
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   rslm_status st = RSLM_OK;
   float* S = nullptr;
-  cudaError_t e = scratch_address(ix->device, &S);
+  e = scratch_address(ix->device, &S);
   if (e != cudaSuccess) {
     st = set_last_error(RSLM_ERR_CUDA, std::string("cudaGetSymbolAddress: ") + cudaGetErrorString(e));
   }

@@ -19,6 +19,15 @@ constexpr int kMaxK = 256;
 constexpr int kMaxNprobe = 4096;
 constexpr int kBatchMinQueries = 16;  // rslm_search: batched scan above this queries/partition
 
+// Event counters of an index (rslm_counters): queries that a search path
+// handed to an exact fallback.
+enum Counter : int {
+  kCtrBatchedShort = 0,     // pass 2 kept fewer than k candidates under a finite threshold
+  kCtrBatchedOverflow = 1,  // the pass-2 candidate buffer overflowed
+  kCtrProbeExact = 2,       // a fused-probe candidate list overflowed
+  kNumCounters = 4,
+};
+
 // Device error codes written to the index's sticky flag.
 enum DeviceError : int {
   kErrNone = 0,
@@ -103,11 +112,12 @@ struct rslm_index {
   uint8_t* codes2 = nullptr;    // rescoring codes, row-major by slot
   uint32_t* scales2 = nullptr;
   int* d_err = nullptr;         // sticky device error flag
+  unsigned long long* d_counters = nullptr;  // [kNumCounters] event counters
   uint8_t* ctiles = nullptr;    // fused probe: centroids * 2^sC as fp16 operand tiles (D <= 128)
   float* cmeta = nullptr;       // fused probe: max|c|, max||c||^2, 2^sC, max||c|| 2^sC
   float* crows = nullptr;       // fused probe: centroids as fp32 rows of Kp floats
   float* crot2 = nullptr;       // rescoring reading A: R2 c of every centroid [nlist * Dp2]
-  void* cublas = nullptr;       // cublasHandle_t
+  uint8_t* cgemm = nullptr;     // probe GEMM: centroids * 2^sC as fp16 hi / lo operand blocks
   int64_t device_bytes = 0;
   // profiling of the dominant scan kernel
   mutable std::mutex prof_mu;

@@ -10,6 +10,7 @@
 // the warp (tile-interleaved layout).  The epilogue applies the scales,
 // s = G (cs + L dot) (Sec. 3.5.2), and feeds a per-warp top-k list; the
 // lists are merged by a block sort at the end.
+#include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <math_constants.h>
 
@@ -17,6 +18,7 @@
 
 #include "device_common.cuh"
 #include "launch.h"
+#include "tcgen05.cuh"
 
 namespace rslm {
 namespace {
@@ -316,6 +318,7 @@ struct ScanArgs {
   float* out_scores;
   int* err;
   int lut_region;  // bytes of the table / merge region
+  int bt_bytes;    // byte-table form: bytes of the per-lane byte table at the start of shared memory (else 0)
 };
 
 template <int CH>
@@ -389,11 +392,33 @@ __device__ __forceinline__ uint32_t nibble_tops(uint32_t w) {
   return (t | (t >> 12)) & 0xFFu;
 }
 
-template <int CH, bool B3>
+// Byte-table form (4-bit codes with one coordinate per code, BT): instead of
+// the per-query table, a query-independent table maps a code byte (two
+// codes) to its two codebook levels as an fp16 pair, one copy per lane
+// (entry (byte, lane) at byte 256 * byte + 4 * lane: the 32 lanes of a read
+// always hit 32 distinct banks).  The levels are exact in fp16; each byte
+// then costs one table read, two conversions and one paired fp32 FMA with
+// the query pair (q[2j], q[2j + 1]) -- half the shared-memory traffic of a
+// 4-byte table entry per code.
+constexpr int kByteTableBytes = 256 * 256;
+
+template <int CH, bool B3, bool BT = false>
 __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanArgs a) {
-  extern __shared__ __align__(16) uint8_t ssm[];
+  extern __shared__ __align__(16) uint8_t ssm_all[];
   __shared__ int scratch[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, W = blockDim.x >> 5;
+  if constexpr (BT) {
+    // the byte table, once per CTA: low half = level of the low nibble
+    // (the even code position), high half = level of the high nibble
+    uint32_t* tb = reinterpret_cast<uint32_t*>(ssm_all);
+    for (int e = tid; e < 256 * 32; e += blockDim.x) {
+      const int byte = e >> 5, ln = e & 31;
+      const uint32_t lo = __half_as_ushort(__float2half_rn(a.cb[byte & 15]));
+      const uint32_t hi = __half_as_ushort(__float2half_rn(a.cb[byte >> 4]));
+      tb[byte * 64 + ln] = lo | (hi << 16);
+    }
+  }
+  uint8_t* ssm = ssm_all + a.bt_bytes;
   const int nrun = a.qlist ? *a.qcount : 1;
   for (int run0 = a.qlist ? int(blockIdx.x) : 0; run0 < nrun; run0 += a.qlist ? int(gridDim.x) : 1) {
   const int64_t q = a.qlist ? int64_t(a.qlist[run0]) : int64_t(blockIdx.x);
@@ -417,6 +442,10 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   // code's shared-memory address is then (block << 8) | (64 k + 4 code):
   // one byte permute per code builds it (see the scan loop).
   const float* qr = a.qrot + q * a.Dp;
+  if constexpr (BT) {
+    // the query itself, zero beyond Dp, one float per code position
+    for (int e = tid; e < a.lut_groups; e += blockDim.x) lut[e] = e < a.Dp ? qr[e] : 0.0f;
+  }
   if constexpr (B3) {
     // Rslm3: T[position][code] at lut[8 position + code]
     for (int e = tid; e < a.lut_groups * 8; e += blockDim.x) {
@@ -424,7 +453,7 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
       lut[e] = pos < a.ngroups ? qr[pos] * a.cb[e & 7] : 0.0f;
     }
   }
-  for (int e = tid; !B3 && e < a.lut_groups * 16; e += blockDim.x) {
+  for (int e = tid; !B3 && !BT && e < a.lut_groups * 16; e += blockDim.x) {
     const int grp = e >> 4, code = e & 15;
     float v = 0.0f;
     if (grp < a.lite_h)
@@ -497,7 +526,45 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
         }
       }
     }
-    for (int c = 0; !B3 && c < nch; ++c) {
+    if constexpr (BT) {
+      // fp32 pairs (even positions, odd positions) per row
+      uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
+      const uint32_t lane4 = uint32_t(lane) * 4u;
+#pragma unroll 1
+      for (int c = 0; c < nch; ++c) {
+        uint32_t w[4][4];
+#pragma unroll
+        for (int r = 0; r < 4; ++r) load_chunk<16>(tp + (size_t(c) * kTile + r * 32 + lane) * 16, w[r]);
+        // the 32 query values of this chunk's positions, as 16 (even, odd) pairs
+        const ulonglong2* qc = reinterpret_cast<const ulonglong2*>(lut + 32 * c);
+        uint64_t qp[16];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const ulonglong2 v = qc[i];
+          qp[2 * i] = v.x;
+          qp[2 * i + 1] = v.y;
+        }
+#pragma unroll
+        for (int v = 0; v < 4; ++v)
+#pragma unroll
+          for (int k = 0; k < 4; ++k)
+#pragma unroll
+            for (int r = 0; r < 4; ++r) {
+              // entry (byte k of word v, lane): byte 0 = 4 lane, byte 1 = the code byte
+              const uint32_t off = __byte_perm(w[r][v], lane4, 0x5504u + 0x10u * k);
+              const uint32_t h2 = *reinterpret_cast<const uint32_t*>(ssm_all + off);
+              const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&h2));
+              acc2[r] = fma2(f2pack(f.x, f.y), qp[4 * v + k], acc2[r]);
+            }
+      }
+#pragma unroll
+      for (int r = 0; r < 4; ++r) {
+        float e, o;
+        f2unpack(acc2[r], e, o);
+        acc[r] = e + o;
+      }
+    }
+    for (int c = 0; !B3 && !BT && c < nch; ++c) {
       uint32_t w[4][CH / 4];
 #pragma unroll
       for (int r = 0; r < 4; ++r)
@@ -674,17 +741,17 @@ __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ Re
   }
 }
 
-template <int CH, bool B3>
+template <int CH, bool B3, bool BT = false>
 cudaError_t launch_scan_ch(const rslm_index* ix, const ScanArgs& a, int64_t nq, size_t smem,
                            cudaStream_t s) {
   // listed queries: a fixed grid strides over the list, whose length is on the device
   const int64_t grid = a.qlist ? (nq < 2 * 152 ? nq : 2 * 152) : nq;
-  cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH, B3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH, B3, BT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        int(smem));
   if (e != cudaSuccess) return e;
   cudaEvent_t stop =
       a.only_if == nullptr && a.qlist == nullptr && a.nprobe > 1 ? prof_start(ix, s, "scan_kernel") : nullptr;
-  scan_kernel<CH, B3><<<unsigned(grid), 256, smem, s>>>(a);
+  scan_kernel<CH, B3, BT><<<unsigned(grid), 256, smem, s>>>(a);
   prof_stop(stop, s);
   return cudaGetLastError();
 }
@@ -766,13 +833,18 @@ cudaError_t launch_scan_impl(const rslm_index* ix, const float* qrot, int64_t nq
   const int W = 8;
   int np2 = 1;
   while (np2 < W * k) np2 <<= 1;
-  const size_t lut_bytes = size_t(a.lut_groups) * (b3 ? 8 : 16) * 4;
+  // byte-table form for 4-bit codes of one coordinate in 16-byte chunks
+  const bool bt = !b3 && ix->cs1.g == 1 && ix->cs1.lite_h == 0 && ix->cs1.chunk == 16;
+  const size_t lut_bytes = size_t(a.lut_groups) * (bt ? 1 : b3 ? 8 : 16) * 4;
   const size_t merge_bytes = ((size_t(np2) * 4 + 15) & ~size_t(15)) + size_t(np2) * 8;
   size_t region = lut_bytes > merge_bytes ? lut_bytes : merge_bytes;
   region = (region + 15) & ~size_t(15);
   a.lut_region = int(region);
-  const size_t smem = 256 + region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
+  a.bt_bytes = bt ? kByteTableBytes : 0;
+  const size_t smem =
+      size_t(a.bt_bytes) + 256 + region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
   if (b3) return launch_scan_ch<4, true>(ix, a, nq, smem, s);
+  if (bt) return launch_scan_ch<16, false, true>(ix, a, nq, smem, s);
   switch (ix->cs1.chunk) {
     case 16: return launch_scan_ch<16, false>(ix, a, nq, smem, s);
     case 8: return launch_scan_ch<8, false>(ix, a, nq, smem, s);

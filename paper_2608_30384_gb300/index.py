@@ -113,3 +113,6 @@ class Index:
 
     def sync(self, stream=None):
         B.rslm_sync(self.handle, stream)
+
+    def counters(self) -> dict:
+        return B.rslm_counters(self.handle)

@@ -79,7 +79,20 @@ class Case:
         return float(np.linalg.norm(self.Q[i]))
 
     def xnorm_max(self):
-        return float(np.linalg.norm(self.X.astype(np.float64), axis=1).max())
+        return float(self.xnorm().max())
+
+    def xnorm(self):
+        """||x|| of every row (row ids are row indices)."""
+        if not hasattr(self, "_xn"):
+            self._xn = np.linalg.norm(self.X.astype(np.float64), axis=1)
+        return self._xn
+
+    def score_tol_of(self, i):
+        """tol(score, row id) for query i: 1e-4 relative with the floor
+        0.01 ||q|| ||x|| of that row (the largest ||x|| when the row is not known)."""
+        from tests.lib_util import score_tol
+        xn, qn = self.xnorm(), self.qnorm(i)
+        return lambda s, j=None: float(score_tol(s, qn, xn[j] if j is not None else xn.max()))
 
 
 def check_stage(gpu_codes, gpu_L, gpu_G, enc, X, A, bits, global_scale, name):

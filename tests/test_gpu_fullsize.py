@@ -26,7 +26,7 @@ from oracle import codec, constants as K
 from oracle.rotation import rotation_matrix, rotation_mode
 from paper_2608_30384_gb300 import workloads as W
 from tests.gpu_cases import check_stage
-from tests.lib_util import check_topk, ensure_library, score_tol
+from tests.lib_util import check_topk, ensure_library, kth_of, score_tol
 
 torch = pytest.importorskip("torch")
 pytestmark = pytest.mark.gpu
@@ -88,7 +88,7 @@ class Full:
         mid = (w.N // 2) // BLOCK * BLOCK
         self.blocks = [0, mid, w.N - BLOCK]          # the last block ends at the ragged end
         self.Xb = {b: np.zeros((BLOCK, w.D), dtype=np.float32) for b in self.blocks}
-        xmax2 = 0.0
+        self.xnorm = np.empty(w.N)  # ||x|| of every row (the score tolerance's floor)
         nch = W.n_chunks(w)
         per = ENCODE_ROWS // W.CHUNK
         from concurrent.futures import ThreadPoolExecutor
@@ -98,7 +98,7 @@ class Full:
                 X = np.concatenate(parts)
                 del parts
                 lo, hi = c0 * W.CHUNK, c0 * W.CHUNK + X.shape[0]
-                xmax2 = max(xmax2, float(np.einsum("ij,ij->i", X, X, dtype=np.float64).max()))
+                self.xnorm[lo:hi] = np.sqrt(np.einsum("ij,ij->i", X, X, dtype=np.float64))
                 for b in self.blocks:
                     a0, a1 = max(lo, b), min(hi, b + BLOCK)
                     if a0 < a1:
@@ -106,7 +106,6 @@ class Full:
                 self.ix.encode(torch.from_numpy(X).cuda(), lo)
                 del X
         self.ix.sync()
-        self.xmax = math.sqrt(xmax2)
         self._rot = {}
 
     def rot(self, bits):
@@ -171,17 +170,18 @@ def _search_check(F: Full, nq: int, sampled):
         cs = F.C.astype(np.float64) @ q
         # probe: the nprobe largest <q, c_p> up to near-ties
         kth_p = np.sort(cs)[::-1][w.nprobe - 1]
-        probs = check_topk(gp[i], gcs[i], lambda j: cs[j], kth_p, lambda s: 1e-5 * qn * cmax)
+        probs = check_topk(gp[i], gcs[i], lambda j: cs[j], kth_p, lambda s, j=None: 1e-5 * qn * cmax)
         assert not probs, (i, "probe", probs[:3])
         # stage 1 over every candidate of the GPU's probe lists
         sel = np.nonzero(np.isin(F.A[s1c.rows], gp[i]))[0]
         cand = s1c.rows[sel]
         s1 = s1c.G[sel] * (cs[F.A[cand]] + s1c.L[sel] * s1c.dots(F.qrot(q, w.bits), w.bits, sel))
-        tol = lambda s: float(score_tol(s, qn, F.xmax))  # noqa: E731
+        tol = lambda s, j=None: float(score_tol(s, qn, F.xnorm[j] if j is not None else F.xnorm.max()))  # noqa: E731
         order = np.lexsort((cand, -s1))
         if not w.rescore_bits:
             ref = dict(zip(cand.tolist(), s1.tolist()))
             kth = s1[order[w.k - 1]] if cand.size >= w.k else -np.inf
+            kid = int(cand[order[w.k - 1]]) if cand.size >= w.k else None
         else:
             # stage 2 (reading B): G2 (s1 + L2 <R2 q, uhat2>) of the oracle's
             # survivors and of every id the GPU returned
@@ -192,9 +192,8 @@ def _search_check(F: Full, nq: int, sampled):
             s2 = s2c.G[pos2] * (s1[need] + s2c.L[pos2] * s2c.dots(F.qrot(q, w.rescore_bits),
                                                                  w.rescore_bits, pos2))
             ref = dict(zip(cand[need].tolist(), s2.tolist()))
-            s2_surv = np.sort(np.array([ref[c] for c in cand[surv].tolist()]))[::-1]
-            kth = s2_surv[w.k_final - 1] if s2_surv.size >= w.k_final else -np.inf
-        probs = check_topk(ids[i], sc[i], lambda j: ref[j], kth, tol, allowed_ids=ref)
+            kth, kid = kth_of({c: ref[c] for c in cand[surv].tolist()}, w.k_final)
+        probs = check_topk(ids[i], sc[i], lambda j: ref[j], kth, tol, allowed_ids=ref, kth_id=kid)
         assert not probs, (i, "results", probs[:3])
         assert (ids[i] >= 0).sum() == min(w.k_final, cand.size)
 

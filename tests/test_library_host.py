@@ -73,6 +73,13 @@ def test_argument_checks_need_no_gpu(L):
         assert L.rslm_last_error()
     st = lib.rslm_index_create(64, 4, None, 4, 0, 1, None, ctypes.byref(out))
     assert st == 1 and "centroids" in L.rslm_last_error()
+    # the one-shot encode checks its arguments before any device work
+    st = lib.rslm_encode_all(dummy, dummy, 10, 64, 4, dummy, 4, 0, 1, None, None)
+    assert st == 1 and "out" in L.rslm_last_error()
+    st = lib.rslm_encode_all(None, dummy, 10, 64, 4, dummy, 4, 0, 1, None, ctypes.byref(out))
+    assert st == 1 and "vectors" in L.rslm_last_error() and out.value is None
+    st = lib.rslm_encode_all(dummy, dummy, 10, 0, 4, dummy, 4, 0, 1, None, ctypes.byref(out))
+    assert st == 1 and out.value is None
     assert lib.rslm_e_max(0, ctypes.byref(ctypes.c_double())) == 1
     with pytest.raises(L.RslmError):
         L.rslm_codebook(5)
