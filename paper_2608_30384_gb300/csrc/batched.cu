@@ -959,6 +959,15 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
 // and each tile's scales; the MMAs of a tile accumulate over its chunks.
 // Sequence per item: for group g, for chunk kc, for tile r of the group.
 constexpr int kKR = 3;                                   // tiles per group = accumulators
+// Roles of this kernel (768 threads, like the single-chunk one): decoders
+// warps 0-3, epilogue warps 4-11 (64 query columns each, in two passes of
+// 32), MMA warp 12, TMA warp 13, loader warps 14-23.  Staging a 64 KB B
+// chunk for every K chunk of a group sets this kernel's pace, so it gets
+// ten loader warps (the epilogue works once per group of K chunks).
+constexpr int kKEpiWarps = 8, kKMmaWarp = 12, kKTmaWarp = 13, kKLoadWarp0 = 14;
+constexpr int kKLoadThreads = kPipeThreads - kKLoadWarp0 * 32;
+static_assert(kKLoadThreads >= 2 * kNQ && kKLoadThreads % 32 == 0, "the loader covers the B pieces");
+static_assert(kDecWarps + kKEpiWarps == kKMmaWarp, "the roles are contiguous");
 constexpr int kBStageBytes = 2 * kTileBytes;             // B hi + lo of one K chunk
 constexpr int kKSlot = (kNQ * 16 + int(sizeof(ItemDesc)) + 127) / 128 * 128;  // constants + desc
 constexpr int kKOffQinv = kNQ * 8, kKOffQid = kNQ * 12, kKOffDesc = kNQ * 16;
@@ -1020,9 +1029,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
   if (tid == 0) {
     s_fail = 0;
     for (uint32_t b = 0; b < 2; ++b) {
-      mbar_init(item_full(b), kLoadThreads);
-      mbar_init(item_empty(b), kEpiWarps);
-      mbar_init(b_full(b), kLoadThreads);
+      mbar_init(item_full(b), kKLoadThreads);
+      mbar_init(item_empty(b), kKEpiWarps);
+      mbar_init(b_full(b), kKLoadThreads);
       mbar_init(b_empty(b), 1);
       mbar_init(a_full(b), kDecWarps);
       mbar_init(a_free(b), 1);
@@ -1033,11 +1042,11 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
     }
     for (uint32_t b = 0; b < kKR; ++b) {
       mbar_init(acc_full(b), 1);
-      mbar_init(acc_empty(b), kEpiWarps);
+      mbar_init(acc_empty(b), kKEpiWarps);
     }
     for (uint32_t b = 0; b < kScaleStages; ++b) {
       mbar_init(scale_full(b), 1);
-      mbar_init(scale_empty(b), kEpiWarps);
+      mbar_init(scale_empty(b), kKEpiWarps);
     }
     asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
   }
@@ -1071,9 +1080,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
     atomicExch(&s_fail, 1);
   };
 
-  if (warp >= kLoadWarp0) {
+  if (warp >= kKLoadWarp0) {
     // ---------------- loader: the item's constants, then its B chunks (group, chunk)
-    const int lt = tid - kLoadWarp0 * 32;
+    const int lt = tid - kKLoadWarp0 * 32;
     uint32_t bseq = 0;
     bool ok = true;
     for (uint32_t seq = 0; ok; ++seq) {
@@ -1097,31 +1106,29 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
           d->p = -1;
         }
       }
-      asm volatile("bar.sync 1, %0;" ::"n"(kLoadThreads) : "memory");
+      asm volatile("bar.sync 1, %0;" ::"n"(kKLoadThreads) : "memory");
       const int p = d->p, q0 = d->q0, nqt = d->nqt, nrows = d->nrows;
-      int qs[kNQ / kLoadThreads];
-      if (p >= 0) {
+      int* qid = reinterpret_cast<int*>(sb + kKOffQid);
+      if (p >= 0 && lt < kNQ) {
+        // thread lt: the constants of the item's query lt
         float* qpair = reinterpret_cast<float*>(sb);
         float* qinv = reinterpret_cast<float*>(sb + kKOffQinv);
-        int* qid = reinterpret_cast<int*>(sb + kKOffQid);
-#pragma unroll
-        for (int u = 0; u < kNQ / kLoadThreads; ++u) {
-          const int j = lt + u * kLoadThreads;
-          qs[u] = j < nqt ? __ldg(a.lq + q0 + j) : -1;
-        }
-#pragma unroll
-        for (int u = 0; u < kNQ / kLoadThreads; ++u) {
-          const int j = lt + u * kLoadThreads;
-          const bool v = qs[u] >= 0;
-          const float inv = v ? __ldg(a.qinv + qs[u]) : 1.0f;
-          const float cs = v ? __ldg(a.lcs + q0 + j) : 0.0f;
-          const float th = v ? (a.theta ? __ldg(a.theta + qs[u]) : -CUDART_INF_F) : CUDART_INF_F;
-          qpair[(j >> 1) * 4 + (j & 1)] = cs / inv;  // exact: inv is a power of two
-          qpair[(j >> 1) * 4 + 2 + (j & 1)] = -th / inv;
-          qinv[j] = inv;
-          qid[j] = qs[u];
-        }
+        const int j = lt;
+        const int qj = j < nqt ? __ldg(a.lq + q0 + j) : -1;
+        const bool v = qj >= 0;
+        const float inv = v ? __ldg(a.qinv + qj) : 1.0f;
+        const float cs = v ? __ldg(a.lcs + q0 + j) : 0.0f;
+        const float th = v ? (a.theta ? __ldg(a.theta + qj) : -CUDART_INF_F) : CUDART_INF_F;
+        qpair[(j >> 1) * 4 + (j & 1)] = cs / inv;  // exact: inv is a power of two
+        qpair[(j >> 1) * 4 + 2 + (j & 1)] = -th / inv;
+        qinv[j] = inv;
+        qid[j] = qj;
       }
+      asm volatile("bar.sync 1, %0;" ::"n"(kKLoadThreads) : "memory");
+      // B work of thread lt < 2 kNQ: query lt % kNQ, the 16-byte pieces
+      // [8 (lt / kNQ), + 8) of each K chunk (lanes take adjacent queries)
+      const int bj = lt & (kNQ - 1), bh = lt / kNQ;
+      const int bq = (p >= 0 && lt < 2 * kNQ) ? qid[bj] : -1;
       mbar_arrive(item_full(s));
       if (p < 0) break;
       // B chunks, one per (group, chunk), through the two-stage ring
@@ -1138,36 +1145,30 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
           fence_proxy_async();  // the MMAs' reads of this stage (async proxy) before its new generic stores
           uint8_t* dst = bst0 + bs * kBStageBytes;
           const int k8n = klen_of(kc) / 8;
-          // loads in batches of four 16-byte pieces, then shared stores (lane =
-          // query row: a warp's stores fill whole 128-byte rows); see the
-          // single-chunk kernel on why not cp.async
-          // both of a thread's queries in one batch: 16 loads in flight
-          constexpr int U = kNQ / kLoadThreads;
-          for (int k0 = 0; k0 < k8n; k0 += 4) {
-            uint4 hv[U][4], lv[U][4];
+          // one batch of 16 loads per thread (8 pieces of hi and of lo), then
+          // shared stores (lane = query row: a warp's stores fill whole
+          // 128-byte core-matrix rows)
+          if (lt < 2 * kNQ) {
+            const bool v = bq >= 0;
+            const int64_t base = int64_t(v ? bq : 0) * a.Dp16 + kc * kKC;
+            uint4 hv[8], lv[8];
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-              const bool v = qs[u] >= 0;
-              const int64_t base = int64_t(v ? qs[u] : 0) * a.Dp16 + kc * kKC;
-#pragma unroll
-              for (int e = 0; e < 4; ++e) {
-                hv[u][e] = make_uint4(0, 0, 0, 0);
-                lv[u][e] = make_uint4(0, 0, 0, 0);
-                if (v && k0 + e < k8n) {
-                  hv[u][e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + (k0 + e) * 8));
-                  lv[u][e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
-                }
+            for (int e = 0; e < 8; ++e) {
+              const int k8 = 8 * bh + e;
+              hv[e] = make_uint4(0, 0, 0, 0);
+              lv[e] = make_uint4(0, 0, 0, 0);
+              if (v && k8 < k8n) {
+                hv[e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + k8 * 8));
+                lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + k8 * 8));
               }
             }
 #pragma unroll
-            for (int u = 0; u < U; ++u) {
-              const int j = lt + u * kLoadThreads;
-#pragma unroll
-              for (int e = 0; e < 4; ++e)
-                if (k0 + e < k8n) {
-                  *reinterpret_cast<uint4*>(dst + tile_off(j, k0 + e)) = hv[u][e];
-                  *reinterpret_cast<uint4*>(dst + kTileBytes + tile_off(j, k0 + e)) = lv[u][e];
-                }
+            for (int e = 0; e < 8; ++e) {
+              const int k8 = 8 * bh + e;
+              if (k8 < k8n) {
+                *reinterpret_cast<uint4*>(dst + tile_off(bj, k8)) = hv[e];
+                *reinterpret_cast<uint4*>(dst + kTileBytes + tile_off(bj, k8)) = lv[e];
+              }
             }
           }
           fence_proxy_async();  // B is read by the tensor cores (async proxy)
@@ -1175,7 +1176,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
         }
       }
     }
-  } else if (warp == kTmaWarp) {
+  } else if (warp == kKTmaWarp) {
     // ---------------- TMA: (tile, chunk) code slabs in the group order, and each tile's scales
     if (lane == 0) {
       uint32_t sseq = 0, cseq = 0;
@@ -1229,7 +1230,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
         mbar_wait(scale_full(ss), ((cseq - 1 - ss) / kScaleStages) & 1);
     }
     __syncwarp();
-  } else if (warp == kMmaWarp) {
+  } else if (warp == kKMmaWarp) {
     // ---------------- MMA issue: per group, per chunk, per tile
     if (lane == 0) {
       uint32_t bseq = 0, aseq = 0, accu[kKR] = {0, 0, 0}, last_acc = 0;
@@ -1343,7 +1344,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
       }
     }
   } else {
-    // ---------------- epilogue: thread = row of quadrant warp % 4, columns eh * 32 ..
+    // ---------------- epilogue: thread = row of quadrant warp % 4, columns
+    // eh * 64 .. eh * 64 + 63 in two passes of 32
     const int quad = warp & 3;
     const int eh = (warp - kDecWarps) >> 2;
     const int row = quad * 32 + lane;
@@ -1363,7 +1365,6 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
       const float* qpair = reinterpret_cast<const float*>(slot(s));
       const float* qinv_s = reinterpret_cast<const float*>(slot(s) + kKOffQinv);
       const int* qid_s = reinterpret_cast<const int*>(slot(s) + kKOffQid);
-      const bool active = eh * 32 < nqt;
       for (int t = 0; t < ntiles && ok; ++t, ++cseq) {
         const int r = t % kKR;
         const int nvalid = min(kMR, nrows - t * kMR);
@@ -1392,13 +1393,22 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
         }
         ++accu[r];
         fence_after_sync();
-        float vall[32];
-        if (active) tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(r) + uint32_t(eh * 32), vall);
-        fence_before_sync();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(acc_empty(r));
-        if (active && row < nvalid)
-          epilogue_row<DENSE>(a, vall, L, Gs, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s);
+#pragma unroll 1
+        for (int c2 = 0; c2 < 2; ++c2) {
+          const int ec = 2 * eh + c2;  // 32-column group
+          const bool active = ec * 32 < nqt;
+          float vall[32];
+          if (active) tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(r) + uint32_t(ec * 32), vall);
+          if (c2 == 1) {
+            // the accumulator is in registers: release it to the next group's MMAs
+            fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(acc_empty(r));
+          }
+          if (active && row < nvalid)
+            epilogue_row<DENSE>(a, vall, L, Gs, row, t, nrows, nqt, ec, pos, qpair, qinv_s, qid_s);
+          __syncwarp();
+        }
       }
       __syncwarp();
       if (ok && lane == 0) mbar_arrive(item_empty(s));

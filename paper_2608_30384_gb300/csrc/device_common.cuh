@@ -46,8 +46,46 @@ __device__ __forceinline__ bool sign_neg(const uint32_t* bits, int i) {
 
 // Orthonormal FWHT H_B = Hhat_B / sqrt(B) of one block (Sec. 3.1.1), in
 // place, by one warp: log2(B) butterfly stages, then the 1/sqrt(B) scale.
+// In float (the query rotation), blocks of 32, 64 or 128 run in registers:
+// lane l holds x[32 j + l] (j < B / 32); the stages of span h < 32 pair
+// lanes l and l ^ h (warp shuffles), the spans 32 and 64 pair the lane's own
+// values j and j ^ h / 32.  The stages are Kronecker factors of Hhat_B and
+// commute, so their order is free.  Smaller blocks, and float64 (the
+// encoder, where a shuffle moves two 32-bit halves and measured slower), go
+// through shared memory stage by stage.
 template <typename T>
 __device__ __forceinline__ void warp_fwht(T* x, int B, int logB, T scale, int lane) {
+  if (sizeof(T) == 4 && B >= 32) {
+    const int J = B >> 5;
+    T v[4];
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (j < J) v[j] = x[32 * j + lane];
+#pragma unroll
+    for (int h = 1; h < 32; h <<= 1) {
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (j < J) {
+          const T o = __shfl_xor_sync(kFull, v[j], h);
+          v[j] = (lane & h) ? o - v[j] : v[j] + o;
+        }
+    }
+#pragma unroll
+    for (int hj = 1; hj < 4; hj <<= 1)
+#pragma unroll
+      for (int j = 0; j < 4; ++j)
+        if (j < J && hj < J && !(j & hj)) {
+          const T a = v[j], b = v[j | hj];
+          v[j] = a + b;
+          v[j | hj] = a - b;
+        }
+    __syncwarp();  // every lane has read its block values before any is overwritten
+#pragma unroll
+    for (int j = 0; j < 4; ++j)
+      if (j < J) x[32 * j + lane] = v[j] * scale;
+    __syncwarp();
+    return;
+  }
   for (int s = 0; s < logB; ++s) {
     const int h = 1 << s;
     for (int t = lane; t < (B >> 1); t += 32) {
