@@ -48,6 +48,8 @@ CLOCK_FIELDS = ["index", "clocks.sm", "clocks.max.sm", "power.draw", "clocks_eve
                 "clocks_event_reasons.sw_thermal_slowdown", "clocks_event_reasons.sw_power_cap"]
 SCAN_SOURCES = {
     "scan_kernel": ["paper_2608_30384_gb300/csrc/search.cu", "paper_2608_30384_gb300/csrc/device_common.cuh"],
+    "scan_bt_kernel": ["paper_2608_30384_gb300/csrc/search.cu", "paper_2608_30384_gb300/csrc/device_common.cuh",
+                       "paper_2608_30384_gb300/csrc/tcgen05.cuh"],
     "batched_pipe_kernel": ["paper_2608_30384_gb300/csrc/batched.cu",
                             "paper_2608_30384_gb300/csrc/device_common.cuh",
                             "paper_2608_30384_gb300/csrc/tcgen05.cuh"],
@@ -516,9 +518,9 @@ def run_gpu(args):
         g_avg = g_ms / max(1, g_n) / 1e3
         g_bytes = cand_g * bytes_per_cand
         g_ach = g_bytes / g_avg / 1e9
-        g_trec = traffic_record(w.name + ("-lite" if args.lite else ""), "scan_kernel") \
+        g_trec = traffic_record(w.name + ("-lite" if args.lite else "") + "-gemv", g_name) \
             if not args.score_bits else None
-        gemv = {"workload": f"first {ng} queries of {w.name}, single-query scan (one CTA per query)",
+        gemv = {"workload": f"first {ng} queries of {w.name}, single-query scan (no cross-query reuse)",
                 "kernel": g_name, "bound": "hbm", "achieved": g_ach, "peak": hbm_peak, "unit": "GB/s",
                 "frac": g_ach / hbm_peak, "peak_kind": peak_kind,
                 "algorithmic_bytes": g_bytes, "bytes_per_candidate": bytes_per_cand, "candidates": cand_g,

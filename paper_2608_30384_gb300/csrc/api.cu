@@ -534,6 +534,7 @@ rslm_status rslm_sync(const rslm_index* ix, void* stream) {
       return fail(RSLM_ERR_TIMEOUT, "a bounded wait for the tensor-core pipeline expired");
     const char* what = h == kErrBadProbe ? "probe list holds a partition id outside [0, nlist)"
                        : h == kErrBadCandidate ? "candidate id outside [-1, n_rows)"
+                       : h == kErrSmemLayout   ? "a scan kernel's shared-memory layout did not fit its launch"
                                                : "device-side check failed";
     return fail(RSLM_ERR_DEVICE, what);
   }

@@ -35,6 +35,7 @@ enum DeviceError : int {
   kErrBadCandidate = 2,  // candidate id out of range in rescoring
   kErrBadAssignment = 3,
   kErrTimeout = 4,       // a bounded wait on the tensor-core pipeline gave up
+  kErrSmemLayout = 5,    // a kernel's shared-memory layout did not fit its launch
 };
 
 // Block-wise cascaded FWHT rotation (Sec. 3.1.1-3.1.3).

@@ -14,6 +14,7 @@
 #include <cuda_runtime.h>
 #include <math_constants.h>
 
+#include <algorithm>
 #include <climits>
 
 #include "device_common.cuh"
@@ -318,7 +319,10 @@ struct ScanArgs {
   float* out_scores;
   int* err;
   int lut_region;  // bytes of the table / merge region
-  int bt_bytes;    // byte-table form: bytes of the per-lane byte table at the start of shared memory (else 0)
+  int parts;       // scan_bt_kernel: work units per query, each over a contiguous range of its probes
+  int stages;      // scan_bt_kernel: shared-memory stages of tiles (kBtStages when it runs)
+  int stages_pre;  // scan_bt_kernel: stages placed below the byte table
+  int64_t nq;      // scan_bt_kernel: queries (unlisted)
 };
 
 template <int CH>
@@ -392,33 +396,11 @@ __device__ __forceinline__ uint32_t nibble_tops(uint32_t w) {
   return (t | (t >> 12)) & 0xFFu;
 }
 
-// Byte-table form (4-bit codes with one coordinate per code, BT): instead of
-// the per-query table, a query-independent table maps a code byte (two
-// codes) to its two codebook levels as an fp16 pair, one copy per lane
-// (entry (byte, lane) at byte 256 * byte + 4 * lane: the 32 lanes of a read
-// always hit 32 distinct banks).  The levels are exact in fp16; each byte
-// then costs one table read, two conversions and one paired fp32 FMA with
-// the query pair (q[2j], q[2j + 1]) -- half the shared-memory traffic of a
-// 4-byte table entry per code.
-constexpr int kByteTableBytes = 256 * 256;
-
-template <int CH, bool B3, bool BT = false>
+template <int CH, bool B3>
 __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanArgs a) {
-  extern __shared__ __align__(16) uint8_t ssm_all[];
+  extern __shared__ __align__(16) uint8_t ssm[];
   __shared__ int scratch[32];
   const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, W = blockDim.x >> 5;
-  if constexpr (BT) {
-    // the byte table, once per CTA: low half = level of the low nibble
-    // (the even code position), high half = level of the high nibble
-    uint32_t* tb = reinterpret_cast<uint32_t*>(ssm_all);
-    for (int e = tid; e < 256 * 32; e += blockDim.x) {
-      const int byte = e >> 5, ln = e & 31;
-      const uint32_t lo = __half_as_ushort(__float2half_rn(a.cb[byte & 15]));
-      const uint32_t hi = __half_as_ushort(__float2half_rn(a.cb[byte >> 4]));
-      tb[byte * 64 + ln] = lo | (hi << 16);
-    }
-  }
-  uint8_t* ssm = ssm_all + a.bt_bytes;
   const int nrun = a.qlist ? *a.qcount : 1;
   for (int run0 = a.qlist ? int(blockIdx.x) : 0; run0 < nrun; run0 += a.qlist ? int(gridDim.x) : 1) {
   const int64_t q = a.qlist ? int64_t(a.qlist[run0]) : int64_t(blockIdx.x);
@@ -442,10 +424,6 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   // code's shared-memory address is then (block << 8) | (64 k + 4 code):
   // one byte permute per code builds it (see the scan loop).
   const float* qr = a.qrot + q * a.Dp;
-  if constexpr (BT) {
-    // the query itself, zero beyond Dp, one float per code position
-    for (int e = tid; e < a.lut_groups; e += blockDim.x) lut[e] = e < a.Dp ? qr[e] : 0.0f;
-  }
   if constexpr (B3) {
     // Rslm3: T[position][code] at lut[8 position + code]
     for (int e = tid; e < a.lut_groups * 8; e += blockDim.x) {
@@ -453,7 +431,7 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
       lut[e] = pos < a.ngroups ? qr[pos] * a.cb[e & 7] : 0.0f;
     }
   }
-  for (int e = tid; !B3 && !BT && e < a.lut_groups * 16; e += blockDim.x) {
+  for (int e = tid; !B3 && e < a.lut_groups * 16; e += blockDim.x) {
     const int grp = e >> 4, code = e & 15;
     float v = 0.0f;
     if (grp < a.lite_h)
@@ -526,45 +504,7 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
         }
       }
     }
-    if constexpr (BT) {
-      // fp32 pairs (even positions, odd positions) per row
-      uint64_t acc2[4] = {0ull, 0ull, 0ull, 0ull};
-      const uint32_t lane4 = uint32_t(lane) * 4u;
-#pragma unroll 1
-      for (int c = 0; c < nch; ++c) {
-        uint32_t w[4][4];
-#pragma unroll
-        for (int r = 0; r < 4; ++r) load_chunk<16>(tp + (size_t(c) * kTile + r * 32 + lane) * 16, w[r]);
-        // the 32 query values of this chunk's positions, as 16 (even, odd) pairs
-        const ulonglong2* qc = reinterpret_cast<const ulonglong2*>(lut + 32 * c);
-        uint64_t qp[16];
-#pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          const ulonglong2 v = qc[i];
-          qp[2 * i] = v.x;
-          qp[2 * i + 1] = v.y;
-        }
-#pragma unroll
-        for (int v = 0; v < 4; ++v)
-#pragma unroll
-          for (int k = 0; k < 4; ++k)
-#pragma unroll
-            for (int r = 0; r < 4; ++r) {
-              // entry (byte k of word v, lane): byte 0 = 4 lane, byte 1 = the code byte
-              const uint32_t off = __byte_perm(w[r][v], lane4, 0x5504u + 0x10u * k);
-              const uint32_t h2 = *reinterpret_cast<const uint32_t*>(ssm_all + off);
-              const float2 f = __half22float2(*reinterpret_cast<const __half2*>(&h2));
-              acc2[r] = fma2(f2pack(f.x, f.y), qp[4 * v + k], acc2[r]);
-            }
-      }
-#pragma unroll
-      for (int r = 0; r < 4; ++r) {
-        float e, o;
-        f2unpack(acc2[r], e, o);
-        acc[r] = e + o;
-      }
-    }
-    for (int c = 0; !B3 && !BT && c < nch; ++c) {
+    for (int c = 0; !B3 && c < nch; ++c) {
       uint32_t w[4][CH / 4];
 #pragma unroll
       for (int r = 0; r < 4; ++r)
@@ -659,6 +599,490 @@ __global__ void __launch_bounds__(256) scan_kernel(const __grid_constant__ ScanA
   }
 }
 
+// ------------------------------------------------ single-query scan, 4-bit
+// The single-query scan for 4-bit codes of one coordinate each (g = 1, no
+// Rslm4Lite head, 16-byte chunks, padded D <= 128).  The dot products
+// <R q, uhat_j> of 16 rows at a time run on the warp-level tensor-core
+// instruction mma.sync.m16n8k16 (fp16 operands, fp32 accumulation), used
+// here as the multiply-add engine of a memory-bound loop (a 16 x 16 x 2
+// product per instruction; tcgen05 would need the decoded codes staged in
+// shared or tensor memory, which doubles the shared-memory traffic that
+// bounds this loop):
+//   A (16 rows x 16 code positions) = decoded codes.  A query-independent
+//     table maps a code byte (two codes) to its two codebook levels as an
+//     fp16 pair (the levels are binary16-exact), one copy per lane: entry
+//     (byte, lane) at shared address kBtTableAddr + 256 byte + 4 lane, so
+//     one byte permute of a code word forms the whole address and the 32
+//     lanes of a read hit 32 distinct banks; the pair is one A register.
+//   B (16 x 8) = the query scaled by 2^s (max |q| 2^s in [1024, 2048)) and
+//     split into q_hi = fp16(q) (column 0) and q_lo = fp16(q - q_hi)
+//     (column 1); the other columns are zero.
+//   D column 0 + column 1 = 2^s <q, uhat> to about 22 bits of the query.
+// The dot product is order-free in its positions, so each lane takes the
+// codes that ldmatrix hands it: one ldmatrix.x4 reads four 8-row x 16-byte
+// blocks of a staged tile (rows 16 P .. + 7 and + 8 .. + 15 of two chunk
+// columns; each block is one conflict-free 128-byte row of banks) and gives
+// lane (g, t) = (lane / 4, lane % 4) word t of rows g and g + 8 of each
+// chunk column.  In the MMAs of chunk c the lane supplies bytes (0, 1), then
+// (2, 3), of its words -- code positions 32 c + 8 t + 4 m .. + 3 for MMA m
+// -- as the fragment columns (2 t, 2 t + 1) and (2 t + 8, 2 t + 9).  The B
+// fragment of lane (g, t) holds the same positions of column g, so a lane's
+// query fragments depend only on t and stay in registers.  Per code byte
+// that is one permute and one 4-byte shared read, and one MMA per 256
+// codes.
+//
+// Streaming: one persistent CTA of 16 warps per SM (four per SM
+// sub-partition, so 128 registers per thread).  Its producer warp turns
+// each work unit (a query, or a contiguous part of its probe list) into a
+// list of 128-row tiles, keeping each probe's row offset, row count and cs
+// in the unit's shared-memory descriptor (double-buffered); then 15 of its
+// lanes copy the tiles -- the codes (a contiguous slab of the
+// tile-interleaved layout) and the scale words -- into 15 shared-memory
+// stages with 1-D bulk copies (one issuing thread sustains only about one
+// copy per 600 cycles).  Tile T of the CTA's sequence goes to stage T mod
+// 15, issued by producer lane T mod 15 and scored by consumer warp T mod
+// 15: every stage has one issuing lane and one consumer warp, which use its
+// phases in order (an mbarrier parity wait is only sound for the current
+// phase), and no warp waits behind another's copies.  A consumer warp reads
+// its tile's codes into registers (ldmatrix), releases the stage, and
+// scores the 128 rows in 8 passes of 16; after each pass the row dots sit
+// in lanes t = 0, and a shuffle hands pass P's dots to lanes t = P mod 4,
+// so that after each 4 passes every lane holds two rows and the epilogue
+// (scales, s = G (cs + L dot), per-warp top-k list) runs on all 32 lanes.
+// At the end of a unit each warp writes its own list (no barrier between
+// the consumer warps); merge_parts_kernel merges the 15 lists of every unit
+// of a query (a query has `parts` > 1 units when the batch is too small to
+// fill the SMs).
+constexpr int kBtTableBytes = 256 * 256;
+constexpr uint32_t kBtTableAddr = 0x10000u;
+constexpr uint32_t kBtLowReserve = 4096;  // static + reserved shared memory below the dynamic allocation, at most
+constexpr int kBtWarps = 15;                     // consumer warps
+constexpr int kBtThreads = (kBtWarps + 1) * 32;  // + the producer warp: 4 warps per SM sub-partition
+constexpr int kBtStages = kBtWarps;              // stage w: consumer warp w, issuing lane w
+constexpr int kBtMaxChunks = 4;                  // padded D <= 128
+constexpr int kBtHalf = kTile / 2;
+
+__device__ __forceinline__ void mma_16816(float (&d)[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3,
+                                          uint32_t b0, uint32_t b1) {
+  asm volatile(
+      "mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, "
+      "{%0,%1,%2,%3};"
+      : "+f"(d[0]), "+f"(d[1]), "+f"(d[2]), "+f"(d[3])
+      : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1));
+}
+
+// Byte-table entry of byte KB (0..3) of code word w for this lane.  The
+// table sits at shared address kBtTableAddr (64 KB aligned) and tbl holds
+// kBtTableAddr | 4 lane, so one byte permute forms the entry's whole
+// address kBtTableAddr + 256 byte + 4 lane (bytes: 4 lane, the code byte,
+// then the table's upper address bytes).
+template <int KB>
+__device__ __forceinline__ uint32_t bt_entry(uint32_t w, uint32_t tbl) {
+  uint32_t v;
+  asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(__byte_perm(w, tbl, 0x7604u | (uint32_t(KB) << 4))));
+  return v;
+}
+
+// The 8 MMAs of four chunk columns: word t of rows g and g + 8 of column
+// c in w0[c] / w1[c], query fragments bq[2 c + m][0..1]; even and odd MMAs
+// accumulate separately.
+__device__ __forceinline__ void bt_group_mma(uint32_t tbl, const uint32_t (&w0)[4],
+                                             const uint32_t (&w1)[4], const uint32_t (&bq)[8][2], float (&d)[4],
+                                             float (&e)[4]) {
+#pragma unroll
+  for (int wi = 0; wi < 4; ++wi) {
+    // MMA 2 wi: bytes 0, 1 of the column's words; MMA 2 wi + 1: bytes 2, 3
+    mma_16816(d, bt_entry<0>(w0[wi], tbl), bt_entry<0>(w1[wi], tbl), bt_entry<1>(w0[wi], tbl),
+              bt_entry<1>(w1[wi], tbl), bq[2 * wi][0], bq[2 * wi][1]);
+    mma_16816(e, bt_entry<2>(w0[wi], tbl), bt_entry<2>(w1[wi], tbl), bt_entry<3>(w0[wi], tbl),
+              bt_entry<3>(w1[wi], tbl), bq[2 * wi + 1][0], bq[2 * wi + 1][1]);
+  }
+}
+
+// A work unit as the producer publishes it (double-buffered).  Per probe
+// j of the unit the same buffer holds, after this header: the partition's
+// first row slot off[j] (int64), its rows n[j], cs[j] and the prefix tile
+// count tpref[j] (tpref[np] = total).
+struct BtUnit {
+  int64_t q;     // the query
+  int64_t orow;  // output row: the query, or its part
+  int np;        // probes of the unit
+  int total;     // tiles of the unit
+  int valid;     // 0: no more units
+};
+constexpr int kBtUnitHead = 32;
+static_assert(sizeof(BtUnit) <= kBtUnitHead, "unit header");
+__host__ __device__ constexpr int bt_unit_bytes(int nprobe) { return (kBtUnitHead + 20 * nprobe + 4 + 15) & ~15; }
+
+__global__ void __launch_bounds__(kBtThreads, 1) scan_bt_kernel(const __grid_constant__ ScanArgs a) {
+  extern __shared__ __align__(128) uint8_t bsm[];
+  __shared__ __align__(8) uint64_t bars[2 * kBtStages + 4];
+  __shared__ int s_fail;
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
+  const int nch = a.stride / 16;
+  const uint32_t stage_bytes = uint32_t(nch) * 2048u + 512u;
+  // dynamic shared memory: stages 0 .. stages_pre - 1, the byte table at
+  // shared address kBtTableAddr, the other stages, the unit descriptors and
+  // the warps' lists
+  const uint32_t dyn0 = uint32_t(__cvta_generic_to_shared(bsm));
+  uint8_t* table = bsm + (kBtTableAddr - dyn0);
+  uint8_t* stage_hi = table + kBtTableBytes;
+  const int npre = a.stages_pre;
+  auto stage_at = [&](uint32_t s) {
+    return int(s) < npre ? bsm + size_t(s) * stage_bytes : stage_hi + size_t(int(s) - npre) * stage_bytes;
+  };
+  const int ubytes = bt_unit_bytes(a.nprobe);
+  uint8_t* ubuf0 = stage_hi + size_t(kBtStages - npre) * stage_bytes;
+  if (dyn0 + uint32_t(npre) * stage_bytes > kBtTableAddr) {
+    // the stages below the table would overlap it (more static shared
+    // memory than the host assumed): nothing is scanned
+    if (tid == 0) set_device_error(a.err, kErrSmemLayout);
+    return;
+  }
+  float* wsc = reinterpret_cast<float*>(ubuf0 + 2 * ubytes);  // the warps' top-k lists
+  int* wps = reinterpret_cast<int*>(wsc + kBtWarps * a.k);
+  const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
+  auto stage_full = [&](uint32_t s) { return bar0 + 8u * s; };
+  auto stage_empty = [&](uint32_t s) { return bar0 + 8u * (kBtStages + s); };
+  auto unit_full = [&](int b) { return bar0 + 8u * (2 * kBtStages + b); };
+  auto unit_empty = [&](int b) { return bar0 + 8u * (2 * kBtStages + 2 + b); };
+  // unit buffer b: header, off[nprobe], n[nprobe], cs[nprobe], tpref[nprobe + 1]
+  auto unit_at = [&](int b) { return ubuf0 + b * ubytes; };
+  auto u_off = [&](int b) { return reinterpret_cast<int64_t*>(unit_at(b) + kBtUnitHead); };
+  auto u_n = [&](int b) { return reinterpret_cast<int*>(u_off(b) + a.nprobe); };
+  auto u_cs = [&](int b) { return reinterpret_cast<float*>(u_n(b) + a.nprobe); };
+  auto u_tpref = [&](int b) { return reinterpret_cast<int*>(u_cs(b) + a.nprobe); };
+  auto failed = [&]() { return *reinterpret_cast<volatile int*>(&s_fail) != 0; };
+  auto fail = [&]() {
+    set_device_error(a.err, kErrTimeout);
+    atomicExch(&s_fail, 1);
+  };
+  {
+    // the byte table: low half = level of the low nibble (the even code
+    // position), high half = level of the high nibble
+    uint32_t* tb = reinterpret_cast<uint32_t*>(table);
+    for (int e = tid; e < 256 * 32; e += blockDim.x) {
+      const int byte = e >> 5, ln = e & 31;
+      const uint32_t lo = __half_as_ushort(__float2half_rn(a.cb[byte & 15]));
+      const uint32_t hi = __half_as_ushort(__float2half_rn(a.cb[byte >> 4]));
+      tb[byte * 64 + ln] = lo | (hi << 16);
+    }
+  }
+  if (tid == 0) {
+    s_fail = 0;
+    for (int s = 0; s < kBtStages; ++s) {
+      mbar_init(stage_full(s), 1);
+      mbar_init(stage_empty(s), 1);
+    }
+    for (int b = 0; b < 2; ++b) {
+      mbar_init(unit_full(b), 1);
+      mbar_init(unit_empty(b), kBtWarps);
+    }
+    asm volatile("fence.mbarrier_init.release.cluster;" ::: "memory");
+  }
+  __syncthreads();
+  const int parts = a.parts;
+  const int64_t nunits = a.nq * parts;
+
+  if (warp == kBtWarps) {
+    // ---------------- producer: unit descriptors, then the unit's tiles by bulk copy
+    uint32_t T = 0;     // tiles of the units so far
+    uint32_t tend = 0;  // this lane: 1 + the last tile it issued
+    for (int ui = 0;; ++ui) {
+      const int ub = ui & 1;
+      if (ui >= 2 && !mbar_wait_warp(unit_empty(ub), ((ui >> 1) - 1) & 1)) {
+        fail();
+        break;
+      }
+      BtUnit* hd = reinterpret_cast<BtUnit*>(unit_at(ub));
+      int64_t* uoff = u_off(ub);
+      int* un = u_n(ub);
+      float* ucs = u_cs(ub);
+      int* tpref = u_tpref(ub);
+      const int64_t u = int64_t(blockIdx.x) + int64_t(ui) * gridDim.x;
+      const bool more = u < nunits && !failed();
+      int run = 0;
+      if (more) {
+        const int64_t q = u / parts;
+        const int part = int(u % parts);
+        const int j0 = int(int64_t(part) * a.nprobe / parts), j1 = int(int64_t(part + 1) * a.nprobe / parts);
+        const int np = j1 - j0;
+        // probes [j0, j1) -> tiles (a warp-wide running prefix sum)
+        for (int base = 0; base < np; base += 32) {
+          const int jj = base + lane;
+          int nt = 0;
+          if (jj < np) {
+            const int p = a.probes[q * a.probe_stride + j0 + jj];
+            int64_t off = 0;
+            int n = 0;
+            if (p < 0 || p >= a.nlist) {
+              set_device_error(a.err, kErrBadProbe);
+            } else {
+              off = a.part_off[p];
+              n = a.part_n[p];
+              nt = (n + kTile - 1) / kTile;
+            }
+            uoff[jj] = off;
+            un[jj] = n;
+            ucs[jj] = a.cs ? a.cs[q * a.probe_stride + j0 + jj] : 0.0f;  // no cs: full-vector codes
+          }
+          int x = nt;
+#pragma unroll
+          for (int o = 1; o < 32; o <<= 1) {
+            const int y = __shfl_up_sync(kFull, x, o);
+            if (lane >= o) x += y;
+          }
+          if (jj < np) tpref[jj] = run + x - nt;
+          run += __shfl_sync(kFull, x, 31);
+        }
+        if (lane == 0) {
+          tpref[np] = run;
+          hd->q = q;
+          hd->orow = u;
+          hd->np = np;
+          hd->total = run;
+          hd->valid = 1;
+        }
+      } else if (lane == 0) {
+        hd->valid = 0;
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(unit_full(ub));
+      if (!more) break;
+      int ok = 1;
+      if (lane < kBtWarps) {
+        // lane L issues the unit's tiles T with T mod kBtStages = L, into stage L
+        int jc = 0;
+        const uint32_t s = uint32_t(lane);
+        const uint32_t dst = uint32_t(__cvta_generic_to_shared(stage_at(s)));
+        for (int i = int((s + kBtStages - T % kBtStages) % kBtStages); i < run; i += kBtStages) {
+          while (tpref[jc + 1] <= i) ++jc;
+          const int t = i - tpref[jc];
+          const int64_t slot0 = uoff[jc] + int64_t(t) * kTile;  // the tile's first row slot
+          const bool both = un[jc] - t * kTile > kBtHalf;      // rows in its second half
+          const uint32_t Ti = T + uint32_t(i);
+          const uint32_t n = Ti / kBtStages;
+          if (n > 0 && !mbar_wait(stage_empty(s), (n - 1) & 1)) {
+            fail();
+            ok = 0;
+            break;
+          }
+          // the codes (when the partition ends in the first half, up to the
+          // end of the last chunk column's first half), then the scales
+          const uint32_t cbytes = both ? uint32_t(nch) * 2048u : uint32_t(nch - 1) * 2048u + 1024u;
+          const uint32_t sbytes = both ? 512u : 256u;
+          mbar_arrive_expect(stage_full(s), cbytes + sbytes);
+          bulk_copy_1d(dst, a.codes + slot0 * a.stride, cbytes, stage_full(s));
+          bulk_copy_1d(dst + uint32_t(nch) * 2048u, a.scales + slot0, sbytes, stage_full(s));
+          tend = Ti + 1;
+        }
+      }
+      T += uint32_t(run);
+      if (__any_sync(kFull, ok == 0)) break;
+    }
+    // no copy may still be landing when the CTA exits: each lane waits for
+    // the last phase of its stage (the phases before it completed before
+    // that copy was issued)
+    if (lane < kBtWarps && tend > uint32_t(lane))
+      mbar_wait(stage_full(uint32_t(lane)), ((tend - 1 - uint32_t(lane)) / kBtStages) & 1);
+    __syncwarp();
+  } else {
+    // ---------------- consumers: warp w scores the tiles T with T mod kBtStages = w, from stage w
+    const int cw = warp;
+    const uint32_t lane4 = uint32_t(lane) * 4u;
+    const uint32_t tbl = kBtTableAddr | lane4;
+    const int tq = lane & 3, gq = lane >> 2;
+    const uint8_t* st = stage_at(uint32_t(cw));
+    const uint32_t st_addr = uint32_t(__cvta_generic_to_shared(st));
+    float* msc = wsc + cw * a.k;
+    int* mps = wps + cw * a.k;
+    uint32_t T0 = 0;  // sequence number of the unit's first tile
+    for (int ui = 0;; ++ui) {
+      const int ub = ui & 1;
+      const bool got = mbar_wait_warp(unit_full(ub), (ui >> 1) & 1);
+      const BtUnit* hd = reinterpret_cast<const BtUnit*>(unit_at(ub));
+      if (!got) fail();
+      if (!got || failed() || hd->valid == 0) break;
+      const int64_t* uoff = u_off(ub);
+      const int* un = u_n(ub);
+      const float* ucs = u_cs(ub);
+      const int* tpref = u_tpref(ub);
+      const int64_t q = hd->q, orow = hd->orow;
+      const int total = hd->total;
+      const float* qr = a.qrot + q * a.Dp;
+      // 2^s with max |q| 2^s in [1024, 2048)
+      float m = 0.0f;
+      for (int d = lane; d < a.Dp; d += 32) m = fmaxf(m, fabsf(qr[d]));
+#pragma unroll
+      for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
+      int ex = 0;
+      if (m > 0.0f) frexpf(m, &ex);
+      const float qsc = ldexpf(1.0f, 11 - ex), qinv = ldexpf(1.0f, ex - 11);
+      // this lane's query fragments: column gq (0: hi, 1: lo, else 0); for
+      // MMA m of chunk column c (index 2 c + m) the positions
+      // 32 c + 8 tq + 4 m + {0, 1} (register 0) and + {2, 3} (register 1)
+      uint32_t bq[8][2];
+#pragma unroll
+      for (int i = 0; i < 8; ++i)
+#pragma unroll
+        for (int r = 0; r < 2; ++r) {
+          const int c = i >> 1;
+          uint32_t wv = 0;
+          if (gq < 2 && c < nch) {
+            const int k0 = 32 * c + 8 * tq + 4 * (i & 1) + 2 * r;
+            __half h2[2];
+#pragma unroll
+            for (int x = 0; x < 2; ++x) {
+              const float v = (k0 + x < a.Dp ? __ldg(qr + k0 + x) : 0.0f) * qsc;
+              const __half hi = __float2half_rn(v);
+              h2[x] = gq == 0 ? hi : __float2half_rn(v - __half2float(hi));
+            }
+            wv = uint32_t(__half_as_ushort(h2[0])) | (uint32_t(__half_as_ushort(h2[1])) << 16);
+          }
+          bq[i][r] = wv;
+        }
+      int cnt = 0;
+      float thr = -CUDART_INF_F;
+      int thr_pos = INT_MAX;
+      // candidates (s, pos) of the lane's rows -> the warp's top-k list
+      auto offer = [&](float sc, int pos, bool valid) {
+        const bool cand = valid && (cnt < a.k || sc > thr || (sc == thr && pos < thr_pos));
+        unsigned mk = __ballot_sync(kFull, cand);
+        while (mk) {
+          const int src = __ffs(mk) - 1;
+          mk &= mk - 1;
+          const float s2 = __shfl_sync(kFull, sc, src);
+          const int p2 = __shfl_sync(kFull, pos, src);
+          if (cnt < a.k || s2 > thr || (s2 == thr && p2 < thr_pos)) {
+            warp_insert(msc, mps, cnt, a.k, s2, p2, lane);
+            if (cnt == a.k) {
+              thr = msc[a.k - 1];
+              thr_pos = mps[a.k - 1];
+            }
+          }
+        }
+      };
+      int jc = 0;
+      for (int i = int((uint32_t(cw) + kBtStages - T0 % kBtStages) % kBtStages); i < total; i += kBtStages) {
+        const uint32_t T = T0 + uint32_t(i);
+        while (tpref[jc + 1] <= i) ++jc;
+        const int t = i - tpref[jc];
+        const int nvalid = min(kTile, un[jc] - t * kTile);
+        const bool two = nvalid > kBtHalf;  // rows in the second half
+        const int pos0 = int(uoff[jc]) + t * kTile;
+        const float csj = ucs[jc];
+        if (!mbar_wait_warp(stage_full(uint32_t(cw)), (T / kBtStages) & 1)) {
+          fail();
+          break;
+        }
+        // this lane's rows: 16 tq + gq and + 8 of each half
+        const int ra = 16 * tq + gq, rb = ra + 8;
+        const uint32_t* scl = reinterpret_cast<const uint32_t*>(st + nch * 2048);
+        uint32_t sw[2][2];
+        sw[0][0] = scl[ra];
+        sw[0][1] = scl[rb];
+        sw[1][0] = two ? scl[kBtHalf + ra] : 0u;
+        sw[1][1] = two ? scl[kBtHalf + rb] : 0u;
+        // the tile's code words by ldmatrix: for pass P (rows 16 P .. + 15)
+        // and chunk columns (2 x, 2 x + 1), word tq of rows gq and gq + 8
+        uint32_t w[8][2][4];
+        auto load_pass = [&](int P) {
+#pragma unroll
+          for (int x = 0; x < 2; ++x) {
+            int c = 2 * x + (lane >> 4);
+            c = c < nch ? c : 0;  // a column past the row's codes: any staged bytes (the query is 0 there)
+            const int r = 16 * P + 8 * ((lane >> 3) & 1) + (lane & 7);
+            asm volatile("ldmatrix.sync.aligned.m8n8.x4.shared.b16 {%0, %1, %2, %3}, [%4];"
+                         : "=r"(w[P][0][2 * x]), "=r"(w[P][1][2 * x]), "=r"(w[P][0][2 * x + 1]),
+                           "=r"(w[P][1][2 * x + 1])
+                         : "r"(st_addr + uint32_t(c * kTile + r) * 16u)
+                         : "memory");
+          }
+        };
+#pragma unroll
+        for (int P = 0; P < 4; ++P) load_pass(P);
+        if (two) {
+#pragma unroll
+          for (int P = 4; P < 8; ++P) load_pass(P);
+        }
+        // the stage has been read: release it to the producer (the generic
+        // reads before the next bulk copy into it)
+        fence_proxy_async();
+        __syncwarp();
+        if (lane == 0) mbar_arrive(stage_empty(uint32_t(cw)));
+#pragma unroll
+        for (int hh = 0; hh < 2; ++hh) {
+          if (hh == 1 && !two) break;
+          float da = 0.0f, db = 0.0f;
+#pragma unroll
+          for (int pp = 0; pp < 4; ++pp) {
+            const int P = 4 * hh + pp;
+            float d[4] = {0.0f, 0.0f, 0.0f, 0.0f}, e[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+            bt_group_mma(tbl, w[P][0], w[P][1], bq, d, e);
+            // lanes tq = 0: (hi, lo) of rows 16 P + gq (d0, d1) and + 8 (d2, d3)
+            const float x0 = __shfl_sync(kFull, (d[0] + e[0]) + (d[1] + e[1]), lane & ~3);
+            const float x1 = __shfl_sync(kFull, (d[2] + e[2]) + (d[3] + e[3]), lane & ~3);
+            if (tq == pp) {
+              da = x0;
+              db = x1;
+            }
+          }
+          // epilogue of the half's 64 rows: two per lane
+          const int hv = nvalid - kBtHalf * hh;
+          const bool va = ra < hv, vb = rb < hv;
+          const uint32_t swa = sw[hh][0], swb = sw[hh][1];
+          const float sa = va ? ue4m12_to_f32(swa >> 16) * fmaf(ue7m9_to_f32(swa & 0xffffu), da * qinv, csj)
+                              : -CUDART_INF_F;
+          const float sb = vb ? ue4m12_to_f32(swb >> 16) * fmaf(ue7m9_to_f32(swb & 0xffffu), db * qinv, csj)
+                              : -CUDART_INF_F;
+          offer(sa, pos0 + kBtHalf * hh + ra, va);
+          offer(sb, pos0 + kBtHalf * hh + rb, vb);
+        }
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(unit_empty(ub));  // the unit's descriptor is no longer read
+      T0 += uint32_t(total);
+      // this warp's list of the unit -> its row of the partial lists (k
+      // entries, -1 / -inf padded); merge_parts_kernel merges the rows
+      const int64_t prow = orow * kBtWarps + cw;
+      for (int e = lane; e < a.k; e += 32) {
+        const bool ok = e < cnt;
+        a.out_ids[prow * a.k + e] = ok ? a.ids[mps[e]] : -1;
+        a.out_scores[prow * a.k + e] = ok ? msc[e] : -CUDART_INF_F;
+      }
+      __syncwarp();  // the list is read before the next unit's inserts
+    }
+  }
+  __syncthreads();
+}
+
+// Top out_k of a query's `parts` partial lists (k entries each, sorted by
+// (score desc, id asc), -1 / -inf padded): one block per query.
+__global__ void merge_parts_kernel(const int64_t* __restrict__ pid, const float* __restrict__ psc, int64_t nq,
+                                   int parts, int k, int out_k, int64_t* __restrict__ out_ids,
+                                   float* __restrict__ out_scores) {
+  extern __shared__ __align__(16) uint8_t msm[];
+  const int n = parts * k;
+  int np2 = 1;
+  while (np2 < n) np2 <<= 1;
+  float* key = reinterpret_cast<float*>(msm);
+  int64_t* idv = reinterpret_cast<int64_t*>(msm + ((size_t(np2) * 4 + 15) & ~size_t(15)));
+  for (int64_t q = blockIdx.x; q < nq; q += gridDim.x) {
+    for (int e = threadIdx.x; e < np2; e += blockDim.x) {
+      const int64_t id = e < n ? pid[q * n + e] : -1;
+      key[e] = id >= 0 ? psc[q * n + e] : -CUDART_INF_F;
+      idv[e] = id >= 0 ? id : LLONG_MAX;
+    }
+    block_bitonic_sort(key, idv, np2);
+    for (int e = threadIdx.x; e < out_k; e += blockDim.x) {
+      const bool ok = idv[e] != LLONG_MAX;
+      out_ids[q * out_k + e] = ok ? idv[e] : -1;
+      out_scores[q * out_k + e] = ok ? key[e] : -CUDART_INF_F;
+    }
+    __syncthreads();
+  }
+}
+
 // ---------------------------------------------------------------- rescore
 struct RescoreArgs {
   const float* qrot2;
@@ -741,19 +1165,88 @@ __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ Re
   }
 }
 
-template <int CH, bool B3, bool BT = false>
+template <int CH, bool B3>
 cudaError_t launch_scan_ch(const rslm_index* ix, const ScanArgs& a, int64_t nq, size_t smem,
                            cudaStream_t s) {
   // listed queries: a fixed grid strides over the list, whose length is on the device
   const int64_t grid = a.qlist ? (nq < 2 * 152 ? nq : 2 * 152) : nq;
-  cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH, B3, BT>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  cudaError_t e = cudaFuncSetAttribute(scan_kernel<CH, B3>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                        int(smem));
   if (e != cudaSuccess) return e;
   cudaEvent_t stop =
       a.only_if == nullptr && a.qlist == nullptr && a.nprobe > 1 ? prof_start(ix, s, "scan_kernel") : nullptr;
-  scan_kernel<CH, B3, BT><<<unsigned(grid), 256, smem, s>>>(a);
+  scan_kernel<CH, B3><<<unsigned(grid), 256, smem, s>>>(a);
   prof_stop(stop, s);
   return cudaGetLastError();
+}
+
+// Shared memory of scan_bt_kernel for a's k and nprobe: sets a.stages
+// (kBtStages, or 0 when they do not fit) and returns the bytes.
+size_t plan_scan_bt(ScanArgs& a, int dev) {
+  const int k = a.k;
+  const size_t stage_bytes = size_t(a.stride / 16) * 2048 + 512;
+  const size_t ubytes = size_t(bt_unit_bytes(a.nprobe));
+  // below the table: the stages that fit when static and reserved shared
+  // memory take at most kBtLowReserve bytes (the kernel checks); the
+  // dynamic allocation starts at most that far above 0, so reserving the
+  // full 64 KB below the table always suffices
+  const int pre = std::min(kBtStages, int((kBtTableAddr - kBtLowReserve) / stage_bytes));
+  const size_t bytes = size_t(kBtTableAddr) + size_t(kBtTableBytes) + size_t(kBtStages - pre) * stage_bytes +
+                       2 * ubytes + size_t(kBtWarps) * k * 8;
+  int optin = 0;
+  if (cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) != cudaSuccess) optin = 0;
+  const bool fits = bytes + kBtLowReserve <= size_t(optin);
+  a.stages = fits ? kBtStages : 0;
+  a.stages_pre = fits ? pre : 0;
+  return fits ? bytes : 0;
+}
+
+// scan_bt_kernel over nq queries, after plan_scan_bt.  Every (unit, consumer
+// warp) writes a k-entry list into a stream-ordered workspace; batches too
+// small to give every SM several units split each query's probe list into
+// `parts` units.  merge_parts_kernel merges the kBtWarps * parts lists of
+// each query into its top out_k.
+cudaError_t launch_scan_bt(const rslm_index* ix, ScanArgs a, int64_t nq, size_t smem, int sms, cudaStream_t s) {
+  const int k = a.k;
+  int parts = 1;
+  const int64_t want = int64_t(4) * sms;  // units: about four per SM
+  if (nq < want) parts = int(std::min<int64_t>(a.nprobe, (want + nq - 1) / nq));
+  parts = std::max(1, std::min(parts, 4096 / (kBtWarps * k)));  // the merge sorts its lists in shared memory
+  a.parts = parts;
+  a.nq = nq;
+  cudaError_t e = cudaFuncSetAttribute(scan_bt_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(smem));
+  if (e != cudaSuccess) return e;
+  const int nl = parts * kBtWarps;  // lists per query
+  const size_t n = size_t(nq) * nl * k;
+  void* ws = nullptr;
+  e = cudaMallocAsync(&ws, n * 12, s);
+  if (e != cudaSuccess) return e;
+  int64_t* pids = reinterpret_cast<int64_t*>(ws);
+  float* pscs = reinterpret_cast<float*>(pids + n);
+  const int out_k = a.out_k;
+  int64_t* final_ids = a.out_ids;
+  float* final_sc = a.out_scores;
+  a.out_ids = pids;
+  a.out_scores = pscs;
+  a.out_k = k;
+  const int64_t grid = std::min<int64_t>(nq * parts, sms);
+  cudaEvent_t stop = a.nprobe > 1 ? prof_start(ix, s, "scan_bt_kernel") : nullptr;
+  scan_bt_kernel<<<unsigned(grid), kBtThreads, smem, s>>>(a);
+  prof_stop(stop, s);
+  e = cudaGetLastError();
+  if (e == cudaSuccess) {
+    int mp2 = 1;
+    while (mp2 < nl * k) mp2 <<= 1;
+    const size_t msm = ((size_t(mp2) * 4 + 15) & ~size_t(15)) + size_t(mp2) * 8;
+    e = cudaFuncSetAttribute(merge_parts_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(msm));
+    if (e == cudaSuccess) {
+      merge_parts_kernel<<<unsigned(std::min<int64_t>(nq, int64_t(8) * sms)), 256, msm, s>>>(
+          pids, pscs, nq, nl, k, out_k, final_ids, final_sc);
+      e = cudaGetLastError();
+    }
+  }
+  cudaError_t f = cudaFreeAsync(ws, s);
+  return e == cudaSuccess ? f : e;
 }
 
 }  // namespace
@@ -833,18 +1326,23 @@ cudaError_t launch_scan_impl(const rslm_index* ix, const float* qrot, int64_t nq
   const int W = 8;
   int np2 = 1;
   while (np2 < W * k) np2 <<= 1;
-  // byte-table form for 4-bit codes of one coordinate in 16-byte chunks
-  const bool bt = !b3 && ix->cs1.g == 1 && ix->cs1.lite_h == 0 && ix->cs1.chunk == 16;
-  const size_t lut_bytes = size_t(a.lut_groups) * (bt ? 1 : b3 ? 8 : 16) * 4;
+  a.parts = 1;
+  // 4-bit codes of one coordinate in 16-byte chunks, padded D <= 128: the tensor-core form
+  if (!b3 && ix->cs1.g == 1 && ix->cs1.lite_h == 0 && ix->cs1.chunk == 16 &&
+      ix->cs1.stride <= 16 * kBtMaxChunks && only_if == nullptr && qlist == nullptr) {
+    int dev = 0, sms = 152;
+    if (cudaGetDevice(&dev) == cudaSuccess) cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    ScanArgs b = a;
+    const size_t bsmem = plan_scan_bt(b, dev);
+    if (b.stages > 0) return launch_scan_bt(ix, b, nq, bsmem, sms, s);
+  }
+  const size_t lut_bytes = size_t(a.lut_groups) * (b3 ? 8 : 16) * 4;
   const size_t merge_bytes = ((size_t(np2) * 4 + 15) & ~size_t(15)) + size_t(np2) * 8;
   size_t region = lut_bytes > merge_bytes ? lut_bytes : merge_bytes;
   region = (region + 15) & ~size_t(15);
   a.lut_region = int(region);
-  a.bt_bytes = bt ? kByteTableBytes : 0;
-  const size_t smem =
-      size_t(a.bt_bytes) + 256 + region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
+  const size_t smem = 256 + region + size_t(W) * k * 8 + size_t(W) * 4 + size_t(2 * nprobe + 1) * 4;
   if (b3) return launch_scan_ch<4, true>(ix, a, nq, smem, s);
-  if (bt) return launch_scan_ch<16, false, true>(ix, a, nq, smem, s);
   switch (ix->cs1.chunk) {
     case 16: return launch_scan_ch<16, false>(ix, a, nq, smem, s);
     case 8: return launch_scan_ch<8, false>(ix, a, nq, smem, s);
