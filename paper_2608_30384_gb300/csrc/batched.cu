@@ -520,25 +520,23 @@ __device__ __forceinline__ void epilogue_row(const BatchArgs& a, const float (&v
         }
       }
     } else {
-      // its maximum over the part's columns rules out most rows at once
+      // y = G (cs' + L v) - theta' per column (packed pairs, each rounded
+      // as fmaf); its maximum over the part's columns rules out most rows
+      // at once, and the signs of the same y values give the hits
       const uint64_t L2 = f2pack(L, L), G2 = f2pack(Gs, Gs);
+      float y[kPart];
       float m = -CUDART_INF_F;
 #pragma unroll
       for (int i = 0; i < kPart; i += 2) {
         const float4 c = q4[i / 2];
         const uint64_t y2 = fma2(G2, fma2(L2, f2pack(v[i], v[i + 1]), f2pack(c.x, c.y)), f2pack(c.z, c.w));
-        float y0, y1;
-        f2unpack(y2, y0, y1);
-        m = fmax3(m, y0, y1);
+        f2unpack(y2, y[i], y[i + 1]);
+        m = fmax3(m, y[i], y[i + 1]);
       }
       if (m >= 0.0f) {
         uint32_t hit = 0;
 #pragma unroll
-        for (int i = 0; i < kPart; i += 2) {
-          const float4 c = q4[i / 2];
-          hit |= (fmaf(Gs, fmaf(L, v[i], c.x), c.z) >= 0.0f ? 1u : 0u) << i;
-          hit |= (fmaf(Gs, fmaf(L, v[i + 1], c.y), c.w) >= 0.0f ? 2u : 0u) << i;
-        }
+        for (int i = 0; i < kPart; ++i) hit |= (y[i] >= 0.0f ? 1u : 0u) << i;
         while (hit) {
           const int i = __ffs(hit) - 1;
           hit &= hit - 1;
