@@ -223,6 +223,52 @@ def test_scan_parity_on_oracle_codes(case):
         assert (ids[i] >= 0).sum() == min(w.k, len(s1))
 
 
+# Single-query scan of 4-bit codes of one coordinate (padded D <= 128): one
+# unit per query (batches of >= 4 units per SM), units split over probe
+# ranges (small batches), partitions shorter than half a tile and an empty
+# one, chunk columns past the row's codes (D = 96, 33), large k near the
+# shared-memory limit, k = 256 (falls back to the table scan) and
+# nprobe = nlist.
+SINGLE = {
+    "one_unit": Wl("sq1", 20_000, 128, 64, 0.5, False, 0.5, "mean", 700, 4, 0, 4, 10, 10, seed=21),
+    "split_units": Wl("sq2", 20_000, 128, 64, 0.5, False, 0.5, "mean", 3, 4, 0, 16, 10, 10, seed=22),
+    "short_lists": Wl("sq3", 3_000, 128, 64, 0.5, False, None, "true", 40, 4, 0, 8, 10, 10, seed=23),
+    "D96": Wl("sq4", 8_000, 96, 16, 0.5, False, None, "true", 40, 4, 0, 4, 10, 10, seed=24),
+    "D33": Wl("sq5", 8_000, 33, 16, 0.5, False, None, "true", 40, 4, 0, 4, 10, 10, seed=25),
+    "k200": Wl("sq6", 20_000, 128, 32, 0.5, False, None, "mean", 30, 4, 0, 8, 200, 200, seed=26),
+    "k256": Wl("sq7", 20_000, 128, 32, 0.5, False, None, "mean", 30, 4, 0, 8, 256, 256, seed=27),
+    "all_probes": Wl("sq8", 6_000, 128, 16, 0.5, False, None, "true", 20, 4, 0, 16, 20, 20, seed=28),
+}
+
+
+@pytest.mark.parametrize("name", sorted(SINGLE))
+def test_single_query_scan_paths(name):
+    """rslm_scan on 4-bit codes of one coordinate, at the edges of its launch plan."""
+    case = Case(SINGLE[name])
+    if name == "short_lists":
+        A = case.A.copy()
+        A[A == 5] = 6  # partition 5 left empty
+        case.A = A
+        case.oracle = search.build_index(case.X, np.arange(case.w.N), A, case.C, 4, 0)
+    w = case.w
+    ix = case.gpu_index(encode=False)
+    case.import_oracle_codes(ix)
+    probes, cs = _scan_inputs(case)
+    qrot = ix.rotate(torch.from_numpy(case.Q).cuda())
+    ids, sc = ix.scan(qrot, torch.from_numpy(probes.astype(np.int32)).cuda(),
+                      torch.from_numpy(cs.astype(np.float32)).cuda(), w.k)
+    ix.sync()
+    ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
+    for i in range(len(case.Q)):
+        ref, s1 = _oracle_stage1(case, i, probes[i], cs[i])
+        kth, kid = kth_of(ref, w.k)
+        probs = check_topk(ids[i], sc[i], lambda j: ref[j], kth, case.score_tol_of(i), allowed_ids=ref,
+                           kth_id=kid)
+        assert not probs, (i, probs[:3])
+        assert (ids[i] >= 0).sum() == min(w.k, len(s1))
+        assert np.all(np.isneginf(sc[i][ids[i] < 0]))
+
+
 def _scan_parity(case, batched: bool):
     w = case.w
     ix = case.gpu_index(encode=False)
