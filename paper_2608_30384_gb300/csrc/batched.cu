@@ -22,6 +22,7 @@
 #include <math_constants.h>
 
 #include <algorithm>
+#include <cmath>
 #include <climits>
 
 #include "device_common.cuh"
@@ -181,7 +182,7 @@ __global__ void __launch_bounds__(1024) scatter_hist_kernel(const int32_t* __res
 // inv = 2^-s.  Dimensions Dp..Dp16 are zero.
 __global__ void split_queries_kernel(const float* __restrict__ qrot, int64_t nq, int Dp, int Dp16,
                                      __half* __restrict__ qhi, __half* __restrict__ qlo,
-                                     float* __restrict__ qinv) {
+                                     float* __restrict__ qinv, float* __restrict__ qrho, float U) {
   const int lane = threadIdx.x & 31, warp = threadIdx.x >> 5, W = blockDim.x >> 5;
   for (int64_t q = int64_t(blockIdx.x) * W + warp; q < nq; q += int64_t(gridDim.x) * W) {
     const float* src = qrot + q * Dp;
@@ -193,11 +194,21 @@ __global__ void split_queries_kernel(const float* __restrict__ qrot, int64_t nq,
     if (m > 0.0f) frexpf(m, &e);  // m in [2^(e-1), 2^e)
     const int s = 11 - e;
     const float sc = ldexpf(1.0f, s);
+    float l2 = 0.0f;  // ||v - hi||^2 (the exact remainder, before its own rounding)
     for (int d = lane; d < Dp16; d += 32) {
       const float v = d < Dp ? src[d] * sc : 0.0f;
       const __half h = __float2half_rn(v);
+      const float r = v - __half2float(h);
       qhi[q * Dp16 + d] = h;
-      qlo[q * Dp16 + d] = __float2half_rn(v - __half2float(h));
+      qlo[q * Dp16 + d] = __float2half_rn(r);
+      l2 = fmaf(r, r, l2);
+    }
+    if (qrho) {
+#pragma unroll
+      for (int o = 16; o; o >>= 1) l2 += __shfl_xor_sync(kFull, l2, o);
+      // |<v - hi, uhat>| <= ||v - hi|| ||uhat||, ||uhat|| <= U; rounded up
+      // against the float rounding of the norm
+      if (lane == 0) qrho[q] = U * sqrtf(l2) * (1.0f + 1e-5f);
     }
     if (lane == 0) qinv[q] = ldexpf(1.0f, -s);
   }
@@ -297,6 +308,8 @@ struct BatchArgs {
   const __half* qhi;
   const __half* qlo;
   const float* qinv;
+  const float* qrho;  // hi-only mode: per query U ||q_lo||, scaled units (a bound on |<q_lo, uhat>|)
+  float* buf_l;       // hi-only mode, pass 2: lower bound of each kept candidate's score
   const float* theta;  // nullptr: keep every candidate
   float* buf_s;
   int32_t* buf_p;
@@ -376,6 +389,18 @@ constexpr int kOffBl = kTileBytes, kOffQct = 2 * kTileBytes, kOffQinv = kOffQct 
               kOffQid = kOffQinv + kNQ * 4, kOffDesc = kOffQid + kNQ * 4,
               kSlotBytes = (kOffDesc + int(sizeof(ItemDesc)) + 127) / 128 * 128;
 constexpr int kScaleBytes = kMR * 4;  // a tile's (L | G << 16) words
+// Hi-only mode (HI: 4-bit codes of one coordinate): the queries' fp16 hi
+// parts alone are multiplied with the codes, and one more MMA (K = 16) adds
+// each query's margin hU >= |<q - q_hi, uhat>| (pass 2: + hU, an upper
+// bound of the exact dot product; pass 1: - hU, a lower bound).  The lo
+// region of an item slot then holds that MMA's operands and the margins:
+constexpr int kOffBc = kOffBl;         // B: the item's queries x 16 halves, hU in column 0
+constexpr int kOffAc = kOffBl + 4096;  // A: 128 rows x 16 halves, 1 in column 0 (written once)
+constexpr int kOffHu = kOffBl + 8192;  // hU per query column, float
+constexpr int kConstSBO = 256;         // 8-row groups of a K = 16 operand (two 128-byte core matrices)
+__device__ __forceinline__ uint32_t const_off(int row, int k8) {
+  return uint32_t((row >> 3) * kConstSBO + k8 * 128 + (row & 7) * 16);
+}
 // 4-bit codes decode a whole byte (two codes -> two halves) through a
 // 256-entry table held once per lane (entry (byte, lane) at word byte * 32 +
 // lane), so the 32 lookups of a warp always fall into 32 distinct banks.
@@ -493,10 +518,11 @@ __device__ __forceinline__ void decode_half(const uint32_t* wd, int dh, const ui
 // Epilogue of one row (thread) over the warp's 32 query columns of a tile:
 // DENSE stores every score at the row's place in the query's buffer;
 // otherwise G (cs' + L acc) - theta' >= 0 decides and the hits are appended.
-template <bool DENSE>
+template <bool DENSE, bool HI = false>
 __device__ __forceinline__ void epilogue_row(const BatchArgs& a, const float (&vall)[32], float L, float Gs,
                                              int row, int t, int nrows, int nqt, int eh, int32_t pos,
-                                             const float* qpair, const float* qinv_s, const int* qid_s) {
+                                             const float* qpair, const float* qinv_s, const int* qid_s,
+                                             const float* hu_s = nullptr) {
   constexpr int kPart = 16;
 #pragma unroll
   for (int part = 0; part < 32 / kPart; ++part) {
@@ -546,11 +572,14 @@ __device__ __forceinline__ void epilogue_row(const BatchArgs& a, const float (&v
           const int col = cbase + i;
           const int q = qid_s[col];
           if (q < 0) continue;
-          const float sc = Gs * fmaf(L, acc, qpair[(col >> 1) * 4 + (col & 1)]);  // score x 2^s
+          const float csc = qpair[(col >> 1) * 4 + (col & 1)];
+          const float sc = Gs * fmaf(L, acc, csc);  // score x 2^s (HI: its upper bound)
           const int at = atomicAdd(&a.cnt[q], 1);
           if (at < a.cap) {
             a.buf_s[int64_t(q) * a.cap + at] = sc * qinv_s[col];
             a.buf_p[int64_t(q) * a.cap + at] = pos;
+            // HI: the lower bound, with the dot product's margin taken off twice
+            if constexpr (HI) a.buf_l[int64_t(q) * a.cap + at] = Gs * fmaf(L, acc - 2.0f * hu_s[col], csc) * qinv_s[col];
           }
         }
       }
@@ -558,8 +587,9 @@ __device__ __forceinline__ void epilogue_row(const BatchArgs& a, const float (&v
   }
 }
 
-template <int G, bool DENSE, int FMT>
+template <int G, bool DENSE, int FMT, bool HI = false>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
+  static_assert(!HI || (G == 1 && FMT == kFmtNibble), "hi-only mode: 4-bit codes of one coordinate");
   extern __shared__ __align__(128) uint8_t psm[];
   uint8_t* slab0 = psm + 2 * kSlotBytes;
   // the scales of the tile in scale stage b: scl0 + b * kMR
@@ -592,6 +622,16 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       t32[2 * c] = a.cbbits[4 * c] | (a.cbbits[4 * c + 1] << 16);
       t32[2 * c + 1] = a.cbbits[4 * c + 2] | (a.cbbits[4 * c + 3] << 16);
     }
+  }
+  if constexpr (HI) {
+    // the margin MMA's A operand in both item slots: 1.0 (fp16 0x3C00) in
+    // column 0 of every row, zeros elsewhere; read by the tensor core
+    for (int e = tid; e < 2 * kMR * 2; e += blockDim.x) {
+      const int sl = e / (kMR * 2), r = (e >> 1) % kMR, k8 = e & 1;
+      *reinterpret_cast<uint4*>(psm + sl * kSlotBytes + kOffAc + const_off(r, k8)) =
+          make_uint4(k8 == 0 ? 0x3C00u : 0u, 0u, 0u, 0u);
+    }
+    fence_proxy_async();
   }
   const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
   // mbarrier layout: item_full[2], item_empty[2], a_full[2], a_free[2],
@@ -707,6 +747,15 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           qpair[(j >> 1) * 4 + 2 + (j & 1)] = -th / inv;
           qinv[j] = inv;
           qid[j] = qs[u];
+          if constexpr (HI) {
+            // the margin hU >= |<q - q_hi, uhat>| (rounded up to fp16): + in
+            // pass 2 (upper bounds), - in pass 1 (lower bounds, for theta)
+            const __half hh = __float2half_ru(v ? __ldg(a.qrho + qs[u]) : 0.0f);
+            reinterpret_cast<float*>(sb + kOffHu)[j] = __half2float(hh);
+            const uint32_t bits = uint32_t(__half_as_ushort(hh)) ^ (DENSE ? 0x8000u : 0u);
+            *reinterpret_cast<uint4*>(sb + kOffBc + const_off(j, 0)) = make_uint4(bits, 0u, 0u, 0u);
+            *reinterpret_cast<uint4*>(sb + kOffBc + const_off(j, 1)) = make_uint4(0u, 0u, 0u, 0u);
+          }
         }
         // B rows: loads in batches of four 16-byte pieces, then shared stores
         // (lane = query row, so a warp's stores fill whole 128-byte
@@ -726,14 +775,14 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
               lv[e] = make_uint4(0, 0, 0, 0);
               if (v && k0 + e < k8n) {
                 hv[e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + (k0 + e) * 8));
-                lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
+                if (!HI) lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + (k0 + e) * 8));
               }
             }
 #pragma unroll
             for (int e = 0; e < 4; ++e)
               if (k0 + e < k8n) {
                 *reinterpret_cast<uint4*>(sb + tile_off(j, k0 + e)) = hv[e];
-                *reinterpret_cast<uint4*>(sb + kOffBl + tile_off(j, k0 + e)) = lv[e];
+                if (!HI) *reinterpret_cast<uint4*>(sb + kOffBl + tile_off(j, k0 + e)) = lv[e];
               }
           }
         }
@@ -816,8 +865,11 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
             const uint32_t at = tmem + a_col(b) + uint32_t(ks * 8);
             umma_f16_ts(tmem + acc_col(c), at, smem_desc(bh_addr + ks * 256, 128, kSBO), idesc,
                         ks > 0 ? 1u : 0u);
-            umma_f16_ts(tmem + acc_col(c), at, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
+            if (!HI) umma_f16_ts(tmem + acc_col(c), at, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
           }
+          if (HI)  // + (or, pass 1, -) the margin hU of every query column
+            umma_f16(tmem + acc_col(c), smem_desc(bh_addr + kOffAc, 128, kConstSBO),
+                     smem_desc(bh_addr + kOffBc, 128, kConstSBO), idesc, 1u);
           umma_commit(a_free(b));
           umma_commit(acc_full(c));
         }
@@ -932,7 +984,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         __syncwarp();
         if (lane == 0) mbar_arrive(acc_empty(b));
         if (active && row < nvalid)
-          epilogue_row<DENSE>(a, vall, L, Gs, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s);
+          epilogue_row<DENSE, HI>(a, vall, L, Gs, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s,
+                                  reinterpret_cast<const float*>(slot(s) + kOffHu));
       }
       __syncwarp();
       if (ok && lane == 0) mbar_arrive(item_empty(s));
@@ -1542,6 +1595,172 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_warp_kernel(
   }
 }
 
+// Hi-only mode: pass 2 kept every candidate whose upper bound reached theta,
+// with its upper bound s_up (buf_s) and lower bound s_lo (buf_l).  One warp
+// per query: T = the k-th largest s_lo bounds the exact k-th best score from
+// below, so only candidates with s_up >= T can be in the top k; their exact
+// scores are s_up + G L (<r, uhat> - hU) 2^-s (r = 2^s q - q_hi, exact in
+// fp32; the MMA added hU instead of <r, uhat>), from the row's codes, and the
+// top k of those by (score desc, id asc) is the result.  With more than
+// kFinCap candidates T is taken over the first kFinCap of them (still a
+// lower bound).  Buffers that overflowed, came out short under a finite
+// theta, or leave more than kFinCap candidates above T go to the exact
+// single-query re-scan, as in finalize_warp_kernel.
+struct FinHiArgs {
+  const float* buf_s;
+  const float* buf_l;
+  const int32_t* buf_p;
+  const int* cnt;
+  int64_t nq;
+  int cap;
+  const int64_t* ids;
+  int k;
+  const float* theta;
+  const float* qrot;  // rotated queries, nq x Dp
+  int Dp;
+  const float* qrho;
+  const uint8_t* codes;  // 4-bit codes of one coordinate, 16-byte chunks, tile-interleaved
+  const uint32_t* scales;
+  int stride;
+  float cb[16];
+  int* ovf_list;
+  int* counts;
+  unsigned long long* ctr;
+  int64_t* out_ids;
+  float* out_scores;
+};
+
+__global__ void __launch_bounds__(kFinWarps * 32) finalize_hi_kernel(const __grid_constant__ FinHiArgs a) {
+  __shared__ uint32_t fk[kFinWarps][kFinCap];
+  __shared__ int64_t fi[kFinWarps][kFinCap];
+  __shared__ float rq[kFinWarps][kKC];  // r = 2^s q - q_hi of the warp's query
+  __shared__ float cbs[16];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  if (threadIdx.x < 16) cbs[threadIdx.x] = a.cb[threadIdx.x];
+  __syncthreads();
+  const int64_t q = int64_t(blockIdx.x) * kFinWarps + w;
+  if (q >= a.nq) return;
+  const int n = a.cnt[q];
+  const int k = a.k;
+  const bool short_list = n < k && a.theta[q] > -CUDART_INF_F;
+  if (n > a.cap || short_list) {
+    if (lane == 0) {
+      a.ovf_list[atomicAdd(&a.counts[0], 1)] = int(q);
+      atomicAdd(&a.ctr[short_list ? kCtrBatchedShort : kCtrBatchedOverflow], 1ull);
+    }
+    return;
+  }
+  // the query's scaling 2^s (max |q| 2^s in [1024, 2048)) and remainder r
+  const float* src = a.qrot + q * a.Dp;
+  float m = 0.0f;
+  for (int d = lane; d < a.Dp; d += 32) m = fmaxf(m, fabsf(src[d]));
+#pragma unroll
+  for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
+  int e2 = 0;
+  if (m > 0.0f) frexpf(m, &e2);
+  const float sc = ldexpf(1.0f, 11 - e2), inv = ldexpf(1.0f, e2 - 11);
+  const int npos = (a.stride / 16) * 32;  // code positions of a row (<= kKC)
+  for (int d = lane; d < npos; d += 32) {
+    const float v = d < a.Dp ? src[d] * sc : 0.0f;
+    rq[w][d] = v - __half2float(__float2half_rn(v));
+  }
+  __syncwarp();  // rq is read by every lane below
+  const float hu = __half2float(__float2half_ru(a.qrho[q]));
+  const float* su = a.buf_s + q * a.cap;
+  const float* sl = a.buf_l + q * a.cap;
+  const int32_t* pp = a.buf_p + q * a.cap;
+  // T: the k-th largest lower bound (of the first kFinCap; all candidates
+  // when n <= k)
+  uint32_t T = 0u;
+  if (n > k) {
+    const int nt = min(n, kFinCap);
+    int p2 = 1;
+    while (p2 < nt) p2 <<= 1;
+    for (int i = lane; i < p2; i += 32) fk[w][i] = i < nt ? float_order_key(sl[i]) : 0u;
+    __syncwarp();
+    for (int size = 2; size <= p2; size <<= 1)
+      for (int stride = size >> 1; stride > 0; stride >>= 1) {
+        for (int i = lane; i < (p2 >> 1); i += 32) {
+          const int lo = 2 * i - (i & (stride - 1)), hi = lo + stride;
+          const bool asc = (lo & size) == 0;  // sorted descending overall
+          const uint32_t klo = fk[w][lo], khi = fk[w][hi];
+          if (asc ? khi > klo : klo > khi) {
+            fk[w][lo] = khi;
+            fk[w][hi] = klo;
+          }
+        }
+        __syncwarp();
+      }
+    T = fk[w][k - 1];
+    __syncwarp();
+  }
+  // the candidates that can be in the top k, with their exact scores
+  int mcnt = 0;
+  for (int base = 0; base < n; base += 32) {
+    const int i = base + lane;
+    const bool in = i < n && float_order_key(su[i]) >= T;
+    const unsigned bm = __ballot_sync(kFull, in);
+    const int at = mcnt + __popc(bm & ((1u << lane) - 1u));
+    if (in && at < kFinCap) {
+      const int32_t pos = pp[i];
+      const int r = pos & (kMR - 1);
+      const uint8_t* row = a.codes + int64_t(pos - r) * a.stride + r * 16;
+      float dot = 0.0f;
+      for (int c = 0; c < a.stride / 16; ++c) {
+        const uint4 wv = __ldg(reinterpret_cast<const uint4*>(row + size_t(c) * kMR * 16));
+        const uint32_t wd[4] = {wv.x, wv.y, wv.z, wv.w};
+#pragma unroll
+        for (int j = 0; j < 4; ++j)
+#pragma unroll
+          for (int nb = 0; nb < 8; ++nb) dot = fmaf(cbs[(wd[j] >> (4 * nb)) & 15u], rq[w][32 * c + 8 * j + nb], dot);
+      }
+      const uint32_t swd = __ldg(a.scales + pos);
+      const float G = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
+      const float s = su[i] + G * L * (dot - hu) * inv;
+      fk[w][at] = float_order_key(s);
+      fi[w][at] = a.ids[pos];
+    }
+    mcnt += __popc(bm);
+  }
+  if (mcnt > kFinCap) {
+    if (lane == 0) {
+      a.ovf_list[atomicAdd(&a.counts[0], 1)] = int(q);
+      atomicAdd(&a.ctr[kCtrBatchedOverflow], 1ull);
+    }
+    return;
+  }
+  __syncwarp();
+  int p2 = 1;
+  while (p2 < mcnt || p2 < k) p2 <<= 1;
+  for (int i = mcnt + lane; i < p2; i += 32) {
+    fk[w][i] = 0u;
+    fi[w][i] = LLONG_MAX;
+  }
+  __syncwarp();
+  for (int size = 2; size <= p2; size <<= 1)
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      for (int i = lane; i < (p2 >> 1); i += 32) {
+        const int lo = 2 * i - (i & (stride - 1)), hi = lo + stride;
+        const bool asc = (lo & size) == 0;
+        const uint32_t klo = fk[w][lo], khi = fk[w][hi];
+        const int64_t ilo = fi[w][lo], ihi = fi[w][hi];
+        const bool swap = asc ? better(khi, ihi, klo, ilo) : better(klo, ilo, khi, ihi);
+        if (swap) {
+          fk[w][lo] = khi;
+          fk[w][hi] = klo;
+          fi[w][lo] = ihi;
+          fi[w][hi] = ilo;
+        }
+      }
+      __syncwarp();
+    }
+  for (int i = lane; i < k; i += 32) {
+    const bool ok = i < mcnt && fi[w][i] != LLONG_MAX;
+    a.out_ids[q * k + i] = ok ? fi[w][i] : -1;
+    a.out_scores[q * k + i] = ok ? float_from_order_key(fk[w][i]) : -CUDART_INF_F;
+  }
+}
+
 int blocks_for(int64_t n, int per, int maxb) {
   int64_t b = (n + per - 1) / per;
   if (b < 1) b = 1;
@@ -1601,7 +1820,8 @@ cudaError_t build_lists(const rslm_index* ix, const int32_t* probes, const float
 
 cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi, const __half* qlo,
                         const float* qinv, int Dp16, const float* theta, float* bs, int32_t* bp, int* bc,
-                        int cap, int* work, bool profile, cudaStream_t s) {
+                        int cap, int* work, bool profile, cudaStream_t s, const float* qrho = nullptr,
+                        float* bl = nullptr) {
   const CodecSpec& c1 = ix->cs1;
   BatchArgs b;
   b.codes = ix->codes1;
@@ -1625,6 +1845,8 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   b.qhi = qhi;
   b.qlo = qlo;
   b.qinv = qinv;
+  b.qrho = qrho;
+  b.buf_l = bl;
   b.theta = theta;
   b.buf_s = bs;
   b.buf_p = bp;
@@ -1644,7 +1866,9 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   const size_t smem = one ? pipe_smem_bytes(g) : kpipe_smem_bytes(g);
   using K = void (*)(BatchArgs);
   K pk;
-  if (one)
+  if (one && qrho)  // hi-only mode (4-bit codes of one coordinate)
+    pk = theta ? batched_pipe_kernel<1, false, kFmtNibble, true> : batched_pipe_kernel<1, true, kFmtNibble, true>;
+  else if (one)
     pk = c1.bits == 3 ? (theta ? batched_pipe_kernel<1, false, kFmt3> : batched_pipe_kernel<1, true, kFmt3>)
          : b.lite_h   ? (theta ? batched_pipe_kernel<1, false, kFmtLite> : batched_pipe_kernel<1, true, kFmtLite>)
          : theta      ? (g == 1   ? batched_pipe_kernel<1, false, kFmtNibble>
@@ -1703,6 +1927,9 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
     oL[l][5] = take(size_t(np) * 4);
     oL[l][6] = take(size_t(np / kNQ + nlist + 1) * 4);  // at most sum of ceil(cnt / kNQ) items
   }
+  // hi-only mode: 4-bit codes of one coordinate in 16-byte chunks, padded D <= 128
+  const bool hi = c1.g == 1 && c1.bits == 4 && c1.lite_h == 0 && c1.chunk == 16 && Dp16 <= kKC;
+  const size_t o_qrho = take(hi ? size_t(nq) * 4 : 4), o_bl = take(hi ? size_t(nq) * cap * 4 : 4);
   const size_t o_qhi = take(size_t(nq) * Dp16 * 2), o_qlo = take(size_t(nq) * Dp16 * 2),
                o_qinv = take(size_t(nq) * 4), o_theta = take(size_t(nq) * 4),
                o_as = take(size_t(nq) * capA * 4), o_ap = take(size_t(nq) * capA * 4),
@@ -1732,6 +1959,12 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   int* ovf = reinterpret_cast<int*>(ws + o_ovf);
   int* work = reinterpret_cast<int*>(ws + o_work);
   int* fcounts = reinterpret_cast<int*>(ws + o_fcounts);
+  float* qrho = hi ? reinterpret_cast<float*>(ws + o_qrho) : nullptr;
+  float* bl = hi ? reinterpret_cast<float*>(ws + o_bl) : nullptr;
+  // ||uhat|| <= sqrt(Dp) max |codebook level| bounds the dot product with the remainder
+  float maxlev = 0.0f;
+  for (int i = 0; i < 16; ++i) maxlev = std::max(maxlev, std::fabs(c1.cbf[i]));
+  const float U = std::sqrt(float(c1.Dp)) * maxlev * (1.0f + 1e-5f);
 
   // lists: L[0] the first probe of every query, L[1] all probe pairs
   const float* lcs = (ix->flags & RSLM_FULL_VECTOR) ? nullptr : cs;  // full-vector codes: no <q, c> term
@@ -1739,7 +1972,7 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   if (e == cudaSuccess) e = build_lists(ix, probes, lcs, nq, nprobe, nprobe, L[1], s);
   if (e == cudaSuccess) {
     split_queries_kernel<<<blocks_for(nq, 8, 152 * 32), 256, 0, s>>>(qrot, nq, c1.Dp, Dp16, qhi, qlo,
-                                                                      qinv);
+                                                                      qinv, qrho, U);
     e = cudaGetLastError();
   }
   if (e == cudaSuccess) e = cudaMemsetAsync(ac, 0, size_t(nq) * 4, s);
@@ -1747,14 +1980,14 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   // Pass 1: every candidate of each query's first probed partition; k of
   // them reach theta, which bounds the query's k-th best score from below.
   if (e == cudaSuccess)
-    e = run_batched(ix, L[0], qhi, qlo, qinv, Dp16, nullptr, as, ap, ac, capA, work, false, s);
+    e = run_batched(ix, L[0], qhi, qlo, qinv, Dp16, nullptr, as, ap, ac, capA, work, false, s, qrho);
   if (e == cudaSuccess) {
     theta_warp_kernel<<<unsigned((nq + 7) / 8), 256, 0, s>>>(as, ac, nq, capA, k, theta);
     e = cudaGetLastError();
   }
   // Pass 2: all probed partitions, keeping candidates >= theta.
   if (e == cudaSuccess)
-    e = run_batched(ix, L[1], qhi, qlo, qinv, Dp16, theta, bs, bp, bc, cap, work, true, s);
+    e = run_batched(ix, L[1], qhi, qlo, qinv, Dp16, theta, bs, bp, bc, cap, work, true, s, qrho, bl);
   if (e == cudaSuccess) {
     int p2 = 1;
     while (p2 < k + 64) p2 <<= 1;
@@ -1764,7 +1997,32 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
       // ac (the first pass's counts) is free again: it lists the queries
       // handed to the block kernel; ovf lists the overflowed ones
       e = cudaMemsetAsync(fcounts, 0, 2 * sizeof(int), s);
-      if (e == cudaSuccess) {
+      if (e == cudaSuccess && hi) {
+        FinHiArgs fa;
+        fa.buf_s = bs;
+        fa.buf_l = bl;
+        fa.buf_p = bp;
+        fa.cnt = bc;
+        fa.nq = nq;
+        fa.cap = cap;
+        fa.ids = ix->ids;
+        fa.k = k;
+        fa.theta = theta;
+        fa.qrot = qrot;
+        fa.Dp = c1.Dp;
+        fa.qrho = qrho;
+        fa.codes = ix->codes1;
+        fa.scales = ix->scales1;
+        fa.stride = c1.stride;
+        for (int i = 0; i < 16; ++i) fa.cb[i] = c1.cbf[i];
+        fa.ovf_list = ovf;
+        fa.counts = fcounts;
+        fa.ctr = ix->d_counters;
+        fa.out_ids = out_ids;
+        fa.out_scores = out_scores;
+        finalize_hi_kernel<<<unsigned((nq + kFinWarps - 1) / kFinWarps), kFinWarps * 32, 0, s>>>(fa);
+        e = cudaGetLastError();
+      } else if (e == cudaSuccess) {
         finalize_warp_kernel<<<unsigned((nq + kFinWarps - 1) / kFinWarps), kFinWarps * 32, 0, s>>>(
             bs, bp, bc, nq, cap, ix->ids, k, theta, ovf, ac, fcounts, ix->d_counters, out_ids, out_scores);
         finalize_kernel<<<unsigned(std::min<int64_t>(nq, 2 * 152)), 256, smem, s>>>(
