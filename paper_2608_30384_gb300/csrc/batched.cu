@@ -398,6 +398,17 @@ constexpr int kOffBc = kOffBl;         // B: the item's queries x 16 halves, hU 
 constexpr int kOffAc = kOffBl + 4096;  // A: 128 rows x 16 halves, 1 in column 0 (written once)
 constexpr int kOffHu = kOffBl + 8192;  // hU per query column, float
 constexpr int kConstSBO = 256;         // 8-row groups of a K = 16 operand (two 128-byte core matrices)
+// The hi-only kernel's item slot is the hi B operand, those operands and
+// the per-query constants; its shared memory puts the code slabs, scales
+// and small tables below shared address kHiTableAddr, a 64 KB per-lane byte
+// table there (entry (byte, lane) at kHiTableAddr + 256 byte + 4 lane, so
+// one byte permute forms a lookup's whole address), and the two item slots
+// above the table.
+constexpr int kHOffQct = kOffHu + kNQ * 4, kHOffQinv = kHOffQct + kNQ * 8, kHOffQid = kHOffQinv + kNQ * 4,
+              kHOffDesc = kHOffQid + kNQ * 4,
+              kHSlotBytes = (kHOffDesc + int(sizeof(ItemDesc)) + 127) / 128 * 128;
+constexpr uint32_t kHiTableAddr = 0x10000u;
+constexpr uint32_t kHiLowReserve = 4096;  // static + reserved shared memory below the dynamic allocation, at most
 __device__ __forceinline__ uint32_t const_off(int row, int k8) {
   return uint32_t((row >> 3) * kConstSBO + k8 * 128 + (row & 7) * 16);
 }
@@ -424,6 +435,13 @@ __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
   return size_t(2) * kSlotBytes + size_t(kSlabs) * slab_bytes(g) + size_t(kScaleStages) * kScaleBytes + 32 * 4 +
          (g == 1 ? kByteTableBytes + kLiteTableBytes : 0);
 }
+// Hi-only kernel: the dynamic allocation starts at most kHiLowReserve bytes
+// above shared address 0, so reserving everything up to the table suffices.
+__host__ __device__ constexpr size_t hi_pipe_smem_bytes() { return size_t(kHiTableAddr) + 65536 + size_t(2) * kHSlotBytes; }
+__host__ __device__ constexpr size_t hi_pipe_low_bytes() {
+  return size_t(kSlabs) * slab_bytes(1) + size_t(kScaleStages) * kScaleBytes + 32 * 4;
+}
+static_assert(hi_pipe_low_bytes() + kHiLowReserve <= kHiTableAddr, "slabs and scales fit below the table");
 
 // The NW code words of row r of a slab whose rows are interleaved in
 // chunks of CH bytes (chunk c of row r at (c * kMR + r) * CH; CH is 16, 8
@@ -591,7 +609,14 @@ template <int G, bool DENSE, int FMT, bool HI = false>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
   static_assert(!HI || (G == 1 && FMT == kFmtNibble), "hi-only mode: 4-bit codes of one coordinate");
   extern __shared__ __align__(128) uint8_t psm[];
-  uint8_t* slab0 = psm + 2 * kSlotBytes;
+  // item slot layout (the hi-only kernel's slots are smaller and sit above
+  // its byte table)
+  constexpr int SlotB = HI ? kHSlotBytes : kSlotBytes;
+  constexpr int OffQct = HI ? kHOffQct : kOffQct, OffQinv = HI ? kHOffQinv : kOffQinv,
+                OffQid = HI ? kHOffQid : kOffQid, OffDesc = HI ? kHOffDesc : kOffDesc;
+  const uint32_t dyn0 = uint32_t(__cvta_generic_to_shared(psm));
+  uint8_t* slots = HI ? psm + (2 * kHiTableAddr - dyn0) : psm;
+  uint8_t* slab0 = HI ? psm : psm + 2 * kSlotBytes;
   // the scales of the tile in scale stage b: scl0 + b * kMR
   uint32_t* scl0 = reinterpret_cast<uint32_t*>(slab0 + kSlabs * slab_bytes(G));
   // decode table: G = 1: code -> 1 half; G = 2: code -> 2 halves; G = 4: code -> 4 halves
@@ -604,7 +629,20 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
 
   uint32_t* t256 = t32 + 32;  // G = 1 only
   uint32_t* t64 = t256 + 256 * 32;  // G = 1 only: Rslm4Lite head
-  if (FMT == kFmt3) {
+  if constexpr (HI) {
+    if (dyn0 + uint32_t(hi_pipe_low_bytes()) > kHiTableAddr) {
+      // more static shared memory than assumed: the slabs would overlap the table
+      if (tid == 0) set_device_error(a.err, kErrSmemLayout);
+      return;
+    }
+    // the per-lane byte table: low half = level of the low nibble (the even
+    // code position), high half = level of the high nibble
+    uint32_t* tb = reinterpret_cast<uint32_t*>(psm + (kHiTableAddr - dyn0));
+    for (int e = tid; e < 256 * 32; e += blockDim.x) {
+      const uint32_t byte = uint32_t(e) >> 5;
+      tb[byte * 64 + (e & 31)] = a.cbbits[byte & 15u] | (a.cbbits[byte >> 4] << 16);
+    }
+  } else if (FMT == kFmt3) {
     for (int e = tid; e < 64 * 32; e += blockDim.x) {
       const uint32_t pair = uint32_t(e) >> 5;  // even code in the low 3 bits -> low half
       t256[e] = a.cbbits[pair & 7u] | (a.cbbits[pair >> 3] << 16);
@@ -628,7 +666,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
     // column 0 of every row, zeros elsewhere; read by the tensor core
     for (int e = tid; e < 2 * kMR * 2; e += blockDim.x) {
       const int sl = e / (kMR * 2), r = (e >> 1) % kMR, k8 = e & 1;
-      *reinterpret_cast<uint4*>(psm + sl * kSlotBytes + kOffAc + const_off(r, k8)) =
+      *reinterpret_cast<uint4*>(slots + sl * SlotB + kOffAc + const_off(r, k8)) =
           make_uint4(k8 == 0 ? 0x3C00u : 0u, 0u, 0u, 0u);
     }
     fence_proxy_async();
@@ -683,7 +721,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   __syncthreads();
   fence_after_sync();
   const uint32_t tmem = tmem_base_sh;
-  const uint32_t psm_addr = uint32_t(__cvta_generic_to_shared(psm));
+  const uint32_t slots_addr = uint32_t(__cvta_generic_to_shared(slots));
   const uint32_t slab_addr0 = uint32_t(__cvta_generic_to_shared(slab0));
   const uint32_t scl_addr0 = uint32_t(__cvta_generic_to_shared(scl0));
   const int n_items = a.items[a.nlist];
@@ -691,8 +729,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   const int nbytes = row_bytes(klen, G, FMT);
   const int c1 = min((nbytes + CH - 1) / CH, a.stride / CH);  // code chunks of a row used
   const uint32_t slab_len = uint32_t(c1 * kMR * CH);
-  auto slot = [&](uint32_t s) { return psm + s * kSlotBytes; };
-  auto desc = [&](uint32_t s) { return reinterpret_cast<const volatile ItemDesc*>(slot(s) + kOffDesc); };
+  auto slot = [&](uint32_t s) { return slots + s * SlotB; };
+  auto desc = [&](uint32_t s) { return reinterpret_cast<const volatile ItemDesc*>(slot(s) + OffDesc); };
   auto failed = [&]() { return *reinterpret_cast<volatile int*>(&s_fail) != 0; };
   auto fail = [&]() {
     set_device_error(a.err, kErrTimeout);
@@ -709,7 +747,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       if (!ok) fail();
       fence_proxy_async();  // the MMAs' reads of this slot (async proxy) before its new generic stores
       uint8_t* sb = slot(s);
-      ItemDesc* d = reinterpret_cast<ItemDesc*>(sb + kOffDesc);
+      ItemDesc* d = reinterpret_cast<ItemDesc*>(sb + OffDesc);
       if (lt == 0) {
         const int item = (ok && !failed()) ? atomicAdd(a.work, 1) : n_items;
         if (item < n_items) {
@@ -726,9 +764,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       asm volatile("bar.sync 1, %0;" ::"n"(kLoadThreads) : "memory");
       const int p = d->p, q0 = d->q0, nqt = d->nqt;
       if (p >= 0) {
-        float* qpair = reinterpret_cast<float*>(sb + kOffQct);
-        float* qinv = reinterpret_cast<float*>(sb + kOffQinv);
-        int* qid = reinterpret_cast<int*>(sb + kOffQid);
+        float* qpair = reinterpret_cast<float*>(sb + OffQct);
+        float* qinv = reinterpret_cast<float*>(sb + OffQinv);
+        int* qid = reinterpret_cast<int*>(sb + OffQid);
         int qs[kNQ / kLoadThreads];
 #pragma unroll
         for (int u = 0; u < kNQ / kLoadThreads; ++u) {
@@ -851,7 +889,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         const int ntiles = (desc(s)->nrows + kMR - 1) / kMR;
         const int nqt = desc(s)->nqt;
         const uint32_t idesc = f16_idesc(kMR, max(16, (nqt + 15) & ~15));
-        const uint32_t bh_addr = psm_addr + s * kSlotBytes, bl_addr = bh_addr + kOffBl;
+        const uint32_t bh_addr = slots_addr + s * SlotB, bl_addr = bh_addr + kOffBl;
         for (int t = 0; t < ntiles; ++t, ++gt) {
           const uint32_t b = gt & 1, u = gt >> 1;             // A buffer
           const uint32_t c = gt % kAccBufs, uc = gt / kAccBufs;  // accumulator
@@ -918,7 +956,23 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
 #pragma unroll
         for (int dh = 0; dh < 2; ++dh) {
           uint32_t av[32];
-          decode_half<G, FMT>(wd, dh, t256, t32, lane, av, dh == 0 ? a.lite_h / 8 : 0, t64);
+          if constexpr (HI) {
+            // byte bb of word w -> one permute forms the entry's address
+            // kHiTableAddr + 256 byte + 4 lane; one shared load
+            const uint32_t tbl = kHiTableAddr | (uint32_t(lane) << 2);
+#pragma unroll
+            for (int w = 0; w < 8; ++w)
+#pragma unroll
+              for (int bb = 0; bb < 4; ++bb) {
+                uint32_t v;
+                asm volatile("ld.shared.b32 %0, [%1];"
+                             : "=r"(v)
+                             : "r"(__byte_perm(wd[8 * dh + w], tbl, 0x7604u | (uint32_t(bb) << 4))));
+                av[4 * w + bb] = v;
+              }
+          } else {
+            decode_half<G, FMT>(wd, dh, t256, t32, lane, av, dh == 0 ? a.lite_h / 8 : 0, t64);
+          }
           tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
         }
         fence_before_sync();
@@ -944,9 +998,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       const int nrows = desc(s)->nrows, nqt = desc(s)->nqt;
       const int64_t slot0 = desc(s)->slot0;
       const int ntiles = (nrows + kMR - 1) / kMR;
-      const float* qpair = reinterpret_cast<const float*>(slot(s) + kOffQct);
-      const float* qinv_s = reinterpret_cast<const float*>(slot(s) + kOffQinv);
-      const int* qid_s = reinterpret_cast<const int*>(slot(s) + kOffQid);
+      const float* qpair = reinterpret_cast<const float*>(slot(s) + OffQct);
+      const float* qinv_s = reinterpret_cast<const float*>(slot(s) + OffQinv);
+      const int* qid_s = reinterpret_cast<const int*>(slot(s) + OffQid);
       // this warp's 32 columns [eh * 32, eh * 32 + 32) hold queries when eh * 32 < nqt
       const bool active = eh * 32 < nqt;
       for (int t = 0; t < ntiles; ++t, ++gt) {
@@ -1863,7 +1917,7 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
   // padded D <= 128: the whole K range per item (B once per item);
   // otherwise K chunks of 128 with B streamed per group of tiles
   const bool one = b.nkc == 1;
-  const size_t smem = one ? pipe_smem_bytes(g) : kpipe_smem_bytes(g);
+  const size_t smem = one ? (qrho ? hi_pipe_smem_bytes() : pipe_smem_bytes(g)) : kpipe_smem_bytes(g);
   using K = void (*)(BatchArgs);
   K pk;
   if (one && qrho)  // hi-only mode (4-bit codes of one coordinate)
