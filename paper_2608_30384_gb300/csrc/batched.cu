@@ -17,6 +17,7 @@
 //      a per-query buffer,
 //   4. takes the exact top-k of every buffer, ordered by (score desc, id asc);
 //      a query whose buffer overflowed is re-scanned by the single-query path.
+#include <cuda_bf16.h>
 #include <cuda_fp16.h>
 #include <cuda_runtime.h>
 #include <math_constants.h>
@@ -390,13 +391,24 @@ constexpr int kOffBl = kTileBytes, kOffQct = 2 * kTileBytes, kOffQinv = kOffQct 
               kSlotBytes = (kOffDesc + int(sizeof(ItemDesc)) + 127) / 128 * 128;
 constexpr int kScaleBytes = kMR * 4;  // a tile's (L | G << 16) words
 // Hi-only mode (HI: 4-bit codes of one coordinate): the queries' fp16 hi
-// parts alone are multiplied with the codes, and one more MMA (K = 16) adds
-// each query's margin hU >= |<q - q_hi, uhat>| (pass 2: + hU, an upper
-// bound of the exact dot product; pass 1: - hU, a lower bound).  The lo
-// region of an item slot then holds that MMA's operands and the margins:
-constexpr int kOffBc = kOffBl;         // B: the item's queries x 16 halves, hU in column 0
-constexpr int kOffAc = kOffBl + 4096;  // A: 128 rows x 16 halves, 1 in column 0 (written once)
-constexpr int kOffHu = kOffBl + 8192;  // hU per query column, float
+// parts alone are multiplied with the codes, and one more MMA (K = 16,
+// bf16 operands: the fold MMA) adds, per (row, query),
+//   hU + cs' / L - theta' / (G L)     (pass 1: -hU + cs' / L)
+// so that the accumulator holds (G (cs' + L (v + hU)) - theta') / (G L): a
+// candidate's upper bound reaches theta exactly when it is >= 0, and G L
+// times it plus theta' is that upper bound.  hU >= |<q - q_hi, uhat>| + 1
+// bounds the hi part's error (the + 1 covers the fold's rounding); the
+// products 1/L cs' and -1/(G L) theta' are each formed from three-part
+// bf16 splits (six partial products, within 2^-24 of the product).
+// Columns of the fold operands (A: per row, written by the decoders; B: per
+// query, staged by the loader):
+//   0: 1 x hU;  1-6: (a1 a1 a2 a1 a2 a3) x (c1 c2 c1 c3 c2 c1) = cs' / L;
+//   7-12: (b1 b1 b2 b1 b2 b3) x (t1 t2 t1 t3 t2 t1) = -theta' / (G L);
+// a = 1 / L, b = -1 / (G L), c = cs', t = theta' split into bf16 parts.
+// The lo region of an item slot holds the B operand and the margins:
+constexpr int kOffBc = kOffBl;           // fold B: the item's queries x 16 bf16
+constexpr int kOffKeep = kOffBl + 4096;  // columns whose theta is -inf (keep every row): 128-bit mask
+constexpr int kOffHu = kOffBl + 8192;    // hU per query column, float
 constexpr int kConstSBO = 256;         // 8-row groups of a K = 16 operand (two 128-byte core matrices)
 // The hi-only kernel's item slot is the hi B operand, those operands and
 // the per-query constants; its shared memory puts the code slabs, scales
@@ -408,6 +420,7 @@ constexpr int kHOffQct = kOffHu + kNQ * 4, kHOffQinv = kHOffQct + kNQ * 8, kHOff
               kHOffDesc = kHOffQid + kNQ * 4,
               kHSlotBytes = (kHOffDesc + int(sizeof(ItemDesc)) + 127) / 128 * 128;
 constexpr uint32_t kHiTableAddr = 0x10000u;
+constexpr int kFoldABytes = kMR * 32;  // a tile's fold A operand (128 rows x 16 bf16), two buffers after the slots
 constexpr uint32_t kHiLowReserve = 4096;  // static + reserved shared memory below the dynamic allocation, at most
 __device__ __forceinline__ uint32_t const_off(int row, int k8) {
   return uint32_t((row >> 3) * kConstSBO + k8 * 128 + (row & 7) * 16);
@@ -437,7 +450,9 @@ __host__ __device__ constexpr size_t pipe_smem_bytes(int g) {
 }
 // Hi-only kernel: the dynamic allocation starts at most kHiLowReserve bytes
 // above shared address 0, so reserving everything up to the table suffices.
-__host__ __device__ constexpr size_t hi_pipe_smem_bytes() { return size_t(kHiTableAddr) + 65536 + size_t(2) * kHSlotBytes; }
+__host__ __device__ constexpr size_t hi_pipe_smem_bytes() {
+  return size_t(kHiTableAddr) + 65536 + size_t(2) * kHSlotBytes + size_t(2) * kFoldABytes;
+}
 __host__ __device__ constexpr size_t hi_pipe_low_bytes() {
   return size_t(kSlabs) * slab_bytes(1) + size_t(kScaleStages) * kScaleBytes + 32 * 4;
 }
@@ -533,6 +548,28 @@ __device__ __forceinline__ void decode_half(const uint32_t* wd, int dh, const ui
   }
 }
 
+// x = b0 + b1 + b2 in bf16 parts (nearest at each step); the sum is within
+// 2^-24 |x| of x.
+__device__ __forceinline__ void bf16_split3(float x, uint32_t (&b)[3]) {
+  float r = x;
+#pragma unroll
+  for (int i = 0; i < 3; ++i) {
+    const __nv_bfloat16 h = __float2bfloat16_rn(r);
+    b[i] = __bfloat16_as_ushort(h);
+    r -= __bfloat162float(h);
+  }
+}
+__device__ __forceinline__ uint32_t bf16_pair(uint32_t lo, uint32_t hi) { return lo | (hi << 16); }
+__device__ __forceinline__ float rcp_approx(float x) {
+  float r;
+  asm("rcp.approx.ftz.f32 %0, %1;" : "=f"(r) : "f"(x));
+  return r;
+}
+// The margin hU of a query as the fold operands hold it (bf16, rounded up).
+__device__ __forceinline__ float fold_margin(float rho) {
+  return __bfloat162float(__float2bfloat16_ru(rho + 1.0f));
+}
+
 // Epilogue of one row (thread) over the warp's 32 query columns of a tile:
 // DENSE stores every score at the row's place in the query's buffer;
 // otherwise G (cs' + L acc) - theta' >= 0 decides and the hits are appended.
@@ -605,6 +642,63 @@ __device__ __forceinline__ void epilogue_row(const BatchArgs& a, const float (&v
   }
 }
 
+// Epilogue of one row in the hi-only mode, for a row with L > 0 and G > 0:
+// the fold MMA left a = (G (cs' + L (v +- hU)) - theta') / (G L) per query
+// column (pass 1, and columns whose theta is -inf: theta' = 0; pass 1:
+// -hU).  DENSE stores G L a (the lower bound) for every column; otherwise
+// a >= 0 (or a column of the keep mask) is a hit, with upper bound
+// G L a + theta' and lower bound that minus 2 G L hU (scores x 2^s).
+template <bool DENSE>
+__device__ __forceinline__ void epilogue_row_fold(const BatchArgs& a, const float (&vall)[32], float GL, int row,
+                                                  int t, int nrows, int nqt, int eh, int32_t pos,
+                                                  const float* qpair, const float* qinv_s, const int* qid_s,
+                                                  const float* hu_s, const uint32_t* keep_s) {
+  constexpr int kPart = 16;
+#pragma unroll
+  for (int part = 0; part < 32 / kPart; ++part) {
+    const int cbase = eh * 32 + part * kPart;
+    if constexpr (DENSE) {
+      float* dst = a.buf_s + int64_t(t) * kMR + row;
+#pragma unroll
+      for (int i = 0; i < kPart; ++i) {
+        const int col = cbase + i;
+        if (col < nqt) {
+          dst[int64_t(qid_s[col]) * a.cap] = GL * vall[part * kPart + i] * qinv_s[col];
+          if (t == 0 && row == 0) a.cnt[qid_s[col]] = nrows;
+        }
+      }
+    } else {
+      float m = -CUDART_INF_F;
+#pragma unroll
+      for (int i = 0; i < kPart; i += 2) m = fmax3(m, vall[part * kPart + i], vall[part * kPart + i + 1]);
+      const uint32_t keep = (keep_s[cbase >> 5] >> (cbase & 31)) & 0xFFFFu;
+      if (m >= 0.0f || keep) {
+        uint32_t hit = keep;
+#pragma unroll
+        for (int i = 0; i < kPart; ++i) hit |= (vall[part * kPart + i] >= 0.0f ? 1u : 0u) << i;
+        while (hit) {
+          const int i = __ffs(hit) - 1;
+          hit &= hit - 1;
+          float acc = 0.0f;
+#pragma unroll
+          for (int kk = 0; kk < kPart; ++kk) acc = kk == i ? vall[part * kPart + kk] : acc;
+          const int col = cbase + i;
+          const int q = qid_s[col];
+          if (q < 0) continue;
+          const float thq = -qpair[(col >> 1) * 4 + 2 + (col & 1)];
+          const float sup = fmaf(GL, acc, thq > -CUDART_INF_F ? thq : 0.0f);  // upper bound x 2^s
+          const int at = atomicAdd(&a.cnt[q], 1);
+          if (at < a.cap) {
+            a.buf_s[int64_t(q) * a.cap + at] = sup * qinv_s[col];
+            a.buf_p[int64_t(q) * a.cap + at] = pos;
+            a.buf_l[int64_t(q) * a.cap + at] = fmaf(-2.0f * GL, hu_s[col], sup) * qinv_s[col];
+          }
+        }
+      }
+    }
+  }
+}
+
 template <int G, bool DENSE, int FMT, bool HI = false>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __grid_constant__ BatchArgs a) {
   static_assert(!HI || (G == 1 && FMT == kFmtNibble), "hi-only mode: 4-bit codes of one coordinate");
@@ -661,16 +755,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       t32[2 * c + 1] = a.cbbits[4 * c + 2] | (a.cbbits[4 * c + 3] << 16);
     }
   }
-  if constexpr (HI) {
-    // the margin MMA's A operand in both item slots: 1.0 (fp16 0x3C00) in
-    // column 0 of every row, zeros elsewhere; read by the tensor core
-    for (int e = tid; e < 2 * kMR * 2; e += blockDim.x) {
-      const int sl = e / (kMR * 2), r = (e >> 1) % kMR, k8 = e & 1;
-      *reinterpret_cast<uint4*>(slots + sl * SlotB + kOffAc + const_off(r, k8)) =
-          make_uint4(k8 == 0 ? 0x3C00u : 0u, 0u, 0u, 0u);
-    }
-    fence_proxy_async();
-  }
+  // HI: the two fold A buffers (tile gt uses buffer gt & 1, like A)
+  uint8_t* afold = slots + 2 * SlotB;
   const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
   // mbarrier layout: item_full[2], item_empty[2], a_full[2], a_free[2],
   // slab_full / slab_empty[kSlabs], acc_full / acc_empty[kAccBufs],
@@ -722,6 +808,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
   fence_after_sync();
   const uint32_t tmem = tmem_base_sh;
   const uint32_t slots_addr = uint32_t(__cvta_generic_to_shared(slots));
+  const uint32_t afold_addr = uint32_t(__cvta_generic_to_shared(afold));
   const uint32_t slab_addr0 = uint32_t(__cvta_generic_to_shared(slab0));
   const uint32_t scl_addr0 = uint32_t(__cvta_generic_to_shared(scl0));
   const int n_items = a.items[a.nlist];
@@ -786,13 +873,28 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           qinv[j] = inv;
           qid[j] = qs[u];
           if constexpr (HI) {
-            // the margin hU >= |<q - q_hi, uhat>| (rounded up to fp16): + in
-            // pass 2 (upper bounds), - in pass 1 (lower bounds, for theta)
-            const __half hh = __float2half_ru(v ? __ldg(a.qrho + qs[u]) : 0.0f);
-            reinterpret_cast<float*>(sb + kOffHu)[j] = __half2float(hh);
-            const uint32_t bits = uint32_t(__half_as_ushort(hh)) ^ (DENSE ? 0x8000u : 0u);
-            *reinterpret_cast<uint4*>(sb + kOffBc + const_off(j, 0)) = make_uint4(bits, 0u, 0u, 0u);
-            *reinterpret_cast<uint4*>(sb + kOffBc + const_off(j, 1)) = make_uint4(0u, 0u, 0u, 0u);
+            // fold B row: the margin hU (+ in pass 2: upper bounds; - in
+            // pass 1: lower bounds, for theta), cs' and theta' in bf16 parts;
+            // a column with theta = -inf folds theta' = 0 and is marked in
+            // the keep mask; a padding column gets a margin of -1e30 (never
+            // a hit)
+            const float hu = v ? fold_margin(__ldg(a.qrho + qs[u])) : 0.0f;
+            reinterpret_cast<float*>(sb + kOffHu)[j] = hu;
+            uint32_t h0 = v ? uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(DENSE ? -hu : hu)))
+                            : uint32_t(__bfloat16_as_ushort(__float2bfloat16_rn(-1e30f)));
+            uint32_t c[3] = {0u, 0u, 0u}, t3[3] = {0u, 0u, 0u};
+            const bool keep = v && !(th > -CUDART_INF_F);  // theta = -inf: every row is kept
+            if (v) {
+              bf16_split3(cs / inv, c);
+              if (!DENSE && !keep) bf16_split3(th / inv, t3);
+            }
+            const unsigned km = __ballot_sync(kFull, keep);
+            if ((lt & 31) == 0) reinterpret_cast<uint32_t*>(sb + kOffKeep)[j >> 5] = km;
+            *reinterpret_cast<uint4*>(sb + kOffBc + const_off(j, 0)) =
+                make_uint4(bf16_pair(h0, c[0]), bf16_pair(c[1], c[0]), bf16_pair(c[2], c[1]),
+                           bf16_pair(c[0], t3[0]));
+            *reinterpret_cast<uint4*>(sb + kOffBc + const_off(j, 1)) =
+                make_uint4(bf16_pair(t3[1], t3[0]), bf16_pair(t3[2], t3[1]), bf16_pair(t3[0], 0u), 0u);
           }
         }
         // B rows: loads in batches of four 16-byte pieces, then shared stores
@@ -905,9 +1007,9 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
                         ks > 0 ? 1u : 0u);
             if (!HI) umma_f16_ts(tmem + acc_col(c), at, smem_desc(bl_addr + ks * 256, 128, kSBO), idesc, 1u);
           }
-          if (HI)  // + (or, pass 1, -) the margin hU of every query column
-            umma_f16(tmem + acc_col(c), smem_desc(bh_addr + kOffAc, 128, kConstSBO),
-                     smem_desc(bh_addr + kOffBc, 128, kConstSBO), idesc, 1u);
+          if (HI)  // the fold: margin, cs' / L and -theta' / (G L), bf16 operands
+            umma_f16(tmem + acc_col(c), smem_desc(afold_addr + b * uint32_t(kFoldABytes), 128, kConstSBO),
+                     smem_desc(bh_addr + kOffBc, 128, kConstSBO), idesc | kIdescBf16AB, 1u);
           umma_commit(a_free(b));
           umma_commit(acc_full(c));
         }
@@ -936,6 +1038,11 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
           fail();
           ok = false;
           break;
+        }
+        // HI: the row's scale word, loaded now and used after the decode
+        uint32_t swd = 0u;
+        if constexpr (HI) {
+          if (t * kMR + r < desc(s)->nrows) swd = __ldg(a.scales + desc(s)->slot0 + int64_t(t) * kMR + r);
         }
         // the code words of row r (half dh: words dh * NW / 2 ..)
         constexpr int NW = row_words(G, FMT);
@@ -974,6 +1081,28 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
             decode_half<G, FMT>(wd, dh, t256, t32, lane, av, dh == 0 ? a.lite_h / 8 : 0, t64);
           }
           tmem_st32(tmem + (uint32_t(warp * 32) << 16) + a_col(b) + uint32_t(dh * 32), av);
+        }
+        if constexpr (HI) {
+          fence_proxy_async();  // the earlier MMAs' reads of this buffer before the new stores
+          // fold A row: 1, then 1 / L and -1 / (G L) in bf16 parts; a row
+          // past the partition's end or with L = 0 or G = 0 keeps the margin
+          // column only (its epilogue uses the explicit formula)
+          // (the hardware reciprocal: its ~2^-22 relative error is far
+          // inside the margin's + 1)
+          const float Lr = ue7m9_to_f32(swd & 0xffffu), Gr = ue4m12_to_f32(swd >> 16);
+          uint32_t al[3] = {0u, 0u, 0u}, be[3] = {0u, 0u, 0u};
+          if (Lr > 0.0f && Gr > 0.0f) {
+            const float ra = rcp_approx(Lr);
+            bf16_split3(ra, al);
+            bf16_split3(-ra * rcp_approx(Gr), be);
+          }
+          uint8_t* fa = afold + b * kFoldABytes;
+          *reinterpret_cast<uint4*>(fa + const_off(r, 0)) =
+              make_uint4(bf16_pair(0x3F80u, al[0]), bf16_pair(al[0], al[1]), bf16_pair(al[0], al[1]),
+                         bf16_pair(al[2], be[0]));
+          *reinterpret_cast<uint4*>(fa + const_off(r, 1)) =
+              make_uint4(bf16_pair(be[0], be[1]), bf16_pair(be[0], be[1]), bf16_pair(be[2], 0u), 0u);
+          fence_proxy_async();  // generic stores, read by the tensor core
         }
         fence_before_sync();
         __syncwarp();
@@ -1038,8 +1167,14 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         __syncwarp();
         if (lane == 0) mbar_arrive(acc_empty(b));
         if (active && row < nvalid)
-          epilogue_row<DENSE, HI>(a, vall, L, Gs, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s,
-                                  reinterpret_cast<const float*>(slot(s) + kOffHu));
+        {
+          const float* hu_s = reinterpret_cast<const float*>(slot(s) + kOffHu);
+          if (HI && L > 0.0f && Gs > 0.0f)
+            epilogue_row_fold<DENSE>(a, vall, Gs * L, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s, hu_s,
+                                     reinterpret_cast<const uint32_t*>(slot(s) + kOffKeep));
+          else
+            epilogue_row<DENSE, HI>(a, vall, L, Gs, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s, hu_s);
+        }
       }
       __syncwarp();
       if (ok && lane == 0) mbar_arrive(item_empty(s));
@@ -1719,7 +1854,7 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_hi_kernel(const __gri
     rq[w][d] = v - __half2float(__float2half_rn(v));
   }
   __syncwarp();  // rq is read by every lane below
-  const float hu = __half2float(__float2half_ru(a.qrho[q]));
+  const float hu = fold_margin(a.qrho[q]);  // the margin the fold MMA added
   const float* su = a.buf_s + q * a.cap;
   const float* sl = a.buf_l + q * a.cap;
   const int32_t* pp = a.buf_p + q * a.cap;

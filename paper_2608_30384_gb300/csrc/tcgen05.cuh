@@ -24,6 +24,10 @@ __host__ __device__ constexpr uint32_t f16_idesc(int M, int N) {
   return (1u << 4) | (uint32_t(N >> 3) << 17) | (uint32_t(M >> 4) << 24);
 }
 
+// The same instruction with A and B both bf16 (A type bits 7-9 and B type
+// bits 10-12 = 1): OR into an f16_idesc.
+constexpr uint32_t kIdescBf16AB = (1u << 7) | (1u << 10);
+
 __device__ __forceinline__ void umma_f16(uint32_t d_tmem, uint64_t adesc, uint64_t bdesc,
                                          uint32_t idesc, uint32_t accumulate) {
   asm volatile(
