@@ -638,6 +638,9 @@ def run_gpu(args):
             "gpu_launches": launches_per_step(w, nq, batched) * args.steps,
             "clocks": clocks,
             "recall": recall,
+            # index event counters over the whole run (warm-up and timed
+            # steps): queries answered by the exact re-scan fallback
+            "events": ix.counters(),
         }
         print(json.dumps(line), flush=True)
     if ws > 1:

@@ -1216,8 +1216,9 @@ __host__ __device__ constexpr size_t kpipe_smem_bytes(int g) {
          size_t(kScaleStages) * kScaleBytes + 32 * 4 + (g == 1 ? kByteTableBytes + kLiteTableBytes : 0);
 }
 
-template <int G, bool DENSE, int FMT>
+template <int G, bool DENSE, int FMT, bool HI = false>
 __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __grid_constant__ BatchArgs a) {
+  static_assert(!HI || FMT == kFmtNibble, "hi-only mode: 4-bit codes");
   extern __shared__ __align__(128) uint8_t psm[];
   uint8_t* bst0 = psm;                               // B ring
   uint8_t* islot0 = psm + 2 * kBStageBytes;          // item constants + descriptor
@@ -1249,6 +1250,18 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
       t32[2 * c] = a.cbbits[4 * c] | (a.cbbits[4 * c + 1] << 16);
       t32[2 * c + 1] = a.cbbits[4 * c + 2] | (a.cbbits[4 * c + 3] << 16);
     }
+  }
+  // HI: the lo half of each B ring stage is free; the first 4 KB of stage
+  // 0's hold the margin MMA's A operand (1 in column 0 of every row, fp16),
+  // and stage s's [4 KB, 8.5 KB) item slot s's margin B rows and margins
+  auto margin_b = [&](uint32_t s) { return bst0 + s * kBStageBytes + kTileBytes + 4096; };
+  auto margin_hu = [&](uint32_t s) { return reinterpret_cast<float*>(bst0 + s * kBStageBytes + kTileBytes + 8192); };
+  if constexpr (HI) {
+    for (int e = tid; e < kMR * 2; e += blockDim.x) {
+      const int r = e >> 1, k8 = e & 1;
+      *reinterpret_cast<uint4*>(bst0 + kTileBytes + const_off(r, k8)) = make_uint4(k8 == 0 ? 0x3C00u : 0u, 0u, 0u, 0u);
+    }
+    fence_proxy_async();
   }
   const uint32_t bar0 = uint32_t(__cvta_generic_to_shared(&bars[0]));
   // mbarriers: item_full[2], item_empty[2], b_full[2], b_empty[2], a_full[2],
@@ -1363,6 +1376,17 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
         qpair[(j >> 1) * 4 + 2 + (j & 1)] = -th / inv;
         qinv[j] = inv;
         qid[j] = qj;
+        if constexpr (HI) {
+          // the margin hU >= |<q - q_hi, uhat>| (rounded up to fp16): + in
+          // pass 2 (upper bounds), - in pass 1 (lower bounds, for theta)
+          fence_proxy_async();  // the previous item's margin MMAs read these rows
+          const __half hh = __float2half_ru(v ? __ldg(a.qrho + qj) : 0.0f);
+          margin_hu(s)[j] = __half2float(hh);
+          const uint32_t bits = uint32_t(__half_as_ushort(hh)) ^ (DENSE ? 0x8000u : 0u);
+          *reinterpret_cast<uint4*>(margin_b(s) + const_off(j, 0)) = make_uint4(bits, 0u, 0u, 0u);
+          *reinterpret_cast<uint4*>(margin_b(s) + const_off(j, 1)) = make_uint4(0u, 0u, 0u, 0u);
+          fence_proxy_async();  // read by the tensor core
+        }
       }
       asm volatile("bar.sync 1, %0;" ::"n"(kKLoadThreads) : "memory");
       // B work of thread lt < 2 kNQ: query lt % kNQ, the 16-byte pieces
@@ -1399,7 +1423,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
               lv[e] = make_uint4(0, 0, 0, 0);
               if (v && k8 < k8n) {
                 hv[e] = __ldg(reinterpret_cast<const uint4*>(a.qhi + base + k8 * 8));
-                lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + k8 * 8));
+                if (!HI) lv[e] = __ldg(reinterpret_cast<const uint4*>(a.qlo + base + k8 * 8));
               }
             }
 #pragma unroll
@@ -1407,7 +1431,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
               const int k8 = 8 * bh + e;
               if (k8 < k8n) {
                 *reinterpret_cast<uint4*>(dst + tile_off(bj, k8)) = hv[e];
-                *reinterpret_cast<uint4*>(dst + kTileBytes + tile_off(bj, k8)) = lv[e];
+                if (!HI) *reinterpret_cast<uint4*>(dst + kTileBytes + tile_off(bj, k8)) = lv[e];
               }
             }
           }
@@ -1510,7 +1534,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
                 const uint32_t at = tmem + a_col(ab) + uint32_t(ks * 8);
                 umma_f16_ts(tmem + acc_col(r), at, smem_desc(bh + ks * 256, 128, kSBO), idesc,
                             (kc > 0 || ks > 0) ? 1u : 0u);
-                umma_f16_ts(tmem + acc_col(r), at, smem_desc(bl + ks * 256, 128, kSBO), idesc, 1u);
+                if (!HI) umma_f16_ts(tmem + acc_col(r), at, smem_desc(bl + ks * 256, 128, kSBO), idesc, 1u);
               }
               umma_commit(a_free(ab));
             }
@@ -1518,6 +1542,13 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
             umma_commit(b_empty(bs));
           }
           if (!ok) break;
+          if (HI) {
+            // + (or, pass 1, -) the margin hU of every query column
+            const uint32_t mb = uint32_t(__cvta_generic_to_shared(margin_b(s)));
+            for (int r = 0; r < R; ++r)
+              umma_f16(tmem + acc_col(r), smem_desc(bst_addr0 + uint32_t(kTileBytes), 128, kConstSBO),
+                       smem_desc(mb, 128, kConstSBO), idesc, 1u);
+          }
           for (int r = 0; r < R; ++r) {
             umma_commit(acc_full(r));
             ++accu[r];
@@ -1646,7 +1677,8 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_kpipe_kernel(const __
             if (lane == 0) mbar_arrive(acc_empty(r));
           }
           if (active && row < nvalid)
-            epilogue_row<DENSE>(a, vall, L, Gs, row, t, nrows, nqt, ec, pos, qpair, qinv_s, qid_s);
+            epilogue_row<DENSE, HI>(a, vall, L, Gs, row, t, nrows, nqt, ec, pos, qpair, qinv_s, qid_s,
+                                    margin_hu(s));
           __syncwarp();
         }
       }
@@ -1789,12 +1821,12 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_warp_kernel(
 // per query: T = the k-th largest s_lo bounds the exact k-th best score from
 // below, so only candidates with s_up >= T can be in the top k; their exact
 // scores are s_up + G L (<r, uhat> - hU) 2^-s (r = 2^s q - q_hi, exact in
-// fp32; the MMA added hU instead of <r, uhat>), from the row's codes, and the
-// top k of those by (score desc, id asc) is the result.  With more than
-// kFinCap candidates T is taken over the first kFinCap of them (still a
-// lower bound).  Buffers that overflowed, came out short under a finite
-// theta, or leave more than kFinCap candidates above T go to the exact
-// single-query re-scan, as in finalize_warp_kernel.
+// fp32; the MMAs added the margin hU instead of <r, uhat>), from the row's
+// codes (4-bit codes of g coordinates, tile-interleaved chunks), and the top
+// k of those by (score desc, id asc) is the result; T comes from a warp
+// radix select over all the candidates.  Buffers that overflowed, came out
+// short under a finite theta, or leave more than fcap candidates above T go
+// to the exact single-query re-scan, as in finalize_warp_kernel.
 struct FinHiArgs {
   const float* buf_s;
   const float* buf_l;
@@ -1808,26 +1840,145 @@ struct FinHiArgs {
   const float* qrot;  // rotated queries, nq x Dp
   int Dp;
   const float* qrho;
-  const uint8_t* codes;  // 4-bit codes of one coordinate, 16-byte chunks, tile-interleaved
+  int fold;              // the margin as the fold MMA holds it (else the fp16 margin MMA's)
+  const uint8_t* codes;  // 4-bit codes of g coordinates each, tile-interleaved chunks
   const uint32_t* scales;
-  int stride;
-  float cb[16];
+  int stride, chunk, g;
+  int npos;  // coordinates covered by a row's codes: 2 g stride
+  int fcap;  // candidates per warp in shared memory (a power of two >= 512)
+  float cb[64];
   int* ovf_list;
   int* counts;
   unsigned long long* ctr;
   int64_t* out_ids;
   float* out_scores;
 };
+__host__ __device__ constexpr size_t fin_hi_warp_bytes(int fcap, int npos) {
+  return size_t(fcap) * 12 + 256 * 4 + size_t(npos) * 4;  // window, radix histogram, r
+}
 
-__global__ void __launch_bounds__(kFinWarps * 32) finalize_hi_kernel(const __grid_constant__ FinHiArgs a) {
-  __shared__ uint32_t fk[kFinWarps][kFinCap];
-  __shared__ int64_t fi[kFinWarps][kFinCap];
-  __shared__ float rq[kFinWarps][kKC];  // r = 2^s q - q_hi of the warp's query
-  __shared__ float cbs[16];
-  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
-  if (threadIdx.x < 16) cbs[threadIdx.x] = a.cb[threadIdx.x];
+// <r, uhat> of the row at slot pos (r in shared memory, codebook cb:
+// component j of codeword c at cb[G c + j]).
+template <int G>
+__device__ __forceinline__ float fin_word_dot(uint32_t wd, const float* rv, const float* cb, float dot) {
+#pragma unroll
+  for (int nb = 0; nb < 8; ++nb) {
+    const float* cv = cb + G * ((wd >> (4 * nb)) & 15u);
+#pragma unroll
+    for (int j = 0; j < G; ++j) dot = fmaf(cv[j], rv[G * nb + j], dot);
+  }
+  return dot;
+}
+template <int G>
+__device__ __forceinline__ float fin_row_dot(const FinHiArgs& a, int32_t pos, const float* rq, const float* cb) {
+  const int r = pos & (kMR - 1);
+  const uint8_t* tile = a.codes + int64_t(pos - r) * a.stride;
+  const int CH = a.chunk;
+  float dot = 0.0f;
+  if (CH == 16) {
+    const int nch = a.stride / 16;
+    int c = 0;
+    for (; c + 4 <= nch; c += 4) {  // four 16-byte loads in flight
+      uint4 wv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) wv[u] = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c + u) * kMR + r) * 16));
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const float* rv = rq + G * 32 * (c + u);
+        dot = fin_word_dot<G>(wv[u].x, rv, cb, dot);
+        dot = fin_word_dot<G>(wv[u].y, rv + 8 * G, cb, dot);
+        dot = fin_word_dot<G>(wv[u].z, rv + 16 * G, cb, dot);
+        dot = fin_word_dot<G>(wv[u].w, rv + 24 * G, cb, dot);
+      }
+    }
+    for (; c < nch; ++c) {
+      const uint4 wv = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c) * kMR + r) * 16));
+      const float* rv = rq + G * 32 * c;
+      dot = fin_word_dot<G>(wv.x, rv, cb, dot);
+      dot = fin_word_dot<G>(wv.y, rv + 8 * G, cb, dot);
+      dot = fin_word_dot<G>(wv.z, rv + 16 * G, cb, dot);
+      dot = fin_word_dot<G>(wv.w, rv + 24 * G, cb, dot);
+    }
+    return dot;
+  }
+  for (int c = 0; c < a.stride / CH; ++c) {
+    const uint8_t* chp = tile + (size_t(c) * kMR + r) * CH;
+    for (int w = 0; w < CH / 4; ++w)
+      dot = fin_word_dot<G>(__ldg(reinterpret_cast<const uint32_t*>(chp) + w), rq + G * 2 * (c * CH + 4 * w), cb,
+                            dot);
+  }
+  return dot;
+}
+
+// The k-th largest order key of s[0 .. n) (n > k) by one warp: four 8-bit
+// radix passes over a 256-bin histogram in shared memory.
+__device__ uint32_t warp_kth_key(const float* s, int n, int k, uint32_t* hist) {
+  const int lane = threadIdx.x & 31;
+  uint32_t prefix = 0u, mask = 0u;
+  int rem = k;
+  for (int pass = 0; pass < 4; ++pass) {
+    const int shift = 24 - 8 * pass;
+    for (int i = lane; i < 256; i += 32) hist[i] = 0u;
+    __syncwarp();
+    for (int base = 0; base < n; base += 32) {
+      const int i = base + lane;
+      const uint32_t key = i < n ? float_order_key(__ldg(s + i)) : 0u;
+      warp_hist_add(hist, (key >> shift) & 255u, i < n && (key & mask) == prefix);
+    }
+    __syncwarp();
+    // lane l holds bins 255 - 8 l .. 248 - 8 l (from the top); the first
+    // bin, from the top, where the count reaches rem
+    uint32_t c8[8], tot = 0u;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      c8[j] = hist[255 - 8 * lane - j];
+      tot += c8[j];
+    }
+    uint32_t incl = tot;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+      const uint32_t y = __shfl_up_sync(kFull, incl, o);
+      if (lane >= o) incl += y;
+    }
+    const uint32_t excl = incl - tot;
+    const unsigned hit = __ballot_sync(kFull, excl < uint32_t(rem) && incl >= uint32_t(rem));
+    const int src = __ffs(hit) - 1;
+    int bin = 0, newrem = rem;
+    if (lane == src) {
+      uint32_t cum = excl;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        if (cum + c8[j] >= uint32_t(rem)) {
+          bin = 255 - 8 * lane - j;
+          newrem = rem - int(cum);
+          break;
+        }
+        cum += c8[j];
+      }
+    }
+    bin = __shfl_sync(kFull, bin, src);
+    rem = __shfl_sync(kFull, newrem, src);
+    prefix |= uint32_t(bin) << shift;
+    mask |= 255u << shift;
+    __syncwarp();
+  }
+  return prefix;
+}
+
+template <int G>
+__global__ void __launch_bounds__(128) finalize_hi_kernel(const __grid_constant__ FinHiArgs a) {
+  extern __shared__ __align__(16) uint8_t fsm_hi[];
+  float* cbs = reinterpret_cast<float*>(fsm_hi);
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, W = blockDim.x >> 5;
+  const int fcap = a.fcap;
+  uint8_t* wb = fsm_hi + 256 + size_t(w) * fin_hi_warp_bytes(fcap, a.npos);
+  int64_t* fi = reinterpret_cast<int64_t*>(wb);
+  uint32_t* fk = reinterpret_cast<uint32_t*>(wb + size_t(fcap) * 8);
+  uint32_t* hist = fk + fcap;  // 256 bins
+  float* rq = reinterpret_cast<float*>(hist + 256);
+  if (threadIdx.x < 64) cbs[threadIdx.x] = a.cb[threadIdx.x];
   __syncthreads();
-  const int64_t q = int64_t(blockIdx.x) * kFinWarps + w;
+  const int64_t q = int64_t(blockIdx.x) * W + w;
   if (q >= a.nq) return;
   const int n = a.cnt[q];
   const int k = a.k;
@@ -1848,41 +1999,17 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_hi_kernel(const __gri
   int e2 = 0;
   if (m > 0.0f) frexpf(m, &e2);
   const float sc = ldexpf(1.0f, 11 - e2), inv = ldexpf(1.0f, e2 - 11);
-  const int npos = (a.stride / 16) * 32;  // code positions of a row (<= kKC)
-  for (int d = lane; d < npos; d += 32) {
+  for (int d = lane; d < a.npos; d += 32) {
     const float v = d < a.Dp ? src[d] * sc : 0.0f;
-    rq[w][d] = v - __half2float(__float2half_rn(v));
+    rq[d] = v - __half2float(__float2half_rn(v));
   }
   __syncwarp();  // rq is read by every lane below
-  const float hu = fold_margin(a.qrho[q]);  // the margin the fold MMA added
+  // the margin the MMAs added
+  const float hu = a.fold ? fold_margin(a.qrho[q]) : __half2float(__float2half_ru(a.qrho[q]));
   const float* su = a.buf_s + q * a.cap;
-  const float* sl = a.buf_l + q * a.cap;
   const int32_t* pp = a.buf_p + q * a.cap;
-  // T: the k-th largest lower bound (of the first kFinCap; all candidates
-  // when n <= k)
-  uint32_t T = 0u;
-  if (n > k) {
-    const int nt = min(n, kFinCap);
-    int p2 = 1;
-    while (p2 < nt) p2 <<= 1;
-    for (int i = lane; i < p2; i += 32) fk[w][i] = i < nt ? float_order_key(sl[i]) : 0u;
-    __syncwarp();
-    for (int size = 2; size <= p2; size <<= 1)
-      for (int stride = size >> 1; stride > 0; stride >>= 1) {
-        for (int i = lane; i < (p2 >> 1); i += 32) {
-          const int lo = 2 * i - (i & (stride - 1)), hi = lo + stride;
-          const bool asc = (lo & size) == 0;  // sorted descending overall
-          const uint32_t klo = fk[w][lo], khi = fk[w][hi];
-          if (asc ? khi > klo : klo > khi) {
-            fk[w][lo] = khi;
-            fk[w][hi] = klo;
-          }
-        }
-        __syncwarp();
-      }
-    T = fk[w][k - 1];
-    __syncwarp();
-  }
+  // T: the k-th largest lower bound (all candidates when n <= k)
+  const uint32_t T = n > k ? warp_kth_key(a.buf_l + q * a.cap, n, k, hist) : 0u;
   // the candidates that can be in the top k, with their exact scores
   int mcnt = 0;
   for (int base = 0; base < n; base += 32) {
@@ -1890,28 +2017,18 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_hi_kernel(const __gri
     const bool in = i < n && float_order_key(su[i]) >= T;
     const unsigned bm = __ballot_sync(kFull, in);
     const int at = mcnt + __popc(bm & ((1u << lane) - 1u));
-    if (in && at < kFinCap) {
+    if (in && at < fcap) {
       const int32_t pos = pp[i];
-      const int r = pos & (kMR - 1);
-      const uint8_t* row = a.codes + int64_t(pos - r) * a.stride + r * 16;
-      float dot = 0.0f;
-      for (int c = 0; c < a.stride / 16; ++c) {
-        const uint4 wv = __ldg(reinterpret_cast<const uint4*>(row + size_t(c) * kMR * 16));
-        const uint32_t wd[4] = {wv.x, wv.y, wv.z, wv.w};
-#pragma unroll
-        for (int j = 0; j < 4; ++j)
-#pragma unroll
-          for (int nb = 0; nb < 8; ++nb) dot = fmaf(cbs[(wd[j] >> (4 * nb)) & 15u], rq[w][32 * c + 8 * j + nb], dot);
-      }
+      const float dot = fin_row_dot<G>(a, pos, rq, cbs);
       const uint32_t swd = __ldg(a.scales + pos);
-      const float G = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
-      const float s = su[i] + G * L * (dot - hu) * inv;
-      fk[w][at] = float_order_key(s);
-      fi[w][at] = a.ids[pos];
+      const float Gs = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
+      const float s = su[i] + Gs * L * (dot - hu) * inv;
+      fk[at] = float_order_key(s);
+      fi[at] = a.ids[pos];
     }
     mcnt += __popc(bm);
   }
-  if (mcnt > kFinCap) {
+  if (mcnt > fcap) {
     if (lane == 0) {
       a.ovf_list[atomicAdd(&a.counts[0], 1)] = int(q);
       atomicAdd(&a.ctr[kCtrBatchedOverflow], 1ull);
@@ -1922,8 +2039,8 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_hi_kernel(const __gri
   int p2 = 1;
   while (p2 < mcnt || p2 < k) p2 <<= 1;
   for (int i = mcnt + lane; i < p2; i += 32) {
-    fk[w][i] = 0u;
-    fi[w][i] = LLONG_MAX;
+    fk[i] = 0u;
+    fi[i] = LLONG_MAX;
   }
   __syncwarp();
   for (int size = 2; size <= p2; size <<= 1)
@@ -1931,22 +2048,22 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_hi_kernel(const __gri
       for (int i = lane; i < (p2 >> 1); i += 32) {
         const int lo = 2 * i - (i & (stride - 1)), hi = lo + stride;
         const bool asc = (lo & size) == 0;
-        const uint32_t klo = fk[w][lo], khi = fk[w][hi];
-        const int64_t ilo = fi[w][lo], ihi = fi[w][hi];
+        const uint32_t klo = fk[lo], khi = fk[hi];
+        const int64_t ilo = fi[lo], ihi = fi[hi];
         const bool swap = asc ? better(khi, ihi, klo, ilo) : better(klo, ilo, khi, ihi);
         if (swap) {
-          fk[w][lo] = khi;
-          fk[w][hi] = klo;
-          fi[w][lo] = ihi;
-          fi[w][hi] = ilo;
+          fk[lo] = khi;
+          fk[hi] = klo;
+          fi[lo] = ihi;
+          fi[hi] = ilo;
         }
       }
       __syncwarp();
     }
   for (int i = lane; i < k; i += 32) {
-    const bool ok = i < mcnt && fi[w][i] != LLONG_MAX;
-    a.out_ids[q * k + i] = ok ? fi[w][i] : -1;
-    a.out_scores[q * k + i] = ok ? float_from_order_key(fk[w][i]) : -CUDART_INF_F;
+    const bool ok = i < mcnt && fi[i] != LLONG_MAX;
+    a.out_ids[q * k + i] = ok ? fi[i] : -1;
+    a.out_scores[q * k + i] = ok ? float_from_order_key(fk[i]) : -CUDART_INF_F;
   }
 }
 
@@ -2066,6 +2183,13 @@ cudaError_t run_batched(const rslm_index* ix, const Lists& L, const __half* qhi,
                       : (g == 1   ? batched_pipe_kernel<1, true, kFmtNibble>
                          : g == 2 ? batched_pipe_kernel<2, true, kFmtNibble>
                                   : batched_pipe_kernel<4, true, kFmtNibble>);
+  else if (qrho)  // hi-only mode, K chunks of 128 (4-bit codes, no Rslm4Lite head)
+    pk = theta ? (g == 1   ? batched_kpipe_kernel<1, false, kFmtNibble, true>
+                  : g == 2 ? batched_kpipe_kernel<2, false, kFmtNibble, true>
+                           : batched_kpipe_kernel<4, false, kFmtNibble, true>)
+               : (g == 1   ? batched_kpipe_kernel<1, true, kFmtNibble, true>
+                  : g == 2 ? batched_kpipe_kernel<2, true, kFmtNibble, true>
+                           : batched_kpipe_kernel<4, true, kFmtNibble, true>);
   else
     pk = c1.bits == 3 ? (theta ? batched_kpipe_kernel<1, false, kFmt3> : batched_kpipe_kernel<1, true, kFmt3>)
          : b.lite_h   ? (theta ? batched_kpipe_kernel<1, false, kFmtLite> : batched_kpipe_kernel<1, true, kFmtLite>)
@@ -2116,8 +2240,11 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
     oL[l][5] = take(size_t(np) * 4);
     oL[l][6] = take(size_t(np / kNQ + nlist + 1) * 4);  // at most sum of ceil(cnt / kNQ) items
   }
-  // hi-only mode: 4-bit codes of one coordinate in 16-byte chunks, padded D <= 128
-  const bool hi = c1.g == 1 && c1.bits == 4 && c1.lite_h == 0 && c1.chunk == 16 && Dp16 <= kKC;
+  // hi-only mode: 4-bit codes (of g = 1, 2 or 4 coordinates), no Rslm4Lite
+  // head; padded D <= 128 (the fold kernel) needs 16-byte chunks of one
+  // coordinate, larger D (the margin MMA in the K-chunk kernel) any of them
+  const bool hi = c1.bits != 3 && c1.lite_h == 0 &&
+                  (Dp16 <= kKC ? (c1.g == 1 && c1.chunk == 16) : true);
   const size_t o_qrho = take(hi ? size_t(nq) * 4 : 4), o_bl = take(hi ? size_t(nq) * cap * 4 : 4);
   const size_t o_qhi = take(size_t(nq) * Dp16 * 2), o_qlo = take(size_t(nq) * Dp16 * 2),
                o_qinv = take(size_t(nq) * 4), o_theta = take(size_t(nq) * 4),
@@ -2150,10 +2277,16 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
   int* fcounts = reinterpret_cast<int*>(ws + o_fcounts);
   float* qrho = hi ? reinterpret_cast<float*>(ws + o_qrho) : nullptr;
   float* bl = hi ? reinterpret_cast<float*>(ws + o_bl) : nullptr;
-  // ||uhat|| <= sqrt(Dp) max |codebook level| bounds the dot product with the remainder
-  float maxlev = 0.0f;
-  for (int i = 0; i < 16; ++i) maxlev = std::max(maxlev, std::fabs(c1.cbf[i]));
-  const float U = std::sqrt(float(c1.Dp)) * maxlev * (1.0f + 1e-5f);
+  // ||uhat|| <= sqrt(codes per row x max ||codeword||^2) bounds the dot
+  // product with the remainder
+  float maxcw = 0.0f;
+  for (int c = 0; c < 16; ++c) {
+    float n2 = 0.0f;
+    for (int j = 0; j < c1.g; ++j) n2 += c1.cbf[c1.g * c + j] * c1.cbf[c1.g * c + j];
+    maxcw = std::max(maxcw, n2);
+  }
+  const int ncodes = (c1.Dp + c1.g - 1) / c1.g;
+  const float U = std::sqrt(float(ncodes) * maxcw) * (1.0f + 1e-5f);
 
   // lists: L[0] the first probe of every query, L[1] all probe pairs
   const float* lcs = (ix->flags & RSLM_FULL_VECTOR) ? nullptr : cs;  // full-vector codes: no <q, c> term
@@ -2200,17 +2333,31 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
         fa.qrot = qrot;
         fa.Dp = c1.Dp;
         fa.qrho = qrho;
+        fa.fold = Dp16 <= kKC ? 1 : 0;
         fa.codes = ix->codes1;
         fa.scales = ix->scales1;
         fa.stride = c1.stride;
-        for (int i = 0; i < 16; ++i) fa.cb[i] = c1.cbf[i];
+        fa.chunk = c1.chunk;
+        fa.g = c1.g;
+        fa.npos = 2 * c1.g * c1.stride;
+        int fcap = 512;
+        while (fcap < 4 * k) fcap <<= 1;
+        fa.fcap = fcap;
+        for (int i = 0; i < 64; ++i) fa.cb[i] = c1.cbf[i];
         fa.ovf_list = ovf;
         fa.counts = fcounts;
         fa.ctr = ix->d_counters;
         fa.out_ids = out_ids;
         fa.out_scores = out_scores;
-        finalize_hi_kernel<<<unsigned((nq + kFinWarps - 1) / kFinWarps), kFinWarps * 32, 0, s>>>(fa);
-        e = cudaGetLastError();
+        const int fw = 4;  // warps (queries) per block
+        const size_t fsm = 256 + size_t(fw) * fin_hi_warp_bytes(fcap, fa.npos);
+        using FK = void (*)(FinHiArgs);
+        const FK fk = c1.g == 1 ? finalize_hi_kernel<1> : c1.g == 2 ? finalize_hi_kernel<2> : finalize_hi_kernel<4>;
+        e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(fsm));
+        if (e == cudaSuccess) {
+          fk<<<unsigned((nq + fw - 1) / fw), fw * 32, fsm, s>>>(fa);
+          e = cudaGetLastError();
+        }
       } else if (e == cudaSuccess) {
         finalize_warp_kernel<<<unsigned((nq + kFinWarps - 1) / kFinWarps), kFinWarps * 32, 0, s>>>(
             bs, bp, bc, nq, cap, ix->ids, k, theta, ovf, ac, fcounts, ix->d_counters, out_ids, out_scores);
