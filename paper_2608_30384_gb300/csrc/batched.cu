@@ -230,15 +230,35 @@ __device__ uint32_t block_kth_key(const float* s, int n, int k, uint32_t* hist, 
       warp_hist_add(hist, (kk >> shift) & 255u, i < n && (kk & mask) == prefix);
     }
     __syncthreads();
-    if (tid == 0) {
-      uint32_t cum = 0;
-      int b = 255;
-      for (; b > 0; --b) {
-        if (cum + hist[b] >= rem) break;
-        cum += hist[b];
+    if (tid < 32) {
+      // lane l holds bins 255 - 8 l .. 248 - 8 l (from the top); the first
+      // bin, from the top, where the count reaches rem
+      uint32_t c8[8], tot = 0u;
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        c8[j] = hist[255 - 8 * tid - j];
+        tot += c8[j];
       }
-      sh[0] = rem - cum;
-      sh[1] = prefix | (uint32_t(b) << shift);
+      uint32_t incl = tot;
+#pragma unroll
+      for (int o = 1; o < 32; o <<= 1) {
+        const uint32_t y = __shfl_up_sync(kFull, incl, o);
+        if (tid >= o) incl += y;
+      }
+      const uint32_t excl = incl - tot;
+      const unsigned hit = __ballot_sync(kFull, excl < rem && incl >= rem);
+      if (tid == __ffs(hit) - 1) {
+        uint32_t cum = excl;
+#pragma unroll
+        for (int j = 0; j < 8; ++j) {
+          if (cum + c8[j] >= rem) {
+            sh[0] = rem - cum;
+            sh[1] = prefix | (uint32_t(255 - 8 * tid - j) << shift);
+            break;
+          }
+          cum += c8[j];
+        }
+      }
     }
     __syncthreads();
     rem = sh[0];
@@ -1817,8 +1837,8 @@ __global__ void __launch_bounds__(kFinWarps * 32) finalize_warp_kernel(
 }
 
 // Hi-only mode: pass 2 kept every candidate whose upper bound reached theta,
-// with its upper bound s_up (buf_s) and lower bound s_lo (buf_l).  One warp
-// per query: T = the k-th largest s_lo bounds the exact k-th best score from
+// with its upper bound s_up (buf_s) and lower bound s_lo (buf_l).  Per
+// query, T = the k-th largest s_lo bounds the exact k-th best score from
 // below, so only candidates with s_up >= T can be in the top k; their exact
 // scores are s_up + G L (<r, uhat> - hU) 2^-s (r = 2^s q - q_hi, exact in
 // fp32; the MMAs added the margin hU instead of <r, uhat>), from the row's
@@ -1845,7 +1865,7 @@ struct FinHiArgs {
   const uint32_t* scales;
   int stride, chunk, g;
   int npos;  // coordinates covered by a row's codes: 2 g stride
-  int fcap;  // candidates per warp in shared memory (a power of two >= 512)
+  int fcap;  // candidates per query in shared memory (a power of two >= 512)
   float cb[64];
   int* ovf_list;
   int* counts;
@@ -1855,6 +1875,9 @@ struct FinHiArgs {
 };
 __host__ __device__ constexpr size_t fin_hi_warp_bytes(int fcap, int npos) {
   return size_t(fcap) * 12 + 256 * 4 + size_t(npos) * 4;  // window, radix histogram, r
+}
+__host__ __device__ constexpr size_t fin_hi_block_bytes(int fcap, int npos) {
+  return 256 + size_t(fcap) * 12 + 256 * 4 + size_t(npos) * 4;  // codebook, window, radix histogram, r
 }
 
 // <r, uhat> of the row at slot pos (r in shared memory, codebook cb:
@@ -1965,8 +1988,10 @@ __device__ uint32_t warp_kth_key(const float* s, int n, int k, uint32_t* hist) {
   return prefix;
 }
 
+// One warp per query (the shorter rows: window decode is cheap, the select
+// and sort dominate).
 template <int G>
-__global__ void __launch_bounds__(128) finalize_hi_kernel(const __grid_constant__ FinHiArgs a) {
+__global__ void __launch_bounds__(128) finalize_hi_warp_kernel(const __grid_constant__ FinHiArgs a) {
   extern __shared__ __align__(16) uint8_t fsm_hi[];
   float* cbs = reinterpret_cast<float*>(fsm_hi);
   const int lane = threadIdx.x & 31, w = threadIdx.x >> 5, W = blockDim.x >> 5;
@@ -2064,6 +2089,98 @@ __global__ void __launch_bounds__(128) finalize_hi_kernel(const __grid_constant_
     const bool ok = i < mcnt && fi[i] != LLONG_MAX;
     a.out_ids[q * k + i] = ok ? fi[i] : -1;
     a.out_scores[q * k + i] = ok ? float_from_order_key(fk[i]) : -CUDART_INF_F;
+  }
+}
+
+// One block of kFinHiThreads per query (grid-strided): the remainder r and
+// the window live in the block's shared memory; a block radix select finds
+// T, every thread scores window rows, and a block sort orders them.
+constexpr int kFinHiThreads = 128;
+template <int G>
+__global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const __grid_constant__ FinHiArgs a) {
+  extern __shared__ __align__(16) uint8_t fsm_hi[];
+  const int fcap = a.fcap;
+  float* cbs = reinterpret_cast<float*>(fsm_hi);                 // 64 floats
+  int64_t* fi = reinterpret_cast<int64_t*>(fsm_hi + 256);        // fcap ids
+  uint32_t* fk = reinterpret_cast<uint32_t*>(fi + fcap);         // fcap keys
+  uint32_t* hist = fk + fcap;                                    // 256 bins
+  float* rq = reinterpret_cast<float*>(hist + 256);              // npos
+  __shared__ int sh_m;
+  __shared__ float sh_max[kFinHiThreads / 32];
+  __shared__ uint32_t sh_sel[2];
+  const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
+  if (tid < 64) cbs[tid] = a.cb[tid];
+  const int k = a.k;
+  for (int64_t q = blockIdx.x; q < a.nq; q += gridDim.x) {
+    __syncthreads();  // the previous query's buffers are read
+    const int n = a.cnt[q];
+    const bool short_list = n < k && a.theta[q] > -CUDART_INF_F;
+    if (n > a.cap || short_list) {
+      if (tid == 0) {
+        a.ovf_list[atomicAdd(&a.counts[0], 1)] = int(q);
+        atomicAdd(&a.ctr[short_list ? kCtrBatchedShort : kCtrBatchedOverflow], 1ull);
+      }
+      continue;
+    }
+    // the query's scaling 2^s (max |q| 2^s in [1024, 2048)) and remainder r
+    const float* src = a.qrot + q * a.Dp;
+    float m = 0.0f;
+    for (int d = tid; d < a.Dp; d += kFinHiThreads) m = fmaxf(m, fabsf(src[d]));
+#pragma unroll
+    for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
+    if (lane == 0) sh_max[w] = m;
+    if (tid == 0) sh_m = 0;
+    __syncthreads();
+    m = sh_max[0];
+#pragma unroll
+    for (int i = 1; i < kFinHiThreads / 32; ++i) m = fmaxf(m, sh_max[i]);
+    int e2 = 0;
+    if (m > 0.0f) frexpf(m, &e2);
+    const float sc = ldexpf(1.0f, 11 - e2), inv = ldexpf(1.0f, e2 - 11);
+    for (int d = tid; d < a.npos; d += kFinHiThreads) {
+      const float v = d < a.Dp ? src[d] * sc : 0.0f;
+      rq[d] = v - __half2float(__float2half_rn(v));
+    }
+    // T: the k-th largest lower bound (all candidates when n <= k)
+    const uint32_t T = n > k ? block_kth_key(a.buf_l + q * a.cap, n, k, hist, sh_sel) : 0u;
+    __syncthreads();  // r is written
+    // the margin the MMAs added
+    const float hu = a.fold ? fold_margin(a.qrho[q]) : __half2float(__float2half_ru(a.qrho[q]));
+    const float* su = a.buf_s + q * a.cap;
+    const int32_t* pp = a.buf_p + q * a.cap;
+    // the candidates that can be in the top k, with their exact scores
+    for (int i = tid; i < n; i += kFinHiThreads) {
+      if (float_order_key(su[i]) < T) continue;
+      const int at = atomicAdd(&sh_m, 1);
+      if (at >= fcap) continue;
+      const int32_t pos = pp[i];
+      const float dot = fin_row_dot<G>(a, pos, rq, cbs);
+      const uint32_t swd = __ldg(a.scales + pos);
+      const float Gs = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
+      fk[at] = float_order_key(su[i] + Gs * L * (dot - hu) * inv);
+      fi[at] = a.ids[pos];
+    }
+    __syncthreads();
+    const int mcnt = sh_m;
+    if (mcnt > fcap) {
+      if (tid == 0) {
+        a.ovf_list[atomicAdd(&a.counts[0], 1)] = int(q);
+        atomicAdd(&a.ctr[kCtrBatchedOverflow], 1ull);
+      }
+      continue;
+    }
+    int p2 = 1;
+    while (p2 < mcnt || p2 < k) p2 <<= 1;
+    for (int i = mcnt + tid; i < p2; i += kFinHiThreads) {
+      fk[i] = 0u;
+      fi[i] = LLONG_MAX;
+    }
+    block_bitonic_sort(fk, fi, p2);
+    for (int i = tid; i < k; i += kFinHiThreads) {
+      const bool ok = i < mcnt && fi[i] != LLONG_MAX;
+      a.out_ids[q * k + i] = ok ? fi[i] : -1;
+      a.out_scores[q * k + i] = ok ? float_from_order_key(fk[i]) : -CUDART_INF_F;
+    }
   }
 }
 
@@ -2349,13 +2466,25 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
         fa.ctr = ix->d_counters;
         fa.out_ids = out_ids;
         fa.out_scores = out_scores;
-        const int fw = 4;  // warps (queries) per block
-        const size_t fsm = 256 + size_t(fw) * fin_hi_warp_bytes(fcap, fa.npos);
+        // rows of at most 256 coordinates: one warp per query; longer rows:
+        // one block per query, whose threads share the window's row decode
         using FK = void (*)(FinHiArgs);
-        const FK fk = c1.g == 1 ? finalize_hi_kernel<1> : c1.g == 2 ? finalize_hi_kernel<2> : finalize_hi_kernel<4>;
+        const bool per_warp = fa.npos <= 256;
+        const int fw = 4;  // warps (queries) per block of the per-warp kernel
+        const size_t fsm = per_warp ? 256 + size_t(fw) * fin_hi_warp_bytes(fcap, fa.npos)
+                                    : fin_hi_block_bytes(fcap, fa.npos);
+        const FK fk = per_warp ? (c1.g == 1   ? finalize_hi_warp_kernel<1>
+                                  : c1.g == 2 ? finalize_hi_warp_kernel<2>
+                                              : finalize_hi_warp_kernel<4>)
+                               : (c1.g == 1   ? finalize_hi_block_kernel<1>
+                                  : c1.g == 2 ? finalize_hi_block_kernel<2>
+                                              : finalize_hi_block_kernel<4>);
         e = cudaFuncSetAttribute(fk, cudaFuncAttributeMaxDynamicSharedMemorySize, int(fsm));
         if (e == cudaSuccess) {
-          fk<<<unsigned((nq + fw - 1) / fw), fw * 32, fsm, s>>>(fa);
+          if (per_warp)
+            fk<<<unsigned((nq + fw - 1) / fw), fw * 32, fsm, s>>>(fa);
+          else
+            fk<<<unsigned(std::min<int64_t>(nq, 152 * 16)), kFinHiThreads, fsm, s>>>(fa);
           e = cudaGetLastError();
         }
       } else if (e == cudaSuccess) {

@@ -1106,6 +1106,11 @@ struct RescoreArgs {
   int64_t* out_ids;
   float* out_scores;
   int* err;
+  // rescore_mma_kernel: queries, warps whose region sits below the byte
+  // table, bytes per warp region
+  int64_t nq;
+  int warps_pre;
+  int region;
 };
 
 __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ RescoreArgs a) {
@@ -1165,6 +1170,211 @@ __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ Re
   }
 }
 
+// Rescoring on the tensor cores, for 4-bit rescoring codes of one
+// coordinate each scored by reading B (<q, a2> = the stage-1 score) or as
+// full-vector codes: one warp per query in persistent CTAs of up to
+// kRsWarps warps, one CTA per SM.  The warp-level MMA m16n8k16 (fp16
+// operands, fp32 accumulation) is the multiply-add engine, as in the
+// single-query scan:
+//   A (16 candidate rows x 16 code positions) = the codes' levels, looked
+//     up through the per-lane byte table at kBtTableAddr (a byte = two codes
+//     -> their two binary16-exact levels, one A register);
+//   B (16 x 8) = the rotated query scaled by 2^s (max |q| 2^s in [1024,
+//     2048)) and split into q_hi = fp16(q) (column 0) and q_lo = fp16(q -
+//     q_hi) (column 1);
+//   D column 0 + column 1 = 2^s <R2 q, u2hat> of each row.
+// A rescoring row is contiguous (stride2 bytes, a multiple of 16).  Lane (g,
+// t) = (lane / 4, lane % 4) loads bytes 64 J + 16 t .. + 15 of rows g and g
+// + 8 of a 16-row group: code positions 128 J + 32 t + 8 w + {0..7} in its
+// word w, and MMA i = 2 w + m of segment J takes bytes 2 m and 2 m + 1 of
+// word w, i.e. positions 128 J + 32 t + 4 i + {0..3}.  The dot product is
+// order-free, so the B fragment of lane (g, t) holds those same positions of
+// column g; the warp's query block keeps them as one 16-byte entry (J, i,
+// t) = (hi, lo) halves of the four positions, so the eight lanes that read
+// an entry set touch 64 contiguous bytes.  A pass scores 32 candidates (two
+// 16-row groups share the B fragments); s2 = G2 (<q, a2> + L2 <R2 q,
+// u2hat>) (Sec. 3.5, Sec. 5.2) is stored in place of the stage-1 score, and
+// a warp bitonic sort of the query's k candidates by (score desc, id asc)
+// gives the top k_final.  Per warp: the query block (stride2 x 8 bytes
+// rounded to 512), then np2 keys and np2 ids.
+constexpr int kRsWarps = 16;
+
+
+__device__ __forceinline__ void warp_bitonic_sort(float* key, int64_t* id, int n) {
+  const int lane = threadIdx.x & 31;
+  for (int size = 2; size <= n; size <<= 1) {
+    for (int stride = size >> 1; stride > 0; stride >>= 1) {
+      __syncwarp();
+      for (int i = lane; i < (n >> 1); i += 32) {
+        const int lo = 2 * i - (i & (stride - 1));
+        const int hi = lo + stride;
+        const bool asc = (lo & size) == 0;
+        const float klo = key[lo], khi = key[hi];
+        const int64_t ilo = id[lo], ihi = id[hi];
+        const bool swap = asc ? better(khi, ihi, klo, ilo) : better(klo, ilo, khi, ihi);
+        if (swap) {
+          key[lo] = khi;
+          key[hi] = klo;
+          id[lo] = ihi;
+          id[hi] = ilo;
+        }
+      }
+    }
+  }
+  __syncwarp();
+}
+
+__global__ void __launch_bounds__(kRsWarps * 32, 1) rescore_mma_kernel(const __grid_constant__ RescoreArgs a) {
+  extern __shared__ __align__(128) uint8_t rsm[];
+  const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5, nw = blockDim.x >> 5;
+  const uint32_t dyn0 = uint32_t(__cvta_generic_to_shared(rsm));
+  uint8_t* table = rsm + (kBtTableAddr - dyn0);
+  if (dyn0 + uint32_t(a.warps_pre) * uint32_t(a.region) > kBtTableAddr) {
+    // the regions below the table would overlap it (more static shared
+    // memory than the host assumed): nothing is rescored
+    if (tid == 0) set_device_error(a.err, kErrSmemLayout);
+    return;
+  }
+  {
+    // the byte table: low half = level of the low nibble (the even code
+    // position), high half = level of the high nibble
+    uint32_t* tb = reinterpret_cast<uint32_t*>(table);
+    for (int e = tid; e < 256 * 32; e += blockDim.x) {
+      const int byte = e >> 5, ln = e & 31;
+      const uint32_t lo = __half_as_ushort(__float2half_rn(a.lv[byte & 15]));
+      const uint32_t hi = __half_as_ushort(__float2half_rn(a.lv[byte >> 4]));
+      tb[byte * 64 + ln] = lo | (hi << 16);
+    }
+  }
+  __syncthreads();
+  uint8_t* reg = warp < a.warps_pre ? rsm + size_t(warp) * a.region
+                                    : table + kBtTableBytes + size_t(warp - a.warps_pre) * a.region;
+  const int nj = (a.stride2 + 63) / 64;
+  int np2 = 2;
+  while (np2 < a.k) np2 <<= 1;
+  const uint8_t* qblk = reg;
+  float* key = reinterpret_cast<float*>(reg + size_t(nj) * 512);
+  int64_t* idv = reinterpret_cast<int64_t*>(key + np2);
+  const uint32_t tbl = kBtTableAddr | (uint32_t(lane) * 4u);
+  const int t = lane & 3, g = lane >> 2;
+  const int64_t nwt = int64_t(gridDim.x) * nw;
+  for (int64_t q = int64_t(blockIdx.x) * nw + warp; q < a.nq; q += nwt) {
+    // 2^s with max |q| 2^s in [1024, 2048)
+    const float* qr = a.qrot2 + q * a.Dp2;
+    float m = 0.0f;
+    for (int d = lane; d < a.Dp2; d += 32) m = fmaxf(m, fabsf(__ldg(qr + d)));
+#pragma unroll
+    for (int o = 16; o; o >>= 1) m = fmaxf(m, __shfl_xor_sync(kFull, m, o));
+    int ex = 0;
+    if (m > 0.0f) frexpf(m, &ex);
+    const float qsc = ldexpf(1.0f, 11 - ex), qinv = ldexpf(1.0f, ex - 11);
+    // the query block: entry (J, i, t) at 16 ((8 J + i) 4 + t) holds the hi
+    // halves, then the lo halves, of positions 128 J + 32 t + 4 i + {0..3}
+    for (int e = lane; e < nj * 32; e += 32) {
+      const int p = 128 * (e >> 5) + 32 * (e & 3) + 4 * ((e >> 2) & 7);
+      uint32_t h2[2], l2[2];
+#pragma unroll
+      for (int x = 0; x < 2; ++x) {
+        __half hh[2], ll[2];
+#pragma unroll
+        for (int y = 0; y < 2; ++y) {
+          const int d = p + 2 * x + y;
+          const float v = d < a.Dp2 ? __ldg(qr + d) * qsc : 0.0f;
+          hh[y] = __float2half_rn(v);
+          ll[y] = __float2half_rn(v - __half2float(hh[y]));
+        }
+        h2[x] = uint32_t(__half_as_ushort(hh[0])) | (uint32_t(__half_as_ushort(hh[1])) << 16);
+        l2[x] = uint32_t(__half_as_ushort(ll[0])) | (uint32_t(__half_as_ushort(ll[1])) << 16);
+      }
+      *reinterpret_cast<uint4*>(reg + size_t(e) * 16) = make_uint4(h2[0], h2[1], l2[0], l2[1]);
+    }
+    // the candidates: ids (LLONG_MAX: none) and <q, a2>
+    for (int j = lane; j < np2; j += 32) {
+      int64_t id = LLONG_MAX;
+      float s1 = -CUDART_INF_F;
+      if (j < a.k) {
+        const int64_t cid = a.cand_ids[q * a.k + j];
+        if (cid >= a.n_rows || cid < -1) set_device_error(a.err, kErrBadCandidate);
+        if (cid >= 0 && cid < a.n_rows) {
+          id = cid;
+          s1 = a.zero_a ? 0.0f : a.cand_scores[q * a.k + j];
+        }
+      }
+      idv[j] = id;
+      key[j] = s1;
+    }
+    __syncwarp();
+    // lane L holds the slot (-1: no candidate) and the scale word of row j0
+    // + L of the current pass, loaded while the previous pass is scored
+    auto slot_of = [&](int j) -> int64_t {
+      const int64_t id = j < a.k ? idv[j] : LLONG_MAX;
+      return id != LLONG_MAX ? int64_t(__ldg(a.slot_of_row + id)) : int64_t(-1);
+    };
+    int64_t slot_cur = slot_of(lane);
+    uint32_t sc_cur = slot_cur >= 0 ? __ldg(a.scales2 + slot_cur) : 0u;
+    for (int j0 = 0; j0 < a.k; j0 += 32) {
+      const int64_t slot_next = slot_of(j0 + 32 + lane);
+      uint32_t sc_next = 0u;
+      // this lane's rows j0 + g + 8 h (h = 0, 1: group 0; 2, 3: group 1),
+      // at its 16-byte column of each 64-byte segment
+      const uint8_t* rp[4];
+#pragma unroll
+      for (int h = 0; h < 4; ++h) {
+        const int64_t sl = __shfl_sync(kFull, slot_cur, g + 8 * h);
+        rp[h] = sl >= 0 ? a.codes2 + sl * a.stride2 + 16 * t : nullptr;
+      }
+      float d0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, e0[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      float d1[4] = {0.0f, 0.0f, 0.0f, 0.0f}, e1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+      uint4 w[4], wn[4];
+      auto load = [&](int J, uint4(&o)[4]) {
+        const bool in = 64 * J + 16 * t < a.stride2;  // rows are whole 16-byte columns
+#pragma unroll
+        for (int h = 0; h < 4; ++h)
+          o[h] = rp[h] != nullptr && in ? __ldg(reinterpret_cast<const uint4*>(rp[h] + 64 * J))
+                                        : make_uint4(0u, 0u, 0u, 0u);
+      };
+      load(0, w);
+      for (int J = 0; J < nj; ++J) {
+        if (J + 1 < nj) load(J + 1, wn);
+        if (J == 0 && slot_next >= 0) sc_next = __ldg(a.scales2 + slot_next);
+        uint32_t bq[8][2];
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          uint2 v = make_uint2(0u, 0u);
+          if (g < 2) v = *reinterpret_cast<const uint2*>(qblk + ((8 * J + i) * 4 + t) * 16 + 8 * g);
+          bq[i][0] = v.x;
+          bq[i][1] = v.y;
+        }
+        const uint32_t w0[4] = {w[0].x, w[0].y, w[0].z, w[0].w}, w1[4] = {w[1].x, w[1].y, w[1].z, w[1].w};
+        const uint32_t w2[4] = {w[2].x, w[2].y, w[2].z, w[2].w}, w3[4] = {w[3].x, w[3].y, w[3].z, w[3].w};
+        bt_group_mma(tbl, w0, w1, bq, d0, e0);
+        bt_group_mma(tbl, w2, w3, bq, d1, e1);
+#pragma unroll
+        for (int h = 0; h < 4; ++h) w[h] = wn[h];
+      }
+      // lanes t = 0 hold (hi, lo) of rows g, g + 8 (group 0) and g + 16,
+      // g + 24 (group 1); lane L takes row j0 + L
+      const float r0 = (d0[0] + e0[0]) + (d0[1] + e0[1]), r1 = (d0[2] + e0[2]) + (d0[3] + e0[3]);
+      const float r2 = (d1[0] + e1[0]) + (d1[1] + e1[1]), r3 = (d1[2] + e1[2]) + (d1[3] + e1[3]);
+      const int src = 4 * (lane & 7), part = lane >> 3;
+      const float x0 = __shfl_sync(kFull, r0, src), x1 = __shfl_sync(kFull, r1, src);
+      const float x2 = __shfl_sync(kFull, r2, src), x3 = __shfl_sync(kFull, r3, src);
+      const float dot = part == 0 ? x0 : part == 1 ? x1 : part == 2 ? x2 : x3;
+      const int j = j0 + lane;
+      if (slot_cur >= 0)
+        key[j] = ue4m12_to_f32(sc_cur >> 16) * fmaf(ue7m9_to_f32(sc_cur & 0xffffu), dot * qinv, key[j]);
+      slot_cur = slot_next;
+      sc_cur = sc_next;
+    }
+    warp_bitonic_sort(key, idv, np2);
+    for (int e = lane; e < a.kf; e += 32) {
+      const bool ok = idv[e] != LLONG_MAX;
+      a.out_ids[q * a.kf + e] = ok ? idv[e] : -1;
+      a.out_scores[q * a.kf + e] = ok ? key[e] : -CUDART_INF_F;
+    }
+    __syncwarp();  // the region is read before the next query's stores
+  }
+}
 template <int CH, bool B3>
 cudaError_t launch_scan_ch(const rslm_index* ix, const ScanArgs& a, int64_t nq, size_t smem,
                            cudaStream_t s) {
@@ -1391,6 +1601,33 @@ cudaError_t launch_rescore(const rslm_index* ix, const float* qrot2, int64_t nq,
   a.out_ids = out_ids;
   a.out_scores = out_scores;
   a.err = ix->d_err;
+  if (a.crot2 == nullptr && ix->cs2.g == 1 && ix->cs2.stride % 16 == 0 && k <= 256) {
+    // the tensor-core kernel: per-warp regions below and above the byte table
+    int np2m = 2;
+    while (np2m < k) np2m <<= 1;
+    const size_t region =
+        (size_t((ix->cs2.stride + 63) / 64) * 512 + size_t(np2m) * 12 + 15) & ~size_t(15);
+    int dev = 0, optin = 0, sms = 0;
+    cudaError_t e = cudaGetDevice(&dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+    if (e == cudaSuccess) e = cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+    if (e != cudaSuccess) return e;
+    const int pre = int(std::min<size_t>(kRsWarps, (kBtTableAddr - kBtLowReserve) / region));
+    const long above = long(optin) - long(kBtLowReserve) - long(kBtTableAddr) - long(kBtTableBytes);
+    const int post = above > 0 ? int(std::min<long>(kRsWarps - pre, above / long(region))) : 0;
+    const int nw = pre + post;
+    if (nw >= 4) {
+      a.nq = nq;
+      a.warps_pre = pre;
+      a.region = int(region);
+      const size_t bytes = size_t(kBtTableAddr) + size_t(kBtTableBytes) + size_t(post) * region;
+      e = cudaFuncSetAttribute(rescore_mma_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, int(bytes));
+      if (e != cudaSuccess) return e;
+      const int64_t grid = std::min<int64_t>(sms, (nq + nw - 1) / nw);
+      rescore_mma_kernel<<<unsigned(grid), unsigned(nw * 32), bytes, s>>>(a);
+      return cudaGetLastError();
+    }
+  }
   int np2 = 1;
   while (np2 < k) np2 <<= 1;
   const size_t smem = ((size_t(2 * a.stride2 + np2) * 4 + 15) & ~size_t(15)) + size_t(np2) * 8;

@@ -503,6 +503,42 @@ def test_rescore_parity_on_oracle_codes(case):
         assert not probs, (i, probs[:3])
 
 
+# (case, stage-1 k, k_final, share of candidate slots set to -1): the
+# largest k, a ragged k returned whole, holes in the lists, D = 1536
+RESCORE_PATHS = {
+    "k256": ("C2s", 256, 10, 0.0),
+    "ragged_all": ("C2s", 45, 45, 0.0),
+    "holes": ("C2s", 100, 10, 0.3),
+    "D1536_holes": ("C5s", 200, 20, 0.1),
+}
+
+
+@pytest.mark.parametrize("name", sorted(RESCORE_PATHS))
+def test_rescore_paths(name):
+    cname, k, kf, holes = RESCORE_PATHS[name]
+    case = Case(CASES[cname])
+    w = case.w
+    ix = case.gpu_index(encode=False)
+    case.import_oracle_codes(ix)
+    res = search.search(case.oracle, case.Q, w.nprobe, k, kf)
+    s1_ids, s1_sc = res["s1_ids"].copy(), res["s1_scores"].copy()
+    if holes:
+        s1_ids[np.random.default_rng(11).random(s1_ids.shape) < holes] = -1
+    q2 = ix.rotate(torch.from_numpy(case.Q).cuda(), which=2)
+    ids, sc = ix.rescore(q2, torch.from_numpy(s1_ids).cuda(), torch.from_numpy(s1_sc.astype(np.float32)).cuda(), kf)
+    ix.sync()
+    ids, sc = ids.cpu().numpy(), sc.cpu().numpy()
+    assert ids.shape == (len(case.Q), kf)
+    for i in range(len(case.Q)):
+        _, _, s2 = search.rescore(case.oracle, case.Q[i], s1_ids[i], s1_sc[i], k)
+        cid = s1_ids[i][s1_ids[i] >= 0]
+        ref = dict(zip(cid.tolist(), s2.tolist()))
+        kth, kid = kth_of(ref, kf)
+        probs = check_topk(ids[i], sc[i], lambda j: ref[j], kth, case.score_tol_of(i), allowed_ids=ref,
+                           kth_id=kid)
+        assert not probs, (i, probs[:3])
+
+
 def _end_to_end(case, ix, code_ok=None):
     w = case.w
     Qt = torch.from_numpy(case.Q).cuda()
