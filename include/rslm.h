@@ -317,7 +317,9 @@ rslm_status rslm_sync(const rslm_index* index, void* stream);
  *          the threshold); also answered by the exact scan (expected, rare);
  *   out[2] queries whose fused-probe candidate list overflowed (many
  *          centroid scores tied at the bound); answered by the exact probe;
- *   out[3] reserved, 0.
+ *   out[3] rows whose exact score the tensor-core scan's hi-only mode
+ *          recomputed after its bounded pass (the candidates whose upper
+ *          bound reached the k-th largest lower bound; a cost figure).
  * RSLM_ERR_INVALID_ARG for a NULL argument or n outside [1, 4]. */
 rslm_status rslm_counters(const rslm_index* index, int64_t* out, int32_t n);
 

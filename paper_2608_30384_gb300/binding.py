@@ -303,7 +303,7 @@ def rslm_sync(index, stream=None):
     _check(lib().rslm_sync(_ptr(index), _stream(stream)))
 
 
-COUNTERS = ("batched_short_rescans", "batched_overflow_rescans", "probe_exact_fallbacks")
+COUNTERS = ("batched_short_rescans", "batched_overflow_rescans", "probe_exact_fallbacks", "hi_exact_rescores")
 
 
 def rslm_counters(index) -> dict:

@@ -355,22 +355,23 @@ __device__ __forceinline__ uint32_t tile_off(int row, int k8) {
 // The same computation for a single K chunk (padded D <= 128), as one
 // persistent CTA per SM whose warps each take one stage, overlapped across
 // the 128-row tiles of an item and across items:
-//   warps 18-19 load: fetch the next item (partition, up to 128 of its
+//   warps 22-23 load: fetch the next item (partition, up to 128 of its
 //              queries) and stage its per-query epilogue constants and its B
 //              operands (the queries' fp16 hi / lo parts in the no-swizzle
 //              K-major layout) into one of two item slots while the other
 //              slot's item computes;
-//   warp 17    lane 0 streams each tile's codes (one contiguous slab of the
+//   warp 21    lane 0 streams each tile's codes (one contiguous slab of the
 //              tile-interleaved layout) and its scales by TMA into rings
 //              of kSlabs and kScaleStages buffers;
-//   warps 0-7  decode: thread = (row, half of the row's columns); take the
-//              tile's codes from the slab, decode them through a 16-entry
-//              table and store them into one of two A operands in TMEM
-//              (tcgen05.st; lane = row, two halves per 32-bit column);
-//   warp 16    lane 0 issues the MMAs (A from TMEM, B hi / lo from the item
+//   warps 0-3  decode: thread = row; take the row's codes from the slab,
+//              decode them through the per-lane byte table (or the code
+//              tables of the other formats) and store them into one of two
+//              A operands in TMEM (tcgen05.st; lane = row, two halves per
+//              32-bit column);
+//   warp 20    lane 0 issues the MMAs (A from TMEM, B hi / lo from the item
 //              slot, N = the item's query count rounded up to 16) into one
-//              of two TMEM accumulators;
-//   warps 8-15 epilogue: thread = (row, half of the query columns); read its
+//              of three TMEM accumulators;
+//   warps 4-19 epilogue: thread = (row, 32 of the query columns); read its
 //              accumulator part, apply s = G (cs + L dot) and append the
 //              candidates with s >= theta_q.
 // A warp reaches only its TMEM lane quadrant (warp index mod 4), so the
@@ -1866,6 +1867,7 @@ struct FinHiArgs {
   int stride, chunk, g;
   int npos;  // coordinates covered by a row's codes: 2 g stride
   int fcap;  // candidates per query in shared memory (a power of two >= 512)
+  int tbl;   // block kernel: score window rows through the per-query code table
   float cb[64];
   int* ovf_list;
   int* counts;
@@ -1876,8 +1878,10 @@ struct FinHiArgs {
 __host__ __device__ constexpr size_t fin_hi_warp_bytes(int fcap, int npos) {
   return size_t(fcap) * 12 + 256 * 4 + size_t(npos) * 4;  // window, radix histogram, r
 }
-__host__ __device__ constexpr size_t fin_hi_block_bytes(int fcap, int npos) {
-  return 256 + size_t(fcap) * 12 + 256 * 4 + size_t(npos) * 4;  // codebook, window, radix histogram, r
+// codebook, window, radix histogram, then r (npos floats) or the code table
+// (npos / g groups x 16 codes)
+__host__ __device__ constexpr size_t fin_hi_block_bytes(int fcap, int npos, int g, bool tbl) {
+  return 256 + size_t(fcap) * 12 + 256 * 4 + (tbl ? size_t(npos / g) * 64 : size_t(npos) * 4);
 }
 
 // <r, uhat> of the row at slot pos (r in shared memory, codebook cb:
@@ -1899,30 +1903,34 @@ __device__ __forceinline__ float fin_row_dot(const FinHiArgs& a, int32_t pos, co
   const int CH = a.chunk;
   float dot = 0.0f;
   if (CH == 16) {
+    // eight 16-byte loads in flight, four partial sums
     const int nch = a.stride / 16;
+    float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
     int c = 0;
-    for (; c + 4 <= nch; c += 4) {  // four 16-byte loads in flight
-      uint4 wv[4];
+    for (; c + 8 <= nch; c += 8) {
+      uint4 wv[8];
 #pragma unroll
-      for (int u = 0; u < 4; ++u) wv[u] = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c + u) * kMR + r) * 16));
+      for (int u = 0; u < 8; ++u) wv[u] = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c + u) * kMR + r) * 16));
 #pragma unroll
-      for (int u = 0; u < 4; ++u) {
+      for (int u = 0; u < 8; ++u) {
         const float* rv = rq + G * 32 * (c + u);
-        dot = fin_word_dot<G>(wv[u].x, rv, cb, dot);
-        dot = fin_word_dot<G>(wv[u].y, rv + 8 * G, cb, dot);
-        dot = fin_word_dot<G>(wv[u].z, rv + 16 * G, cb, dot);
-        dot = fin_word_dot<G>(wv[u].w, rv + 24 * G, cb, dot);
+        float& d = acc[u & 3];
+        d = fin_word_dot<G>(wv[u].x, rv, cb, d);
+        d = fin_word_dot<G>(wv[u].y, rv + 8 * G, cb, d);
+        d = fin_word_dot<G>(wv[u].z, rv + 16 * G, cb, d);
+        d = fin_word_dot<G>(wv[u].w, rv + 24 * G, cb, d);
       }
     }
     for (; c < nch; ++c) {
       const uint4 wv = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c) * kMR + r) * 16));
       const float* rv = rq + G * 32 * c;
-      dot = fin_word_dot<G>(wv.x, rv, cb, dot);
-      dot = fin_word_dot<G>(wv.y, rv + 8 * G, cb, dot);
-      dot = fin_word_dot<G>(wv.z, rv + 16 * G, cb, dot);
-      dot = fin_word_dot<G>(wv.w, rv + 24 * G, cb, dot);
+      float& d = acc[c & 3];
+      d = fin_word_dot<G>(wv.x, rv, cb, d);
+      d = fin_word_dot<G>(wv.y, rv + 8 * G, cb, d);
+      d = fin_word_dot<G>(wv.z, rv + 16 * G, cb, d);
+      d = fin_word_dot<G>(wv.w, rv + 24 * G, cb, d);
     }
-    return dot;
+    return (acc[0] + acc[1]) + (acc[2] + acc[3]) + dot;
   }
   for (int c = 0; c < a.stride / CH; ++c) {
     const uint8_t* chp = tile + (size_t(c) * kMR + r) * CH;
@@ -1931,6 +1939,53 @@ __device__ __forceinline__ float fin_row_dot(const FinHiArgs& a, int32_t pos, co
                             dot);
   }
   return dot;
+}
+
+// <r, uhat> of the row at slot pos through the query's code table T:
+// T[16 i + c] = <r restricted to group i, codeword c>, so a code costs one
+// shared load and one add (four partial sums, eight 16-byte loads in
+// flight for 16-byte chunks).
+__device__ __forceinline__ float fin_row_dot_t(const FinHiArgs& a, int32_t pos, const float* T) {
+  const int r = pos & (kMR - 1);
+  const uint8_t* tile = a.codes + int64_t(pos - r) * a.stride;
+  const int CH = a.chunk;
+  float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
+  auto word = [&](uint32_t wd, int gi, float& d) {  // gi: group of the word's first code
+#pragma unroll
+    for (int nb = 0; nb < 8; ++nb) d += T[((gi + nb) << 4) | ((wd >> (4 * nb)) & 15u)];
+  };
+  if (CH == 16) {
+    const int nch = a.stride / 16;
+    int c = 0;
+    for (; c + 8 <= nch; c += 8) {
+      uint4 wv[8];
+#pragma unroll
+      for (int u = 0; u < 8; ++u) wv[u] = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c + u) * kMR + r) * 16));
+#pragma unroll
+      for (int u = 0; u < 8; ++u) {
+        const int gi = 32 * (c + u);
+        word(wv[u].x, gi, acc[u & 3]);
+        word(wv[u].y, gi + 8, acc[u & 3]);
+        word(wv[u].z, gi + 16, acc[u & 3]);
+        word(wv[u].w, gi + 24, acc[u & 3]);
+      }
+    }
+    for (; c < nch; ++c) {
+      const uint4 wv = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c) * kMR + r) * 16));
+      const int gi = 32 * c;
+      word(wv.x, gi, acc[c & 3]);
+      word(wv.y, gi + 8, acc[c & 3]);
+      word(wv.z, gi + 16, acc[c & 3]);
+      word(wv.w, gi + 24, acc[c & 3]);
+    }
+  } else {
+    for (int c = 0; c < a.stride / CH; ++c) {
+      const uint8_t* chp = tile + (size_t(c) * kMR + r) * CH;
+      for (int w = 0; w < CH / 4; ++w)
+        word(__ldg(reinterpret_cast<const uint32_t*>(chp) + w), 2 * (c * CH + 4 * w), acc[w & 3]);
+    }
+  }
+  return (acc[0] + acc[1]) + (acc[2] + acc[3]);
 }
 
 // The k-th largest order key of s[0 .. n) (n > k) by one warp: four 8-bit
@@ -2060,6 +2115,7 @@ __global__ void __launch_bounds__(128) finalize_hi_warp_kernel(const __grid_cons
     }
     return;
   }
+  if (lane == 0) atomicAdd(&a.ctr[kCtrHiExact], (unsigned long long)mcnt);
   __syncwarp();
   int p2 = 1;
   while (p2 < mcnt || p2 < k) p2 <<= 1;
@@ -2095,7 +2151,7 @@ __global__ void __launch_bounds__(128) finalize_hi_warp_kernel(const __grid_cons
 // One block of kFinHiThreads per query (grid-strided): the remainder r and
 // the window live in the block's shared memory; a block radix select finds
 // T, every thread scores window rows, and a block sort orders them.
-constexpr int kFinHiThreads = 128;
+constexpr int kFinHiThreads = 256;
 template <int G>
 __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const __grid_constant__ FinHiArgs a) {
   extern __shared__ __align__(16) uint8_t fsm_hi[];
@@ -2104,7 +2160,7 @@ __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const 
   int64_t* fi = reinterpret_cast<int64_t*>(fsm_hi + 256);        // fcap ids
   uint32_t* fk = reinterpret_cast<uint32_t*>(fi + fcap);         // fcap keys
   uint32_t* hist = fk + fcap;                                    // 256 bins
-  float* rq = reinterpret_cast<float*>(hist + 256);              // npos
+  float* rq = reinterpret_cast<float*>(hist + 256);              // npos (r), or the code table
   __shared__ int sh_m;
   __shared__ float sh_max[kFinHiThreads / 32];
   __shared__ uint32_t sh_sel[2];
@@ -2137,13 +2193,39 @@ __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const 
     int e2 = 0;
     if (m > 0.0f) frexpf(m, &e2);
     const float sc = ldexpf(1.0f, 11 - e2), inv = ldexpf(1.0f, e2 - 11);
-    for (int d = tid; d < a.npos; d += kFinHiThreads) {
-      const float v = d < a.Dp ? src[d] * sc : 0.0f;
-      rq[d] = v - __half2float(__float2half_rn(v));
+    if (a.tbl) {
+      // the code table: group gi's remainder r_gi against each codeword
+      for (int gi = tid; gi < a.npos / G; gi += kFinHiThreads) {
+        float rv[G];
+#pragma unroll
+        for (int j = 0; j < G; ++j) {
+          const int d = G * gi + j;
+          const float v = d < a.Dp ? src[d] * sc : 0.0f;
+          rv[j] = v - __half2float(__float2half_rn(v));
+        }
+        float4* tg = reinterpret_cast<float4*>(rq + 16 * gi);
+#pragma unroll
+        for (int c4 = 0; c4 < 4; ++c4) {
+          float e[4];
+#pragma unroll
+          for (int x = 0; x < 4; ++x) {
+            float t = 0.0f;
+#pragma unroll
+            for (int j = 0; j < G; ++j) t = fmaf(cbs[G * (4 * c4 + x) + j], rv[j], t);
+            e[x] = t;
+          }
+          tg[c4] = make_float4(e[0], e[1], e[2], e[3]);
+        }
+      }
+    } else {
+      for (int d = tid; d < a.npos; d += kFinHiThreads) {
+        const float v = d < a.Dp ? src[d] * sc : 0.0f;
+        rq[d] = v - __half2float(__float2half_rn(v));
+      }
     }
     // T: the k-th largest lower bound (all candidates when n <= k)
     const uint32_t T = n > k ? block_kth_key(a.buf_l + q * a.cap, n, k, hist, sh_sel) : 0u;
-    __syncthreads();  // r is written
+    __syncthreads();  // r or the code table is written
     // the margin the MMAs added
     const float hu = a.fold ? fold_margin(a.qrho[q]) : __half2float(__float2half_ru(a.qrho[q]));
     const float* su = a.buf_s + q * a.cap;
@@ -2154,7 +2236,7 @@ __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const 
       const int at = atomicAdd(&sh_m, 1);
       if (at >= fcap) continue;
       const int32_t pos = pp[i];
-      const float dot = fin_row_dot<G>(a, pos, rq, cbs);
+      const float dot = a.tbl ? fin_row_dot_t(a, pos, rq) : fin_row_dot<G>(a, pos, rq, cbs);
       const uint32_t swd = __ldg(a.scales + pos);
       const float Gs = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
       fk[at] = float_order_key(su[i] + Gs * L * (dot - hu) * inv);
@@ -2169,6 +2251,7 @@ __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const 
       }
       continue;
     }
+    if (tid == 0) atomicAdd(&a.ctr[kCtrHiExact], (unsigned long long)mcnt);
     int p2 = 1;
     while (p2 < mcnt || p2 < k) p2 <<= 1;
     for (int i = mcnt + tid; i < p2; i += kFinHiThreads) {
@@ -2471,8 +2554,14 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
         using FK = void (*)(FinHiArgs);
         const bool per_warp = fa.npos <= 256;
         const int fw = 4;  // warps (queries) per block of the per-warp kernel
+        int dev = 0, sms = 152, optin = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess) {
+          cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev);
+          cudaDeviceGetAttribute(&optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev);
+        }
+        fa.tbl = fin_hi_block_bytes(fcap, fa.npos, c1.g, true) <= size_t(optin) / 2 ? 1 : 0;
         const size_t fsm = per_warp ? 256 + size_t(fw) * fin_hi_warp_bytes(fcap, fa.npos)
-                                    : fin_hi_block_bytes(fcap, fa.npos);
+                                    : fin_hi_block_bytes(fcap, fa.npos, c1.g, fa.tbl != 0);
         const FK fk = per_warp ? (c1.g == 1   ? finalize_hi_warp_kernel<1>
                                   : c1.g == 2 ? finalize_hi_warp_kernel<2>
                                               : finalize_hi_warp_kernel<4>)
@@ -2483,8 +2572,14 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
         if (e == cudaSuccess) {
           if (per_warp)
             fk<<<unsigned((nq + fw - 1) / fw), fw * 32, fsm, s>>>(fa);
-          else
-            fk<<<unsigned(std::min<int64_t>(nq, 152 * 16)), kFinHiThreads, fsm, s>>>(fa);
+          else {
+            // as many blocks as stay resident (each strides over the queries)
+            int per_sm = 1;
+            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fk, kFinHiThreads, fsm) != cudaSuccess ||
+                per_sm < 1)
+              per_sm = 1;
+            fk<<<unsigned(std::min<int64_t>(nq, int64_t(sms) * per_sm)), kFinHiThreads, fsm, s>>>(fa);
+          }
           e = cudaGetLastError();
         }
       } else if (e == cudaSuccess) {

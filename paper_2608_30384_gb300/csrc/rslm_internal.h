@@ -20,11 +20,12 @@ constexpr int kMaxNprobe = 4096;
 constexpr int kBatchMinQueries = 16;  // rslm_search: batched scan above this queries/partition
 
 // Event counters of an index (rslm_counters): queries that a search path
-// handed to an exact fallback.
+// handed to an exact fallback, and the hi-only finalize's exact rescores.
 enum Counter : int {
   kCtrBatchedShort = 0,     // pass 2 kept fewer than k candidates under a finite threshold
   kCtrBatchedOverflow = 1,  // the pass-2 candidate buffer overflowed
   kCtrProbeExact = 2,       // a fused-probe candidate list overflowed
+  kCtrHiExact = 3,          // rows whose exact score the hi-only finalize recomputed
   kNumCounters = 4,
 };
 

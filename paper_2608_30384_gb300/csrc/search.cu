@@ -1304,24 +1304,15 @@ __global__ void __launch_bounds__(kRsWarps * 32, 1) rescore_mma_kernel(const __g
       key[j] = s1;
     }
     __syncwarp();
-    // lane L holds the slot (-1: no candidate) and the scale word of row j0
-    // + L of the current pass, loaded while the previous pass is scored
-    auto slot_of = [&](int j) -> int64_t {
-      const int64_t id = j < a.k ? idv[j] : LLONG_MAX;
-      return id != LLONG_MAX ? int64_t(__ldg(a.slot_of_row + id)) : int64_t(-1);
-    };
-    int64_t slot_cur = slot_of(lane);
-    uint32_t sc_cur = slot_cur >= 0 ? __ldg(a.scales2 + slot_cur) : 0u;
     for (int j0 = 0; j0 < a.k; j0 += 32) {
-      const int64_t slot_next = slot_of(j0 + 32 + lane);
-      uint32_t sc_next = 0u;
       // this lane's rows j0 + g + 8 h (h = 0, 1: group 0; 2, 3: group 1),
       // at its 16-byte column of each 64-byte segment
       const uint8_t* rp[4];
 #pragma unroll
       for (int h = 0; h < 4; ++h) {
-        const int64_t sl = __shfl_sync(kFull, slot_cur, g + 8 * h);
-        rp[h] = sl >= 0 ? a.codes2 + sl * a.stride2 + 16 * t : nullptr;
+        const int j = j0 + g + 8 * h;
+        const int64_t id = j < a.k ? idv[j] : LLONG_MAX;
+        rp[h] = id != LLONG_MAX ? a.codes2 + int64_t(__ldg(a.slot_of_row + id)) * a.stride2 + 16 * t : nullptr;
       }
       float d0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, e0[4] = {0.0f, 0.0f, 0.0f, 0.0f};
       float d1[4] = {0.0f, 0.0f, 0.0f, 0.0f}, e1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
@@ -1336,7 +1327,6 @@ __global__ void __launch_bounds__(kRsWarps * 32, 1) rescore_mma_kernel(const __g
       load(0, w);
       for (int J = 0; J < nj; ++J) {
         if (J + 1 < nj) load(J + 1, wn);
-        if (J == 0 && slot_next >= 0) sc_next = __ldg(a.scales2 + slot_next);
         uint32_t bq[8][2];
 #pragma unroll
         for (int i = 0; i < 8; ++i) {
@@ -1361,10 +1351,10 @@ __global__ void __launch_bounds__(kRsWarps * 32, 1) rescore_mma_kernel(const __g
       const float x2 = __shfl_sync(kFull, r2, src), x3 = __shfl_sync(kFull, r3, src);
       const float dot = part == 0 ? x0 : part == 1 ? x1 : part == 2 ? x2 : x3;
       const int j = j0 + lane;
-      if (slot_cur >= 0)
-        key[j] = ue4m12_to_f32(sc_cur >> 16) * fmaf(ue7m9_to_f32(sc_cur & 0xffffu), dot * qinv, key[j]);
-      slot_cur = slot_next;
-      sc_cur = sc_next;
+      if (j < a.k && idv[j] != LLONG_MAX) {
+        const uint32_t sc = __ldg(a.scales2 + __ldg(a.slot_of_row + idv[j]));
+        key[j] = ue4m12_to_f32(sc >> 16) * fmaf(ue7m9_to_f32(sc & 0xffffu), dot * qinv, key[j]);
+      }
     }
     warp_bitonic_sort(key, idv, np2);
     for (int e = lane; e < a.kf; e += 32) {
