@@ -1868,6 +1868,8 @@ struct FinHiArgs {
   int npos;  // coordinates covered by a row's codes: 2 g stride
   int fcap;  // candidates per query in shared memory (a power of two >= 512)
   int tbl;   // block kernel: score window rows through the per-query code table
+  uint32_t* tq;  // block kernel: T per query (finalize_hi_select_kernel)
+  uint32_t zero;  // 0: makes the table lookups depend on a row's loads (all issued first)
   float cb[64];
   int* ovf_list;
   int* counts;
@@ -1878,10 +1880,10 @@ struct FinHiArgs {
 __host__ __device__ constexpr size_t fin_hi_warp_bytes(int fcap, int npos) {
   return size_t(fcap) * 12 + 256 * 4 + size_t(npos) * 4;  // window, radix histogram, r
 }
-// codebook, window, radix histogram, then r (npos floats) or the code table
-// (npos / g groups x 16 codes)
+// codebook, window (ids, keys, candidate indices), then r (npos floats) or
+// the code table (npos / g groups x 16 codes)
 __host__ __device__ constexpr size_t fin_hi_block_bytes(int fcap, int npos, int g, bool tbl) {
-  return 256 + size_t(fcap) * 12 + 256 * 4 + (tbl ? size_t(npos / g) * 64 : size_t(npos) * 4);
+  return 256 + size_t(fcap) * 16 + (tbl ? size_t(npos / g) * 64 : size_t(npos) * 4);
 }
 
 // <r, uhat> of the row at slot pos (r in shared memory, codebook cb:
@@ -1950,9 +1952,9 @@ __device__ __forceinline__ float fin_row_dot_t(const FinHiArgs& a, int32_t pos, 
   const uint8_t* tile = a.codes + int64_t(pos - r) * a.stride;
   const int CH = a.chunk;
   float acc[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-  auto word = [&](uint32_t wd, int gi, float& d) {  // gi: group of the word's first code
+  auto word = [&](const float* Tw, uint32_t wd, int gi, float& d) {  // gi: group of the word's first code
 #pragma unroll
-    for (int nb = 0; nb < 8; ++nb) d += T[((gi + nb) << 4) | ((wd >> (4 * nb)) & 15u)];
+    for (int nb = 0; nb < 8; ++nb) d += Tw[((gi + nb) << 4) | ((wd >> (4 * nb)) & 15u)];
   };
   if (CH == 16) {
     const int nch = a.stride / 16;
@@ -1961,28 +1963,34 @@ __device__ __forceinline__ float fin_row_dot_t(const FinHiArgs& a, int32_t pos, 
       uint4 wv[8];
 #pragma unroll
       for (int u = 0; u < 8; ++u) wv[u] = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c + u) * kMR + r) * 16));
+      // the lookups' base depends on every word (a.zero = 0), so the eight
+      // loads are all issued before the first lookup
+      uint32_t dep = 0u;
+#pragma unroll
+      for (int u = 0; u < 8; ++u) dep |= wv[u].x | wv[u].y | wv[u].z | wv[u].w;
+      const float* Tb = T + (dep & a.zero);
 #pragma unroll
       for (int u = 0; u < 8; ++u) {
         const int gi = 32 * (c + u);
-        word(wv[u].x, gi, acc[u & 3]);
-        word(wv[u].y, gi + 8, acc[u & 3]);
-        word(wv[u].z, gi + 16, acc[u & 3]);
-        word(wv[u].w, gi + 24, acc[u & 3]);
+        word(Tb, wv[u].x, gi, acc[u & 3]);
+        word(Tb, wv[u].y, gi + 8, acc[u & 3]);
+        word(Tb, wv[u].z, gi + 16, acc[u & 3]);
+        word(Tb, wv[u].w, gi + 24, acc[u & 3]);
       }
     }
     for (; c < nch; ++c) {
       const uint4 wv = __ldg(reinterpret_cast<const uint4*>(tile + (size_t(c) * kMR + r) * 16));
       const int gi = 32 * c;
-      word(wv.x, gi, acc[c & 3]);
-      word(wv.y, gi + 8, acc[c & 3]);
-      word(wv.z, gi + 16, acc[c & 3]);
-      word(wv.w, gi + 24, acc[c & 3]);
+      word(T, wv.x, gi, acc[c & 3]);
+      word(T, wv.y, gi + 8, acc[c & 3]);
+      word(T, wv.z, gi + 16, acc[c & 3]);
+      word(T, wv.w, gi + 24, acc[c & 3]);
     }
   } else {
     for (int c = 0; c < a.stride / CH; ++c) {
       const uint8_t* chp = tile + (size_t(c) * kMR + r) * CH;
       for (int w = 0; w < CH / 4; ++w)
-        word(__ldg(reinterpret_cast<const uint32_t*>(chp) + w), 2 * (c * CH + 4 * w), acc[w & 3]);
+        word(T, __ldg(reinterpret_cast<const uint32_t*>(chp) + w), 2 * (c * CH + 4 * w), acc[w & 3]);
     }
   }
   return (acc[0] + acc[1]) + (acc[2] + acc[3]);
@@ -2148,9 +2156,31 @@ __global__ void __launch_bounds__(128) finalize_hi_warp_kernel(const __grid_cons
   }
 }
 
-// One block of kFinHiThreads per query (grid-strided): the remainder r and
-// the window live in the block's shared memory; a block radix select finds
-// T, every thread scores window rows, and a block sort orders them.
+// T per query by one warp (a radix select over the candidates' lower
+// bounds), then one block of kFinHiThreads per query (grid-strided): the
+// remainder r (or its code table) and the window live in the block's shared
+// memory, every thread scores window rows, and each row's rank among them
+// is its place in the result.
+constexpr uint32_t kFinSkip = 0xffffffffu;  // T of a query listed for the exact re-scan
+__global__ void __launch_bounds__(128) finalize_hi_select_kernel(const __grid_constant__ FinHiArgs a) {
+  __shared__ uint32_t hist[4][256];
+  const int lane = threadIdx.x & 31, w = threadIdx.x >> 5;
+  const int64_t q = int64_t(blockIdx.x) * 4 + w;
+  if (q >= a.nq) return;
+  const int n = a.cnt[q], k = a.k;
+  const bool short_list = n < k && a.theta[q] > -CUDART_INF_F;
+  if (n > a.cap || short_list) {
+    if (lane == 0) {
+      a.ovf_list[atomicAdd(&a.counts[0], 1)] = int(q);
+      atomicAdd(&a.ctr[short_list ? kCtrBatchedShort : kCtrBatchedOverflow], 1ull);
+      a.tq[q] = kFinSkip;
+    }
+    return;
+  }
+  const uint32_t T = n > k ? warp_kth_key(a.buf_l + q * a.cap, n, k, hist[w]) : 0u;
+  if (lane == 0) a.tq[q] = T;
+}
+
 constexpr int kFinHiThreads = 256;
 template <int G>
 __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const __grid_constant__ FinHiArgs a) {
@@ -2159,25 +2189,20 @@ __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const 
   float* cbs = reinterpret_cast<float*>(fsm_hi);                 // 64 floats
   int64_t* fi = reinterpret_cast<int64_t*>(fsm_hi + 256);        // fcap ids
   uint32_t* fk = reinterpret_cast<uint32_t*>(fi + fcap);         // fcap keys
-  uint32_t* hist = fk + fcap;                                    // 256 bins
-  float* rq = reinterpret_cast<float*>(hist + 256);              // npos (r), or the code table
+  int* wl = reinterpret_cast<int*>(fk + fcap);                   // fcap window indices
+  float* rq = reinterpret_cast<float*>(wl + fcap);               // npos (r), or the code table
   __shared__ int sh_m;
   __shared__ float sh_max[kFinHiThreads / 32];
-  __shared__ uint32_t sh_sel[2];
   const int tid = threadIdx.x, lane = tid & 31, w = tid >> 5;
   if (tid < 64) cbs[tid] = a.cb[tid];
   const int k = a.k;
   for (int64_t q = blockIdx.x; q < a.nq; q += gridDim.x) {
     __syncthreads();  // the previous query's buffers are read
+    // T (finalize_hi_select_kernel): the k-th largest lower bound, 0 when
+    // n <= k, kFinSkip for a query already listed for the exact re-scan
+    const uint32_t T = a.tq[q];
+    if (T == kFinSkip) continue;
     const int n = a.cnt[q];
-    const bool short_list = n < k && a.theta[q] > -CUDART_INF_F;
-    if (n > a.cap || short_list) {
-      if (tid == 0) {
-        a.ovf_list[atomicAdd(&a.counts[0], 1)] = int(q);
-        atomicAdd(&a.ctr[short_list ? kCtrBatchedShort : kCtrBatchedOverflow], 1ull);
-      }
-      continue;
-    }
     // the query's scaling 2^s (max |q| 2^s in [1024, 2048)) and remainder r
     const float* src = a.qrot + q * a.Dp;
     float m = 0.0f;
@@ -2223,24 +2248,28 @@ __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const 
         rq[d] = v - __half2float(__float2half_rn(v));
       }
     }
-    // T: the k-th largest lower bound (all candidates when n <= k)
-    const uint32_t T = n > k ? block_kth_key(a.buf_l + q * a.cap, n, k, hist, sh_sel) : 0u;
     __syncthreads();  // r or the code table is written
     // the margin the MMAs added
     const float hu = a.fold ? fold_margin(a.qrho[q]) : __half2float(__float2half_ru(a.qrho[q]));
     const float* su = a.buf_s + q * a.cap;
     const int32_t* pp = a.buf_p + q * a.cap;
-    // the candidates that can be in the top k, with their exact scores
-    for (int i = tid; i < n; i += kFinHiThreads) {
-      if (float_order_key(su[i]) < T) continue;
-      const int at = atomicAdd(&sh_m, 1);
-      if (at >= fcap) continue;
-      const int32_t pos = pp[i];
-      const float dot = a.tbl ? fin_row_dot_t(a, pos, rq) : fin_row_dot<G>(a, pos, rq, cbs);
-      const uint32_t swd = __ldg(a.scales + pos);
-      const float Gs = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
-      fk[at] = float_order_key(su[i] + Gs * L * (dot - hu) * inv);
-      fi[at] = a.ids[pos];
+    // the window: the candidates that can be in the top k (upper bound >= T),
+    // listed with four loads in flight per thread
+    for (int i0 = tid; i0 < n; i0 += 4 * kFinHiThreads) {
+      float sv[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * kFinHiThreads;
+        sv[u] = i < n ? su[i] : 0.0f;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = i0 + u * kFinHiThreads;
+        if (i < n && float_order_key(sv[u]) >= T) {
+          const int at = atomicAdd(&sh_m, 1);
+          if (at < fcap) wl[at] = i;
+        }
+      }
     }
     __syncthreads();
     const int mcnt = sh_m;
@@ -2251,18 +2280,34 @@ __global__ void __launch_bounds__(kFinHiThreads) finalize_hi_block_kernel(const 
       }
       continue;
     }
-    if (tid == 0) atomicAdd(&a.ctr[kCtrHiExact], (unsigned long long)mcnt);
-    int p2 = 1;
-    while (p2 < mcnt || p2 < k) p2 <<= 1;
-    for (int i = mcnt + tid; i < p2; i += kFinHiThreads) {
-      fk[i] = 0u;
-      fi[i] = LLONG_MAX;
+    // their exact scores
+    for (int w = tid; w < mcnt; w += kFinHiThreads) {
+      const int i = wl[w];
+      const int32_t pos = pp[i];
+      const uint32_t swd = __ldg(a.scales + pos);
+      const int64_t id = a.ids[pos];
+      const float dot = a.tbl ? fin_row_dot_t(a, pos, rq) : fin_row_dot<G>(a, pos, rq, cbs);
+      const float Gs = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
+      fk[w] = float_order_key(su[i] + Gs * L * (dot - hu) * inv);
+      fi[w] = id;
     }
-    block_bitonic_sort(fk, fi, p2);
-    for (int i = tid; i < k; i += kFinHiThreads) {
-      const bool ok = i < mcnt && fi[i] != LLONG_MAX;
-      a.out_ids[q * k + i] = ok ? fi[i] : -1;
-      a.out_scores[q * k + i] = ok ? float_from_order_key(fk[i]) : -CUDART_INF_F;
+    __syncthreads();
+    if (tid == 0) atomicAdd(&a.ctr[kCtrHiExact], (unsigned long long)mcnt);
+    // the top k by rank: (score desc, id asc) is a strict order, so each
+    // window entry's count of better entries is its place
+    for (int i = tid; i < mcnt; i += kFinHiThreads) {
+      const uint32_t ki = fk[i];
+      const int64_t ii = fi[i];
+      int rank = 0;
+      for (int j = 0; j < mcnt; ++j) rank += better(fk[j], fi[j], ki, ii) ? 1 : 0;
+      if (rank < k) {
+        a.out_ids[q * k + rank] = ii;
+        a.out_scores[q * k + rank] = float_from_order_key(ki);
+      }
+    }
+    for (int i = mcnt + tid; i < k; i += kFinHiThreads) {
+      a.out_ids[q * k + i] = -1;
+      a.out_scores[q * k + i] = -CUDART_INF_F;
     }
   }
 }
@@ -2451,7 +2496,8 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
                o_as = take(size_t(nq) * capA * 4), o_ap = take(size_t(nq) * capA * 4),
                o_ac = take(size_t(nq) * 4), o_bs = take(size_t(nq) * cap * 4),
                o_bp = take(size_t(nq) * cap * 4), o_bc = take(size_t(nq) * 4),
-               o_ovf = take(size_t(nq) * 4), o_work = take(4), o_fcounts = take(8);
+               o_ovf = take(size_t(nq) * 4), o_work = take(4), o_fcounts = take(8),
+               o_tq = take(hi ? size_t(nq) * 4 : 4);
   uint8_t* ws = nullptr;
   cudaError_t e = cudaMallocAsync(reinterpret_cast<void**>(&ws), bytes, s);
   if (e != cudaSuccess) return e;
@@ -2549,6 +2595,8 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
         fa.ctr = ix->d_counters;
         fa.out_ids = out_ids;
         fa.out_scores = out_scores;
+        fa.tq = reinterpret_cast<uint32_t*>(ws + o_tq);
+        fa.zero = 0u;
         // rows of at most 256 coordinates: one warp per query; longer rows:
         // one block per query, whose threads share the window's row decode
         using FK = void (*)(FinHiArgs);
@@ -2573,6 +2621,7 @@ cudaError_t launch_scan_batched(const rslm_index* ix, const float* qrot, int64_t
           if (per_warp)
             fk<<<unsigned((nq + fw - 1) / fw), fw * 32, fsm, s>>>(fa);
           else {
+            finalize_hi_select_kernel<<<unsigned((nq + 3) / 4), 128, 0, s>>>(fa);
             // as many blocks as stay resident (each strides over the queries)
             int per_sm = 1;
             if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, fk, kFinHiThreads, fsm) != cudaSuccess ||

@@ -1111,6 +1111,7 @@ struct RescoreArgs {
   int64_t nq;
   int warps_pre;
   int region;
+  uint32_t zero;  // 0: makes the table lookups depend on a segment pair's loads (all issued first)
 };
 
 __global__ void __launch_bounds__(256) rescore_kernel(const __grid_constant__ RescoreArgs a) {
@@ -1316,31 +1317,42 @@ __global__ void __launch_bounds__(kRsWarps * 32, 1) rescore_mma_kernel(const __g
       }
       float d0[4] = {0.0f, 0.0f, 0.0f, 0.0f}, e0[4] = {0.0f, 0.0f, 0.0f, 0.0f};
       float d1[4] = {0.0f, 0.0f, 0.0f, 0.0f}, e1[4] = {0.0f, 0.0f, 0.0f, 0.0f};
-      uint4 w[4], wn[4];
-      auto load = [&](int J, uint4(&o)[4]) {
-        const bool in = 64 * J + 16 * t < a.stride2;  // rows are whole 16-byte columns
+      // two 64-byte segments per step: their eight loads are issued together
+      // (the lookups' table address depends on all of them; a.zero = 0)
+      for (int J = 0; J < nj; J += 2) {
+        uint4 w[2][4];
 #pragma unroll
-        for (int h = 0; h < 4; ++h)
-          o[h] = rp[h] != nullptr && in ? __ldg(reinterpret_cast<const uint4*>(rp[h] + 64 * J))
-                                        : make_uint4(0u, 0u, 0u, 0u);
-      };
-      load(0, w);
-      for (int J = 0; J < nj; ++J) {
-        if (J + 1 < nj) load(J + 1, wn);
-        uint32_t bq[8][2];
+        for (int jj = 0; jj < 2; ++jj) {
+          const bool in = J + jj < nj && 64 * (J + jj) + 16 * t < a.stride2;  // rows are whole 16-byte columns
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          uint2 v = make_uint2(0u, 0u);
-          if (g < 2) v = *reinterpret_cast<const uint2*>(qblk + ((8 * J + i) * 4 + t) * 16 + 8 * g);
-          bq[i][0] = v.x;
-          bq[i][1] = v.y;
+          for (int h = 0; h < 4; ++h)
+            w[jj][h] = rp[h] != nullptr && in ? __ldg(reinterpret_cast<const uint4*>(rp[h] + 64 * (J + jj)))
+                                              : make_uint4(0u, 0u, 0u, 0u);
         }
-        const uint32_t w0[4] = {w[0].x, w[0].y, w[0].z, w[0].w}, w1[4] = {w[1].x, w[1].y, w[1].z, w[1].w};
-        const uint32_t w2[4] = {w[2].x, w[2].y, w[2].z, w[2].w}, w3[4] = {w[3].x, w[3].y, w[3].z, w[3].w};
-        bt_group_mma(tbl, w0, w1, bq, d0, e0);
-        bt_group_mma(tbl, w2, w3, bq, d1, e1);
+        uint32_t dep = 0u;
 #pragma unroll
-        for (int h = 0; h < 4; ++h) w[h] = wn[h];
+        for (int jj = 0; jj < 2; ++jj)
+#pragma unroll
+          for (int h = 0; h < 4; ++h) dep |= w[jj][h].x | w[jj][h].y | w[jj][h].z | w[jj][h].w;
+        const uint32_t tblj = tbl | (dep & a.zero);
+#pragma unroll
+        for (int jj = 0; jj < 2; ++jj) {
+          if (J + jj >= nj) break;
+          uint32_t bq[8][2];
+#pragma unroll
+          for (int i = 0; i < 8; ++i) {
+            uint2 v = make_uint2(0u, 0u);
+            if (g < 2) v = *reinterpret_cast<const uint2*>(qblk + ((8 * (J + jj) + i) * 4 + t) * 16 + 8 * g);
+            bq[i][0] = v.x;
+            bq[i][1] = v.y;
+          }
+          const uint32_t w0[4] = {w[jj][0].x, w[jj][0].y, w[jj][0].z, w[jj][0].w};
+          const uint32_t w1[4] = {w[jj][1].x, w[jj][1].y, w[jj][1].z, w[jj][1].w};
+          const uint32_t w2[4] = {w[jj][2].x, w[jj][2].y, w[jj][2].z, w[jj][2].w};
+          const uint32_t w3[4] = {w[jj][3].x, w[jj][3].y, w[jj][3].z, w[jj][3].w};
+          bt_group_mma(tblj, w0, w1, bq, d0, e0);
+          bt_group_mma(tblj, w2, w3, bq, d1, e1);
+        }
       }
       // lanes t = 0 hold (hi, lo) of rows g, g + 8 (group 0) and g + 16,
       // g + 24 (group 1); lane L takes row j0 + L
@@ -1608,6 +1620,7 @@ cudaError_t launch_rescore(const rslm_index* ix, const float* qrot2, int64_t nq,
     const int nw = pre + post;
     if (nw >= 4) {
       a.nq = nq;
+      a.zero = 0u;
       a.warps_pre = pre;
       a.region = int(region);
       const size_t bytes = size_t(kBtTableAddr) + size_t(kBtTableBytes) + size_t(post) * region;
