@@ -1131,7 +1131,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       }
     }
   } else {
-    // ---------------- epilogue: thread = row of quadrant warp % 4, columns eh * 32 ..
+    // ---------------- epilogue: thread = row of quadrant warp % 4, columns chunk * 32 ..
     const int quad = warp & 3;
     const int eh = (warp - kDecWarps) >> 2;
     const int row = quad * 32 + lane;
@@ -1151,9 +1151,16 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
       const float* qpair = reinterpret_cast<const float*>(slot(s) + OffQct);
       const float* qinv_s = reinterpret_cast<const float*>(slot(s) + OffQinv);
       const int* qid_s = reinterpret_cast<const int*>(slot(s) + OffQid);
-      // this warp's 32 columns [eh * 32, eh * 32 + 32) hold queries when eh * 32 < nqt
-      const bool active = eh * 32 < nqt;
+      // the item's 32-column chunks: with one (two) of them the four warps
+      // of a quadrant take every fourth (second) tile in turn, so that a
+      // warp's TMEM load and epilogue get several tiles of time
+      const int nch = (nqt + 31) >> 5;
+      const int rot = nch <= 1 ? 4 : nch == 2 ? 2 : 1;
+      const int chunk = nch <= 1 ? 0 : nch == 2 ? (eh & 1) : eh;
+      const int phase = nch <= 1 ? eh : nch == 2 ? (eh >> 1) : 0;
+      const bool has_cols = chunk * 32 < nqt;
       for (int t = 0; t < ntiles; ++t, ++gt) {
+        const bool active = has_cols && int(gt % uint32_t(rot)) == phase;
         const uint32_t b = gt % kAccBufs, u = gt / kAccBufs;  // accumulator
         const int nvalid = min(kMR, nrows - t * kMR);
         const int32_t pos = int32_t(slot0 + int64_t(t) * kMR + row);
@@ -1182,7 +1189,7 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         }
         fence_after_sync();
         float vall[32];
-        if (active) tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(b) + uint32_t(eh * 32), vall);
+        if (active) tmem_ld32(tmem + (uint32_t(quad * 32) << 16) + acc_col(b) + uint32_t(chunk * 32), vall);
         // the accumulator is in registers: release it to the next tile's MMAs
         fence_before_sync();
         __syncwarp();
@@ -1191,10 +1198,10 @@ __global__ void __launch_bounds__(kPipeThreads, 1) batched_pipe_kernel(const __g
         {
           const float* hu_s = reinterpret_cast<const float*>(slot(s) + kOffHu);
           if (HI && L > 0.0f && Gs > 0.0f)
-            epilogue_row_fold<DENSE>(a, vall, Gs * L, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s, hu_s,
+            epilogue_row_fold<DENSE>(a, vall, Gs * L, row, t, nrows, nqt, chunk, pos, qpair, qinv_s, qid_s, hu_s,
                                      reinterpret_cast<const uint32_t*>(slot(s) + kOffKeep));
           else
-            epilogue_row<DENSE, HI>(a, vall, L, Gs, row, t, nrows, nqt, eh, pos, qpair, qinv_s, qid_s, hu_s);
+            epilogue_row<DENSE, HI>(a, vall, L, Gs, row, t, nrows, nqt, chunk, pos, qpair, qinv_s, qid_s, hu_s);
         }
       }
       __syncwarp();
