@@ -2013,10 +2013,18 @@ __device__ uint32_t warp_kth_key(const float* s, int n, int k, uint32_t* hist) {
     const int shift = 24 - 8 * pass;
     for (int i = lane; i < 256; i += 32) hist[i] = 0u;
     __syncwarp();
-    for (int base = 0; base < n; base += 32) {
-      const int i = base + lane;
-      const uint32_t key = i < n ? float_order_key(__ldg(s + i)) : 0u;
-      warp_hist_add(hist, (key >> shift) & 255u, i < n && (key & mask) == prefix);
+    for (int base = 0; base < n; base += 128) {  // four loads in flight per lane
+      uint32_t key[4];
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = base + 32 * u + lane;
+        key[u] = i < n ? float_order_key(__ldg(s + i)) : 0u;
+      }
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int i = base + 32 * u + lane;
+        warp_hist_add(hist, (key[u] >> shift) & 255u, i < n && (key[u] & mask) == prefix);
+      }
     }
     __syncwarp();
     // lane l holds bins 255 - 8 l .. 248 - 8 l (from the top); the first
@@ -2107,21 +2115,24 @@ __global__ void __launch_bounds__(128) finalize_hi_warp_kernel(const __grid_cons
   const uint32_t T = n > k ? warp_kth_key(a.buf_l + q * a.cap, n, k, hist) : 0u;
   // the candidates that can be in the top k, with their exact scores
   int mcnt = 0;
-  for (int base = 0; base < n; base += 32) {
-    const int i = base + lane;
-    const bool in = i < n && float_order_key(su[i]) >= T;
-    const unsigned bm = __ballot_sync(kFull, in);
-    const int at = mcnt + __popc(bm & ((1u << lane) - 1u));
-    if (in && at < fcap) {
-      const int32_t pos = pp[i];
-      const float dot = fin_row_dot<G>(a, pos, rq, cbs);
-      const uint32_t swd = __ldg(a.scales + pos);
-      const float Gs = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
-      const float s = su[i] + Gs * L * (dot - hu) * inv;
-      fk[at] = float_order_key(s);
-      fi[at] = a.ids[pos];
+  // the window's candidate indices (four loads in flight per lane), then
+  // their exact scores in place
+  for (int base = 0; base < n; base += 128) {
+    float sv[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = base + 32 * u + lane;
+      sv[u] = i < n ? su[i] : 0.0f;
     }
-    mcnt += __popc(bm);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+      const int i = base + 32 * u + lane;
+      const bool in = i < n && float_order_key(sv[u]) >= T;
+      const unsigned bm = __ballot_sync(kFull, in);
+      const int at = mcnt + __popc(bm & ((1u << lane) - 1u));
+      if (in && at < fcap) fk[at] = uint32_t(i);
+      mcnt += __popc(bm);
+    }
   }
   if (mcnt > fcap) {
     if (lane == 0) {
@@ -2129,6 +2140,17 @@ __global__ void __launch_bounds__(128) finalize_hi_warp_kernel(const __grid_cons
       atomicAdd(&a.ctr[kCtrBatchedOverflow], 1ull);
     }
     return;
+  }
+  __syncwarp();
+  for (int w = lane; w < mcnt; w += 32) {
+    const int i = int(fk[w]);
+    const int32_t pos = pp[i];
+    const uint32_t swd = __ldg(a.scales + pos);
+    const int64_t id = a.ids[pos];
+    const float dot = fin_row_dot<G>(a, pos, rq, cbs);
+    const float Gs = ue4m12_to_f32(swd >> 16), L = ue7m9_to_f32(swd & 0xffffu);
+    fk[w] = float_order_key(su[i] + Gs * L * (dot - hu) * inv);
+    fi[w] = id;
   }
   if (lane == 0) atomicAdd(&a.ctr[kCtrHiExact], (unsigned long long)mcnt);
   __syncwarp();

@@ -274,17 +274,6 @@ __device__ __forceinline__ void warp_hist_add(uint32_t* hist, uint32_t bin, bool
   if ((threadIdx.x & 31) == __ffs(peers) - 1) atomicAdd(&hist[bin], uint32_t(__popc(peers)));
 }
 
-// A 16-byte read-only global load issued in program order with the other
-// volatile asm of the caller, so that loads meant to be in flight together
-// are issued before the code that consumes earlier ones.
-__device__ __forceinline__ uint4 ldg_v4_ordered(const void* p) {
-  uint4 v;
-  asm volatile("ld.global.nc.v4.u32 {%0, %1, %2, %3}, [%4];"
-               : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w)
-               : "l"(p));
-  return v;
-}
-
 __device__ __forceinline__ void set_device_error(int* err, int code) {
   if (err) atomicCAS(err, 0, code);
 }
