@@ -107,3 +107,24 @@ def test_exact_topk_and_recall_at():
     r = ex.recall(truth[:, :10], found)
     assert r["recall_k_at_k"] == 1.0 and r["recall_1_at_k"] == 1.0
     assert (r["recall_20_at_20"], r["recall_20_at_30"], r["recall_20_at_40"]) == (0.75, 0.75, 0.75)
+
+
+def test_traffic_records_are_consistent():
+    """Each ncu traffic record states its bytes per candidate as (read +
+    write) / candidates, names the command that captured it, and is looked
+    up only while its kernel's sources are unchanged (hash match)."""
+    b = _bench()
+    with open(os.path.join(ROOT, "profiles", "scan_kernel_traffic.json")) as f:
+        recs = json.load(f)
+    assert recs
+    for key, r in recs.items():
+        cfg, _, kernel = key.partition("/")
+        assert kernel in b.SCAN_SOURCES, key
+        assert r["command"].startswith("ncu ") and "--clock-control none" in r["command"], key
+        per = (r["dram_bytes_read"] + r["dram_bytes_write"]) / r["candidates"]
+        assert abs(per - r["dram_bytes_per_candidate"]) <= 1e-9 * per, key
+        got = b.traffic_record(cfg, kernel)
+        if r.get("kernel_hash") == b.scan_source_hash(kernel):
+            assert got is not None and got["dram_bytes_per_candidate"] == r["dram_bytes_per_candidate"], key
+        else:
+            assert got is None, key
