@@ -339,8 +339,22 @@ def run_reference(args):
 
 
 # ------------------------------------------------------------------- GPU arm
-def launches_per_step(w: W.Workload, nq: int, batched: bool) -> int:
-    """Kernels of librslm launched by one step."""
+def finalize_launches(desc: dict, lite: bool) -> int:
+    """Finalize kernels of the batched regime: the hi-only mode (4-bit codes
+    without the Rslm4Lite head; padded D <= 128 also needs one coordinate
+    per code in 16-byte chunks) finalizes rows of at most 256 coordinates
+    with one warp kernel and longer rows with a select kernel and a block
+    kernel; the other formats take the warp kernel and its block fallback."""
+    g, bits = desc["group"], desc["score_bits"]
+    dp16 = (desc["padded_dim"] + 15) // 16 * 16
+    stride = (desc["code_bytes"] + 3) // 4 * 4
+    chunk = 16 if stride % 16 == 0 else 8 if stride % 8 == 0 else 4
+    hi = bits != 3 and not lite and ((g == 1 and chunk == 16) if dp16 <= 128 else True)
+    return 1 if hi and 2 * g * stride <= 256 else 2
+
+
+def launches_per_step(w: W.Workload, nq: int, batched: bool, fin: int = 2) -> int:
+    """Kernels of librslm launched by one step (fin: finalize kernels)."""
     if (w.D + 15) // 16 * 16 <= 128 and w.P >= 32 * w.nprobe and w.nprobe <= 256:
         n = 4                # fused probe: query operands, two-pass probe, list selection,
                              # exact fallback for overflowed lists
@@ -352,10 +366,10 @@ def launches_per_step(w: W.Workload, nq: int, batched: bool) -> int:
         # hands over (nprobe <= 256)
         n = math.ceil(nq / qc) * (4 if w.nprobe <= 256 else 3)
     n += 1                   # query rotation
-    # batched: two probe-list inversions (count, list scan, item table,
-    # scatter), query split, first-probe pass, threshold, tensor-core scan,
-    # finalize (warp kernel + block fallback), overflow re-scan; else one scan
-    n += 8 + 1 + 1 + 1 + 1 + 2 + 1 if batched else 1
+    # batched: two probe-list inversions (pair histograms, segment sums,
+    # prefix, scatter, list scan, item table), query split, first-probe pass,
+    # threshold, tensor-core scan, finalize, overflow re-scan; else one scan
+    n += 12 + 1 + 1 + 1 + 1 + fin + 1 if batched else 1
     if w.rescore_bits:
         n += 2               # second rotation + rescore
     return n
@@ -635,7 +649,7 @@ def run_gpu(args):
             "gemv": gemv,
             "cpu_baseline": cpu,
             "e2e": e2e,
-            "gpu_launches": launches_per_step(w, nq, batched) * args.steps,
+            "gpu_launches": launches_per_step(w, nq, batched, finalize_launches(desc, args.lite)) * args.steps,
             "clocks": clocks,
             "recall": recall,
             # index event counters over the whole run (warm-up and timed
