@@ -128,3 +128,21 @@ def test_traffic_records_are_consistent():
             assert got is not None and got["dram_bytes_per_candidate"] == r["dram_bytes_per_candidate"], key
         else:
             assert got is None, key
+
+
+def test_launch_count_matches_the_profiled_lists():
+    """gpu_launches per step for C4 and C5 equals the kernel launches of one
+    search in the committed launch lists (23 and 38: probe, rotation, two
+    list inversions, split, two passes, threshold, finalize, re-scan, and
+    for C5 the GEMM probe chunks, the second rotation and the rescoring)."""
+    b = _bench()
+    import paper_2608_30384_gb300.workloads as W
+
+    def desc(bits, D):
+        g = {1: 4, 2: 2, 4: 1}[bits]
+        Dp = (D + g - 1) // g * g
+        return {"group": g, "score_bits": bits, "padded_dim": Dp, "code_bytes": (Dp // g + 1) // 2}
+
+    for name, want in (("C4", 23), ("C5", 38)):
+        w = W.WORKLOADS[name]
+        assert b.launches_per_step(w, w.nq, True, b.finalize_launches(desc(w.bits, w.D), False)) == want, name
